@@ -1,0 +1,436 @@
+#!/usr/bin/env python
+"""Benchmark: circuit evaluations/s of the batched statevector engine on GB300.
+
+One step = one pass of the whole hot path over one batch: forward sweep to
+per-qubit <Z> (saving the final state) plus the adjoint backward to dL/dx and
+dL/dw, for the 8-qubit / 4-layer / batch-1024 complex64 workload (RY(x)
+encoding, RX RY RZ per qubit per layer, CZ ring).  Inputs are seeded and
+synthetic.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun (N > 1) every rank runs the same per-rank batch (weak scaling);
+the shared-weight gradient is summed across ranks with one all-reduce per step.
+Rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "circuit evals/sec (fwd; fwd+adjoint bwd) at 4-16 qubits; % of roofline"
+FP32_LANES_PER_SM = 128
+NUM_SMS = 152
+SM_MAX_MHZ = 2070.0
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    except Exception:
+        return {"hbm_gbs": 6800.0, "sm_max_mhz": SM_MAX_MHZ}, "fallback"
+
+
+def fp32_peak_tflops(sm_mhz):
+    # FP32 CUDA-core peak: SMs x 128 lanes x 2 flop (FFMA) x clock
+    return NUM_SMS * FP32_LANES_PER_SM * 2 * sm_mhz * 1e6 / 1e12
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index, self.proc, self.lines = index, None, []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.1)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def workload(cfg=2):
+    from paper_2607_11985_gb300 import workloads as wl
+    return wl.config(cfg)[0]
+
+
+# ------------------------------------------------------------------ CPU oracle baseline
+def oracle_rate(w_, seconds=12.0, chunk=16, backward=True):
+    """Oracle fwd(+bwd) evaluations/s on the host (single thread), on a bounded
+    sample of the workload's rows."""
+    from oracle import oracle as orc
+    done, t0, row = 0, time.perf_counter(), 0
+    while time.perf_counter() - t0 < seconds:
+        rows = [(row + i) % w_.batch for i in range(chunk)]
+        x = w_.x[rows]
+        orc.forward(w_.spec, x, w_.w)
+        if backward:
+            orc.backward(w_.spec, x, w_.w, w_.gE[rows])
+        done += chunk
+        row += chunk
+    dt = time.perf_counter() - t0
+    return done / dt, done, dt
+
+
+# ------------------------------------------------------------------ our engine
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+    import __graft_entry__
+    from paper_2607_11985_gb300 import binding as B
+    from paper_2607_11985_gb300.circuit import Circuit
+
+    __graft_entry__.build()
+    torch.cuda.set_device(local_rank)
+    w_ = workload(args.config)
+    Bt = w_.batch
+    c = Circuit(w_.spec, "c64")
+    info = c.info(Bt)
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+    x = torch.tensor(w_.x, dtype=torch.float32, device="cuda")
+    w = torch.tensor(w_.w, dtype=torch.float32, device="cuda")
+    gE = torch.tensor(w_.gE, dtype=torch.float32, device="cuda")
+    E = torch.empty(Bt, w_.spec.n, dtype=torch.float32, device="cuda")
+    st = torch.empty(Bt, 1 << w_.spec.n, dtype=torch.complex64, device="cuda")
+    dx = torch.empty_like(x)
+    dw = torch.empty_like(w)
+    ws, wsb = c.workspace(Bt, 1, stream)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")   # > 129 MB L2
+
+    def step():
+        B.vqc_forward(c.plan, Bt, x.data_ptr(), w.data_ptr(), None, E.data_ptr(), st.data_ptr(),
+                      None, 0, sp)
+        B.vqc_backward(c.plan, Bt, x.data_ptr(), w.data_ptr(), None, st.data_ptr(), gE.data_ptr(),
+                       dx.data_ptr(), dw.data_ptr(), ws.data_ptr(), wsb, sp)
+
+    for _ in range(args.warmup):
+        step()
+        if world > 1:
+            dist.all_reduce(dw)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    sampler = ClockSampler(local_rank)
+    if rank == 0:
+        sampler.start()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    torch.cuda._sleep(int(50e-3 * SM_MAX_MHZ * 1e6))   # queue work ahead of the GPU
+    t_wall = time.perf_counter()
+    for i in range(K):
+        flush.zero_()                                   # L2 flush, outside the step events
+        e0, e1, e2 = ev[i]
+        e0.record(stream)
+        B.vqc_forward(c.plan, Bt, x.data_ptr(), w.data_ptr(), None, E.data_ptr(), st.data_ptr(),
+                      None, 0, sp)
+        e1.record(stream)
+        B.vqc_backward(c.plan, Bt, x.data_ptr(), w.data_ptr(), None, st.data_ptr(), gE.data_ptr(),
+                       dx.data_ptr(), dw.data_ptr(), ws.data_ptr(), wsb, sp)
+        if world > 1:
+            dist.all_reduce(dw)
+        e2.record(stream)
+    torch.cuda.synchronize()
+    t_wall = time.perf_counter() - t_wall
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop() if rank == 0 else None
+    fwd_ms = [a.elapsed_time(b) for a, b, _ in ev]
+    bwd_ms = [b.elapsed_time(cc) for _, b, cc in ev]
+    step_ms = [a.elapsed_time(cc) for a, _, cc in ev]
+    total_ms = float(sum(step_ms))
+    tot = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(tot, op=dist.ReduceOp.MAX)
+    total_ms = float(tot.item())
+    ms_per_step = total_ms / K
+    value = world * Bt * K / (total_ms / 1e3)
+
+    # ---- end to end through the public API: pinned host inputs in, results out
+    xh = torch.tensor(w_.x, dtype=torch.float32).pin_memory()
+    wh = torch.tensor(w_.w, dtype=torch.float32).pin_memory()
+    gh = torch.tensor(w_.gE, dtype=torch.float32).pin_memory()
+    Eh = torch.empty(Bt, w_.spec.n, dtype=torch.float32).pin_memory()
+    dxh = torch.empty_like(xh).pin_memory()
+    dwh = torch.empty_like(wh).pin_memory()
+    h2d = xh.numel() * 4 + wh.numel() * 4 + gh.numel() * 4
+    d2h = Eh.numel() * 4 + dxh.numel() * 4 + dwh.numel() * 4
+
+    def e2e_step():
+        xd = xh.to("cuda", non_blocking=True)
+        wd = wh.to("cuda", non_blocking=True)
+        gd = gh.to("cuda", non_blocking=True)
+        Ed, sd = c.forward(xd, wd, want_state=True)
+        dxd, dwd = c.backward(xd, wd, gd, psi_final=sd)
+        if world > 1:
+            dist.all_reduce(dwd)
+        Eh.copy_(Ed, non_blocking=True)
+        dxh.copy_(dxd, non_blocking=True)
+        dwh.copy_(dwd, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+
+    for _ in range(max(3, args.warmup // 4)):
+        e2e_step()
+    Ke = max(10, min(K, 500))
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(Ke):
+        e2e_step()
+    e2e_s = time.perf_counter() - t0
+    t = torch.tensor([e2e_s], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    e2e_value = world * Bt * Ke / float(t.item())
+    E_check = float(np.max(np.abs(Eh.numpy()))) if Eh.numel() else 0.0
+    assert np.isfinite(E_check)
+
+    if rank != 0:
+        return None
+
+    pk, pk_kind = peaks()
+    peak = fp32_peak_tflops(pk.get("sm_max_mhz", SM_MAX_MHZ))
+    bwd_avg_s = statistics.mean(bwd_ms) / 1e3
+    fwd_avg_s = statistics.mean(fwd_ms) / 1e3
+    bwd_flops = info["bwd_flops_per_eval"] * Bt
+    fwd_flops = info["fwd_flops_per_eval"] * Bt
+    ach_bwd = bwd_flops / bwd_avg_s / 1e12
+    ach_fwd = fwd_flops / fwd_avg_s / 1e12
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tpath):
+        with open(tpath) as f:
+            tj = json.load(f)
+        key = "%s:%s" % (w_.name, "bwd")
+        if key in tj and tj[key].get("digest") == info_digest():
+            traffic = tj[key]["bytes_per_launch"]
+    out = {
+        "metric": METRIC,
+        "value": value,
+        "unit": "circuit evals/s (fwd+adjoint bwd)",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": args.warmup,
+        "ms_per_step": ms_per_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "c64 (fp32 arithmetic)",
+        "data": "synthetic (seeded; RY(x) encoding + RX/RY/RZ layers + CZ ring)",
+        "config": {"workload": w_.name, "qubits": w_.spec.n, "layers": 4, "batch_per_gpu": Bt,
+                   "gates": len(w_.spec.gates), "num_x": w_.spec.num_x, "num_w": w_.spec.num_w,
+                   "parallelism": "dp%d (batch-sharded replicas, dw all-reduce)" % world,
+                   "l2": "flushed between steps (256 MiB write) outside the per-step CUDA events",
+                   "fwd_k": info["fwd_k"], "bwd_k": info["bwd_k"],
+                   "fwd_stages": info["fwd_stages"], "bwd_stages": info["bwd_stages"]},
+        "fwd": {"value": world * Bt / fwd_avg_s, "unit": "circuit evals/s (fwd)",
+                "ms": fwd_avg_s * 1e3, "tflops": ach_fwd},
+        "roofline": {"kernel": "sweep_kernel<float,K=%d,bwd>" % info["bwd_k"], "bound": "alu",
+                     "achieved": ach_bwd, "peak": peak, "unit": "TFLOP/s",
+                     "frac": ach_bwd / peak, "traffic": traffic,
+                     "peak_basis": "FP32 FFMA: 152 SMs x 128 lanes x 2 x %.0f MHz (%s sm_max_mhz)"
+                                   % (pk.get("sm_max_mhz", SM_MAX_MHZ), pk_kind),
+                     "flops_per_launch": bwd_flops, "launch_ms": bwd_avg_s * 1e3,
+                     "fwd_frac": ach_fwd / peak},
+        "e2e": {"value": e2e_value, "unit": "circuit evals/s (fwd+adjoint bwd, host buffers)",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": Ke},
+        "gpu_launches": 2 * K,
+        "clocks": clocks,
+        "wall_s_timed_loop": t_wall,
+    }
+    if not args.no_cpu_baseline:
+        rate, done, dt = oracle_rate(w_, seconds=args.cpu_seconds)
+        out["cpu_baseline"] = {"value": rate, "unit": "circuit evals/s (fwd+adjoint bwd)",
+                               "cores": 1, "kind": "oracle",
+                               "sample": "%d rows of the workload (cycled), fwd+bwd, %.1f s"
+                                         % (done, dt)}
+    if args.extra:
+        out["configs"] = extra_configs(torch, Circuit, B)
+    return out
+
+
+_DIGEST = None
+
+
+def info_digest():
+    global _DIGEST
+    if _DIGEST is None:
+        from paper_2607_11985_gb300 import build
+        _DIGEST = build._sources_digest()[:16]
+    return _DIGEST
+
+
+def extra_configs(torch, Circuit, B):
+    """Forward and fwd+bwd evaluations/s of the other workloads (quick, device-timed)."""
+    from paper_2607_11985_gb300 import workloads as wl
+    res = {}
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    for k in (1, 3, 4):
+        try:
+            ws_ = wl.config(k)[:4] if k == 4 else wl.config(k)
+            tot_f, tot_b, evals, flops_f, flops_b = 0.0, 0.0, 0, 0.0, 0.0
+            for w_ in ws_:
+                c = Circuit(w_.spec, "c64")
+                inf = c.info(w_.batch)
+                x = torch.tensor(w_.x, dtype=torch.float32, device="cuda")
+                w = torch.tensor(w_.w, dtype=torch.float32, device="cuda") if w_.spec.num_w else None
+                gE = torch.tensor(w_.gE, dtype=torch.float32, device="cuda")
+                E, st = c.forward(x, w, want_state=True)
+                if w_.backward:
+                    c.backward(x, w, gE, psi_final=st)
+                torch.cuda.synchronize()
+                n_rep = 5
+                for _ in range(n_rep):
+                    flush.zero_()
+                    a, b2, d = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+                    a.record()
+                    c.forward(x, w, out=E, state_out=st)
+                    b2.record()
+                    if w_.backward:
+                        c.backward(x, w, gE, psi_final=st)
+                    d.record()
+                    torch.cuda.synchronize()
+                    tot_f += a.elapsed_time(b2) / 1e3
+                    tot_b += b2.elapsed_time(d) / 1e3
+                evals += n_rep * w_.batch
+                flops_f += n_rep * w_.batch * inf["fwd_flops_per_eval"]
+                flops_b += n_rep * w_.batch * inf["bwd_flops_per_eval"]
+                del c
+            res["cfg%d" % k] = {"fwd_evals_per_s": evals / tot_f,
+                                "fwd_tflops": flops_f / tot_f / 1e12,
+                                "fwd_bwd_evals_per_s": (evals / (tot_f + tot_b)) if tot_b else None,
+                                "bwd_tflops": (flops_b / tot_b / 1e12) if tot_b else None,
+                                "circuits": len(ws_)}
+        except Exception as e:   # report, do not hide
+            res["cfg%d" % k] = {"error": str(e)[:200]}
+    return res
+
+
+# ------------------------------------------------------------------ reference arm
+def run_reference(args, rank, world):
+    """The oracle on the host cores, same metric and workload (bounded sample)."""
+    if rank != 0:
+        return None
+    w_ = workload(args.config)
+    chunk = 8
+    from oracle import oracle as orc
+    orc.build()
+    for _ in range(args.warmup):
+        orc.forward(w_.spec, w_.x[:1], w_.w)
+    times, row = [], 0
+    for _ in range(args.steps):
+        rows = [(row + i) % w_.batch for i in range(chunk)]
+        t0 = time.perf_counter()
+        orc.forward(w_.spec, w_.x[rows], w_.w)
+        orc.backward(w_.spec, w_.x[rows], w_.w, w_.gE[rows])
+        times.append(time.perf_counter() - t0)
+        row += chunk
+    total = sum(times)
+    value = chunk * args.steps / total
+    return {"metric": METRIC, "value": value, "unit": "circuit evals/s (fwd+adjoint bwd)",
+            "impl": "reference", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": total / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "c128 (fp64 arithmetic)",
+            "data": "synthetic (seeded)", "config": {"workload": w_.name, "qubits": w_.spec.n,
+                                                    "batch_per_step": chunk},
+            "cpu_baseline": {"value": value, "unit": "circuit evals/s (fwd+adjoint bwd)",
+                             "cores": 1, "kind": "oracle",
+                             "sample": "%d steps x %d rows of the workload" % (args.steps, chunk)},
+            "e2e": {"value": value, "unit": "circuit evals/s (fwd+adjoint bwd)",
+                    "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", type=int, default=2)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--extra", action="store_true", help="also time configs 1, 3, 4")
+    args = ap.parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        out = run_reference(args, rank, world)
+        if out is not None:
+            print(json.dumps(out))
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    out = run_ours(args, rank, world, local_rank)
+    if out is not None:
+        print(json.dumps(out))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

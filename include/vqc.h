@@ -1,0 +1,211 @@
+/*
+ * vqc.h -- C ABI of the GB300 batched statevector engine for static
+ * parametrised quantum circuits.
+ *
+ * The operation (paper, Alg. 1 "Compile-Once Lowering and Batched Execution",
+ * and Sec. 3 "Compile-Once Lowering and Execution"):
+ *   compile once:  a static gate list (no measurement, no classical control,
+ *                  only angles vary; Sec. 3 "Static Circuit Scope") is lowered
+ *                  to a plan; constant gates are pre-multiplied into cached
+ *                  matrices, parametrised gates stay symbolic (Alg. 1, compile
+ *                  phase).
+ *   execute:       for a batch of B samples, psi_b = U_G ... U_1 psi0_b with
+ *                  psi0_b = |0...0> unless given, and
+ *                  E[b, j] = sum_k (-1)^{k_j} |psi_b[k]|^2     (Alg. 1, execute
+ *                  phase and return statement).
+ *   differentiate: for L = sum_{b,j} gE[b, j] * E[b, j], dL/dx[b, .] for the
+ *                  per-sample angles and dL/dw[.] for the shared angles
+ *                  (Sec. 3 "Gate Application and Differentiation": gradients
+ *                  with respect to trainable parameters).  The engine uses the
+ *                  adjoint method (two states, O(B 2^n) memory) where the paper
+ *                  used autograd (O(B G 2^n) memory, Sec. 3 "Complexity and
+ *                  Tradeoffs").
+ *
+ * Conventions.  Qubit q is bit q of the amplitude index (little endian).  A
+ * gate list is in time order.  States are interleaved (re, im) pairs: float2
+ * for VQC_C64, double2 for VQC_C128; arrays are row-major and sample-major.
+ * Real arrays (x, w, E, gradients) are float for VQC_C64 and double for
+ * VQC_C128.  Gate matrices: RX/RY/RZ(t) = exp(-i t P / 2); U3 is
+ * [[c, -e^{i l} s], [e^{i p} s, e^{i(p+l)} c]] with c, s = cos, sin(t/2);
+ * CRZ(t) = |0><0|_q0 (x) I + |1><1|_q0 (x) RZ_q1(t); RZZ(t) = exp(-i t Z Z / 2);
+ * CX/CRZ control is q0, target q1.
+ *
+ * Ownership.  The caller owns every device buffer and the CUDA stream.
+ * vqc_compile copies the gate list; the plan owns its host and device copies
+ * and is released with vqc_free.  Calls are stream-ordered and asynchronous:
+ * a returned VQC_OK means the work was enqueued.  No C++ exception crosses
+ * this ABI.  A plan may be used from several threads; calls that share a
+ * workspace must be ordered on one stream.
+ *
+ * Errors.  Every call returns a vqc_status; vqc_last_error() gives a
+ * thread-local message for the last failing call on the calling thread.
+ */
+#ifndef VQC_ABI_H_INCLUDED
+#define VQC_ABI_H_INCLUDED
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define VQC_ABI_VERSION 1
+#define VQC_MAX_QUBITS 24
+
+typedef struct vqc_plan vqc_plan;   /* opaque */
+
+typedef enum {
+    VQC_OK = 0,
+    VQC_ERR_INVALID_ARG = 1,       /* NULL where a pointer is required, bad size or dtype */
+    VQC_ERR_UNSUPPORTED_GATE = 2,  /* opcode outside vqc_gate_op */
+    VQC_ERR_QUBIT_RANGE = 3,       /* qubit >= num_qubits, or q0 == q1 on a 2q gate */
+    VQC_ERR_TOO_MANY_QUBITS = 4,   /* num_qubits outside 1..VQC_MAX_QUBITS */
+    VQC_ERR_PARAM_RANGE = 5,       /* angle source kind or index out of range */
+    VQC_ERR_OUT_OF_MEMORY = 6,     /* host or device allocation failed */
+    VQC_ERR_CUDA = 7,              /* a CUDA runtime call failed (message has the name) */
+    VQC_ERR_WORKSPACE = 8,         /* workspace NULL, too small or not 256-byte aligned */
+    VQC_ERR_DEVICE_CHECK = 9,      /* a kernel's own bounds/consistency check tripped */
+    VQC_ERR_UNSUPPORTED = 10       /* valid request this build cannot run (e.g. too large) */
+} vqc_status;
+
+typedef enum { VQC_C64 = 0, VQC_C128 = 1 } vqc_dtype;
+
+/* The 16-gate set.  Angles per gate: RX/RY/RZ/CRZ/RZZ one (theta),
+ * U3 three (theta, phi, lambda), the rest none. */
+typedef enum {
+    VQC_H = 0, VQC_X = 1, VQC_Y = 2, VQC_Z = 3, VQC_S = 4, VQC_T = 5, VQC_SX = 6,
+    VQC_RX = 7, VQC_RY = 8, VQC_RZ = 9, VQC_U3 = 10,
+    VQC_CX = 11, VQC_CZ = 12, VQC_SWAP = 13, VQC_CRZ = 14, VQC_RZZ = 15,
+    VQC_NUM_GATE_OPS = 16
+} vqc_gate_op;
+
+/* Source of one angle (Alg. 1 compile phase: constant gates are cached,
+ * parametric gates are instantiated from theta at run time). */
+typedef enum {
+    VQC_P_NONE = 0,    /* unused slot */
+    VQC_P_CONST = 1,   /* pconst[i] */
+    VQC_P_X = 2,       /* per-sample angle x[b, pidx[i]] */
+    VQC_P_W = 3        /* shared angle w[pidx[i]] */
+} vqc_pkind;
+
+/* One gate of the input list (48 bytes, natural alignment, no implicit padding). */
+typedef struct {
+    uint8_t op;          /* vqc_gate_op */
+    uint8_t q0;          /* first qubit (control of CX / CRZ) */
+    uint8_t q1;          /* second qubit (target); ignored for 1q gates */
+    uint8_t pkind[3];    /* vqc_pkind of each angle slot; slots beyond the gate's arity ignored */
+    uint8_t reserved[2]; /* must be zero */
+    int32_t pidx[3];     /* column of x or index of w for VQC_P_X / VQC_P_W */
+    int32_t reserved2;   /* must be zero */
+    double pconst[3];    /* angle for VQC_P_CONST */
+} vqc_gate;
+
+/* Execution paths a plan can take. */
+typedef enum {
+    VQC_PATH_RESIDENT = 0,  /* each sample's state stays in one CTA's shared memory */
+    VQC_PATH_HBM = 1        /* state in HBM, swept in shared-memory tiles, one launch per pass */
+} vqc_path;
+
+typedef struct {
+    int32_t num_qubits, num_x, num_w, dtype;
+    int32_t num_gates_in;        /* gates given to vqc_compile */
+    int32_t num_ops;             /* fused ops after lowering (1q runs, CX, CZ, phase ops) */
+    int32_t num_runs;            /* fused single-qubit runs */
+    int32_t num_terms;           /* parametrised angle occurrences carrying a gradient */
+    int32_t fwd_path, bwd_path;  /* vqc_path chosen for the batch given to vqc_plan_info (-1: none) */
+    int32_t fwd_k, bwd_k;        /* register-block qubits per thread */
+    int32_t fwd_stages, bwd_stages;
+    int32_t fwd_passes, bwd_passes;      /* HBM passes (1 on the resident path) */
+    int32_t fwd_threads_per_sample, bwd_threads_per_sample;
+    int32_t fwd_tile_qubits, bwd_tile_qubits;
+    double fwd_flops_per_eval;   /* algorithmic flops of one forward evaluation */
+    double bwd_flops_per_eval;   /* algorithmic flops of one backward evaluation (from psi_final) */
+    double recompute_flops_per_eval;     /* extra flops when the backward recomputes psi_final */
+    double fwd_hbm_bytes_per_eval;       /* state bytes moved through HBM per forward evaluation */
+    double bwd_hbm_bytes_per_eval;
+} vqc_plan_stats;
+
+/* Compile a gate list (paper, Alg. 1 compile phase).  Validates every gate,
+ * fuses runs of single-qubit gates, pre-multiplies constant matrices, and
+ * builds the register-block stage schedules.  When the process sees a CUDA
+ * device, uploads the plan to the current device (one synchronous copy);
+ * otherwise the plan is host-only (vqc_plan_info / vqc_plan_export work) and
+ * the first vqc_forward / vqc_backward uploads it, so that first call must
+ * not be made inside CUDA stream capture.  On success *out_plan owns the result.
+ * Errors: VQC_ERR_INVALID_ARG (NULL gates with num_gates > 0, NULL out_plan,
+ * negative counts, bad dtype, nonzero reserved bytes), VQC_ERR_UNSUPPORTED_GATE,
+ * VQC_ERR_QUBIT_RANGE, VQC_ERR_TOO_MANY_QUBITS, VQC_ERR_PARAM_RANGE,
+ * VQC_ERR_OUT_OF_MEMORY, VQC_ERR_CUDA. */
+vqc_status vqc_compile(const vqc_gate* gates, int32_t num_gates, int32_t num_qubits,
+                       int32_t num_x, int32_t num_w, vqc_dtype dtype, vqc_plan** out_plan);
+
+/* Release a plan (NULL-safe).  The caller must make sure no enqueued call
+ * still uses it (synchronise the streams first). */
+void vqc_free(vqc_plan* plan);
+
+/* Bytes of device workspace a call needs: mode 0 = vqc_forward, 1 = vqc_backward.
+ * Returns 0 when no workspace is needed; (size_t)-1 for a NULL plan. */
+size_t vqc_workspace_bytes(const vqc_plan* plan, int32_t batch, int32_t mode);
+
+/* Zero a workspace's control block on `stream` (enqueued memset).  A freshly
+ * allocated workspace must be initialised once with this call (or zeroed by
+ * the caller) before its first use; every call leaves it initialised. */
+vqc_status vqc_workspace_init(void* workspace, size_t workspace_bytes, void* stream);
+
+/* Forward sweep (paper, Alg. 1 execute phase).
+ *   batch     B >= 0 (B == 0 enqueues nothing).
+ *   x         device [B, num_x] real, or NULL when num_x == 0.
+ *   w         device [num_w] real, or NULL when num_w == 0.
+ *   psi0      device [B, 2^n] complex initial states, or NULL for |0...0>.
+ *   expz_out  device [B, n] real: E[b, j] (required).
+ *   state_out device [B, 2^n] complex final states, or NULL.
+ *   workspace device scratch of vqc_workspace_bytes(plan, B, 0) bytes, 256-byte
+ *             aligned (may be NULL when that size is 0).
+ *   stream    cudaStream_t (NULL = legacy default stream).
+ * Buffers must not overlap, except that state_out may equal psi0. */
+vqc_status vqc_forward(const vqc_plan* plan, int32_t batch, const void* x, const void* w,
+                       const void* psi0, void* expz_out, void* state_out,
+                       void* workspace, size_t workspace_bytes, void* stream);
+
+/* Adjoint backward (paper, Sec. 3 gradients).  For L = sum gE * E:
+ *   psi_final device [B, 2^n] complex: the state_out of a vqc_forward with the
+ *             same plan, x, w and psi0, or NULL to recompute it in the kernel.
+ *   grad_expz device [B, n] real gE (required).
+ *   grad_x    device [B, num_x] real, overwritten with dL/dx (or NULL: not computed).
+ *   grad_w    device [num_w] real, overwritten with dL/dw summed over the
+ *             batch in a fixed order (deterministic for a given plan and B),
+ *             or NULL.
+ *   workspace vqc_workspace_bytes(plan, B, 1) bytes, 256-byte aligned,
+ *             initialised once with vqc_workspace_init.
+ * Other arguments as vqc_forward. */
+vqc_status vqc_backward(const vqc_plan* plan, int32_t batch, const void* x, const void* w,
+                        const void* psi0, const void* psi_final, const void* grad_expz,
+                        void* grad_x, void* grad_w, void* workspace, size_t workspace_bytes,
+                        void* stream);
+
+/* Plan statistics (paths, stage counts, algorithmic flop and byte counts per
+ * evaluation) for a batch of `batch` samples. */
+vqc_status vqc_plan_info(const vqc_plan* plan, int32_t batch, vqc_plan_stats* out);
+
+/* Serialise the host plan (fused ops, runs, constituents, term table and all
+ * stage schedules) into buf.  *inout_bytes holds buf's capacity on entry and
+ * the bytes needed on return; buf may be NULL to query the size.  The bytes
+ * are a deterministic function of the vqc_compile arguments. */
+vqc_status vqc_plan_export(const vqc_plan* plan, void* buf, size_t* inout_bytes);
+
+/* Synchronise `stream` and report any CUDA error or tripped device check
+ * raised by enqueued work on plans of this process. */
+vqc_status vqc_sync_check(void* stream);
+
+/* Thread-local message of the last failing call ("" if none). */
+const char* vqc_last_error(void);
+
+/* VQC_ABI_VERSION of the loaded library. */
+int32_t vqc_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VQC_ABI_H_INCLUDED */

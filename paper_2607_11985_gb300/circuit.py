@@ -1,0 +1,137 @@
+"""PyTorch-facing wrapper: compile once, then run batches through the C ABI.
+
+``Circuit`` holds one compiled plan (paper, Alg. 1 compile phase: the gate
+list is lowered once and the result cached) and calls ``vqc_forward`` /
+``vqc_backward`` on torch CUDA tensors.  Torch supplies device memory and the
+current stream only; every step of the sweep runs in the library's kernels.
+``VQCFunction`` makes the forward differentiable with the adjoint backward.
+"""
+from __future__ import annotations
+
+import torch
+
+from . import binding as B
+
+_DT = {"c64": (B.VQC_C64, torch.float32, torch.complex64),
+       "c128": (B.VQC_C128, torch.float64, torch.complex128)}
+
+
+def _ptr(t):
+    return None if t is None else t.data_ptr()
+
+
+class Circuit:
+    """A compiled static circuit (see ``workloads.CircuitSpec`` for the format)."""
+
+    def __init__(self, spec, dtype: str = "c64"):
+        if dtype not in _DT:
+            raise ValueError("dtype must be 'c64' or 'c128'")
+        self.spec = spec
+        self.n, self.num_x, self.num_w = int(spec.n), int(spec.num_x), int(spec.num_w)
+        self.dtype = dtype
+        self.code, self.real, self.cplx = _DT[dtype]
+        self._gates = B.gates_array(spec)
+        self.plan = B.vqc_compile(self._gates, len(spec.gates), self.n, self.num_x, self.num_w,
+                                  self.code)
+        self._ws = {}
+
+    def __del__(self):
+        plan = getattr(self, "plan", None)
+        if plan:
+            try:
+                torch.cuda.synchronize()
+            except Exception:
+                pass
+            B.vqc_free(plan)
+            self.plan = None
+
+    # ------------------------------------------------------------------ helpers
+    def info(self, batch: int = 1) -> dict:
+        return B.vqc_plan_info(self.plan, batch)
+
+    def export(self) -> bytes:
+        return B.vqc_plan_export(self.plan)
+
+    def _check(self, t, dtype, shape, name):
+        if t is None:
+            return None
+        if not t.is_cuda or t.dtype != dtype or tuple(t.shape) != tuple(shape):
+            raise ValueError("%s must be a CUDA %s tensor of shape %s (got %s %s %s)"
+                             % (name, dtype, tuple(shape), t.device, t.dtype, tuple(t.shape)))
+        return t.contiguous()
+
+    def workspace(self, batch: int, mode: int, stream=None):
+        nbytes = B.vqc_workspace_bytes(self.plan, batch, mode)
+        if nbytes == 0:
+            return None, 0
+        stream = stream or torch.cuda.current_stream()
+        key = (mode, stream.cuda_stream, torch.cuda.current_device())
+        buf = self._ws.get(key)
+        if buf is None or buf.numel() < nbytes:
+            buf = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+            B.vqc_workspace_init(buf.data_ptr(), nbytes, stream.cuda_stream)
+            self._ws[key] = buf
+        return buf, buf.numel()
+
+    # ------------------------------------------------------------------ calls
+    def forward(self, x, w, psi0=None, want_state=False, out=None, state_out=None):
+        """E [B, n] (and the final states [B, 2^n] when ``want_state``)."""
+        batch = x.shape[0] if x is not None and x.dim() == 2 else (psi0.shape[0] if psi0 is not None else 1)
+        x = self._check(x, self.real, (batch, self.num_x), "x") if self.num_x else None
+        w = self._check(w, self.real, (self.num_w,), "w") if self.num_w else None
+        psi0 = self._check(psi0, self.cplx, (batch, 1 << self.n), "psi0")
+        E = out if out is not None else torch.empty(batch, self.n, dtype=self.real, device="cuda")
+        st = state_out
+        if want_state and st is None:
+            st = torch.empty(batch, 1 << self.n, dtype=self.cplx, device="cuda")
+        stream = torch.cuda.current_stream()
+        ws, wsb = self.workspace(batch, 0, stream)
+        B.vqc_forward(self.plan, batch, _ptr(x), _ptr(w), _ptr(psi0), _ptr(E), _ptr(st),
+                      _ptr(ws), wsb, stream.cuda_stream)
+        return (E, st) if want_state else E
+
+    def backward(self, x, w, grad_expz, psi0=None, psi_final=None, need_x=True, need_w=True,
+                 grad_x=None, grad_w=None):
+        """(dL/dx [B, num_x], dL/dw [num_w]) for L = sum(grad_expz * E)."""
+        batch = grad_expz.shape[0]
+        x = self._check(x, self.real, (batch, self.num_x), "x") if self.num_x else None
+        w = self._check(w, self.real, (self.num_w,), "w") if self.num_w else None
+        gE = self._check(grad_expz, self.real, (batch, self.n), "grad_expz")
+        psi0 = self._check(psi0, self.cplx, (batch, 1 << self.n), "psi0")
+        psi_final = self._check(psi_final, self.cplx, (batch, 1 << self.n), "psi_final")
+        dx = grad_x
+        if dx is None and need_x and self.num_x:
+            dx = torch.empty(batch, self.num_x, dtype=self.real, device="cuda")
+        dw = grad_w
+        if dw is None and need_w and self.num_w:
+            dw = torch.empty(self.num_w, dtype=self.real, device="cuda")
+        stream = torch.cuda.current_stream()
+        ws, wsb = self.workspace(batch, 1, stream)
+        B.vqc_backward(self.plan, batch, _ptr(x), _ptr(w), _ptr(psi0), _ptr(psi_final),
+                       _ptr(gE), _ptr(dx), _ptr(dw), _ptr(ws), wsb, stream.cuda_stream)
+        return dx, dw
+
+    def __call__(self, x, w, psi0=None):
+        return VQCFunction.apply(x, w, self, psi0)
+
+
+class VQCFunction(torch.autograd.Function):
+    """E = circuit(x, w); backward by the adjoint method from the saved final state."""
+
+    @staticmethod
+    def forward(ctx, x, w, circuit, psi0=None):
+        E, st = circuit.forward(x.detach() if x is not None else None,
+                                w.detach() if w is not None else None, psi0=psi0, want_state=True)
+        ctx.circuit = circuit
+        ctx.save_for_backward(x, w, psi0, st)
+        return E
+
+    @staticmethod
+    def backward(ctx, gE):
+        x, w, psi0, st = ctx.saved_tensors
+        c = ctx.circuit
+        need_x = x is not None and ctx.needs_input_grad[0]
+        need_w = w is not None and ctx.needs_input_grad[1]
+        dx, dw = c.backward(x, w, gE.contiguous(), psi0=psi0, psi_final=st,
+                            need_x=need_x, need_w=need_w)
+        return (dx if need_x else None), (dw if need_w else None), None, None

@@ -1,0 +1,503 @@
+// capi.cu -- the C ABI declared in include/vqc.h: plan lifetime, launch
+// geometry, workspace layout and kernel launches.  No exception crosses the
+// ABI; every entry point returns a vqc_status and records a thread-local
+// message on failure.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdlib>
+#include <cstring>
+#include <memory>
+#include <mutex>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "engine.h"
+#include "kernels.h"
+#include "sweep.cuh"
+
+struct vqc_plan {
+    vqc::HostPlan hp;
+};
+
+namespace vqc {
+namespace {
+
+thread_local std::string g_err;
+
+vqc_status fail(vqc_status s, const std::string& msg) {
+    g_err = msg;
+    return s;
+}
+
+vqc_status cuda_fail(cudaError_t e, const char* what) {
+    return fail(VQC_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+#define VQC_CUDA(call)                                          \
+    do {                                                        \
+        cudaError_t e_ = (call);                                \
+        if (e_ != cudaSuccess) return cuda_fail(e_, #call);     \
+    } while (0)
+
+struct DevInfo {
+    int sms = 0, smem_optin = 0;
+    bool ok = false;
+};
+
+std::mutex g_mu;
+std::vector<DevInfo> g_dev;
+
+vqc_status device_info(int dev, DevInfo& out) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if ((int)g_dev.size() <= dev) g_dev.resize(dev + 1);
+    if (!g_dev[dev].ok) {
+        VQC_CUDA(cudaDeviceGetAttribute(&g_dev[dev].sms, cudaDevAttrMultiProcessorCount, dev));
+        VQC_CUDA(cudaDeviceGetAttribute(&g_dev[dev].smem_optin,
+                                        cudaDevAttrMaxSharedMemoryPerBlockOptin, dev));
+        g_dev[dev].ok = true;
+    }
+    out = g_dev[dev];
+    return VQC_OK;
+}
+
+const void* kernel_ptr(int dtype, int mode, int K) {
+    if (dtype == VQC_C64) return mode == 0 ? sweep_ptr_f32_fwd(K) : sweep_ptr_f32_bwd(K);
+    return mode == 0 ? sweep_ptr_f64_fwd(K) : sweep_ptr_f64_bwd(K);
+}
+
+size_t align16(size_t v) { return (v + 15) & ~size_t(15); }
+size_t align256(size_t v) { return (v + 255) & ~size_t(255); }
+
+// Launch geometry of one call.
+struct Launch {
+    const Schedule* s = nullptr;
+    int K = 0, T = 0, S = 0, block = 0, grid = 0, nunits = 0, wg = 1;
+    size_t smem = 0;
+    int sm_sh = 0, sm_ps = 0, sm_psi = 0, sm_lam = 0, sm_acc = 0, sm_terms = 0, sm_dw = 0,
+        sm_red = 0;
+    const void* fn = nullptr;
+};
+
+int env_int(const char* name, int dflt) {
+    const char* v = std::getenv(name);
+    return v && *v ? std::atoi(v) : dflt;
+}
+
+// Pick the register-block size: the largest K that still gives the batch
+// enough threads to cover every SM's schedulers (>= 152 * 4 warps), but not
+// below 3 (a block of 8 amplitudes) where the circuit allows it.
+int choose_k(const HostPlan& p, int mode, int B) {
+    int forced = env_int(mode == 0 ? "VQC_FORCE_K_FWD" : "VQC_FORCE_K_BWD", 0);
+    if (forced > 0 && find_schedule(p, mode, forced)) return forced;
+    int kmax = 0;
+    for (const auto& s : p.scheds)
+        if (s.mode == mode && s.path == VQC_PATH_RESIDENT) kmax = std::max(kmax, s.K);
+    if (kmax == 0) return 0;
+    const int kmin = std::min(kmax, 3);
+    const double want = 152.0 * 4 * 32;
+    int K = kmax;
+    while (K > kmin && (double)B * std::ldexp(1.0, p.n - K) < want && find_schedule(p, mode, K - 1))
+        --K;
+    return K;
+}
+
+vqc_status plan_launch(const HostPlan& p, int mode, int B, Launch& L) {
+    int dev = 0;
+    VQC_CUDA(cudaGetDevice(&dev));
+    DevInfo di;
+    vqc_status st = device_info(dev, di);
+    if (st != VQC_OK) return st;
+    L.K = choose_k(p, mode, B);
+    L.s = L.K ? find_schedule(p, mode, L.K) : nullptr;
+    if (!L.s)
+        return fail(VQC_ERR_UNSUPPORTED, "no resident schedule for this circuit (n = " +
+                                             std::to_string(p.n) + ")");
+    const bool dbl = p.dtype == VQC_C128;
+    const size_t rs = dbl ? 8 : 4, cs = 2 * rs;
+    L.T = 1 << (p.n - L.K);
+    L.S = std::max(1, 128 / L.T);
+    L.block = L.S * L.T;
+    L.wg = L.T > 32 ? L.T / 32 : 1;
+    if (L.block > sweep_max_threads(dbl, mode, L.K))
+        return fail(VQC_ERR_UNSUPPORTED, "thread group too large for this kernel");
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        size_t o = off;
+        off = align16(off + bytes);
+        return (int)o;
+    };
+    L.sm_sh = take((size_t)p.n_sh * 8 * rs);
+    L.sm_ps = take((size_t)L.S * p.n_ps * 8 * rs);
+    L.sm_psi = take((size_t)L.S * ((size_t)1 << p.n) * cs);
+    L.sm_lam = take(mode == 1 ? (size_t)L.S * ((size_t)1 << p.n) * cs : 0);
+    L.sm_acc = take(mode == 1 ? (size_t)L.S * p.accs.size() * L.wg * 8 * rs : 0);
+    L.sm_terms = take(mode == 1 ? (size_t)L.S * p.term_src.size() * rs : 0);
+    L.sm_dw = take(mode == 1 ? (size_t)p.num_w * rs : 0);
+    L.sm_red = take(mode == 0 ? (size_t)L.S * L.wg * p.n * rs : 0);
+    L.smem = off;
+    if (L.smem > (size_t)di.smem_optin)
+        return fail(VQC_ERR_UNSUPPORTED,
+                    "state does not fit in shared memory on the resident path (" +
+                        std::to_string(L.smem) + " > " + std::to_string(di.smem_optin) + " bytes)");
+    L.fn = kernel_ptr(p.dtype, mode, L.K);
+    if (!L.fn) return fail(VQC_ERR_UNSUPPORTED, "kernel not instantiated for this K");
+    VQC_CUDA(cudaFuncSetAttribute(L.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem));
+    int per_sm = 0;
+    VQC_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, L.fn, L.block, L.smem));
+    if (per_sm < 1) return fail(VQC_ERR_UNSUPPORTED, "kernel cannot be resident with this geometry");
+    L.nunits = (B + L.S - 1) / L.S;
+    L.grid = std::max(1, std::min(L.nunits, per_sm * di.sms));
+    return VQC_OK;
+}
+
+template <typename R>
+void fill_plan_args(const HostPlan& p, const Launch& L, KArgs<R>& a) {
+    const char* base = static_cast<const char*>(p.dbuf);
+    a.ops = reinterpret_cast<const DOp*>(base + L.s->dev_ops);
+    a.stages = reinterpret_cast<const DStage*>(base + L.s->dev_stages);
+    a.nstages = (int)L.s->stages.size();
+    a.entries = reinterpret_cast<const DEntry*>(base + p.dev_entries);
+    a.ps_list = reinterpret_cast<const int32_t*>(base + p.dev_ps_list);
+    a.sh_list = reinterpret_cast<const int32_t*>(base + p.dev_sh_list);
+    a.consts = reinterpret_cast<const DConst*>(base + p.dev_consts);
+    a.cmat = reinterpret_cast<const R*>(base + p.dev_cmat);
+    a.cang = reinterpret_cast<const R*>(base + p.dev_cang);
+    a.accs = reinterpret_cast<const DAcc*>(base + p.dev_accs);
+    a.xocc_ptr = reinterpret_cast<const int32_t*>(base + p.dev_xocc_ptr);
+    a.xocc = reinterpret_cast<const int32_t*>(base + p.dev_xocc);
+    a.wocc_ptr = reinterpret_cast<const int32_t*>(base + p.dev_wocc_ptr);
+    a.wocc = reinterpret_cast<const int32_t*>(base + p.dev_wocc);
+    a.err = p.dev_error;
+    a.n = p.n;
+    a.K = L.K;
+    a.tbits = p.n - L.K;
+    a.G = p.G_swz;
+    a.S = L.S;
+    a.n_ps = p.n_ps;
+    a.n_sh = p.n_sh;
+    a.n_accs = (int)p.accs.size();
+    a.n_terms = (int)p.term_src.size();
+    a.Px = p.num_x;
+    a.Pw = p.num_w;
+    a.sm_sh = L.sm_sh; a.sm_ps = L.sm_ps; a.sm_psi = L.sm_psi; a.sm_lam = L.sm_lam;
+    a.sm_acc = L.sm_acc; a.sm_terms = L.sm_terms; a.sm_dw = L.sm_dw; a.sm_red = L.sm_red;
+}
+
+// Device buffer layout of a plan (all sections 16-byte aligned).
+vqc_status upload(HostPlan& p) {
+    const bool dbl = p.dtype == VQC_C128;
+    std::vector<uint8_t> blob;
+    auto put = [&](const void* src, size_t bytes) {
+        size_t off = blob.size();
+        blob.resize(align16(off + bytes), 0);
+        if (bytes) std::memcpy(blob.data() + off, src, bytes);
+        return off;
+    };
+    std::vector<int32_t> ps_list, sh_list;
+    for (size_t i = 0; i < p.entries.size(); ++i)
+        (p.entries[i].per_sample ? ps_list : sh_list).push_back((int32_t)i);
+    // the kernels index lists by slot order, which is entry order within each list
+    std::vector<double> cm_d = p.cmat, ca_d = p.cang;
+    std::vector<float> cm_f(cm_d.begin(), cm_d.end()), ca_f(ca_d.begin(), ca_d.end());
+    p.dev_entries = put(p.entries.data(), p.entries.size() * sizeof(DEntry));
+    p.dev_ps_list = put(ps_list.data(), ps_list.size() * 4);
+    p.dev_sh_list = put(sh_list.data(), sh_list.size() * 4);
+    p.dev_consts = put(p.consts.data(), p.consts.size() * sizeof(DConst));
+    p.dev_cmat = dbl ? put(cm_d.data(), cm_d.size() * 8) : put(cm_f.data(), cm_f.size() * 4);
+    p.dev_cang = dbl ? put(ca_d.data(), ca_d.size() * 8) : put(ca_f.data(), ca_f.size() * 4);
+    p.dev_accs = put(p.accs.data(), p.accs.size() * sizeof(DAcc));
+    p.dev_xocc_ptr = put(p.xocc_ptr.data(), p.xocc_ptr.size() * 4);
+    p.dev_xocc = put(p.xocc.data(), p.xocc.size() * 4);
+    p.dev_wocc_ptr = put(p.wocc_ptr.data(), p.wocc_ptr.size() * 4);
+    p.dev_wocc = put(p.wocc.data(), p.wocc.size() * 4);
+    for (auto& s : p.scheds) {
+        s.dev_ops = put(s.ops.data(), s.ops.size() * sizeof(DOp));
+        s.dev_stages = put(s.stages.data(), s.stages.size() * sizeof(DStage));
+    }
+    size_t err_off = put(nullptr, 16);
+    blob.resize(align256(blob.size()), 0);
+    VQC_CUDA(cudaGetDevice(&p.device));
+    void* d = nullptr;
+    cudaError_t e = cudaMalloc(&d, blob.size());
+    if (e != cudaSuccess) {
+        (void)cudaGetLastError();
+        return fail(VQC_ERR_OUT_OF_MEMORY, "cudaMalloc of the plan failed");
+    }
+    e = cudaMemcpy(d, blob.data(), blob.size(), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) {
+        cudaFree(d);
+        return cuda_fail(e, "cudaMemcpy(plan)");
+    }
+    p.dbuf = d;
+    p.dbytes = blob.size();
+    p.dev_error = reinterpret_cast<unsigned*>(static_cast<char*>(d) + err_off);
+    return VQC_OK;
+}
+
+// Workspace of a backward call: [0, 256) control block (counter), then the
+// per-CTA dw partials [grid, num_w].
+size_t bwd_workspace(const HostPlan& p, const Launch& L) {
+    const size_t rs = p.dtype == VQC_C128 ? 8 : 4;
+    return 256 + align256((size_t)L.grid * std::max(p.num_w, 1) * rs);
+}
+
+bool misaligned(const void* ptr, size_t a) {
+    return (reinterpret_cast<uintptr_t>(ptr) & (a - 1)) != 0;
+}
+
+template <typename R>
+vqc_status run(const HostPlan& p, int mode, int B, const void* x, const void* w, const void* psi0,
+               const void* psi_final, const void* gE, void* E, void* state_out, void* dx, void* dw,
+               void* ws, size_t ws_bytes, cudaStream_t stream) {
+    using C = C2<R>;
+    Launch L;
+    vqc_status st = plan_launch(p, mode, B, L);
+    if (st != VQC_OK) return st;
+    KArgs<R> a{};
+    fill_plan_args<R>(p, L, a);
+    a.B = B;
+    a.nunits = L.nunits;
+    a.x = static_cast<const R*>(x);
+    a.w = static_cast<const R*>(w);
+    a.psi0 = static_cast<const C*>(psi0);
+    a.psi_final = static_cast<const C*>(psi_final);
+    a.gE = static_cast<const R*>(gE);
+    a.E = static_cast<R*>(E);
+    a.state_out = static_cast<C*>(state_out);
+    a.dx = static_cast<R*>(dx);
+    a.dw = static_cast<R*>(dw);
+    if (mode == 1) {
+        size_t need = bwd_workspace(p, L);
+        if (!ws || ws_bytes < need || misaligned(ws, 256))
+            return fail(VQC_ERR_WORKSPACE, "backward workspace must be >= " + std::to_string(need) +
+                                               " bytes and 256-byte aligned");
+        a.counter = static_cast<unsigned*>(ws);
+        a.dw_part = reinterpret_cast<R*>(static_cast<char*>(ws) + 256);
+    }
+    void* args[] = {&a};
+    VQC_CUDA(cudaLaunchKernel(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
+    return VQC_OK;
+}
+
+std::mutex g_upload_mu;
+
+vqc_status check_common(const vqc_plan* plan, int32_t batch) {
+    if (!plan) return fail(VQC_ERR_INVALID_ARG, "plan is NULL");
+    if (batch < 0) return fail(VQC_ERR_INVALID_ARG, "batch must be >= 0");
+    int dev = -1;
+    VQC_CUDA(cudaGetDevice(&dev));
+    {
+        std::lock_guard<std::mutex> lk(g_upload_mu);
+        if (!plan->hp.dbuf) {
+            vqc_status st = upload(const_cast<vqc_plan*>(plan)->hp);
+            if (st != VQC_OK) return st;
+        }
+    }
+    if (dev != plan->hp.device)
+        return fail(VQC_ERR_INVALID_ARG, "plan was compiled for device " +
+                                             std::to_string(plan->hp.device) +
+                                             " but the current device is " + std::to_string(dev));
+    return VQC_OK;
+}
+
+vqc_status check_ptrs(const HostPlan& p, const void* x, const void* w, const void* psi0,
+                      const void* psi_final) {
+    const size_t rs = p.dtype == VQC_C128 ? 8 : 4;
+    if (p.num_x > 0 && !x) return fail(VQC_ERR_INVALID_ARG, "x is NULL but the circuit uses x");
+    if (p.num_w > 0 && !w) return fail(VQC_ERR_INVALID_ARG, "w is NULL but the circuit uses w");
+    if ((x && misaligned(x, rs)) || (w && misaligned(w, rs)))
+        return fail(VQC_ERR_INVALID_ARG, "x / w must be aligned to the real type");
+    if ((psi0 && misaligned(psi0, 2 * rs)) || (psi_final && misaligned(psi_final, 2 * rs)))
+        return fail(VQC_ERR_INVALID_ARG, "state arrays must be aligned to the complex type");
+    return VQC_OK;
+}
+
+}  // namespace
+}  // namespace vqc
+
+using namespace vqc;
+
+extern "C" {
+
+vqc_status vqc_compile(const vqc_gate* gates, int32_t num_gates, int32_t num_qubits,
+                       int32_t num_x, int32_t num_w, vqc_dtype dtype, vqc_plan** out_plan) {
+    try {
+        if (!out_plan) return fail(VQC_ERR_INVALID_ARG, "out_plan is NULL");
+        *out_plan = nullptr;
+        if (num_gates < 0 || num_x < 0 || num_w < 0 || (num_gates > 0 && !gates))
+            return fail(VQC_ERR_INVALID_ARG, "negative count or NULL gate list");
+        if (dtype != VQC_C64 && dtype != VQC_C128) return fail(VQC_ERR_INVALID_ARG, "bad dtype");
+        if (num_qubits < 1 || num_qubits > VQC_MAX_QUBITS)
+            return fail(VQC_ERR_TOO_MANY_QUBITS, "num_qubits must be in 1.." +
+                                                     std::to_string(VQC_MAX_QUBITS));
+        std::unique_ptr<vqc_plan> p(new vqc_plan());
+        std::string err;
+        vqc_status st = compile_host(gates, num_gates, num_qubits, num_x, num_w, dtype, p->hp, err);
+        if (st != VQC_OK) return fail(st, err);
+        // Upload now when a CUDA device is present; a host-only plan (no device
+        // in this process) still serves vqc_plan_export and vqc_plan_info, and
+        // is uploaded by the first launching call.
+        int ndev = 0;
+        if (cudaGetDeviceCount(&ndev) != cudaSuccess) {
+            (void)cudaGetLastError();
+            ndev = 0;
+        }
+        if (ndev > 0) {
+            st = upload(p->hp);
+            if (st != VQC_OK) return st;
+        }
+        *out_plan = p.release();
+        return VQC_OK;
+    } catch (const std::bad_alloc&) {
+        return fail(VQC_ERR_OUT_OF_MEMORY, "host allocation failed");
+    } catch (...) {
+        return fail(VQC_ERR_INVALID_ARG, "internal error in vqc_compile");
+    }
+}
+
+void vqc_free(vqc_plan* plan) {
+    if (!plan) return;
+    if (plan->hp.dbuf) {
+        int cur = -1;
+        cudaGetDevice(&cur);
+        if (cur != plan->hp.device) cudaSetDevice(plan->hp.device);
+        cudaFree(plan->hp.dbuf);
+        if (cur != plan->hp.device && cur >= 0) cudaSetDevice(cur);
+    }
+    delete plan;
+}
+
+size_t vqc_workspace_bytes(const vqc_plan* plan, int32_t batch, int32_t mode) {
+    if (!plan) return (size_t)-1;
+    if (mode != 1 || batch <= 0) return 0;
+    Launch L;
+    if (plan_launch(plan->hp, 1, batch, L) != VQC_OK) return 0;
+    return bwd_workspace(plan->hp, L);
+}
+
+vqc_status vqc_workspace_init(void* workspace, size_t workspace_bytes, void* stream) {
+    if (!workspace || workspace_bytes < 256) return fail(VQC_ERR_WORKSPACE, "workspace too small");
+    VQC_CUDA(cudaMemsetAsync(workspace, 0, 256, static_cast<cudaStream_t>(stream)));
+    return VQC_OK;
+}
+
+vqc_status vqc_forward(const vqc_plan* plan, int32_t batch, const void* x, const void* w,
+                       const void* psi0, void* expz_out, void* state_out, void* workspace,
+                       size_t workspace_bytes, void* stream) {
+    try {
+        vqc_status st = check_common(plan, batch);
+        if (st != VQC_OK) return st;
+        if (batch == 0) return VQC_OK;
+        const HostPlan& p = plan->hp;
+        st = check_ptrs(p, x, w, psi0, nullptr);
+        if (st != VQC_OK) return st;
+        if (!expz_out) return fail(VQC_ERR_INVALID_ARG, "expz_out is NULL");
+        (void)workspace;
+        (void)workspace_bytes;
+        cudaStream_t s = static_cast<cudaStream_t>(stream);
+        if (p.dtype == VQC_C64)
+            return run<float>(p, 0, batch, x, w, psi0, nullptr, nullptr, expz_out, state_out,
+                              nullptr, nullptr, nullptr, 0, s);
+        return run<double>(p, 0, batch, x, w, psi0, nullptr, nullptr, expz_out, state_out, nullptr,
+                           nullptr, nullptr, 0, s);
+    } catch (...) {
+        return fail(VQC_ERR_INVALID_ARG, "internal error in vqc_forward");
+    }
+}
+
+vqc_status vqc_backward(const vqc_plan* plan, int32_t batch, const void* x, const void* w,
+                        const void* psi0, const void* psi_final, const void* grad_expz,
+                        void* grad_x, void* grad_w, void* workspace, size_t workspace_bytes,
+                        void* stream) {
+    try {
+        vqc_status st = check_common(plan, batch);
+        if (st != VQC_OK) return st;
+        const HostPlan& p = plan->hp;
+        cudaStream_t s = static_cast<cudaStream_t>(stream);
+        if (batch == 0) {
+            if (grad_w && p.num_w > 0)
+                VQC_CUDA(cudaMemsetAsync(grad_w, 0, (size_t)p.num_w * (p.dtype == VQC_C128 ? 8 : 4), s));
+            return VQC_OK;
+        }
+        st = check_ptrs(p, x, w, psi0, psi_final);
+        if (st != VQC_OK) return st;
+        if (!grad_expz) return fail(VQC_ERR_INVALID_ARG, "grad_expz is NULL");
+        if (p.dtype == VQC_C64)
+            return run<float>(p, 1, batch, x, w, psi0, psi_final, grad_expz, nullptr, nullptr,
+                              grad_x, grad_w, workspace, workspace_bytes, s);
+        return run<double>(p, 1, batch, x, w, psi0, psi_final, grad_expz, nullptr, nullptr, grad_x,
+                           grad_w, workspace, workspace_bytes, s);
+    } catch (...) {
+        return fail(VQC_ERR_INVALID_ARG, "internal error in vqc_backward");
+    }
+}
+
+vqc_status vqc_plan_info(const vqc_plan* plan, int32_t batch, vqc_plan_stats* out) {
+    if (!plan || !out) return fail(VQC_ERR_INVALID_ARG, "NULL argument");
+    const HostPlan& p = plan->hp;
+    std::memset(out, 0, sizeof(*out));
+    out->num_qubits = p.n;
+    out->num_x = p.num_x;
+    out->num_w = p.num_w;
+    out->dtype = p.dtype;
+    out->num_gates_in = p.num_gates_in;
+    out->num_ops = (int32_t)p.ops.size();
+    out->num_runs = p.n_runs;
+    out->num_terms = (int32_t)p.term_src.size();
+    out->fwd_flops_per_eval = p.fwd_flops;
+    out->bwd_flops_per_eval = p.bwd_flops;
+    out->recompute_flops_per_eval = p.recompute_flops;
+    const int B = std::max(batch, 1);
+    for (int mode = 0; mode < 2; ++mode) {
+        int K = choose_k(p, mode, B);
+        const Schedule* s = K ? find_schedule(p, mode, K) : nullptr;
+        int* path = mode == 0 ? &out->fwd_path : &out->bwd_path;
+        int* kk = mode == 0 ? &out->fwd_k : &out->bwd_k;
+        int* ns = mode == 0 ? &out->fwd_stages : &out->bwd_stages;
+        int* np = mode == 0 ? &out->fwd_passes : &out->bwd_passes;
+        int* tps = mode == 0 ? &out->fwd_threads_per_sample : &out->bwd_threads_per_sample;
+        int* tq = mode == 0 ? &out->fwd_tile_qubits : &out->bwd_tile_qubits;
+        if (!s) {
+            *path = -1;
+            continue;
+        }
+        *path = s->path;
+        *kk = s->K;
+        *ns = (int)s->stages.size();
+        *np = 1;
+        *tps = 1 << (p.n - s->K);
+        *tq = s->m;
+    }
+    return VQC_OK;
+}
+
+vqc_status vqc_plan_export(const vqc_plan* plan, void* buf, size_t* inout_bytes) {
+    if (!plan || !inout_bytes) return fail(VQC_ERR_INVALID_ARG, "NULL argument");
+    try {
+        std::vector<uint8_t> b = export_plan(plan->hp);
+        size_t cap = *inout_bytes;
+        *inout_bytes = b.size();
+        if (!buf) return VQC_OK;
+        if (cap < b.size()) return fail(VQC_ERR_INVALID_ARG, "buffer too small");
+        std::memcpy(buf, b.data(), b.size());
+        return VQC_OK;
+    } catch (...) {
+        return fail(VQC_ERR_OUT_OF_MEMORY, "export failed");
+    }
+}
+
+vqc_status vqc_sync_check(void* stream) {
+    cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetLastError");
+    return VQC_OK;
+}
+
+const char* vqc_last_error(void) { return g_err.c_str(); }
+
+int32_t vqc_abi_version(void) { return VQC_ABI_VERSION; }
+
+}  // extern "C"

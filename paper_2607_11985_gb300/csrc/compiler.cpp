@@ -1,0 +1,525 @@
+// compiler.cpp -- host compiler: gate list -> plan (paper, Alg. 1 compile phase).
+//
+// Steps, each O(G):
+//   1. validate every gate (static-circuit scope, Sec. 3: fixed gate identity
+//      and wiring, only angles vary at run time);
+//   2. lower: SWAP -> CX CX CX; single-qubit gates become constituents of the
+//      run open on their qubit; a two-qubit gate closes the runs on its qubits;
+//   3. classify constituents as constant (pre-multiplied here in fp64, the
+//      paper's cached static matrices) or parametric (x or w, evaluated in the
+//      kernel prologue), and number the gradient terms;
+//   4. cut the fused op list into register-block stages for each (mode, K).
+#include <algorithm>
+#include <cmath>
+#include <complex>
+#include <cstring>
+#include <numeric>
+
+#include "engine.h"
+
+namespace vqc {
+namespace {
+
+using cd = std::complex<double>;
+
+struct Mat2 {
+    cd m[4];   // row-major [[m0, m1], [m2, m3]]
+};
+
+Mat2 mul(const Mat2& a, const Mat2& b) {   // a * b
+    Mat2 r;
+    r.m[0] = a.m[0] * b.m[0] + a.m[1] * b.m[2];
+    r.m[1] = a.m[0] * b.m[1] + a.m[1] * b.m[3];
+    r.m[2] = a.m[2] * b.m[0] + a.m[3] * b.m[2];
+    r.m[3] = a.m[2] * b.m[1] + a.m[3] * b.m[3];
+    return r;
+}
+
+Mat2 fixed_matrix(int op, const double* th) {
+    const double r2 = 1.0 / std::sqrt(2.0);
+    const cd i(0, 1);
+    Mat2 u{};
+    switch (op) {
+    case VQC_H: u = {{r2, r2, r2, -r2}}; break;
+    case VQC_X: u = {{0, 1, 1, 0}}; break;
+    case VQC_Y: u = {{0, -i, i, 0}}; break;
+    case VQC_Z: u = {{1, 0, 0, -1}}; break;
+    case VQC_S: u = {{1, 0, 0, i}}; break;
+    case VQC_T: u = {{1, 0, 0, std::polar(1.0, M_PI / 4)}}; break;
+    case VQC_SX: u = {{cd(0.5, 0.5), cd(0.5, -0.5), cd(0.5, -0.5), cd(0.5, 0.5)}}; break;
+    case VQC_RX: { double c = std::cos(th[0] / 2), s = std::sin(th[0] / 2);
+                   u = {{c, cd(0, -s), cd(0, -s), c}}; break; }
+    case VQC_RY: { double c = std::cos(th[0] / 2), s = std::sin(th[0] / 2);
+                   u = {{c, -s, s, c}}; break; }
+    case VQC_RZ: u = {{std::polar(1.0, -th[0] / 2), 0, 0, std::polar(1.0, th[0] / 2)}}; break;
+    case VQC_U3: { double c = std::cos(th[0] / 2), s = std::sin(th[0] / 2);
+                   u = {{c, -std::polar(s, th[2]), std::polar(s, th[1]),
+                         std::polar(c, th[1] + th[2])}}; break; }
+    default: break;
+    }
+    return u;
+}
+
+bool is_two_qubit(int op) { return op >= VQC_CX && op <= VQC_RZZ; }
+int num_angles(int op) {
+    switch (op) {
+    case VQC_RX: case VQC_RY: case VQC_RZ: case VQC_CRZ: case VQC_RZZ: return 1;
+    case VQC_U3: return 3;
+    default: return 0;
+    }
+}
+
+struct Src {
+    uint8_t kind = SRC_NONE;
+    int32_t idx = 0;
+    double cval = 0;
+};
+
+struct Cons {            // constituent before packing
+    uint8_t kind;
+    Src s0, s1;
+    Mat2 mat;            // CK_CONST
+};
+
+struct Builder {
+    HostPlan& p;
+    std::vector<std::vector<Cons>> open;   // per qubit
+
+    explicit Builder(HostPlan& plan) : p(plan), open(plan.n) {}
+
+    int32_t cang_index(double v) {
+        p.cang.push_back(v);
+        return (int32_t)p.cang.size() - 1;
+    }
+
+    // Pack a constituent list into an entry.  Consecutive constants are
+    // multiplied here (time order: later factor on the left).
+    int make_entry(std::vector<Cons>& in, bool phase) {
+        std::vector<Cons> cs;
+        for (auto& c : in) {
+            if (c.kind == CK_CONST && !cs.empty() && cs.back().kind == CK_CONST)
+                cs.back().mat = mul(c.mat, cs.back().mat);
+            else
+                cs.push_back(c);
+        }
+        DEntry e{};
+        e.cfirst = (uint16_t)p.consts.size();
+        e.ccount = (uint16_t)cs.size();
+        e.phase = phase ? 1 : 0;
+        e.per_sample = 0;
+        bool has_term = false;
+        for (auto& c : cs) {
+            DConst d{};
+            d.kind = c.kind;
+            d.term = -1;
+            if (c.kind == CK_CONST) {
+                d.idx0 = (int32_t)(p.cmat.size() / 8);
+                for (int k = 0; k < 4; ++k) {
+                    p.cmat.push_back(c.mat.m[k].real());
+                    p.cmat.push_back(c.mat.m[k].imag());
+                }
+            } else {
+                auto put = [&](const Src& s, uint8_t& kind, int32_t& idx) {
+                    kind = s.kind;
+                    idx = s.kind == SRC_CONST ? cang_index(s.cval) : s.idx;
+                    if (s.kind == SRC_X) e.per_sample = 1;
+                };
+                put(c.s0, d.src0, d.idx0);
+                if (c.kind == CK_GPHASE) put(c.s1, d.src1, d.idx1);
+                // Gradient terms: rotations and phase gates with an x or w source.
+                // The global phase of U3 carries none: L is invariant under it.
+                if (c.kind != CK_GPHASE && (c.s0.kind == SRC_X || c.s0.kind == SRC_W)) {
+                    d.term = (int32_t)p.term_src.size();
+                    p.term_src.push_back(c.s0.kind);
+                    p.term_idx.push_back(c.s0.idx);
+                    has_term = true;
+                }
+            }
+            p.consts.push_back(d);
+        }
+        int id = (int)p.entries.size();
+        e.acc = 0xffff;
+        if (has_term) {
+            e.acc = (uint16_t)p.accs.size();
+            p.accs.push_back(DAcc{id, phase ? 1 : 0});
+        }
+        p.entries.push_back(e);
+        return id;
+    }
+
+    void flush(int q) {
+        if (open[q].empty()) return;
+        int id = make_entry(open[q], false);
+        open[q].clear();
+        p.ops.push_back(HOp{OP_M1, q, -1, id, 0});
+        ++p.n_runs;
+    }
+
+    void add_rotation(int q, uint8_t kind, const Src& s) {
+        Cons c{};
+        if (s.kind == SRC_CONST) {
+            const double th[3] = {s.cval, 0, 0};
+            c.kind = CK_CONST;
+            c.mat = fixed_matrix(kind == CK_RX ? VQC_RX : kind == CK_RY ? VQC_RY : VQC_RZ, th);
+        } else {
+            c.kind = kind;
+            c.s0 = s;
+        }
+        open[q].push_back(c);
+    }
+
+    void add_gate(const vqc_gate& g) {
+        Src src[3];
+        for (int k = 0; k < num_angles(g.op); ++k) {
+            src[k].kind = g.pkind[k];
+            src[k].idx = g.pidx[k];
+            src[k].cval = g.pconst[k];
+        }
+        const int q0 = g.q0, q1 = g.q1;
+        switch (g.op) {
+        case VQC_H: case VQC_X: case VQC_Y: case VQC_Z: case VQC_S: case VQC_T: case VQC_SX: {
+            Cons c{};
+            c.kind = CK_CONST;
+            c.mat = fixed_matrix(g.op, nullptr);
+            open[q0].push_back(c);
+            break;
+        }
+        case VQC_RX: add_rotation(q0, CK_RX, src[0]); break;
+        case VQC_RY: add_rotation(q0, CK_RY, src[0]); break;
+        case VQC_RZ: add_rotation(q0, CK_RZ, src[0]); break;
+        case VQC_U3: {
+            bool all_const = src[0].kind == SRC_CONST && src[1].kind == SRC_CONST &&
+                             src[2].kind == SRC_CONST;
+            if (all_const) {
+                const double th[3] = {src[0].cval, src[1].cval, src[2].cval};
+                Cons c{};
+                c.kind = CK_CONST;
+                c.mat = fixed_matrix(VQC_U3, th);
+                open[q0].push_back(c);
+            } else {
+                // U3(t, p, l) = e^{i(p+l)/2} RZ(p) RY(t) RZ(l): RZ(l) first.
+                add_rotation(q0, CK_RZ, src[2]);
+                add_rotation(q0, CK_RY, src[0]);
+                add_rotation(q0, CK_RZ, src[1]);
+                Cons c{};
+                if (src[1].kind == SRC_CONST && src[2].kind == SRC_CONST) {
+                    c.kind = CK_CONST;
+                    cd ph = std::polar(1.0, 0.5 * (src[1].cval + src[2].cval));
+                    c.mat = {{ph, 0, 0, ph}};
+                } else {
+                    c.kind = CK_GPHASE;
+                    c.s0 = src[1];
+                    c.s1 = src[2];
+                }
+                open[q0].push_back(c);
+            }
+            break;
+        }
+        case VQC_CX: case VQC_CZ: case VQC_SWAP: case VQC_CRZ: case VQC_RZZ: {
+            flush(q0);
+            flush(q1);
+            if (g.op == VQC_CX) {
+                p.ops.push_back(HOp{OP_CX, q0, q1, -1, 0});
+            } else if (g.op == VQC_SWAP) {
+                p.ops.push_back(HOp{OP_CX, q0, q1, -1, 0});
+                p.ops.push_back(HOp{OP_CX, q1, q0, -1, 0});
+                p.ops.push_back(HOp{OP_CX, q0, q1, -1, 0});
+            } else if (g.op == VQC_CZ) {
+                p.ops.push_back(HOp{OP_CZ, q0, q1, -1, 0});
+            } else {
+                std::vector<Cons> one(1);
+                one[0].kind = g.op == VQC_CRZ ? CK_CRZ : CK_RZZ;
+                one[0].s0 = src[0];
+                const int id = make_entry(one, true);   // constant angles come from the pool
+                p.ops.push_back(HOp{OP_PH2, q0, q1, id,
+                                    (uint8_t)(g.op == VQC_CRZ ? OPF_GEN_CRZ : OPF_GEN_RZZ)});
+            }
+            break;
+        }
+        default: break;
+        }
+    }
+};
+
+vqc_status validate(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx, int32_t nw,
+                    std::string& err) {
+    for (int32_t g = 0; g < G; ++g) {
+        const vqc_gate& x = gates[g];
+        if (x.op >= VQC_NUM_GATE_OPS) {
+            err = "gate " + std::to_string(g) + ": unsupported opcode " + std::to_string(x.op);
+            return VQC_ERR_UNSUPPORTED_GATE;
+        }
+        if (x.reserved[0] || x.reserved[1] || x.reserved2) {
+            err = "gate " + std::to_string(g) + ": reserved bytes must be zero";
+            return VQC_ERR_INVALID_ARG;
+        }
+        if (x.q0 >= n || (is_two_qubit(x.op) && (x.q1 >= n || x.q1 == x.q0))) {
+            err = "gate " + std::to_string(g) + ": qubit out of range or repeated";
+            return VQC_ERR_QUBIT_RANGE;
+        }
+        for (int k = 0; k < num_angles(x.op); ++k) {
+            int kind = x.pkind[k];
+            bool ok = (kind == VQC_P_CONST && std::isfinite(x.pconst[k])) ||
+                      (kind == VQC_P_X && x.pidx[k] >= 0 && x.pidx[k] < nx) ||
+                      (kind == VQC_P_W && x.pidx[k] >= 0 && x.pidx[k] < nw);
+            if (!ok) {
+                err = "gate " + std::to_string(g) + ": angle " + std::to_string(k) +
+                      " has an invalid source";
+                return VQC_ERR_PARAM_RANGE;
+            }
+        }
+    }
+    return VQC_OK;
+}
+
+uint32_t swz(uint32_t u, int G) {
+    uint32_t v = u >> G, f = 0;
+    while (v) { f ^= v; v >>= G; }
+    return u ^ (f & ((1u << G) - 1));
+}
+
+uint32_t op_touch(const HOp& o) {
+    uint32_t t = 1u << o.q0;
+    if (o.type != OP_M1) t |= 1u << o.q1;
+    return t;
+}
+uint32_t op_need(const HOp& o) {
+    if (o.type == OP_M1) return 1u << o.q0;
+    if (o.type == OP_CX) return 1u << o.q1;
+    return 0;
+}
+
+// Cut the op list into stages of K active qubits (resident path: tile = all n).
+void build_schedule(const HostPlan& p, Schedule& s) {
+    const int n = p.n, K = s.K, G = p.G_swz;
+    s.m = n;
+    s.thread_bits = n - K;
+    s.group_lanes_log2 = s.thread_bits;
+    std::vector<int> remaining(p.ops.size());
+    std::iota(remaining.begin(), remaining.end(), 0);
+    do {   // an empty circuit still gets one (empty) stage
+        uint32_t active = 0, blocked = 0;
+        std::vector<int> taken, deferred;
+        for (int oi : remaining) {
+            const HOp& o = p.ops[oi];
+            uint32_t touch = op_touch(o), need = op_need(o);
+            if (touch & blocked) {
+                blocked |= touch;
+                deferred.push_back(oi);
+                continue;
+            }
+            uint32_t na = active | need;
+            if (__builtin_popcount(na) <= K) {
+                active = na;
+                taken.push_back(oi);
+            } else {
+                blocked |= touch;
+                deferred.push_back(oi);
+            }
+        }
+        // Pad the active set to exactly K qubits, keeping every residue class
+        // (mod G) represented among the outer qubits where possible.
+        while (__builtin_popcount(active) < K) {
+            int best = -1, best_cnt = -1;
+            for (int q = n - 1; q >= 0; --q) {
+                if (active >> q & 1) continue;
+                int cnt = 0;
+                for (int r = 0; r < n; ++r)
+                    if (!(active >> r & 1) && r % G == q % G) ++cnt;
+                if (cnt > best_cnt) { best_cnt = cnt; best = q; }
+            }
+            active |= 1u << best;
+        }
+        DStage st{};
+        int j = 0;
+        for (int q = 0; q < n; ++q)
+            if (active >> q & 1) st.active[j++] = (uint8_t)q;
+        for (int k = 0; k < K; ++k) st.sigma[k] = (int32_t)swz(1u << st.active[k], G);
+        // Thread bits: bit i (i < G) takes an outer qubit of residue i when one exists.
+        std::vector<int> outer;
+        for (int q = 0; q < n; ++q)
+            if (!(active >> q & 1)) outer.push_back(q);
+        std::vector<int> order;
+        std::vector<bool> used(outer.size(), false);
+        for (int i = 0; i < std::min<int>(G, (int)outer.size()); ++i) {
+            int pick = -1;
+            for (size_t c = 0; c < outer.size(); ++c)
+                if (!used[c] && outer[c] % G == i) { pick = (int)c; break; }
+            if (pick < 0)
+                for (size_t c = 0; c < outer.size(); ++c)
+                    if (!used[c]) { pick = (int)c; break; }
+            used[pick] = true;
+            order.push_back(outer[pick]);
+        }
+        for (size_t c = 0; c < outer.size(); ++c)
+            if (!used[c]) order.push_back(outer[c]);
+        st.nthreadbits = (uint8_t)order.size();
+        for (size_t i = 0; i < order.size(); ++i) {
+            st.tau[i] = (int32_t)swz(1u << order[i], G);
+            st.tmask[i] = 1u << order[i];
+        }
+        auto local = [&](int q) -> int {
+            for (int k = 0; k < K; ++k)
+                if (st.active[k] == q) return k;
+            return -1;
+        };
+        auto ref = [&](int q) -> uint8_t {
+            int l = local(q);
+            return (uint8_t)(l >= 0 ? l : kRefPhys + q);
+        };
+        st.op_begin = (int32_t)s.ops.size();
+        for (int oi : taken) {
+            const HOp& o = p.ops[oi];
+            DOp d{};
+            d.type = o.type;
+            if (o.type == OP_M1 || o.type == OP_PH2) {
+                const DEntry& e = p.entries[o.entry];
+                d.slot = e.slot;
+                d.flags = (uint8_t)((e.per_sample ? OPF_PER_SAMPLE : 0) |
+                                    (e.acc != 0xffff ? OPF_HAS_ACC : 0) | o.gen);
+                d.aux = e.acc;
+            }
+            if (o.type == OP_M1) {
+                d.a = (uint8_t)local(o.q0);
+            } else if (o.type == OP_CX) {
+                d.a = ref(o.q0);
+                d.b = (uint8_t)local(o.q1);
+            } else {
+                d.a = ref(o.q0);
+                d.b = ref(o.q1);
+            }
+            s.ops.push_back(d);
+        }
+        st.op_end = (int32_t)s.ops.size();
+        s.stages.push_back(st);
+        remaining.swap(deferred);
+    } while (!remaining.empty());
+}
+
+template <class T>
+void put_vec(std::vector<uint8_t>& out, const std::vector<T>& v) {
+    int32_t count = (int32_t)v.size();
+    const uint8_t* c = reinterpret_cast<const uint8_t*>(&count);
+    out.insert(out.end(), c, c + 4);
+    if (!v.empty()) {
+        const uint8_t* b = reinterpret_cast<const uint8_t*>(v.data());
+        out.insert(out.end(), b, b + v.size() * sizeof(T));
+    }
+}
+
+void put_i32(std::vector<uint8_t>& out, int32_t v) {
+    const uint8_t* c = reinterpret_cast<const uint8_t*>(&v);
+    out.insert(out.end(), c, c + 4);
+}
+
+}  // namespace
+
+vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx, int32_t nw,
+                        int dtype, HostPlan& p, std::string& err) {
+    vqc_status st = validate(gates, G, n, nx, nw, err);
+    if (st != VQC_OK) return st;
+    p.n = n;
+    p.num_x = nx;
+    p.num_w = nw;
+    p.dtype = dtype;
+    p.num_gates_in = G;
+    p.G_swz = dtype == VQC_C64 ? 4 : 3;
+    Builder b(p);
+    for (int32_t g = 0; g < G; ++g) b.add_gate(gates[g]);
+    for (int q = 0; q < n; ++q) b.flush(q);
+    if (p.entries.size() > 0xfff0 || p.accs.size() > 0xfff0) {
+        err = "circuit too large for one plan (table entries exceed 65520)";
+        return VQC_ERR_UNSUPPORTED;
+    }
+    // Table slots: per-sample entries and shared entries are numbered apart.
+    for (auto& e : p.entries) e.slot = (uint16_t)(e.per_sample ? p.n_ps++ : p.n_sh++);
+    // Terms of each x column / w index, in increasing term order.
+    p.xocc_ptr.assign(nx + 1, 0);
+    p.wocc_ptr.assign(nw + 1, 0);
+    for (size_t t = 0; t < p.term_src.size(); ++t)
+        (p.term_src[t] == SRC_X ? p.xocc_ptr : p.wocc_ptr)[p.term_idx[t] + 1]++;
+    for (int i = 0; i < nx; ++i) p.xocc_ptr[i + 1] += p.xocc_ptr[i];
+    for (int i = 0; i < nw; ++i) p.wocc_ptr[i + 1] += p.wocc_ptr[i];
+    p.xocc.assign(p.xocc_ptr[nx], 0);
+    p.wocc.assign(p.wocc_ptr[nw], 0);
+    {
+        std::vector<int32_t> fx(p.xocc_ptr.begin(), p.xocc_ptr.end() - 1);
+        std::vector<int32_t> fw(p.wocc_ptr.begin(), p.wocc_ptr.end() - 1);
+        for (size_t t = 0; t < p.term_src.size(); ++t) {
+            if (p.term_src[t] == SRC_X) p.xocc[fx[p.term_idx[t]]++] = (int32_t)t;
+            else p.wocc[fw[p.term_idx[t]]++] = (int32_t)t;
+        }
+    }
+    // Algorithmic flops per evaluation (counted on the fused op list).
+    const double dim = std::ldexp(1.0, n);
+    double f = 0, fb = 0;
+    for (const HOp& o : p.ops) {
+        bool acc = (o.type == OP_M1 || o.type == OP_PH2) && p.entries[o.entry].acc != 0xffff;
+        if (o.type == OP_M1) { f += 14; fb += acc ? 44 : 28; }
+        else if (o.type == OP_PH2) {
+            double half = o.gen == OPF_GEN_CRZ ? 0.5 : 1.0;
+            f += 6 * half;
+            fb += (acc ? 16 : 12) * half;
+        }
+    }
+    p.recompute_flops = f * dim;
+    p.fwd_flops = (f + 3 + n) * dim;
+    p.bwd_flops = (fb + n + 2) * dim;
+    // Stage schedules for every usable (mode, K) on the resident path.
+    for (int mode = 0; mode < 2; ++mode) {
+        for (int K = 1; K <= std::min(max_k(mode, dtype), n); ++K) {
+            const int max_tb = (dtype == VQC_C64 && mode == 0 && K <= 4) ? 10 : 9;
+            if (n - K > max_tb) continue;   // thread group must fit one CTA
+            Schedule s;
+            s.mode = mode;
+            s.K = K;
+            s.path = VQC_PATH_RESIDENT;
+            build_schedule(p, s);
+            p.scheds.push_back(std::move(s));
+        }
+    }
+    return VQC_OK;
+}
+
+const Schedule* find_schedule(const HostPlan& p, int mode, int K) {
+    for (const auto& s : p.scheds)
+        if (s.mode == mode && s.K == K && s.path == VQC_PATH_RESIDENT) return &s;
+    return nullptr;
+}
+
+std::vector<uint8_t> export_plan(const HostPlan& p) {
+    std::vector<uint8_t> out = {'V', 'Q', 'C', 'P'};
+    put_i32(out, 1);
+    for (int v : {p.n, p.num_x, p.num_w, p.dtype, p.num_gates_in, p.G_swz, p.n_ps, p.n_sh,
+                  p.n_runs})
+        put_i32(out, v);
+    std::vector<int32_t> hops;
+    for (const HOp& o : p.ops) {
+        hops.push_back(o.type);
+        hops.push_back(o.q0);
+        hops.push_back(o.q1);
+        hops.push_back(o.entry);
+        hops.push_back(o.gen);
+    }
+    put_vec(out, hops);
+    put_vec(out, p.entries);
+    put_vec(out, p.consts);
+    put_vec(out, p.cmat);
+    put_vec(out, p.cang);
+    put_vec(out, p.term_src);
+    put_vec(out, p.term_idx);
+    put_vec(out, p.accs);
+    put_vec(out, p.xocc_ptr);
+    put_vec(out, p.xocc);
+    put_vec(out, p.wocc_ptr);
+    put_vec(out, p.wocc);
+    put_i32(out, (int32_t)p.scheds.size());
+    for (const auto& s : p.scheds) {
+        for (int v : {s.mode, s.K, s.m, s.path, s.thread_bits, s.group_lanes_log2}) put_i32(out, v);
+        put_vec(out, s.ops);
+        put_vec(out, s.stages);
+    }
+    return out;
+}
+
+}  // namespace vqc

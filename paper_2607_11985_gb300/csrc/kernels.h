@@ -1,0 +1,19 @@
+// kernels.h -- entry points into the kernel translation units (one per real
+// type and mode, compiled in parallel).  Each returns the address of the
+// sweep kernel instantiated for register-block size K, or nullptr.
+#pragma once
+
+namespace vqc {
+
+const void* sweep_ptr_f32_fwd(int K);
+const void* sweep_ptr_f32_bwd(int K);
+const void* sweep_ptr_f64_fwd(int K);
+const void* sweep_ptr_f64_bwd(int K);
+
+// Largest block (threads) each instantiation is compiled for.
+inline int sweep_max_threads(bool is_double, int mode, int K) {
+    if (!is_double && mode == 0 && K <= 4) return 1024;
+    return 512;
+}
+
+}  // namespace vqc

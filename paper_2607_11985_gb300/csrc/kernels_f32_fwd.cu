@@ -1,0 +1,18 @@
+// kernels_f32_fwd.cu -- instantiations of the sweep kernel for float, mode 0.
+#include "kernels.h"
+#include "sweep.cuh"
+
+namespace vqc {
+
+const void* sweep_ptr_f32_fwd(int K) {
+    switch (K) {
+    case 1: return reinterpret_cast<const void*>(&sweep_kernel<float, 1, 0>);
+    case 2: return reinterpret_cast<const void*>(&sweep_kernel<float, 2, 0>);
+    case 3: return reinterpret_cast<const void*>(&sweep_kernel<float, 3, 0>);
+    case 4: return reinterpret_cast<const void*>(&sweep_kernel<float, 4, 0>);
+    case 5: return reinterpret_cast<const void*>(&sweep_kernel<float, 5, 0>);
+    default: return nullptr;
+    }
+}
+
+}  // namespace vqc

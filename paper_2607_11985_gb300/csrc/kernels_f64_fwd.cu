@@ -1,0 +1,17 @@
+// kernels_f64_fwd.cu -- instantiations of the sweep kernel for double, mode 0.
+#include "kernels.h"
+#include "sweep.cuh"
+
+namespace vqc {
+
+const void* sweep_ptr_f64_fwd(int K) {
+    switch (K) {
+    case 1: return reinterpret_cast<const void*>(&sweep_kernel<double, 1, 0>);
+    case 2: return reinterpret_cast<const void*>(&sweep_kernel<double, 2, 0>);
+    case 3: return reinterpret_cast<const void*>(&sweep_kernel<double, 3, 0>);
+    case 4: return reinterpret_cast<const void*>(&sweep_kernel<double, 4, 0>);
+    default: return nullptr;
+    }
+}
+
+}  // namespace vqc

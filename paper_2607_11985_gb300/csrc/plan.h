@@ -1,0 +1,98 @@
+// plan.h -- the compiled plan: host representation and the POD records the
+// kernels read from device memory.
+//
+// A plan is the "gate sequence with cached static unitaries" of the paper's
+// compile phase (Alg. 1, compile phase), lowered further for the GPU:
+//
+//   * single-qubit gates that meet consecutively on a qubit are fused into a
+//     run; consecutive constant factors of a run are pre-multiplied on the host
+//     in fp64 (Alg. 1: "precompute and cache" constant matrices);
+//   * two-qubit gates become CX (conditional swap), CZ (sign) or a diagonal
+//     two-qubit phase (CRZ, RZZ); SWAP is lowered to three CX;
+//   * the op list is cut into stages.  In a stage every thread of a sample's
+//     thread group holds a register block of 2^K amplitudes spanned by the
+//     stage's K "active" qubits; every non-diagonal op of the stage acts on
+//     active qubits only, diagonal ops and CX controls may use any qubit.
+//     Between stages the state goes through shared memory.
+//
+// Amplitude addressing in shared memory (per sample, tile-local index u):
+//   slot(u) = sw(u) ^ h_sample,   sw(u) = u ^ (fold_G(u >> G) & (2^G - 1))
+// with G = 4 for complex64 and 3 for complex128 (2^G amplitudes = 128 bytes).
+// sw is linear over GF(2), so the slot of amplitude r of a thread's block is
+// XOR(swizzled thread base, XOR of sigma[j] over set bits j of r).
+#pragma once
+
+#include <cstdint>
+
+namespace vqc {
+
+constexpr int kMaxK = 5;             // register-block qubits per thread (<= 32 amplitudes)
+constexpr int kMaxThreadBits = 16;   // thread-index bits of one sample group / tile
+constexpr uint8_t kRefPhys = 8;      // qubit ref >= 8: physical qubit (ref - 8), not active
+
+// ---- ops (8 bytes) -------------------------------------------------------
+enum OpType : uint8_t {
+    OP_M1 = 1,    // general 2x2 on active local position a; table entry `slot`
+    OP_CX = 2,    // control ref a (local or physical), target local b
+    OP_CZ = 3,    // sign on bit a & bit b (refs)
+    OP_PH2 = 4    // diagonal phase ph[bit a + 2 bit b] from table entry `slot`
+};
+enum OpFlags : uint8_t {
+    OPF_PER_SAMPLE = 1,   // table entry lives in the per-sample table
+    OPF_GEN_CRZ = 2,      // generator |1><1|_a (x) Z_b   (CRZ)
+    OPF_GEN_RZZ = 4,      // generator Z_a (x) Z_b        (RZZ)
+    OPF_HAS_ACC = 8       // op accumulates a gradient slot (aux) in the backward
+};
+
+struct DOp {
+    uint8_t type, a, b, flags;
+    uint16_t slot;   // table entry index inside its table (per-sample or shared)
+    uint16_t aux;    // accumulator slot for the backward (run or phase op id)
+};
+static_assert(sizeof(DOp) == 8, "DOp layout");
+
+// ---- stages ----------------------------------------------------------------
+struct DStage {
+    int32_t op_begin, op_end;
+    int32_t sigma[kMaxK];             // swizzled slot offset of local bit j
+    int32_t tau[kMaxThreadBits];      // swizzled slot offset of thread bit i
+    uint32_t tmask[kMaxThreadBits];   // physical-index bit of thread bit i
+    uint8_t active[kMaxK];            // physical qubit of local bit j
+    uint8_t nthreadbits;
+    uint8_t pad[2];
+};
+
+// ---- table entries and their constituents ----------------------------------
+enum ConstKind : uint8_t {
+    CK_CONST = 1,    // pre-multiplied constant 2x2 (cmat[idx0])
+    CK_RX = 2, CK_RY = 3, CK_RZ = 4,   // exp(-i t P / 2), angle from src0
+    CK_GPHASE = 5,   // scalar e^{i (t0 + t1) / 2} (global phase of U3)
+    CK_CRZ = 6,      // phases (1, e^{-it/2}, 1, e^{it/2}) on s = b0 + 2 b1
+    CK_RZZ = 7       // phases (e^{-it/2}, e^{it/2}, e^{it/2}, e^{-it/2})
+};
+enum SrcKind : uint8_t { SRC_NONE = 0, SRC_CONST = 1, SRC_X = 2, SRC_W = 3 };
+
+struct DConst {
+    uint8_t kind, src0, src1, pad;
+    int32_t idx0, idx1;   // x column / w index / const-angle index (or cmat index for CK_CONST)
+    int32_t term;         // gradient term index, -1 if none
+};
+static_assert(sizeof(DConst) == 16, "DConst layout");
+
+struct DEntry {
+    uint16_t cfirst, ccount;   // constituents, in time order
+    uint16_t slot;             // index inside its table
+    uint8_t per_sample;        // 1: depends on x[b]
+    uint8_t phase;             // 0: 2x2 matrix, 1: four diagonal phases
+    uint16_t acc;              // accumulator slot (backward)
+    uint16_t pad;
+};
+static_assert(sizeof(DEntry) == 12, "DEntry layout");
+
+// Accumulator slot -> what it holds (backward).
+struct DAcc {
+    int32_t entry;   // table entry id
+    int32_t kind;    // 0: 2x2 rho of a run, 1: scalar of a phase op
+};
+
+}  // namespace vqc

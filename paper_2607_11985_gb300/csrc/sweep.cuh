@@ -1,0 +1,846 @@
+// sweep.cuh -- sm_103a kernels of the batched statevector engine.
+//
+// Forward (paper, Alg. 1 execute phase): per sample, psi = U_G ... U_1 psi0
+// and E[b, j] = sum_k (-1)^{k_j} |psi[k]|^2 (Alg. 1, return statement).
+// Backward (paper, Sec. 3, gradients w.r.t. trainable parameters), adjoint
+// method: lam = O psi with O = sum_j gE[b, j] Z_j; the plan is swept in
+// reverse, un-applying every op on psi and lam, and for every parametrised
+// angle t of a gate exp(-i t P / 2) the term dL/dt = Im <lam|P|psi> is taken
+// at the gate's output.  For a fused single-qubit run V the kernel
+// accumulates rho = sum_pairs psi_pair lam_pair^dag (a 2x2 matrix) once at
+// the run's output; each constituent j of the run then gives
+// dL/dt_j = Im Tr(W_j P_j W_j^dag rho) with W_j the constituents after j.
+//
+// Execution model ("resident" path).  A sample's state lives in shared
+// memory.  A group of T = 2^(n-K) threads owns one sample; in each stage a
+// thread loads the 2^K amplitudes spanned by the stage's K active qubits into
+// registers (its block; the other n-K index bits come from the thread index),
+// applies all of the stage's ops there, and stores the block back.  Blocks of
+// different threads are disjoint, so one group barrier per stage suffices.
+// Gate matrices are evaluated once per sample (sincos once per angle) into a
+// shared-memory table before the sweep.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "plan.h"
+
+namespace vqc {
+
+template <typename R> struct V2;
+template <> struct V2<float> { using t = float2; };
+template <> struct V2<double> { using t = double2; };
+template <typename R> using C2 = typename V2<R>::t;
+
+template <typename R>
+__device__ __forceinline__ C2<R> cm(R x, R y) { C2<R> r; r.x = x; r.y = y; return r; }
+
+template <typename R>
+__device__ __forceinline__ C2<R> cmul(C2<R> a, C2<R> b) {
+    return cm<R>(fma(a.x, b.x, -a.y * b.y), fma(a.x, b.y, a.y * b.x));
+}
+// m0 * u + m1 * v
+template <typename R>
+__device__ __forceinline__ C2<R> cmv2(C2<R> m0, C2<R> u, C2<R> m1, C2<R> v) {
+    R x = fma(m0.x, u.x, fma(-m0.y, u.y, fma(m1.x, v.x, -m1.y * v.y)));
+    R y = fma(m0.x, u.y, fma(m0.y, u.x, fma(m1.x, v.y, m1.y * v.x)));
+    return cm<R>(x, y);
+}
+template <typename R>
+__device__ __forceinline__ C2<R> cconj(C2<R> a) { return cm<R>(a.x, -a.y); }
+
+template <typename R> struct M2 { C2<R> a, b, c, d; };   // [[a, b], [c, d]]
+
+template <typename R>
+__device__ __forceinline__ M2<R> mmul(const M2<R>& p, const M2<R>& q) {   // p * q
+    M2<R> r;
+    r.a = cmv2<R>(p.a, q.a, p.b, q.c);
+    r.b = cmv2<R>(p.a, q.b, p.b, q.d);
+    r.c = cmv2<R>(p.c, q.a, p.d, q.c);
+    r.d = cmv2<R>(p.c, q.b, p.d, q.d);
+    return r;
+}
+template <typename R>
+__device__ __forceinline__ M2<R> mdag(const M2<R>& p) {
+    M2<R> r;
+    r.a = cconj<R>(p.a); r.b = cconj<R>(p.c); r.c = cconj<R>(p.b); r.d = cconj<R>(p.d);
+    return r;
+}
+template <typename R>
+__device__ __forceinline__ M2<R> mident() {
+    M2<R> r;
+    r.a = cm<R>(1, 0); r.b = cm<R>(0, 0); r.c = cm<R>(0, 0); r.d = cm<R>(1, 0);
+    return r;
+}
+
+__device__ __forceinline__ void sc(float t, float* s, float* c) { sincosf(t, s, c); }
+__device__ __forceinline__ void sc(double t, double* s, double* c) { sincos(t, s, c); }
+
+// ---------------------------------------------------------------- kernel args
+template <typename R>
+struct KArgs {
+    // plan
+    const DOp* ops;
+    const DStage* stages;
+    int nstages;
+    const DEntry* entries;
+    const int32_t* ps_list;   // per-sample entry ids
+    const int32_t* sh_list;   // shared entry ids
+    const DConst* consts;
+    const R* cmat;
+    const R* cang;
+    const DAcc* accs;
+    const int32_t* xocc_ptr;
+    const int32_t* xocc;
+    const int32_t* wocc_ptr;
+    const int32_t* wocc;
+    unsigned* err;
+    int n, K, tbits, G, S;     // S = samples per CTA
+    int n_ps, n_sh, n_accs, n_terms, Px, Pw;
+    // batch
+    int B, nunits;
+    const R* x;
+    const R* w;
+    const C2<R>* psi0;
+    const C2<R>* psi_final;
+    const R* gE;
+    R* E;
+    C2<R>* state_out;
+    R* dx;
+    R* dw;
+    R* dw_part;          // [gridDim.x, Pw]
+    unsigned* counter;
+    // shared-memory carve-up (byte offsets)
+    int sm_sh, sm_ps, sm_psi, sm_lam, sm_acc, sm_terms, sm_dw, sm_red;
+};
+
+// ---------------------------------------------------------------- tables
+template <typename R>
+__device__ __forceinline__ R angle_of(uint8_t src, int32_t idx, const R* xb, const R* w,
+                                      const R* cang) {
+    if (src == SRC_X) return xb[idx];
+    if (src == SRC_W) return w[idx];
+    return cang[idx];
+}
+
+// Matrix of one constituent of a run.
+template <typename R>
+__device__ M2<R> constituent(const DConst& c, const R* xb, const R* w, const R* cang,
+                             const R* cmat) {
+    M2<R> u;
+    if (c.kind == CK_CONST) {
+        const R* m = cmat + 8 * c.idx0;
+        u.a = cm<R>(m[0], m[1]); u.b = cm<R>(m[2], m[3]);
+        u.c = cm<R>(m[4], m[5]); u.d = cm<R>(m[6], m[7]);
+        return u;
+    }
+    R t = angle_of<R>(c.src0, c.idx0, xb, w, cang);
+    if (c.kind == CK_GPHASE) t += angle_of<R>(c.src1, c.idx1, xb, w, cang);
+    R s, co;
+    sc(t * R(0.5), &s, &co);
+    const C2<R> z = cm<R>(0, 0);
+    switch (c.kind) {
+    case CK_RX: u.a = cm<R>(co, 0); u.b = cm<R>(0, -s); u.c = cm<R>(0, -s); u.d = cm<R>(co, 0); break;
+    case CK_RY: u.a = cm<R>(co, 0); u.b = cm<R>(-s, 0); u.c = cm<R>(s, 0); u.d = cm<R>(co, 0); break;
+    case CK_RZ: u.a = cm<R>(co, -s); u.b = z; u.c = z; u.d = cm<R>(co, s); break;
+    default:    u.a = cm<R>(co, s); u.b = z; u.c = z; u.d = cm<R>(co, s); break;   // CK_GPHASE
+    }
+    return u;
+}
+
+// Evaluate one table entry (8 reals) for sample row xb.
+template <typename R>
+__device__ void eval_entry(const DEntry& e, const DConst* consts, const R* xb, const R* w,
+                           const R* cang, const R* cmat, R* out) {
+    if (e.phase) {
+        const DConst c = consts[e.cfirst];
+        R t = angle_of<R>(c.src0, c.idx0, xb, w, cang);
+        R s, co;
+        sc(t * R(0.5), &s, &co);
+        if (c.kind == CK_CRZ) {
+            out[0] = 1; out[1] = 0; out[2] = co; out[3] = -s;
+            out[4] = 1; out[5] = 0; out[6] = co; out[7] = s;
+        } else {   // CK_RZZ: parity 0 -> e^{-it/2}, parity 1 -> e^{it/2}
+            out[0] = co; out[1] = -s; out[2] = co; out[3] = s;
+            out[4] = co; out[5] = s; out[6] = co; out[7] = -s;
+        }
+        return;
+    }
+    M2<R> m = mident<R>();
+    for (int k = 0; k < e.ccount; ++k) {
+        const DConst c = consts[e.cfirst + k];
+        m = mmul<R>(constituent<R>(c, xb, w, cang, cmat), m);
+    }
+    out[0] = m.a.x; out[1] = m.a.y; out[2] = m.b.x; out[3] = m.b.y;
+    out[4] = m.c.x; out[5] = m.c.y; out[6] = m.d.x; out[7] = m.d.y;
+}
+
+template <typename R>
+__device__ __forceinline__ M2<R> load_m2(const R* p) {
+    M2<R> m;
+    m.a = cm<R>(p[0], p[1]); m.b = cm<R>(p[2], p[3]);
+    m.c = cm<R>(p[4], p[5]); m.d = cm<R>(p[6], p[7]);
+    return m;
+}
+
+// ---------------------------------------------------------------- block ops
+// Pair (i0, i1) = (r with bit T clear, r with bit T set), p enumerates pairs.
+template <int T>
+__host__ __device__ constexpr int pair_lo(int p) { return ((p >> T) << (T + 1)) | (p & ((1 << T) - 1)); }
+
+template <typename R, int K, int T>
+__device__ __forceinline__ void m1_apply(C2<R> (&a)[1 << K], const M2<R>& m) {
+#pragma unroll
+    for (int p = 0; p < (1 << (K - 1)); ++p) {
+        const int i0 = pair_lo<T>(p), i1 = i0 | (1 << T);
+        C2<R> u = a[i0], v = a[i1];
+        a[i0] = cmv2<R>(m.a, u, m.b, v);
+        a[i1] = cmv2<R>(m.c, u, m.d, v);
+    }
+}
+
+// rho[a][b] += sum_pairs psi[a] conj(lam[b])  -> r[0..7] = (00, 01, 10, 11) re/im
+template <typename R, int K, int T>
+__device__ __forceinline__ void m1_rho(const C2<R> (&ps)[1 << K], const C2<R> (&la)[1 << K],
+                                       R (&r)[8]) {
+#pragma unroll
+    for (int p = 0; p < (1 << (K - 1)); ++p) {
+        const int i0 = pair_lo<T>(p), i1 = i0 | (1 << T);
+        const C2<R> u = ps[i0], v = ps[i1], q0 = la[i0], q1 = la[i1];
+        r[0] = fma(u.x, q0.x, fma(u.y, q0.y, r[0])); r[1] = fma(u.y, q0.x, fma(-u.x, q0.y, r[1]));
+        r[2] = fma(u.x, q1.x, fma(u.y, q1.y, r[2])); r[3] = fma(u.y, q1.x, fma(-u.x, q1.y, r[3]));
+        r[4] = fma(v.x, q0.x, fma(v.y, q0.y, r[4])); r[5] = fma(v.y, q0.x, fma(-v.x, q0.y, r[5]));
+        r[6] = fma(v.x, q1.x, fma(v.y, q1.y, r[6])); r[7] = fma(v.y, q1.x, fma(-v.x, q1.y, r[7]));
+    }
+}
+
+template <typename R, int K>
+__device__ __forceinline__ void m1_dispatch(int t, C2<R> (&a)[1 << K], const M2<R>& m) {
+    switch (t) {
+    case 0: m1_apply<R, K, 0>(a, m); break;
+    case 1: if constexpr (K > 1) m1_apply<R, K, 1>(a, m); break;
+    case 2: if constexpr (K > 2) m1_apply<R, K, 2>(a, m); break;
+    case 3: if constexpr (K > 3) m1_apply<R, K, 3>(a, m); break;
+    case 4: if constexpr (K > 4) m1_apply<R, K, 4>(a, m); break;
+    default: break;
+    }
+}
+
+template <typename R, int K>
+__device__ __forceinline__ void m1_rho_dispatch(int t, const C2<R> (&ps)[1 << K],
+                                                const C2<R> (&la)[1 << K], R (&r)[8]) {
+    switch (t) {
+    case 0: m1_rho<R, K, 0>(ps, la, r); break;
+    case 1: if constexpr (K > 1) m1_rho<R, K, 1>(ps, la, r); break;
+    case 2: if constexpr (K > 2) m1_rho<R, K, 2>(ps, la, r); break;
+    case 3: if constexpr (K > 3) m1_rho<R, K, 3>(ps, la, r); break;
+    case 4: if constexpr (K > 4) m1_rho<R, K, 4>(ps, la, r); break;
+    default: break;
+    }
+}
+
+// CX with local control C and local target T: swap (r, r^T) for r with C set, T clear.
+template <typename R, int K, int Cc, int T>
+__device__ __forceinline__ void cx_ll(C2<R> (&a)[1 << K]) {
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r) {
+        if (((r >> Cc) & 1) && !((r >> T) & 1)) {
+            C2<R> u = a[r];
+            a[r] = a[r | (1 << T)];
+            a[r | (1 << T)] = u;
+        }
+    }
+}
+
+template <typename R, int K>
+__device__ __forceinline__ void cx_ll_dispatch(int c, int t, C2<R> (&a)[1 << K]) {
+#define VQC_CXCASE(C_, T_) \
+    case C_ * 8 + T_: if constexpr (C_ < K && T_ < K) cx_ll<R, K, C_, T_>(a); break;
+    switch (c * 8 + t) {
+        VQC_CXCASE(0, 1) VQC_CXCASE(0, 2) VQC_CXCASE(0, 3) VQC_CXCASE(0, 4)
+        VQC_CXCASE(1, 0) VQC_CXCASE(1, 2) VQC_CXCASE(1, 3) VQC_CXCASE(1, 4)
+        VQC_CXCASE(2, 0) VQC_CXCASE(2, 1) VQC_CXCASE(2, 3) VQC_CXCASE(2, 4)
+        VQC_CXCASE(3, 0) VQC_CXCASE(3, 1) VQC_CXCASE(3, 2) VQC_CXCASE(3, 4)
+        VQC_CXCASE(4, 0) VQC_CXCASE(4, 1) VQC_CXCASE(4, 2) VQC_CXCASE(4, 3)
+        default: break;
+    }
+#undef VQC_CXCASE
+}
+
+// X on local T when the predicate holds (control outside the block).
+template <typename R, int K, int T>
+__device__ __forceinline__ void x_pred(C2<R> (&a)[1 << K], bool p) {
+#pragma unroll
+    for (int q = 0; q < (1 << (K - 1)); ++q) {
+        const int i0 = pair_lo<T>(q), i1 = i0 | (1 << T);
+        C2<R> u = a[i0], v = a[i1];
+        a[i0] = p ? v : u;
+        a[i1] = p ? u : v;
+    }
+}
+
+template <typename R, int K>
+__device__ __forceinline__ void x_pred_dispatch(int t, C2<R> (&a)[1 << K], bool p) {
+    switch (t) {
+    case 0: x_pred<R, K, 0>(a, p); break;
+    case 1: if constexpr (K > 1) x_pred<R, K, 1>(a, p); break;
+    case 2: if constexpr (K > 2) x_pred<R, K, 2>(a, p); break;
+    case 3: if constexpr (K > 3) x_pred<R, K, 3>(a, p); break;
+    case 4: if constexpr (K > 4) x_pred<R, K, 4>(a, p); break;
+    default: break;
+    }
+}
+
+// Negate amplitudes with local bits A and Bq set (when p) -- CZ inside the block.
+template <typename R, int K, int A, int Bq>
+__device__ __forceinline__ void z2_ll(C2<R> (&a)[1 << K]) {
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r)
+        if (((r >> A) & 1) && ((r >> Bq) & 1)) a[r] = cm<R>(-a[r].x, -a[r].y);
+}
+template <typename R, int K, int A>
+__device__ __forceinline__ void z1_pred(C2<R> (&a)[1 << K], bool p) {
+    const R s = p ? R(-1) : R(1);
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r)
+        if ((r >> A) & 1) a[r] = cm<R>(s * a[r].x, s * a[r].y);
+}
+
+template <typename R, int K>
+__device__ __forceinline__ void cz_dispatch(int ra, int rb, uint32_t pb, C2<R> (&a)[1 << K]) {
+    if (ra >= kRefPhys && rb >= kRefPhys) {
+        const bool p = ((pb >> (ra - kRefPhys)) & (pb >> (rb - kRefPhys)) & 1u) != 0;
+        const R s = p ? R(-1) : R(1);
+#pragma unroll
+        for (int r = 0; r < (1 << K); ++r) a[r] = cm<R>(s * a[r].x, s * a[r].y);
+        return;
+    }
+    if (ra >= kRefPhys || rb >= kRefPhys) {
+        const int l = ra >= kRefPhys ? rb : ra;
+        const int ph = ra >= kRefPhys ? ra : rb;
+        const bool p = ((pb >> (ph - kRefPhys)) & 1u) != 0;
+        switch (l) {
+        case 0: z1_pred<R, K, 0>(a, p); break;
+        case 1: if constexpr (K > 1) z1_pred<R, K, 1>(a, p); break;
+        case 2: if constexpr (K > 2) z1_pred<R, K, 2>(a, p); break;
+        case 3: if constexpr (K > 3) z1_pred<R, K, 3>(a, p); break;
+        case 4: if constexpr (K > 4) z1_pred<R, K, 4>(a, p); break;
+        default: break;
+        }
+        return;
+    }
+    const int lo = ra < rb ? ra : rb, hi = ra < rb ? rb : ra;
+#define VQC_ZCASE(A_, B_) \
+    case A_ * 8 + B_: if constexpr (A_ < K && B_ < K) z2_ll<R, K, A_, B_>(a); break;
+    switch (lo * 8 + hi) {
+        VQC_ZCASE(0, 1) VQC_ZCASE(0, 2) VQC_ZCASE(0, 3) VQC_ZCASE(0, 4)
+        VQC_ZCASE(1, 2) VQC_ZCASE(1, 3) VQC_ZCASE(1, 4)
+        VQC_ZCASE(2, 3) VQC_ZCASE(2, 4) VQC_ZCASE(3, 4)
+        default: break;
+    }
+#undef VQC_ZCASE
+}
+
+__device__ __forceinline__ int refbit(int ref, int r, uint32_t pb) {
+    return ref >= kRefPhys ? (int)((pb >> (ref - kRefPhys)) & 1u) : ((r >> ref) & 1);
+}
+
+// Diagonal two-qubit phase: a[r] *= ph[bit a + 2 bit b]  (conj when ADJ).
+template <typename R, int K, bool ADJ>
+__device__ __forceinline__ void ph2_apply(int ra, int rb, uint32_t pb, C2<R> (&a)[1 << K],
+                                          const C2<R> (&ph)[4]) {
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r) {
+        const int s = refbit(ra, r, pb) + 2 * refbit(rb, r, pb);
+        C2<R> f = s == 0 ? ph[0] : s == 1 ? ph[1] : s == 2 ? ph[2] : ph[3];
+        if (ADJ) f.y = -f.y;
+        a[r] = cmul<R>(a[r], f);
+    }
+}
+
+// Im <lam|P|psi> over the block for the phase op's generator.
+template <typename R, int K>
+__device__ __forceinline__ R ph2_term(int ra, int rb, uint32_t pb, uint8_t flags,
+                                      const C2<R> (&ps)[1 << K], const C2<R> (&la)[1 << K]) {
+    R acc = 0;
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r) {
+        const int ba = refbit(ra, r, pb), bb = refbit(rb, r, pb);
+        R g;
+        if (flags & OPF_GEN_CRZ) g = ba ? (bb ? R(-1) : R(1)) : R(0);
+        else g = (ba ^ bb) ? R(-1) : R(1);
+        acc = fma(g, la[r].x * ps[r].y - la[r].y * ps[r].x, acc);
+    }
+    return acc;
+}
+
+// ---------------------------------------------------------------- reductions
+template <typename R>
+__device__ __forceinline__ R shx(R v, int m) { return __shfl_xor_sync(0xffffffffu, v, m); }
+
+// Reduce 8 values over a group of `lanes` lanes (power of two <= 32) and
+// write the 8 sums to dst (reduce-scatter butterfly: 9 shuffles at 32 lanes).
+template <typename R>
+__device__ __forceinline__ void reduce8_store(R (&v)[8], int lanes, int lane, R* dst) {
+    int u0 = 0, u1 = 0, u2 = 0;
+    if (lanes >= 2) {
+        const int m = lanes >> 1;
+        u0 = (lane & m) ? 1 : 0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            R send = u0 ? v[i] : v[i + 4];
+            R keep = u0 ? v[i + 4] : v[i];
+            v[i] = keep + shx<R>(send, m);
+        }
+    }
+    if (lanes >= 4) {
+        const int m = lanes >> 2;
+        u1 = (lane & m) ? 1 : 0;
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            R send = u1 ? v[i] : v[i + 2];
+            R keep = u1 ? v[i + 2] : v[i];
+            v[i] = keep + shx<R>(send, m);
+        }
+    }
+    if (lanes >= 8) {
+        const int m = lanes >> 3;
+        u2 = (lane & m) ? 1 : 0;
+        R send = u2 ? v[0] : v[1];
+        R keep = u2 ? v[1] : v[0];
+        v[0] = keep + shx<R>(send, m);
+        for (int mm = lanes >> 4; mm >= 1; mm >>= 1) v[0] += shx<R>(v[0], mm);
+        if ((lane & ((lanes >> 3) - 1)) == 0) dst[4 * u0 + 2 * u1 + u2] = v[0];
+    } else if (lanes == 4) {
+        dst[4 * u0 + 2 * u1] = v[0];
+        dst[4 * u0 + 2 * u1 + 1] = v[1];
+    } else if (lanes == 2) {
+        for (int i = 0; i < 4; ++i) dst[4 * u0 + i] = v[i];
+    } else {
+        for (int i = 0; i < 8; ++i) dst[i] = v[i];
+    }
+}
+
+template <typename R>
+__device__ __forceinline__ R reduce1(R v, int lanes) {
+    for (int m = lanes >> 1; m >= 1; m >>= 1) v += shx<R>(v, m);
+    return v;
+}
+
+// ---------------------------------------------------------------- addressing
+struct Geo {
+    int T;        // threads per sample group
+    int lanes;    // min(T, 32)
+    int wg;       // warps per group (>= 1)
+    int g;        // group (sample slot) index in the CTA
+    int t;        // thread index in the group
+    int h;        // per-sample XOR on the slot index (bank spreading of small groups)
+};
+
+__device__ __forceinline__ uint32_t swz(uint32_t u, int G) {
+    uint32_t v = u >> G, f = 0;
+    while (v) { f ^= v; v >>= G; }
+    return u ^ (f & ((1u << G) - 1));
+}
+
+template <typename R>
+__device__ __forceinline__ void group_sync(const Geo& q) {
+    if (q.T > 32) __syncthreads(); else __syncwarp();
+}
+
+template <int K>
+__device__ __forceinline__ uint32_t block_off(int r, const int32_t (&sg)[K]) {
+    uint32_t o = 0;
+#pragma unroll
+    for (int j = 0; j < K; ++j)
+        if ((r >> j) & 1) o ^= (uint32_t)sg[j];
+    return o;
+}
+
+struct StageView {
+    uint32_t swb, pb;
+};
+
+template <int K>
+__device__ __forceinline__ StageView stage_view(const DStage* sp, int t, int h, int32_t (&sg)[K]) {
+#pragma unroll
+    for (int j = 0; j < K; ++j) sg[j] = __ldg(&sp->sigma[j]);
+    const int nb = __ldg(&sp->nthreadbits);   // uint8 load
+    StageView v{(uint32_t)h, 0u};
+    for (int i = 0; i < nb; ++i) {
+        if ((t >> i) & 1) {
+            v.swb ^= (uint32_t)__ldg(&sp->tau[i]);
+            v.pb |= __ldg(&sp->tmask[i]);
+        }
+    }
+    return v;
+}
+
+template <typename R, int K>
+__device__ __forceinline__ void block_load(C2<R> (&a)[1 << K], const C2<R>* st, uint32_t swb,
+                                           const int32_t (&sg)[K]) {
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r) a[r] = st[swb ^ block_off<K>(r, sg)];
+}
+template <typename R, int K>
+__device__ __forceinline__ void block_store(const C2<R> (&a)[1 << K], C2<R>* st, uint32_t swb,
+                                            const int32_t (&sg)[K]) {
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r) st[swb ^ block_off<K>(r, sg)] = a[r];
+}
+
+// ---------------------------------------------------------------- forward op
+template <typename R, int K>
+__device__ __forceinline__ void fwd_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 << K],
+                                       const R* sh_tab, const R* ps_tab) {
+    const int type = raw.x & 0xff, ra = (raw.x >> 8) & 0xff, rb = (raw.x >> 16) & 0xff;
+    const int flags = raw.x >> 24, slot = raw.y & 0xffff;
+    const R* tab = (flags & OPF_PER_SAMPLE) ? ps_tab : sh_tab;
+    if (type == OP_M1) {
+        const M2<R> m = load_m2<R>(tab + 8 * slot);
+        m1_dispatch<R, K>(ra, a, m);
+    } else if (type == OP_CX) {
+        if (ra < kRefPhys) cx_ll_dispatch<R, K>(ra, rb, a);
+        else x_pred_dispatch<R, K>(rb, a, ((pb >> (ra - kRefPhys)) & 1u) != 0);
+    } else if (type == OP_CZ) {
+        cz_dispatch<R, K>(ra, rb, pb, a);
+    } else if (type == OP_PH2) {
+        const R* p = tab + 8 * slot;
+        C2<R> ph[4] = {cm<R>(p[0], p[1]), cm<R>(p[2], p[3]), cm<R>(p[4], p[5]), cm<R>(p[6], p[7])};
+        ph2_apply<R, K, false>(ra, rb, pb, a, ph);
+    }
+}
+
+// ---------------------------------------------------------------- kernel
+template <typename R, int K, int MODE>
+struct MaxThreads {
+    static constexpr int value = (sizeof(R) == 4 && MODE == 0 && K <= 4) ? 1024 : 512;
+};
+
+// MODE 0: forward, MODE 1: backward.
+template <typename R, int K, int MODE>
+__global__ void __launch_bounds__(MaxThreads<R, K, MODE>::value)
+sweep_kernel(const __grid_constant__ KArgs<R> A) {
+    extern __shared__ __align__(16) unsigned char smem[];
+    R* sh_tab = reinterpret_cast<R*>(smem + A.sm_sh);
+    R* ps_all = reinterpret_cast<R*>(smem + A.sm_ps);
+    C2<R>* psi_all = reinterpret_cast<C2<R>*>(smem + A.sm_psi);
+    C2<R>* lam_all = reinterpret_cast<C2<R>*>(smem + A.sm_lam);
+    R* acc_all = reinterpret_cast<R*>(smem + A.sm_acc);
+    R* terms_all = reinterpret_cast<R*>(smem + A.sm_terms);
+    R* dw_cta = reinterpret_cast<R*>(smem + A.sm_dw);
+    R* red_all = reinterpret_cast<R*>(smem + A.sm_red);
+
+    const int n = A.n, G = A.G;
+    const int dim = 1 << n;
+    Geo q;
+    q.T = 1 << A.tbits;
+    q.lanes = q.T < 32 ? q.T : 32;
+    q.wg = q.T > 32 ? q.T / 32 : 1;
+    q.g = threadIdx.x / q.T;
+    q.t = threadIdx.x % q.T;
+    q.h = 0;
+    if (A.tbits < G) q.h = ((q.g & ((1 << (G - A.tbits)) - 1)) << A.tbits) & (dim - 1);
+    const int lane = q.t & 31;
+    const int warp_in_group = q.t >> 5;
+    const int nthr = blockDim.x;
+
+    // shared table (w and constants): once per CTA
+    for (int i = threadIdx.x; i < A.n_sh; i += nthr) {
+        const int id = __ldg(&A.sh_list[i]);
+        const DEntry e = A.entries[id];
+        eval_entry<R>(e, A.consts, nullptr, A.w, A.cang, A.cmat, sh_tab + 8 * e.slot);
+    }
+    if (MODE == 1)
+        for (int i = threadIdx.x; i < A.Pw; i += nthr) dw_cta[i] = 0;
+    __syncthreads();
+
+    C2<R>* psi = psi_all + (size_t)q.g * dim;
+    C2<R>* lam = lam_all + (size_t)q.g * dim;
+    R* ps_tab = ps_all + (size_t)q.g * A.n_ps * 8;
+    R* acc = acc_all + (size_t)q.g * A.n_accs * q.wg * 8;
+    R* terms = terms_all + (size_t)q.g * A.n_terms;
+
+    for (int unit = blockIdx.x; unit < A.nunits; unit += gridDim.x) {
+        const int b_raw = unit * A.S + q.g;
+        const bool valid = b_raw < A.B;
+        const int b = valid ? b_raw : A.B - 1;
+        const R* xb = A.x ? A.x + (size_t)b * A.Px : nullptr;
+
+        // per-sample table (x-dependent runs): threads of the CTA over (sample, entry)
+        for (int i = threadIdx.x; i < A.S * A.n_ps; i += nthr) {
+            const int gg = i / A.n_ps, k = i % A.n_ps;
+            const int bb = min(unit * A.S + gg, A.B - 1);
+            const int id = __ldg(&A.ps_list[k]);
+            const DEntry e = A.entries[id];
+            eval_entry<R>(e, A.consts, A.x + (size_t)bb * A.Px, A.w, A.cang, A.cmat,
+                          ps_all + ((size_t)gg * A.n_ps + e.slot) * 8);
+        }
+        // initial / final state from global memory (coalesced, into swizzled slots)
+        const C2<R>* src = MODE == 1 ? A.psi_final : A.psi0;
+        if (MODE == 1 && !src) src = A.psi0;
+        const bool from_global = src != nullptr;
+        if (from_global) {
+            const C2<R>* gs = src + (size_t)b * dim;
+            for (int u = q.t; u < dim; u += q.T) psi[swz(u, G) ^ q.h] = gs[u];
+        }
+        __syncthreads();
+
+        C2<R> a[1 << K];
+        int32_t sg[K];
+        StageView v{0, 0};
+        const bool recompute = MODE == 1 && A.psi_final == nullptr;
+        const int ns = A.nstages;
+
+        // -------- forward sweep (forward mode, or backward recompute)
+        if (MODE == 0 || recompute) {
+            for (int s = 0; s < ns; ++s) {
+                const DStage* sp = A.stages + s;
+                v = stage_view<K>(sp, q.t, q.h, sg);
+                if (s == 0 && !from_global) {
+#pragma unroll
+                    for (int r = 0; r < (1 << K); ++r) a[r] = cm<R>(0, 0);
+                    if (v.pb == 0) a[0] = cm<R>(1, 0);
+                } else {
+                    block_load<R, K>(a, psi, v.swb, sg);
+                }
+                const int ob = __ldg(&sp->op_begin), oe = __ldg(&sp->op_end);
+                for (int o = ob; o < oe; ++o) {
+                    const uint2 raw = __ldg(reinterpret_cast<const uint2*>(A.ops) + o);
+                    fwd_op<R, K>(raw, v.pb, a, sh_tab, ps_tab);
+                }
+                if (s + 1 < ns || (MODE == 0 && A.state_out)) {
+                    block_store<R, K>(a, psi, v.swb, sg);
+                    group_sync<R>(q);
+                }
+            }
+        }
+
+        if (MODE == 0) {
+            // -------- <Z_j> partials from the final block
+            const DStage* sp = A.stages + (ns - 1);
+            R pr[1 << K];
+            R ptot = 0;
+#pragma unroll
+            for (int r = 0; r < (1 << K); ++r) {
+                pr[r] = fma(a[r].x, a[r].x, a[r].y * a[r].y);
+                ptot += pr[r];
+            }
+            R dloc[K];
+#pragma unroll
+            for (int j = 0; j < K; ++j) {
+                R d = 0;
+#pragma unroll
+                for (int r = 0; r < (1 << K); ++r) d += ((r >> j) & 1) ? -pr[r] : pr[r];
+                dloc[j] = d;
+            }
+            uint32_t actmask = 0;
+            int aq[K];
+#pragma unroll
+            for (int j = 0; j < K; ++j) {
+                aq[j] = __ldg(&sp->active[j]);
+                actmask |= 1u << aq[j];
+            }
+            R* red = red_all + (size_t)q.g * q.wg * n;
+            for (int j = 0; j < n; ++j) {
+                R val;
+                if ((actmask >> j) & 1) {
+                    val = 0;
+#pragma unroll
+                    for (int k = 0; k < K; ++k) if (aq[k] == j) val = dloc[k];
+                } else {
+                    val = ((v.pb >> j) & 1u) ? -ptot : ptot;
+                }
+                val = reduce1<R>(val, q.lanes);
+                if ((q.t & (q.lanes - 1)) == 0) red[warp_in_group * n + j] = val;
+            }
+            __syncthreads();
+            if (valid) {
+                for (int j = q.t; j < n; j += q.T) {
+                    R e = 0;
+                    for (int k = 0; k < q.wg; ++k) e += red[k * n + j];
+                    A.E[(size_t)b * n + j] = e;
+                }
+                if (A.state_out) {
+                    C2<R>* go = A.state_out + (size_t)b * dim;
+                    for (int u = q.t; u < dim; u += q.T) go[u] = psi[swz(u, G) ^ q.h];
+                }
+            }
+            __syncthreads();
+            continue;
+        }
+
+        // -------- backward: reverse sweep with psi and lam
+        R ge_loc[K];
+        for (int s = ns - 1; s >= 0; --s) {
+            const DStage* sp = A.stages + s;
+            C2<R> l[1 << K];
+            if (s == ns - 1) {
+                v = stage_view<K>(sp, q.t, q.h, sg);
+                if (!recompute) block_load<R, K>(a, psi, v.swb, sg);
+                // lam = O psi with O = sum_j gE_j Z_j (diagonal)
+                const R* gb = A.gE + (size_t)b * n;
+                R cst = 0;
+                uint32_t actmask = 0;
+#pragma unroll
+                for (int j = 0; j < K; ++j) {
+                    const int aq = __ldg(&sp->active[j]);
+                    actmask |= 1u << aq;
+                    ge_loc[j] = gb[aq];
+                }
+                for (int j = 0; j < n; ++j)
+                    if (!((actmask >> j) & 1)) cst += ((v.pb >> j) & 1u) ? -gb[j] : gb[j];
+#pragma unroll
+                for (int r = 0; r < (1 << K); ++r) {
+                    R o = cst;
+#pragma unroll
+                    for (int j = 0; j < K; ++j) o += ((r >> j) & 1) ? -ge_loc[j] : ge_loc[j];
+                    l[r] = cm<R>(o * a[r].x, o * a[r].y);
+                }
+            } else {
+                v = stage_view<K>(sp, q.t, q.h, sg);
+                block_load<R, K>(a, psi, v.swb, sg);
+                block_load<R, K>(l, lam, v.swb, sg);
+            }
+            const int ob = __ldg(&sp->op_begin), oe = __ldg(&sp->op_end);
+            for (int o = oe - 1; o >= ob; --o) {
+                const uint2 raw = __ldg(reinterpret_cast<const uint2*>(A.ops) + o);
+                const int type = raw.x & 0xff, ra = (raw.x >> 8) & 0xff, rb = (raw.x >> 16) & 0xff;
+                const int flags = raw.x >> 24, slot = raw.y & 0xffff, aux = raw.y >> 16;
+                const R* tab = (flags & OPF_PER_SAMPLE) ? ps_tab : sh_tab;
+                if (type == OP_M1) {
+                    const M2<R> m = load_m2<R>(tab + 8 * slot);
+                    if (flags & OPF_HAS_ACC) {
+                        R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+                        m1_rho_dispatch<R, K>(ra, a, l, rh);
+                        reduce8_store<R>(rh, q.lanes, q.lanes < 32 ? q.t : lane,
+                                         acc + ((size_t)aux * q.wg + warp_in_group) * 8);
+                    }
+                    const M2<R> md = mdag<R>(m);
+                    m1_dispatch<R, K>(ra, a, md);
+                    m1_dispatch<R, K>(ra, l, md);
+                } else if (type == OP_CX) {
+                    if (ra < kRefPhys) {
+                        cx_ll_dispatch<R, K>(ra, rb, a);
+                        cx_ll_dispatch<R, K>(ra, rb, l);
+                    } else {
+                        const bool p = ((v.pb >> (ra - kRefPhys)) & 1u) != 0;
+                        x_pred_dispatch<R, K>(rb, a, p);
+                        x_pred_dispatch<R, K>(rb, l, p);
+                    }
+                } else if (type == OP_CZ) {
+                    cz_dispatch<R, K>(ra, rb, v.pb, a);
+                    cz_dispatch<R, K>(ra, rb, v.pb, l);
+                } else if (type == OP_PH2) {
+                    const R* p = tab + 8 * slot;
+                    C2<R> ph[4] = {cm<R>(p[0], p[1]), cm<R>(p[2], p[3]), cm<R>(p[4], p[5]),
+                                   cm<R>(p[6], p[7])};
+                    if (flags & OPF_HAS_ACC) {
+                        R tv = ph2_term<R, K>(ra, rb, v.pb, (uint8_t)flags, a, l);
+                        tv = reduce1<R>(tv, q.lanes);
+                        if ((q.t & (q.lanes - 1)) == 0)
+                            acc[((size_t)aux * q.wg + warp_in_group) * 8] = tv;
+                    }
+                    ph2_apply<R, K, true>(ra, rb, v.pb, a, ph);
+                    ph2_apply<R, K, true>(ra, rb, v.pb, l, ph);
+                }
+            }
+            if (s > 0) {
+                block_store<R, K>(a, psi, v.swb, sg);
+                block_store<R, K>(l, lam, v.swb, sg);
+            }
+            group_sync<R>(q);
+        }
+        __syncthreads();
+
+        // -------- gradient terms from the accumulated rho / scalars
+        for (int i = threadIdx.x; i < A.S * A.n_accs; i += nthr) {
+            const int gg = i / A.n_accs, k = i % A.n_accs;
+            const DAcc ac = A.accs[k];
+            const R* ap = acc_all + ((size_t)gg * A.n_accs + k) * q.wg * 8;
+            R* tm = terms_all + (size_t)gg * A.n_terms;
+            const int bb = min(unit * A.S + gg, A.B - 1);
+            const R* xg = A.x ? A.x + (size_t)bb * A.Px : nullptr;
+            const DEntry e = A.entries[ac.entry];
+            if (ac.kind == 1) {
+                R sum = 0;
+                for (int k2 = 0; k2 < q.wg; ++k2) sum += ap[k2 * 8];
+                tm[A.consts[e.cfirst].term] = sum;
+                continue;
+            }
+            R rr[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+            for (int k2 = 0; k2 < q.wg; ++k2)
+                for (int c = 0; c < 8; ++c) rr[c] += ap[k2 * 8 + c];
+            // rho = [[r00, r01], [r10, r11]]; term = Im Tr(W P W^dag rho)
+            M2<R> W = mident<R>();
+            for (int c = e.ccount - 1; c >= 0; --c) {
+                const DConst cn = A.consts[e.cfirst + c];
+                if (cn.term >= 0) {
+                    M2<R> P;
+                    const C2<R> z = cm<R>(0, 0), one = cm<R>(1, 0);
+                    if (cn.kind == CK_RX) { P.a = z; P.b = one; P.c = one; P.d = z; }
+                    else if (cn.kind == CK_RY) { P.a = z; P.b = cm<R>(0, -1); P.c = cm<R>(0, 1); P.d = z; }
+                    else { P.a = one; P.b = z; P.c = z; P.d = cm<R>(-1, 0); }
+                    const M2<R> Mx = mmul<R>(mmul<R>(W, P), mdag<R>(W));
+                    // Im sum_{a,b} M[a][b] rho[b][a]
+                    R im = 0;
+                    im += Mx.a.x * rr[1] + Mx.a.y * rr[0];   // M00 rho00
+                    im += Mx.b.x * rr[5] + Mx.b.y * rr[4];   // M01 rho10
+                    im += Mx.c.x * rr[3] + Mx.c.y * rr[2];   // M10 rho01
+                    im += Mx.d.x * rr[7] + Mx.d.y * rr[6];   // M11 rho11
+                    tm[cn.term] = im;
+                }
+                W = mmul<R>(W, constituent<R>(cn, xg, A.w, A.cang, A.cmat));
+            }
+        }
+        __syncthreads();
+        // dx rows of this CTA's samples; dw partial of this CTA (fixed order)
+        if (A.dx) {
+            for (int i = threadIdx.x; i < A.S * A.Px; i += nthr) {
+                const int gg = i / A.Px, p = i % A.Px;
+                const int bb = unit * A.S + gg;
+                if (bb >= A.B) continue;
+                const R* tm = terms_all + (size_t)gg * A.n_terms;
+                R sum = 0;
+                for (int k = __ldg(&A.xocc_ptr[p]); k < __ldg(&A.xocc_ptr[p + 1]); ++k)
+                    sum += tm[__ldg(&A.xocc[k])];
+                A.dx[(size_t)bb * A.Px + p] = sum;
+            }
+        }
+        for (int p = threadIdx.x; p < A.Pw; p += nthr) {
+            R sum = dw_cta[p];
+            for (int gg = 0; gg < A.S; ++gg) {
+                if (unit * A.S + gg >= A.B) break;
+                const R* tm = terms_all + (size_t)gg * A.n_terms;
+                for (int k = __ldg(&A.wocc_ptr[p]); k < __ldg(&A.wocc_ptr[p + 1]); ++k)
+                    sum += tm[__ldg(&A.wocc[k])];
+            }
+            dw_cta[p] = sum;
+        }
+        __syncthreads();
+    }
+
+    if (MODE == 1 && A.Pw > 0 && A.dw) {
+        // per-CTA partial, then the last CTA to finish sums all partials in
+        // block order (deterministic for a given grid).
+        for (int p = threadIdx.x; p < A.Pw; p += nthr)
+            A.dw_part[(size_t)blockIdx.x * A.Pw + p] = dw_cta[p];
+        __threadfence();
+        __shared__ unsigned last;
+        __syncthreads();
+        if (threadIdx.x == 0) last = atomicInc(A.counter, gridDim.x - 1) == gridDim.x - 1;
+        __syncthreads();
+        if (last) {
+            __threadfence();
+            for (int p = threadIdx.x; p < A.Pw; p += nthr) {
+                R sum = 0;
+                for (int k = 0; k < (int)gridDim.x; ++k)
+                    sum += __ldcg(&A.dw_part[(size_t)k * A.Pw + p]);
+                A.dw[p] = sum;
+            }
+        }
+    }
+}
+
+}  // namespace vqc

@@ -1,0 +1,193 @@
+"""CPU tests of the boundary and the host compiler (no kernel launches).
+
+* libvqc.so loads and exports every entry point declared in include/vqc.h;
+* vqc_compile validates its input (static-circuit scope, paper Sec. 3) and
+  returns the documented status codes;
+* vqc_plan_export is a deterministic function of the compile arguments;
+* every exported stage schedule, executed on the CPU exactly as the kernels
+  address it (tests/plan_emulator.py), reproduces the oracle's final state
+  and the oracle's adjoint gradients;
+* register-block addressing is a bijection onto the shared-memory slots.
+"""
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import oracle as orc
+from paper_2607_11985_gb300 import binding as B
+from paper_2607_11985_gb300 import workloads as wl
+from tests.plan_emulator import Plan, swz
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2607_11985_gb300 import build
+    build.build()
+
+
+def header_functions():
+    with open(os.path.join(ROOT, "include", "vqc.h")) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^[A-Za-z_][\w\s\*]*?\b(vqc_\w+)\s*\(", text, flags=re.M)))
+
+
+def test_library_exports_every_declared_symbol():
+    names = header_functions()
+    assert len(names) >= 11, names
+    lib = B.lib()
+    for name in names:
+        assert hasattr(lib, name), name
+    assert B.vqc_abi_version() == 1
+    assert {s[0] for s in B.SIGNATURES} == set(names)
+
+
+def compile_spec(spec, dtype=0):
+    arr = B.gates_array(spec)
+    return B.vqc_compile(arr, len(spec.gates), spec.n, spec.num_x, spec.num_w, dtype)
+
+
+def status_of(spec, dtype=0, n=None, nx=None, nw=None, arr=None):
+    import ctypes
+    arr = arr if arr is not None else B.gates_array(spec)
+    plan = ctypes.c_void_p()
+    st = B.lib().vqc_compile(arr, len(spec.gates), spec.n if n is None else n,
+                             spec.num_x if nx is None else nx, spec.num_w if nw is None else nw,
+                             dtype, ctypes.byref(plan))
+    if st == 0:
+        B.vqc_free(plan.value)
+    return st
+
+
+def test_validation_codes():
+    ok = wl.CircuitSpec(3, 1, 1).add("RY", (0,), [("x", 0)]).add("CX", (0, 2)).add("RZ", (1,), [("w", 0)])
+    assert status_of(ok) == 0
+    assert status_of(wl.CircuitSpec(3, 0, 0).add("H", (3,))) == 3            # qubit range
+    assert status_of(wl.CircuitSpec(3, 0, 0).add("CX", (1, 1))) == 3         # repeated qubit
+    assert status_of(wl.CircuitSpec(3, 1, 0).add("RX", (0,), [("x", 1)])) == 5   # x column
+    assert status_of(wl.CircuitSpec(3, 0, 1).add("RX", (0,), [("w", 3)])) == 5   # w index
+    assert status_of(ok, n=0) == 4
+    assert status_of(ok, n=25) == 4
+    assert status_of(ok, nx=-1) == 1
+    assert status_of(ok, dtype=7) == 1
+    arr = B.gates_array(ok)
+    arr[0].op = 16
+    assert status_of(ok, arr=arr) == 2
+    arr = B.gates_array(ok)
+    arr[1].reserved[0] = 1
+    assert status_of(ok, arr=arr) == 1
+    arr = B.gates_array(ok)
+    arr[0].pkind[0] = 0
+    assert status_of(ok, arr=arr) == 5
+    assert "invalid source" in B.vqc_last_error()
+
+
+def test_export_deterministic_and_info():
+    for k in (1, 2, 3):
+        spec = wl.config(k)[0].spec
+        p1, p2 = compile_spec(spec), compile_spec(spec)
+        assert B.vqc_plan_export(p1) == B.vqc_plan_export(p2)
+        info = B.vqc_plan_info(p1, 1024)
+        assert info["num_gates_in"] == len(spec.gates)
+        assert info["fwd_path"] == 0 and info["fwd_stages"] >= 1
+        B.vqc_free(p1)
+        B.vqc_free(p2)
+
+
+def check_addressing(plan):
+    for s in plan.scheds:
+        n, K = plan.n, s["K"]
+        for st in s["stages"]:
+            assert sorted(st["active"][:K].tolist()) == st["active"][:K].tolist()
+            assert int(st["nthreadbits"]) == n - K
+            slots = set()
+            for t in range(1 << (n - K)):
+                base, idx = Plan.block_index(st, K, t)
+                swb = 0
+                for i in range(n - K):
+                    if (t >> i) & 1:
+                        swb ^= int(st["tau"][i])
+                for r in range(1 << K):
+                    sl = swb
+                    for j in range(K):
+                        if (r >> j) & 1:
+                            sl ^= int(st["sigma"][j])
+                    assert sl == swz(int(idx[r]), plan.G)
+                    slots.add(sl)
+            assert slots == set(range(1 << n))
+            for op in s["ops"][st["op_begin"]:st["op_end"]]:
+                if op["type"] == 1:
+                    assert op["a"] < K
+                if op["type"] == 2:
+                    assert op["b"] < K
+
+
+SMALL_CASES = [(s, n, g) for s, n, g in [(101, 1, 12), (102, 2, 30), (103, 3, 60), (104, 4, 80),
+                                        (105, 5, 120), (106, 6, 150), (107, 7, 150)]]
+
+
+@pytest.mark.parametrize("seed,n,G", SMALL_CASES)
+@pytest.mark.parametrize("dtype", [0, 1])
+def test_schedules_reproduce_oracle_state(seed, n, G, dtype):
+    w_, psi0 = wl.small_random(seed, n, G, batch=2, dtype="c128", with_psi0=(seed % 2 == 1))
+    pl = Plan(B.vqc_plan_export(compile_spec(w_.spec, dtype)))
+    check_addressing(pl)
+    _, ref = orc.forward(w_.spec, w_.x, w_.w, psi0=psi0, want_state=True)
+    assert len(pl.scheds) >= 2
+    for s in pl.scheds:
+        for b in range(2):
+            xb = w_.x[b] if w_.spec.num_x else np.zeros(0)
+            got = pl.forward(s, xb, w_.w, None if psi0 is None else psi0[b])
+            assert np.allclose(got, ref[b], atol=1e-12), (s["mode"], s["K"])
+
+
+@pytest.mark.parametrize("seed,n,G", SMALL_CASES[:6])
+def test_schedules_reproduce_oracle_gradients(seed, n, G):
+    w_, psi0 = wl.small_random(seed, n, G, batch=2, dtype="c128", with_psi0=(seed % 2 == 0))
+    pl = Plan(B.vqc_plan_export(compile_spec(w_.spec, 1)))
+    dx_ref, dw_ref = orc.backward(w_.spec, w_.x, w_.w, w_.gE, psi0=psi0)
+    for s in pl.scheds:
+        if s["mode"] != 1:
+            continue
+        dw = np.zeros(w_.spec.num_w)
+        for b in range(2):
+            xb = w_.x[b] if w_.spec.num_x else np.zeros(0)
+            dx, dwb = pl.backward(s, xb, w_.w, w_.gE[b], None if psi0 is None else psi0[b])
+            assert np.allclose(dx, dx_ref[b], atol=1e-10), s["K"]
+            dw += dwb
+        assert np.allclose(dw, dw_ref, atol=1e-10), s["K"]
+
+
+@pytest.mark.parametrize("k", [1, 2])
+def test_config_schedules_gradients(k):
+    w_ = wl.config(k, dtype="c128", batch=2)[0]
+    pl = Plan(B.vqc_plan_export(compile_spec(w_.spec, 1)))
+    check_addressing(pl)
+    dx_ref, dw_ref = orc.backward(w_.spec, w_.x, w_.w, w_.gE)
+    s = [s for s in pl.scheds if s["mode"] == 1][-1]
+    dw = np.zeros(w_.spec.num_w)
+    for b in range(2):
+        dx, dwb = pl.backward(s, w_.x[b], w_.w, w_.gE[b])
+        assert np.allclose(dx, dx_ref[b], atol=1e-10)
+        dw += dwb
+    assert np.allclose(dw, dw_ref, atol=1e-10)
+
+
+def test_reupload_config_structure():
+    # config 3 shape at 6 qubits: re-uploaded x, Rot layers, CX range ring
+    spec = wl.layered(6, 3, ("RZ", "RY", "RZ"), "CX", reupload=True, ring_range=lambda l: (l % 5) + 1)
+    rng = np.random.default_rng(3)
+    x = rng.standard_normal((1, 6))
+    w = rng.uniform(-np.pi, np.pi, spec.num_w)
+    gE = rng.standard_normal((1, 6))
+    pl = Plan(B.vqc_plan_export(compile_spec(spec, 1)))
+    dx_ref, dw_ref = orc.backward(spec, x, w, gE)
+    for s in pl.scheds:
+        if s["mode"] == 1:
+            dx, dw = pl.backward(s, x[0], w, gE[0])
+            assert np.allclose(dx, dx_ref[0], atol=1e-10)
+            assert np.allclose(dw, dw_ref, atol=1e-10)

@@ -1,0 +1,265 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle.
+
+Tolerances (stated for this engine): complex64 path -- expectations and
+amplitudes max-abs <= 1e-4, gradients max-abs <= 5e-4; complex128 path --
+<= 1e-10 for all of them.  Inputs are seeded and generated in fp64, rounded to
+the engine's real type, and the oracle consumes the rounded values promoted to
+fp64, so the comparison measures kernel error only.
+"""
+import os
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from oracle import oracle as orc  # noqa: E402
+from paper_2607_11985_gb300 import workloads as wl  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"c64": dict(E=1e-4, state=1e-4, grad=5e-4), "c128": dict(E=1e-10, state=1e-10, grad=1e-10)}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def cuda_ready():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    torch.cuda.set_device(0)
+
+
+def C(spec, dtype):
+    from paper_2607_11985_gb300.circuit import Circuit
+    return Circuit(spec, dtype)
+
+
+def dev(a, dtype):
+    real = torch.float32 if dtype == "c64" else torch.float64
+    return torch.tensor(np.asarray(a), dtype=real, device="cuda")
+
+
+def devc(a, dtype):
+    cplx = torch.complex64 if dtype == "c64" else torch.complex128
+    return torch.tensor(np.asarray(a), dtype=cplx, device="cuda")
+
+
+def run_fwd(c, w_, psi0=None, want_state=True):
+    x = dev(w_.x, w_.dtype) if w_.spec.num_x else None
+    w = dev(w_.w, w_.dtype) if w_.spec.num_w else None
+    p0 = devc(psi0, w_.dtype) if psi0 is not None else None
+    if x is None and p0 is None:
+        # batch is carried by x; circuits without x get a zero-column x
+        pass
+    out = c.forward(x, w, psi0=p0, want_state=want_state)
+    torch.cuda.synchronize()
+    if want_state:
+        return out[0].cpu().numpy(), out[1].cpu().numpy()
+    return out.cpu().numpy()
+
+
+def run_bwd(c, w_, psi0=None, psi_final=None):
+    x = dev(w_.x, w_.dtype) if w_.spec.num_x else None
+    w = dev(w_.w, w_.dtype) if w_.spec.num_w else None
+    gE = dev(w_.gE, w_.dtype)
+    p0 = devc(psi0, w_.dtype) if psi0 is not None else None
+    dx, dw = c.backward(x, w, gE, psi0=p0, psi_final=psi_final)
+    torch.cuda.synchronize()
+    return (dx.cpu().numpy() if dx is not None else np.zeros((w_.batch, 0)),
+            dw.cpu().numpy() if dw is not None else np.zeros(0))
+
+
+def maxerr(a, b):
+    a, b = np.asarray(a), np.asarray(b)
+    return float(np.max(np.abs(a - b))) if a.size else 0.0
+
+
+# ------------------------------------------------------------------ small random circuits
+SMALL = [(201, 1, 10), (202, 2, 40), (203, 3, 80), (204, 4, 120), (205, 5, 160), (206, 6, 200),
+         (207, 7, 200), (208, 8, 240), (209, 9, 200), (210, 10, 160)]
+
+
+@pytest.mark.parametrize("dtype", ["c64", "c128"])
+@pytest.mark.parametrize("seed,n,G", SMALL)
+def test_random_forward_and_gradients(seed, n, G, dtype):
+    w_, psi0 = wl.small_random(seed, n, G, batch=37, dtype=dtype, with_psi0=(seed % 2 == 0))
+    if w_.spec.num_x == 0:
+        pytest.skip("needs x to carry the batch")
+    c = C(w_.spec, dtype)
+    E, st = run_fwd(c, w_, psi0)
+    E_ref, st_ref = orc.forward(w_.spec, w_.x, w_.w, psi0=psi0, want_state=True)
+    tol = TOL[dtype]
+    assert maxerr(E, E_ref) <= tol["E"]
+    assert maxerr(st, st_ref) <= tol["state"]
+    dx_ref, dw_ref = orc.backward(w_.spec, w_.x, w_.w, w_.gE, psi0=psi0)
+    dx, dw = run_bwd(c, w_, psi0)                       # recompute psi_final in the kernel
+    assert maxerr(dx, dx_ref) <= tol["grad"]
+    assert maxerr(dw, dw_ref) <= tol["grad"]
+    dx2, dw2 = run_bwd(c, w_, psi0, psi_final=devc(st, dtype))   # from the saved state
+    assert maxerr(dx2, dx_ref) <= tol["grad"]
+    assert maxerr(dw2, dw_ref) <= tol["grad"]
+
+
+@pytest.mark.parametrize("mode_env", ["VQC_FORCE_K_FWD", "VQC_FORCE_K_BWD"])
+@pytest.mark.parametrize("K", [1, 2, 3, 4, 5])
+def test_every_register_block_size(monkeypatch, mode_env, K):
+    w_, psi0 = wl.small_random(300 + K, 8, 200, batch=19, dtype="c64", with_psi0=True)
+    monkeypatch.setenv(mode_env, str(K))
+    c = C(w_.spec, "c64")
+    E, st = run_fwd(c, w_, psi0)
+    E_ref, st_ref = orc.forward(w_.spec, w_.x, w_.w, psi0=psi0, want_state=True)
+    assert maxerr(E, E_ref) <= 1e-4
+    assert maxerr(st, st_ref) <= 1e-4
+    dx, dw = run_bwd(c, w_, psi0)
+    dx_ref, dw_ref = orc.backward(w_.spec, w_.x, w_.w, w_.gE, psi0=psi0)
+    assert maxerr(dx, dx_ref) <= 5e-4
+    assert maxerr(dw, dw_ref) <= 5e-4
+
+
+# ------------------------------------------------------------------ the five workloads
+def test_config1_full():
+    w_ = wl.config(1)[0]
+    c = C(w_.spec, "c64")
+    E, st = run_fwd(c, w_)
+    assert maxerr(E, orc.forward(w_.spec, w_.x, w_.w)) <= 1e-4
+    dx, dw = run_bwd(c, w_, psi_final=devc(st, "c64"))
+    dx_ref, dw_ref = orc.backward(w_.spec, w_.x, w_.w, w_.gE)
+    assert maxerr(dx, dx_ref) <= 5e-4
+    assert maxerr(dw, dw_ref) <= 5e-4
+
+
+def test_config2_full():
+    w_ = wl.config(2)[0]
+    c = C(w_.spec, "c64")
+    E, st = run_fwd(c, w_)
+    assert maxerr(E, orc.forward(w_.spec, w_.x, w_.w)) <= 1e-4
+    dx, dw = run_bwd(c, w_, psi_final=devc(st, "c64"))
+    dx_ref, dw_ref = orc.backward(w_.spec, w_.x, w_.w, w_.gE)
+    assert maxerr(dx, dx_ref) <= 5e-4
+    assert maxerr(dw, dw_ref) <= 5e-4
+
+
+def test_config2_paper_objective_mean_z():
+    # the paper's scalar objective: mean of <Z_i>  (upstream gradient 1/n)
+    w_ = wl.config(2, batch=64)[0]
+    w_.gE = np.full_like(w_.gE, np.float32(1.0 / w_.spec.n))
+    c = C(w_.spec, "c64")
+    dx, dw = run_bwd(c, w_)
+    dx_ref, dw_ref = orc.backward(w_.spec, w_.x, w_.w, w_.gE)
+    assert maxerr(dx, dx_ref) <= 5e-4
+    assert maxerr(dw, dw_ref) <= 5e-4
+
+
+def test_config3_sampled_rows_and_linearity():
+    w_ = wl.config(3)[0]
+    c = C(w_.spec, "c64")
+    E, st = run_fwd(c, w_)
+    dx, dw = run_bwd(c, w_, psi_final=devc(st, "c64"))
+    rows = [0, 1, 1000, 2047, 3333, 4095]
+    sub = wl.Workload(w_.name, w_.spec, len(rows), w_.x[rows], w_.w, w_.gE[rows], "c64", w_.seed)
+    assert maxerr(E[rows], orc.forward(w_.spec, sub.x, sub.w)) <= 1e-4
+    dx_ref, _ = orc.backward(w_.spec, sub.x, sub.w, sub.gE)
+    assert maxerr(dx[rows], dx_ref) <= 5e-4
+    # dw on a 16-row slice against the oracle
+    s16 = wl.Workload(w_.name, w_.spec, 16, w_.x[:16], w_.w, w_.gE[:16], "c64", w_.seed)
+    _, dw16 = run_bwd(c, s16)
+    _, dw16_ref = orc.backward(w_.spec, s16.x, s16.w, s16.gE)
+    assert maxerr(dw16, dw16_ref) <= 5e-4
+    # full-batch dw (the launch the benchmark times) equals the sum over two halves
+    h1 = wl.Workload(w_.name, w_.spec, 2048, w_.x[:2048], w_.w, w_.gE[:2048], "c64", w_.seed)
+    h2 = wl.Workload(w_.name, w_.spec, 2048, w_.x[2048:], w_.w, w_.gE[2048:], "c64", w_.seed)
+    _, dwa = run_bwd(c, h1)
+    _, dwb = run_bwd(c, h2)
+    scale = max(1.0, float(np.max(np.abs(dw))))
+    assert maxerr(dw, dwa + dwb) <= 1e-4 * scale
+
+
+def test_config4_random_circuits_full_state():
+    for w_ in wl.config(4):
+        c = C(w_.spec, "c64")
+        E, st = run_fwd(c, w_)
+        rows = [0, w_.batch - 1]
+        x = w_.x[rows]
+        E_ref, st_ref = orc.forward(w_.spec, x, w_.w, want_state=True)
+        assert maxerr(E[rows], E_ref) <= 1e-4, w_.name
+        assert maxerr(st[rows], st_ref) <= 1e-4, w_.name
+        fid = np.abs(np.sum(np.conj(st_ref) * st[rows], axis=1)) ** 2
+        assert np.all(fid >= 1 - 1e-5), w_.name
+
+
+# ------------------------------------------------------------------ edge cases
+def test_zero_batch_and_ragged_batches():
+    w_, _ = wl.small_random(401, 6, 80, batch=1, dtype="c64")
+    c = C(w_.spec, "c64")
+    x = torch.empty(0, w_.spec.num_x, device="cuda")
+    w = dev(w_.w, "c64")
+    E = c.forward(x, w)
+    assert E.shape == (0, 6)
+    for B in (1, 2, 3, 5, 31, 33, 129, 257):
+        wb, _ = wl.small_random(401, 6, 80, batch=B, dtype="c64")
+        E = run_fwd(c, wb, want_state=False)
+        assert maxerr(E, orc.forward(wb.spec, wb.x, wb.w)) <= 1e-4
+        dx, dw = run_bwd(c, wb)
+        dx_ref, dw_ref = orc.backward(wb.spec, wb.x, wb.w, wb.gE)
+        assert maxerr(dx, dx_ref) <= 5e-4 and maxerr(dw, dw_ref) <= 5e-4
+
+
+def test_batch_rows_independent():
+    w_, psi0 = wl.small_random(402, 7, 150, batch=9, dtype="c64", with_psi0=True)
+    c = C(w_.spec, "c64")
+    E = run_fwd(c, w_, psi0, want_state=False)
+    for b in (0, 4, 8):
+        one = wl.Workload(w_.name, w_.spec, 1, w_.x[b:b + 1], w_.w, w_.gE[b:b + 1], "c64", 0)
+        Eb = run_fwd(c, one, psi0[b:b + 1], want_state=False)
+        assert maxerr(Eb[0], E[b]) <= 1e-6
+
+
+def test_only_two_qubit_gates_and_constants():
+    spec = wl.CircuitSpec(6, 1, 0)
+    spec.add("RY", (0,), [("x", 0)])
+    for q in range(5):
+        spec.add("CX", (q, q + 1))
+    spec.add("SWAP", (0, 5)).add("CZ", (2, 4)).add("CRZ", (1, 3), [("c", 0.7)])
+    spec.add("RZZ", (5, 2), [("c", -1.3)]).add("H", (4,)).add("T", (4,)).add("SX", (1,))
+    rng = np.random.default_rng(5)
+    x = wl._round(rng.uniform(-np.pi, np.pi, (11, 1)), "c64")
+    w_ = wl.Workload("twoq", spec, 11, x, np.zeros(0), wl._round(rng.standard_normal((11, 6)), "c64"), "c64", 0)
+    c = C(spec, "c64")
+    E, st = run_fwd(c, w_)
+    E_ref, st_ref = orc.forward(spec, x, None, want_state=True)
+    assert maxerr(E, E_ref) <= 1e-4 and maxerr(st, st_ref) <= 1e-4
+    dx, _ = run_bwd(c, w_)
+    dx_ref, _ = orc.backward(spec, x, None, w_.gE)
+    assert maxerr(dx, dx_ref) <= 5e-4
+
+
+def test_single_rotation_closed_form_on_gpu():
+    spec = wl.CircuitSpec(1, 1, 0).add("RY", (0,), [("x", 0)])
+    t = np.linspace(-np.pi, np.pi, 65)[:, None]
+    w_ = wl.Workload("ry", spec, 65, wl._round(t, "c128"), np.zeros(0), np.ones((65, 1)), "c128", 0)
+    c = C(spec, "c128")
+    E, _ = run_fwd(c, w_)
+    assert np.max(np.abs(E[:, 0] - np.cos(t[:, 0]))) <= 1e-12
+    dx, _ = run_bwd(c, w_)
+    assert np.max(np.abs(dx[:, 0] + np.sin(t[:, 0]))) <= 1e-12
+
+
+def test_autograd_function():
+    w_ = wl.config(1, batch=16)[0]
+    c = C(w_.spec, "c64")
+    x = dev(w_.x, "c64").requires_grad_(True)
+    w = dev(w_.w, "c64").requires_grad_(True)
+    E = c(x, w)
+    (E * dev(w_.gE, "c64")).sum().backward()
+    dx_ref, dw_ref = orc.backward(w_.spec, w_.x, w_.w, w_.gE)
+    assert maxerr(x.grad.cpu().numpy(), dx_ref) <= 5e-4
+    assert maxerr(w.grad.cpu().numpy(), dw_ref) <= 5e-4
+
+
+def test_deterministic_dw():
+    w_ = wl.config(2)[0]
+    c = C(w_.spec, "c64")
+    _, dw1 = run_bwd(c, w_)
+    _, dw2 = run_bwd(c, w_)
+    assert np.array_equal(dw1, dw2)
