@@ -192,7 +192,7 @@ vqc_status upload(HostPlan& p) {
     auto put = [&](const void* src, size_t bytes) {
         size_t off = blob.size();
         blob.resize(align16(off + bytes), 0);
-        if (bytes) std::memcpy(blob.data() + off, src, bytes);
+        if (bytes && src) std::memcpy(blob.data() + off, src, bytes);
         return off;
     };
     std::vector<int32_t> ps_list, sh_list;
