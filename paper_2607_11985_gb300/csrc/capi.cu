@@ -117,9 +117,29 @@ vqc_status plan_launch(const HostPlan& p, int mode, int B, Launch& L) {
     const bool dbl = p.dtype == VQC_C128;
     const size_t rs = dbl ? 8 : 4, cs = 2 * rs;
     L.T = 1 << (p.n - L.K);
-    L.S = std::max(1, 128 / L.T);
-    L.block = L.S * L.T;
     L.wg = L.T > 32 ? L.T / 32 : 1;
+    // Shared memory: a fixed part per CTA and a part per resident sample.
+    const size_t dim = (size_t)1 << p.n;
+    const size_t fixed = align16((size_t)p.n_sh * 8 * rs) + align16(mode == 1 ? (size_t)p.num_w * rs : 0) + 8 * 16;
+    const size_t per_sample = (size_t)p.n_ps * 8 * rs + dim * cs * (mode == 1 ? 2 : 1) +
+                              (mode == 1 ? p.accs.size() * L.wg * 8 * rs + p.term_src.size() * rs
+                                         : (size_t)L.wg * p.n * rs);
+    int S = std::max(1, 128 / L.T);
+    if ((size_t)di.smem_optin > fixed) {
+        size_t fit = ((size_t)di.smem_optin - fixed) / per_sample;
+        S = (int)std::min<size_t>((size_t)S, fit);
+    } else {
+        S = 0;
+    }
+    if (S < 1)
+        return fail(VQC_ERR_UNSUPPORTED,
+                    "state does not fit in shared memory on the resident path (" +
+                        std::to_string(fixed + per_sample) + " > " +
+                        std::to_string(di.smem_optin) + " bytes)");
+    // Groups smaller than a warp fill whole warps when the CTA spans more than one.
+    if (L.T < 32 && S * L.T > 32) S -= S % (32 / L.T);
+    L.S = S;
+    L.block = L.S * L.T;
     if (L.block > sweep_max_threads(dbl, mode, L.K))
         return fail(VQC_ERR_UNSUPPORTED, "thread group too large for this kernel");
     size_t off = 0;
@@ -130,17 +150,15 @@ vqc_status plan_launch(const HostPlan& p, int mode, int B, Launch& L) {
     };
     L.sm_sh = take((size_t)p.n_sh * 8 * rs);
     L.sm_ps = take((size_t)L.S * p.n_ps * 8 * rs);
-    L.sm_psi = take((size_t)L.S * ((size_t)1 << p.n) * cs);
-    L.sm_lam = take(mode == 1 ? (size_t)L.S * ((size_t)1 << p.n) * cs : 0);
+    L.sm_psi = take((size_t)L.S * dim * cs);
+    L.sm_lam = take(mode == 1 ? (size_t)L.S * dim * cs : 0);
     L.sm_acc = take(mode == 1 ? (size_t)L.S * p.accs.size() * L.wg * 8 * rs : 0);
     L.sm_terms = take(mode == 1 ? (size_t)L.S * p.term_src.size() * rs : 0);
     L.sm_dw = take(mode == 1 ? (size_t)p.num_w * rs : 0);
     L.sm_red = take(mode == 0 ? (size_t)L.S * L.wg * p.n * rs : 0);
     L.smem = off;
     if (L.smem > (size_t)di.smem_optin)
-        return fail(VQC_ERR_UNSUPPORTED,
-                    "state does not fit in shared memory on the resident path (" +
-                        std::to_string(L.smem) + " > " + std::to_string(di.smem_optin) + " bytes)");
+        return fail(VQC_ERR_UNSUPPORTED, "shared-memory layout exceeds the per-CTA limit");
     L.fn = kernel_ptr(p.dtype, mode, L.K);
     if (!L.fn) return fail(VQC_ERR_UNSUPPORTED, "kernel not instantiated for this K");
     VQC_CUDA(cudaFuncSetAttribute(L.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem));

@@ -377,12 +377,13 @@ __device__ __forceinline__ R ph2_term(int ra, int rb, uint32_t pb, uint8_t flags
 
 // ---------------------------------------------------------------- reductions
 template <typename R>
-__device__ __forceinline__ R shx(R v, int m) { return __shfl_xor_sync(0xffffffffu, v, m); }
+__device__ __forceinline__ R shx(R v, int m, unsigned mask) { return __shfl_xor_sync(mask, v, m); }
 
 // Reduce 8 values over a group of `lanes` lanes (power of two <= 32) and
 // write the 8 sums to dst (reduce-scatter butterfly: 9 shuffles at 32 lanes).
 template <typename R>
-__device__ __forceinline__ void reduce8_store(R (&v)[8], int lanes, int lane, R* dst) {
+__device__ __forceinline__ void reduce8_store(R (&v)[8], int lanes, int lane, R* dst,
+                                              unsigned mask) {
     int u0 = 0, u1 = 0, u2 = 0;
     if (lanes >= 2) {
         const int m = lanes >> 1;
@@ -391,7 +392,7 @@ __device__ __forceinline__ void reduce8_store(R (&v)[8], int lanes, int lane, R*
         for (int i = 0; i < 4; ++i) {
             R send = u0 ? v[i] : v[i + 4];
             R keep = u0 ? v[i + 4] : v[i];
-            v[i] = keep + shx<R>(send, m);
+            v[i] = keep + shx<R>(send, m, mask);
         }
     }
     if (lanes >= 4) {
@@ -401,7 +402,7 @@ __device__ __forceinline__ void reduce8_store(R (&v)[8], int lanes, int lane, R*
         for (int i = 0; i < 2; ++i) {
             R send = u1 ? v[i] : v[i + 2];
             R keep = u1 ? v[i + 2] : v[i];
-            v[i] = keep + shx<R>(send, m);
+            v[i] = keep + shx<R>(send, m, mask);
         }
     }
     if (lanes >= 8) {
@@ -409,8 +410,8 @@ __device__ __forceinline__ void reduce8_store(R (&v)[8], int lanes, int lane, R*
         u2 = (lane & m) ? 1 : 0;
         R send = u2 ? v[0] : v[1];
         R keep = u2 ? v[1] : v[0];
-        v[0] = keep + shx<R>(send, m);
-        for (int mm = lanes >> 4; mm >= 1; mm >>= 1) v[0] += shx<R>(v[0], mm);
+        v[0] = keep + shx<R>(send, m, mask);
+        for (int mm = lanes >> 4; mm >= 1; mm >>= 1) v[0] += shx<R>(v[0], mm, mask);
         if ((lane & ((lanes >> 3) - 1)) == 0) dst[4 * u0 + 2 * u1 + u2] = v[0];
     } else if (lanes == 4) {
         dst[4 * u0 + 2 * u1] = v[0];
@@ -423,8 +424,8 @@ __device__ __forceinline__ void reduce8_store(R (&v)[8], int lanes, int lane, R*
 }
 
 template <typename R>
-__device__ __forceinline__ R reduce1(R v, int lanes) {
-    for (int m = lanes >> 1; m >= 1; m >>= 1) v += shx<R>(v, m);
+__device__ __forceinline__ R reduce1(R v, int lanes, unsigned mask) {
+    for (int m = lanes >> 1; m >= 1; m >>= 1) v += shx<R>(v, m, mask);
     return v;
 }
 
@@ -436,6 +437,7 @@ struct Geo {
     int g;        // group (sample slot) index in the CTA
     int t;        // thread index in the group
     int h;        // per-sample XOR on the slot index (bank spreading of small groups)
+    unsigned mask;   // lanes of this warp that exist (a CTA smaller than a warp)
 };
 
 __device__ __forceinline__ uint32_t swz(uint32_t u, int G) {
@@ -446,7 +448,7 @@ __device__ __forceinline__ uint32_t swz(uint32_t u, int G) {
 
 template <typename R>
 __device__ __forceinline__ void group_sync(const Geo& q) {
-    if (q.T > 32) __syncthreads(); else __syncwarp();
+    if (q.T > 32) __syncthreads(); else __syncwarp(q.mask);
 }
 
 template <int K>
@@ -542,6 +544,7 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
     q.t = threadIdx.x % q.T;
     q.h = 0;
     if (A.tbits < G) q.h = ((q.g & ((1 << (G - A.tbits)) - 1)) << A.tbits) & (dim - 1);
+    q.mask = blockDim.x >= 32 ? 0xffffffffu : ((1u << blockDim.x) - 1u);
     const int lane = q.t & 31;
     const int warp_in_group = q.t >> 5;
     const int nthr = blockDim.x;
@@ -652,7 +655,7 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
                 } else {
                     val = ((v.pb >> j) & 1u) ? -ptot : ptot;
                 }
-                val = reduce1<R>(val, q.lanes);
+                val = reduce1<R>(val, q.lanes, q.mask);
                 if ((q.t & (q.lanes - 1)) == 0) red[warp_in_group * n + j] = val;
             }
             __syncthreads();
@@ -715,7 +718,7 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
                         R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};
                         m1_rho_dispatch<R, K>(ra, a, l, rh);
                         reduce8_store<R>(rh, q.lanes, q.lanes < 32 ? q.t : lane,
-                                         acc + ((size_t)aux * q.wg + warp_in_group) * 8);
+                                         acc + ((size_t)aux * q.wg + warp_in_group) * 8, q.mask);
                     }
                     const M2<R> md = mdag<R>(m);
                     m1_dispatch<R, K>(ra, a, md);
@@ -738,7 +741,7 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
                                    cm<R>(p[6], p[7])};
                     if (flags & OPF_HAS_ACC) {
                         R tv = ph2_term<R, K>(ra, rb, v.pb, (uint8_t)flags, a, l);
-                        tv = reduce1<R>(tv, q.lanes);
+                        tv = reduce1<R>(tv, q.lanes, q.mask);
                         if ((q.t & (q.lanes - 1)) == 0)
                             acc[((size_t)aux * q.wg + warp_in_group) * 8] = tv;
                     }
