@@ -104,9 +104,10 @@ class ClockSampler:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
-def workload(cfg=2):
+def workload(cfg=2, rank=0, world=1):
+    """This rank's shard of the global batch (world x per-rank batch rows)."""
     from paper_2607_11985_gb300 import workloads as wl
-    return wl.config(cfg)[0]
+    return wl.config(cfg, rank=rank, world=world)[0]
 
 
 # ------------------------------------------------------------------ CPU oracle baseline
@@ -137,7 +138,7 @@ def run_ours(args, rank, world, local_rank):
 
     __graft_entry__.build()
     torch.cuda.set_device(local_rank)
-    w_ = workload(args.config)
+    w_ = workload(args.config, rank, world)
     Bt = w_.batch
     c = Circuit(w_.spec, "c64")
     info = c.info(Bt)
@@ -256,13 +257,14 @@ def run_ours(args, rank, world, local_rank):
     ach_bwd = bwd_flops / bwd_avg_s / 1e12
     ach_fwd = fwd_flops / fwd_avg_s / 1e12
     traffic = None
-    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    tpath = os.path.join(ROOT, "profiles", "traffic.txt")
     if os.path.exists(tpath):
         with open(tpath) as f:
-            tj = json.load(f)
-        key = "%s:%s" % (w_.name, "bwd")
-        if key in tj and tj[key].get("digest") == info_digest():
-            traffic = tj[key]["bytes_per_launch"]
+            for line in f:
+                parts = line.split()
+                if len(parts) >= 4 and not line.startswith("#") and parts[0] == w_.name.split("_rank")[0] \
+                        and parts[1] == "bwd" and parts[2] == info_digest():
+                    traffic = float(parts[3])
     out = {
         "metric": METRIC,
         "value": value,
@@ -276,7 +278,8 @@ def run_ours(args, rank, world, local_rank):
         "vs_baseline": None,
         "dtype": "c64 (fp32 arithmetic)",
         "data": "synthetic (seeded; RY(x) encoding + RX/RY/RZ layers + CZ ring)",
-        "config": {"workload": w_.name, "qubits": w_.spec.n, "layers": 4, "batch_per_gpu": Bt,
+        "config": {"workload": w_.name.split("_rank")[0], "qubits": w_.spec.n, "layers": 4,
+                   "batch_per_gpu": Bt,
                    "gates": len(w_.spec.gates), "num_x": w_.spec.num_x, "num_w": w_.spec.num_w,
                    "parallelism": "dp%d (batch-sharded replicas, dw all-reduce)" % world,
                    "l2": "flushed between steps (256 MiB write) outside the per-step CUDA events",
@@ -353,12 +356,13 @@ def extra_configs(torch, Circuit, B):
                     tot_b += b2.elapsed_time(d) / 1e3
                 evals += n_rep * w_.batch
                 flops_f += n_rep * w_.batch * inf["fwd_flops_per_eval"]
-                flops_b += n_rep * w_.batch * inf["bwd_flops_per_eval"]
+                if w_.backward:
+                    flops_b += n_rep * w_.batch * inf["bwd_flops_per_eval"]
                 del c
             res["cfg%d" % k] = {"fwd_evals_per_s": evals / tot_f,
                                 "fwd_tflops": flops_f / tot_f / 1e12,
-                                "fwd_bwd_evals_per_s": (evals / (tot_f + tot_b)) if tot_b else None,
-                                "bwd_tflops": (flops_b / tot_b / 1e12) if tot_b else None,
+                                "fwd_bwd_evals_per_s": (evals / (tot_f + tot_b)) if flops_b else None,
+                                "bwd_tflops": (flops_b / tot_b / 1e12) if flops_b else None,
                                 "circuits": len(ws_)}
         except Exception as e:   # report, do not hide
             res["cfg%d" % k] = {"error": str(e)[:200]}

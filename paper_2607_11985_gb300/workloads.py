@@ -137,19 +137,27 @@ CONFIG_NAMES = {
 }
 
 
-def config(k: int, dtype: Optional[str] = None, batch: Optional[int] = None) -> List[Workload]:
-    """The five workloads.  Returns a list (config 4 holds 32 circuits)."""
+def config(k: int, dtype: Optional[str] = None, batch: Optional[int] = None,
+           rank: int = 0, world: int = 1) -> List[Workload]:
+    """The five workloads.  Returns a list (config 4 holds 32 circuits).
+
+    With ``world`` > 1 the global batch is ``world`` x batch rows and this returns
+    rank ``rank``'s contiguous shard; rank 0 of any world sees the same rows as
+    world = 1 (each array has its own PCG64 stream, filled row by row)."""
     if k == 1:
         spec = layered(4, 2, ("RY", "RZ"), "CX")
-        return [_draw("cfg1_" + CONFIG_NAMES[1], spec, batch or 64, dtype or "c64", 1001, "uniform")]
+        return [_draw("cfg1_" + CONFIG_NAMES[1], spec, batch or 64, dtype or "c64", 1001,
+                      "uniform", rank, world)]
     if k == 2:
         spec = layered(8, 4, ("RX", "RY", "RZ"), "CZ")
-        return [_draw("cfg2_" + CONFIG_NAMES[2], spec, batch or 1024, dtype or "c64", 1002, "uniform")]
+        return [_draw("cfg2_" + CONFIG_NAMES[2], spec, batch or 1024, dtype or "c64", 1002,
+                      "uniform", rank, world)]
     if k == 3:
         # Rot(phi, theta, omega) = RZ(omega) RY(theta) RZ(phi): RZ(phi) first.
         spec = layered(12, 6, ("RZ", "RY", "RZ"), "CX", reupload=True,
                        ring_range=lambda l: (l % 11) + 1)
-        return [_draw("cfg3_" + CONFIG_NAMES[3], spec, batch or 4096, dtype or "c64", 1003, "normal")]
+        return [_draw("cfg3_" + CONFIG_NAMES[3], spec, batch or 4096, dtype or "c64", 1003,
+                      "normal", rank, world)]
     if k == 4:
         out = []
         B = batch or 256
@@ -167,18 +175,23 @@ def config(k: int, dtype: Optional[str] = None, batch: Optional[int] = None) -> 
     if k == 5:
         spec = layered(16, 8, ("RX", "RY", "RZ"), "CX")
         return [_draw("cfg5_" + CONFIG_NAMES[5] + "_" + (dtype or "c64"), spec, batch or 512,
-                      dtype or "c64", 1005, "uniform")]
+                      dtype or "c64", 1005, "uniform", rank, world)]
     raise ValueError("config must be 1..5")
 
 
-def _draw(name, spec, B, dtype, seed, xdist) -> Workload:
-    rng = np.random.Generator(np.random.PCG64(seed))
+def _draw(name, spec, B, dtype, seed, xdist, rank=0, world=1) -> Workload:
+    sx, sw, sg = np.random.SeedSequence(seed).spawn(3)
+    rx, rw, rg = (np.random.Generator(np.random.PCG64(s)) for s in (sx, sw, sg))
+    rows = B * (rank + 1)            # fill up to the end of this rank's shard
     if xdist == "normal":
-        x = rng.standard_normal((B, spec.num_x))
+        x = rx.standard_normal((rows, spec.num_x))
     else:
-        x = rng.uniform(-np.pi, np.pi, (B, spec.num_x))
-    w = rng.uniform(-np.pi, np.pi, spec.num_w)
-    gE = rng.standard_normal((B, spec.n))
+        x = rx.uniform(-np.pi, np.pi, (rows, spec.num_x))
+    w = rw.uniform(-np.pi, np.pi, spec.num_w)
+    gE = rg.standard_normal((rows, spec.n))
+    x, gE = x[B * rank:], gE[B * rank:]
+    if world > 1:
+        name = "%s_rank%dof%d" % (name, rank, world)
     return Workload(name, spec, B, _round(x, dtype), _round(w, dtype), _round(gE, dtype),
                     dtype, seed)
 
