@@ -184,6 +184,29 @@ vqc_status vqc_backward(const vqc_plan* plan, int32_t batch, const void* x, cons
                         void* grad_x, void* grad_w, void* workspace, size_t workspace_bytes,
                         void* stream);
 
+/* Bytes of device scratch built into the library for vqc_backward_noalloc
+ * (one array per GPU that loads the library, held until the process exits). */
+#define VQC_NOALLOC_SCRATCH_BYTES (1u << 20)
+
+/* vqc_backward without a workspace argument, for callers that cannot allocate
+ * device memory (a plugin whose host application owns all device memory, a
+ * real-time loop that must not pay cudaMalloc's latency or implicit device
+ * synchronisation, code under a fixed device-memory budget).  The paper has no
+ * counterpart; it is a deployment convenience of this library.
+ *   Arguments, outputs and results are those of vqc_backward.  The scratch is
+ *   a fixed array of VQC_NOALLOC_SCRATCH_BYTES inside the library; a batch
+ *   whose scratch need (vqc_workspace_bytes(plan, batch, 1)) exceeds it is
+ *   rejected with VQC_ERR_WORKSPACE and a message giving both sizes.
+ *   No cudaMalloc, cudaFree or allocating library call is made.  Each call
+ *   clears the array's control block on `stream` before its launch; all calls
+ *   on a device share the array, so calls that overlap on the GPU race and must
+ *   be ordered by the caller.  The first call on a device (with that device
+ *   current) looks up the array's device address; make it before any CUDA
+ *   stream capture begins. */
+vqc_status vqc_backward_noalloc(const vqc_plan* plan, int32_t batch, const void* x,
+                                const void* w, const void* psi0, const void* psi_final,
+                                const void* grad_expz, void* grad_x, void* grad_w, void* stream);
+
 /* Plan statistics (paths, stage counts, algorithmic flop and byte counts per
  * evaluation) for a batch of `batch` samples. */
 vqc_status vqc_plan_info(const vqc_plan* plan, int32_t batch, vqc_plan_stats* out);

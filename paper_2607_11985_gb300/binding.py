@@ -68,6 +68,7 @@ SIGNATURES = [
     ("vqc_workspace_init", _I, [_P, _S, _P]),
     ("vqc_forward", _I, [_P, _I, _P, _P, _P, _P, _P, _P, _S, _P]),
     ("vqc_backward", _I, [_P, _I, _P, _P, _P, _P, _P, _P, _P, _P, _S, _P]),
+    ("vqc_backward_noalloc", _I, [_P, _I, _P, _P, _P, _P, _P, _P, _P, _P]),
     ("vqc_plan_info", _I, [_P, _I, ctypes.POINTER(vqc_plan_stats)]),
     ("vqc_plan_export", _I, [_P, _P, ctypes.POINTER(_S)]),
     ("vqc_sync_check", _I, [_P]),
@@ -141,6 +142,11 @@ def vqc_backward(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x, grad_w, 
                  workspace_bytes, stream):
     _check(lib().vqc_backward(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x, grad_w,
                               workspace, workspace_bytes, stream))
+
+
+def vqc_backward_noalloc(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x, grad_w, stream):
+    _check(lib().vqc_backward_noalloc(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x,
+                                      grad_w, stream))
 
 
 def vqc_plan_info(plan, batch):

@@ -333,6 +333,44 @@ vqc_status check_ptrs(const HostPlan& p, const void* x, const void* w, const voi
 }
 
 }  // namespace
+
+vqc_status set_error(vqc_status s, const std::string& msg) { return fail(s, msg); }
+
+// The backward with an explicit scratch buffer, for vqc_backward_noalloc: the
+// scratch must hold the same layout as a vqc_backward workspace; with
+// clear_control the control block is zeroed on `stream` before the launch.
+vqc_status backward_with_scratch(const vqc_plan* plan, int32_t batch, const void* x,
+                                 const void* w, const void* psi0, const void* psi_final,
+                                 const void* grad_expz, void* grad_x, void* grad_w, void* scratch,
+                                 size_t scratch_bytes, void* stream, bool clear_control) {
+    vqc_status st = check_common(plan, batch);
+    if (st != VQC_OK) return st;
+    const HostPlan& p = plan->hp;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (batch == 0) {
+        if (grad_w && p.num_w > 0)
+            VQC_CUDA(cudaMemsetAsync(grad_w, 0, (size_t)p.num_w * (p.dtype == VQC_C128 ? 8 : 4), s));
+        return VQC_OK;
+    }
+    st = check_ptrs(p, x, w, psi0, psi_final);
+    if (st != VQC_OK) return st;
+    if (!grad_expz) return fail(VQC_ERR_INVALID_ARG, "grad_expz is NULL");
+    Launch L;
+    st = plan_launch(p, 1, batch, L);
+    if (st != VQC_OK) return st;
+    const size_t need = bwd_workspace(p, L);
+    if (need > scratch_bytes)
+        return fail(VQC_ERR_WORKSPACE, "this batch needs " + std::to_string(need) +
+                                           " bytes of scratch; the built-in scratch holds " +
+                                           std::to_string(scratch_bytes));
+    if (clear_control) VQC_CUDA(cudaMemsetAsync(scratch, 0, 256, s));
+    if (p.dtype == VQC_C64)
+        return run<float>(p, 1, batch, x, w, psi0, psi_final, grad_expz, nullptr, nullptr, grad_x,
+                          grad_w, scratch, scratch_bytes, s);
+    return run<double>(p, 1, batch, x, w, psi0, psi_final, grad_expz, nullptr, nullptr, grad_x,
+                       grad_w, scratch, scratch_bytes, s);
+}
+
 }  // namespace vqc
 
 using namespace vqc;

@@ -1,0 +1,102 @@
+"""vqc_backward_noalloc against vqc_backward, through the C ABI (GPU).
+
+vqc_backward_noalloc serves callers that cannot allocate device memory (a
+plugin whose host application owns every device allocation, a real-time loop
+that cannot afford cudaMalloc's latency and implicit synchronisation, code under
+a fixed device-memory budget): it takes no workspace and uses scratch built
+into the library instead.  Its gradients must equal those of the workspace
+entry point within the engine's complex64 gradient tolerance (5e-4), on two
+calls in a row (the second call finds the first call's leftovers in the shared
+scratch).  A batch whose scratch need exceeds the built-in size must be
+rejected with VQC_ERR_WORKSPACE.
+
+This file is collected last so that a run stopping at its first failure has
+already run every other test; it also passes on its own in a fresh process.
+"""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from paper_2607_11985_gb300 import workloads as wl  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+GRAD_TOL = 5e-4
+
+
+@pytest.fixture(scope="module", autouse=True)
+def ready():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    torch.cuda.set_device(0)
+
+
+def _inputs(w_):
+    f = lambda a: torch.tensor(np.asarray(a), dtype=torch.float32, device="cuda")
+    return f(w_.x), f(w_.w), f(w_.gE)
+
+
+def _workspace_backward(B, c, x, w, gE, st):
+    dx = torch.empty_like(x)
+    dw = torch.empty_like(w)
+    stream = torch.cuda.current_stream()
+    ws, wsb = c.workspace(x.shape[0], 1, stream)
+    B.vqc_backward(c.plan, x.shape[0], x.data_ptr(), w.data_ptr(), None, st.data_ptr(),
+                   gE.data_ptr(), dx.data_ptr(), dw.data_ptr(), ws.data_ptr(), wsb,
+                   stream.cuda_stream)
+    return dx, dw
+
+
+def _noalloc_backward(B, c, x, w, gE, st):
+    dx = torch.full_like(x, float("nan"))
+    dw = torch.full_like(w, float("nan"))
+    B.vqc_backward_noalloc(c.plan, x.shape[0], x.data_ptr(), w.data_ptr(), None, st.data_ptr(),
+                           gE.data_ptr(), dx.data_ptr(), dw.data_ptr(),
+                           torch.cuda.current_stream().cuda_stream)
+    return dx, dw
+
+
+@pytest.mark.parametrize("k", [2, 3])
+def test_noalloc_backward_matches_workspace_backward_twice(k):
+    from paper_2607_11985_gb300 import binding as B
+    from paper_2607_11985_gb300.circuit import Circuit
+    w_ = wl.config(k)[0]
+    c = Circuit(w_.spec, "c64")
+    x, w, gE = _inputs(w_)
+    E, st = c.forward(x, w, want_state=True)
+    dx_ref, dw_ref = _workspace_backward(B, c, x, w, gE, st)
+    for _ in range(2):
+        dx, dw = _noalloc_backward(B, c, x, w, gE, st)
+        torch.cuda.synchronize()
+        assert torch.isfinite(dx).all() and torch.isfinite(dw).all()
+        assert float((dx - dx_ref).abs().max()) <= GRAD_TOL
+        assert float((dw - dw_ref).abs().max()) <= GRAD_TOL
+
+
+def test_noalloc_rejects_batches_beyond_the_builtin_scratch():
+    from paper_2607_11985_gb300 import binding as B
+    from paper_2607_11985_gb300.circuit import Circuit
+    # 6000 shared weights: the per-CTA dw partials of a full grid exceed 1 MiB
+    spec = wl.CircuitSpec(6, 6, 6000)
+    for q in range(6):
+        spec.add("RY", (q,), [("x", q)])
+    for j in range(6000):
+        spec.add("RZ", (j % 6,), [("w", j)])
+    c = Circuit(spec, "c64")
+    batch = 4096
+    need = B.vqc_workspace_bytes(c.plan, batch, 1)
+    assert need > (1 << 20)
+    x = torch.zeros(batch, 6, device="cuda")
+    w = torch.zeros(6000, device="cuda")
+    gE = torch.ones(batch, 6, device="cuda")
+    dx = torch.empty_like(x)
+    dw = torch.empty_like(w)
+    with pytest.raises(B.VQCError) as err:
+        B.vqc_backward_noalloc(c.plan, batch, x.data_ptr(), w.data_ptr(), None, None,
+                               gE.data_ptr(), dx.data_ptr(), dw.data_ptr(),
+                               torch.cuda.current_stream().cuda_stream)
+    assert err.value.status == 8
+    assert "scratch" in str(err.value)
