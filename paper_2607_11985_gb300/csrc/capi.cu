@@ -15,6 +15,7 @@
 
 #include "engine.h"
 #include "kernels.h"
+#include "pass.cuh"
 #include "sweep.cuh"
 
 struct vqc_plan {
@@ -233,6 +234,9 @@ vqc_status upload(HostPlan& p) {
     for (auto& s : p.scheds) {
         s.dev_ops = put(s.ops.data(), s.ops.size() * sizeof(DOp));
         s.dev_stages = put(s.stages.data(), s.stages.size() * sizeof(DStage));
+        s.dev_passes = put(s.passes.data(), s.passes.size() * sizeof(DPass));
+        s.dev_pass_entries = put(s.pass_entries.data(), s.pass_entries.size() * 4);
+        s.dev_pass_accs = put(s.pass_accs.data(), s.pass_accs.size() * 4);
     }
     size_t err_off = put(nullptr, 16);
     blob.resize(align256(blob.size()), 0);
@@ -297,6 +301,270 @@ vqc_status run(const HostPlan& p, int mode, int B, const void* x, const void* w,
     void* args[] = {&a};
     VQC_CUDA(cudaLaunchKernel(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
     return VQC_OK;
+}
+
+
+// ---------------------------------------------------------------- HBM path
+struct PassGeo {
+    const Schedule* s = nullptr;
+    int K = 0, T = 0, S = 0, block = 0, grid = 0, wg = 1, ntiles = 1;
+    long long nunits = 0;
+    size_t smem = 0;
+    int sm_sh = 0, sm_ps = 0, sm_psi = 0, sm_lam = 0, sm_acc = 0, sm_red = 0;
+    const void* fn = nullptr;
+};
+
+vqc_status plan_hbm(const HostPlan& p, int mode, int B, PassGeo& L) {
+    L.s = find_hbm_schedule(p, mode);
+    if (!L.s) return fail(VQC_ERR_UNSUPPORTED, "no HBM-tiled schedule for this circuit");
+    int dev = 0;
+    VQC_CUDA(cudaGetDevice(&dev));
+    DevInfo di;
+    vqc_status st = device_info(dev, di);
+    if (st != VQC_OK) return st;
+    const bool dbl = p.dtype == VQC_C128;
+    const size_t rs = dbl ? 8 : 4, cs = 2 * rs;
+    const int m = L.s->m;
+    L.K = L.s->K;
+    L.T = 1 << (m - L.K);
+    L.wg = L.T > 32 ? L.T / 32 : 1;
+    L.ntiles = 1 << (p.n - m);
+    int ps_max = 0, sh_max = 0, acc_max = 0;
+    for (const DPass& ps : L.s->passes) {
+        ps_max = std::max(ps_max, ps.ps_count);
+        sh_max = std::max(sh_max, ps.sh_count);
+        acc_max = std::max(acc_max, ps.acc_count);
+    }
+    const size_t tdim = (size_t)1 << m;
+    const size_t fixed = align16((size_t)sh_max * 8 * rs) + 8 * 16;
+    const size_t per_tile = (size_t)ps_max * 8 * rs + tdim * cs * (mode == 1 ? 2 : 1) +
+                            (mode == 1 ? (size_t)acc_max * L.wg * 8 * rs : (size_t)L.wg * p.n * rs);
+    int S = std::max(1, 128 / L.T);
+    if ((size_t)di.smem_optin <= fixed + per_tile)
+        S = (size_t)di.smem_optin >= fixed + per_tile ? 1 : 0;
+    else
+        S = (int)std::min<size_t>((size_t)S, ((size_t)di.smem_optin - fixed) / per_tile);
+    if (S < 1) return fail(VQC_ERR_UNSUPPORTED, "HBM tile does not fit in shared memory");
+    if (L.T < 32 && S * L.T > 32) S -= S % (32 / L.T);
+    L.S = S;
+    L.block = S * L.T;
+    if (L.block > 512) return fail(VQC_ERR_UNSUPPORTED, "HBM tile group too large");
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        size_t o = off;
+        off = align16(off + bytes);
+        return (int)o;
+    };
+    L.sm_sh = take((size_t)sh_max * 8 * rs);
+    L.sm_ps = take((size_t)S * ps_max * 8 * rs);
+    L.sm_psi = take((size_t)S * tdim * cs);
+    L.sm_lam = take(mode == 1 ? (size_t)S * tdim * cs : 0);
+    L.sm_acc = take(mode == 1 ? (size_t)S * acc_max * L.wg * 8 * rs : 0);
+    L.sm_red = take(mode == 0 ? (size_t)S * L.wg * p.n * rs : 0);
+    L.smem = off;
+    L.fn = pass_ptr(dbl, mode, L.K);
+    if (!L.fn) return fail(VQC_ERR_UNSUPPORTED, "pass kernel not instantiated for this K");
+    VQC_CUDA(cudaFuncSetAttribute(L.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem));
+    int per_sm = 0;
+    VQC_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, L.fn, L.block, L.smem));
+    if (per_sm < 1) return fail(VQC_ERR_UNSUPPORTED, "pass kernel cannot be resident");
+    L.nunits = ((long long)B * L.ntiles + S - 1) / S;
+    L.grid = (int)std::max<long long>(1, std::min<long long>(L.nunits, (long long)per_sm * di.sms));
+    return VQC_OK;
+}
+
+// Workspace of the HBM path.  Forward: [control | working state | <Z> partials].
+// Backward: [control | psi | lam | gradient-term partials].
+struct HbmWs {
+    size_t state = 0, lam = 0, part = 0, total = 0;
+};
+
+HbmWs hbm_layout(const HostPlan& p, int mode, int B, int ntiles) {
+    const size_t rs = p.dtype == VQC_C128 ? 8 : 4, cs = 2 * rs;
+    const size_t sbytes = align256((size_t)B * ((size_t)1 << p.n) * cs);
+    HbmWs w;
+    w.state = 256;
+    if (mode == 0) {
+        w.part = w.state + sbytes;
+        w.total = w.part + align256((size_t)B * ntiles * p.n * rs);
+    } else {
+        w.lam = w.state + sbytes;
+        w.part = w.lam + sbytes;
+        w.total = w.part + align256((size_t)B * ntiles * std::max<size_t>(p.term_src.size(), 1) * rs);
+    }
+    return w;
+}
+
+template <typename R>
+void fill_pass_args(const HostPlan& p, const PassGeo& L, const DPass& ps, PArgs<R>& a) {
+    const char* base = static_cast<const char*>(p.dbuf);
+    a.ops = reinterpret_cast<const DOp*>(base + L.s->dev_ops);
+    a.stages = reinterpret_cast<const DStage*>(base + L.s->dev_stages);
+    a.pass_entries = reinterpret_cast<const int32_t*>(base + L.s->dev_pass_entries);
+    a.pass_accs = reinterpret_cast<const int32_t*>(base + L.s->dev_pass_accs);
+    a.entries = reinterpret_cast<const DEntry*>(base + p.dev_entries);
+    a.consts = reinterpret_cast<const DConst*>(base + p.dev_consts);
+    a.cmat = reinterpret_cast<const R*>(base + p.dev_cmat);
+    a.cang = reinterpret_cast<const R*>(base + p.dev_cang);
+    a.accs = reinterpret_cast<const DAcc*>(base + p.dev_accs);
+    a.n = p.n;
+    a.m = L.s->m;
+    a.K = L.K;
+    a.tbits = L.s->m - L.K;
+    a.G = p.G_swz;
+    a.S = L.S;
+    a.nout = p.n - L.s->m;
+    a.ntiles = L.ntiles;
+    a.stage_begin = ps.stage_begin;
+    a.stage_end = ps.stage_end;
+    a.ps_begin = ps.ps_begin;
+    a.ps_count = ps.ps_count;
+    a.sh_begin = ps.sh_begin;
+    a.sh_count = ps.sh_count;
+    a.acc_begin = ps.acc_begin;
+    a.acc_count = ps.acc_count;
+    a.n_terms = (int)p.term_src.size();
+    a.Px = p.num_x;
+    a.nunits = L.nunits;
+    for (int i = 0; i < 24; ++i) {
+        a.tile_q[i] = ps.tile_q[i];
+        a.out_q[i] = ps.out_q[i];
+    }
+    a.sm_sh = L.sm_sh; a.sm_ps = L.sm_ps; a.sm_psi = L.sm_psi; a.sm_lam = L.sm_lam;
+    a.sm_acc = L.sm_acc; a.sm_red = L.sm_red;
+}
+
+template <typename R>
+vqc_status run_hbm_forward(const HostPlan& p, int B, const void* x, const void* w,
+                           const void* psi0, void* E, void* state_out, void* ws, size_t ws_bytes,
+                           cudaStream_t stream, bool want_E) {
+    using C = C2<R>;
+    PassGeo L;
+    vqc_status st = plan_hbm(p, 0, B, L);
+    if (st != VQC_OK) return st;
+    const HbmWs lay = hbm_layout(p, 0, B, L.ntiles);
+    if (!ws || ws_bytes < lay.total || misaligned(ws, 256))
+        return fail(VQC_ERR_WORKSPACE, "forward workspace must be >= " + std::to_string(lay.total) +
+                                           " bytes and 256-byte aligned");
+    char* wsc = static_cast<char*>(ws);
+    C* W = state_out ? static_cast<C*>(state_out) : reinterpret_cast<C*>(wsc + lay.state);
+    R* E_part = reinterpret_cast<R*>(wsc + lay.part);
+    const int np = (int)L.s->passes.size();
+    for (int i = 0; i < np; ++i) {
+        PArgs<R> a{};
+        fill_pass_args<R>(p, L, L.s->passes[i], a);
+        a.B = B;
+        a.x = static_cast<const R*>(x);
+        a.w = static_cast<const R*>(w);
+        a.src_psi = i == 0 ? static_cast<const C*>(psi0) : W;
+        const bool last = i == np - 1;
+        a.dst_psi = (last && want_E && !state_out) ? nullptr : W;
+        a.E_part = (last && want_E) ? E_part : nullptr;
+        void* args[] = {&a};
+        VQC_CUDA(cudaLaunchKernel(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
+    }
+    if (want_E) {
+        const R* Ep = E_part;
+        R* Eo = static_cast<R*>(E);
+        int Bi = B, nt = L.ntiles, n = p.n;
+        void* args[] = {&Ep, &Bi, &nt, &n, &Eo};
+        const int blocks = (int)std::min<long long>(4096, ((long long)B * n + 255) / 256);
+        VQC_CUDA(cudaLaunchKernel(reduce_expz_ptr(p.dtype == VQC_C128), dim3(std::max(blocks, 1)),
+                                  dim3(256), args, 0, stream));
+    }
+    return VQC_OK;
+}
+
+template <typename R>
+vqc_status run_hbm_backward(const HostPlan& p, int B, const void* x, const void* w,
+                            const void* psi0, const void* psi_final, const void* gE, void* dx,
+                            void* dw, void* ws, size_t ws_bytes, cudaStream_t stream) {
+    using C = C2<R>;
+    PassGeo L;
+    vqc_status st = plan_hbm(p, 1, B, L);
+    if (st != VQC_OK) return st;
+    const HbmWs lay = hbm_layout(p, 1, B, L.ntiles);
+    size_t need = lay.total;
+    if (!ws || ws_bytes < need || misaligned(ws, 256))
+        return fail(VQC_ERR_WORKSPACE, "backward workspace must be >= " + std::to_string(need) +
+                                           " bytes and 256-byte aligned");
+    char* wsc = static_cast<char*>(ws);
+    C* Psi = reinterpret_cast<C*>(wsc + lay.state);
+    C* Lam = reinterpret_cast<C*>(wsc + lay.lam);
+    R* terms = reinterpret_cast<R*>(wsc + lay.part);
+    const C* src0 = static_cast<const C*>(psi_final);
+    if (!src0) {
+        // recompute the final state into Psi (the forward passes need no <Z>)
+        PassGeo Lf;
+        st = plan_hbm(p, 0, B, Lf);
+        if (st != VQC_OK) return st;
+        const int npf = (int)Lf.s->passes.size();
+        for (int i = 0; i < npf; ++i) {
+            PArgs<R> a{};
+            fill_pass_args<R>(p, Lf, Lf.s->passes[i], a);
+            a.B = B;
+            a.x = static_cast<const R*>(x);
+            a.w = static_cast<const R*>(w);
+            a.src_psi = i == 0 ? static_cast<const C*>(psi0) : Psi;
+            a.dst_psi = Psi;
+            void* args[] = {&a};
+            VQC_CUDA(cudaLaunchKernel(Lf.fn, dim3(Lf.grid), dim3(Lf.block), args, Lf.smem, stream));
+        }
+        src0 = Psi;
+    }
+    const int np = (int)L.s->passes.size();
+    for (int i = np - 1; i >= 0; --i) {
+        PArgs<R> a{};
+        fill_pass_args<R>(p, L, L.s->passes[i], a);
+        a.B = B;
+        a.x = static_cast<const R*>(x);
+        a.w = static_cast<const R*>(w);
+        a.gE = static_cast<const R*>(gE);
+        const bool first = i == np - 1, last = i == 0;
+        a.src_psi = first ? src0 : Psi;
+        a.src_lam = first ? nullptr : Lam;
+        a.dst_psi = last ? nullptr : Psi;
+        a.dst_lam = last ? nullptr : Lam;
+        a.terms = terms;
+        void* args[] = {&a};
+        VQC_CUDA(cudaLaunchKernel(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
+    }
+    const char* base = static_cast<const char*>(p.dbuf);
+    const bool dbl = p.dtype == VQC_C128;
+    int nt = (int)p.term_src.size();
+    if (dx && p.num_x > 0) {
+        const R* t = terms;
+        int Bi = B, ntl = L.ntiles, Px = p.num_x;
+        const int32_t* ptr = reinterpret_cast<const int32_t*>(base + p.dev_xocc_ptr);
+        const int32_t* occ = reinterpret_cast<const int32_t*>(base + p.dev_xocc);
+        R* o = static_cast<R*>(dx);
+        void* args[] = {&t, &Bi, &ntl, &nt, &ptr, &occ, &Px, &o};
+        const int blocks = (int)std::min<long long>(4096, ((long long)B * Px + 255) / 256);
+        VQC_CUDA(cudaLaunchKernel(reduce_dx_ptr(dbl), dim3(std::max(blocks, 1)), dim3(256), args, 0,
+                                  stream));
+    }
+    if (dw && p.num_w > 0) {
+        const R* t = terms;
+        long long rows = (long long)B * L.ntiles;
+        const int32_t* ptr = reinterpret_cast<const int32_t*>(base + p.dev_wocc_ptr);
+        const int32_t* occ = reinterpret_cast<const int32_t*>(base + p.dev_wocc);
+        R* o = static_cast<R*>(dw);
+        void* args[] = {&t, &rows, &nt, &ptr, &occ, &o};
+        VQC_CUDA(cudaLaunchKernel(reduce_dw_ptr(dbl), dim3(p.num_w), dim3(256), args, 0, stream));
+    }
+    return VQC_OK;
+}
+
+// The resident path when it can take the batch (and VQC_FORCE_PATH does not
+// ask for the HBM path), else the HBM path.
+bool use_hbm(const HostPlan& p, int mode, int B) {
+    const char* f = std::getenv("VQC_FORCE_PATH");
+    if (f && std::string(f) == "hbm" && find_hbm_schedule(p, mode)) return true;
+    Launch L;
+    std::string saved = g_err;
+    if (plan_launch(p, mode, B, L) == VQC_OK) return false;
+    g_err = saved;
+    return find_hbm_schedule(p, mode) != nullptr;
 }
 
 std::mutex g_upload_mu;
@@ -427,10 +695,17 @@ void vqc_free(vqc_plan* plan) {
 
 size_t vqc_workspace_bytes(const vqc_plan* plan, int32_t batch, int32_t mode) {
     if (!plan) return (size_t)-1;
-    if (mode != 1 || batch <= 0) return 0;
+    if ((mode != 0 && mode != 1) || batch <= 0) return 0;
+    const HostPlan& p = plan->hp;
+    if (use_hbm(p, mode, batch)) {
+        PassGeo L;
+        if (plan_hbm(p, mode, batch, L) != VQC_OK) return 0;
+        return hbm_layout(p, mode, batch, L.ntiles).total;
+    }
+    if (mode == 0) return 0;
     Launch L;
-    if (plan_launch(plan->hp, 1, batch, L) != VQC_OK) return 0;
-    return bwd_workspace(plan->hp, L);
+    if (plan_launch(p, 1, batch, L) != VQC_OK) return 0;
+    return bwd_workspace(p, L);
 }
 
 vqc_status vqc_workspace_init(void* workspace, size_t workspace_bytes, void* stream) {
@@ -450,9 +725,14 @@ vqc_status vqc_forward(const vqc_plan* plan, int32_t batch, const void* x, const
         st = check_ptrs(p, x, w, psi0, nullptr);
         if (st != VQC_OK) return st;
         if (!expz_out) return fail(VQC_ERR_INVALID_ARG, "expz_out is NULL");
-        (void)workspace;
-        (void)workspace_bytes;
         cudaStream_t s = static_cast<cudaStream_t>(stream);
+        if (use_hbm(p, 0, batch)) {
+            if (p.dtype == VQC_C64)
+                return run_hbm_forward<float>(p, batch, x, w, psi0, expz_out, state_out, workspace,
+                                              workspace_bytes, s, true);
+            return run_hbm_forward<double>(p, batch, x, w, psi0, expz_out, state_out, workspace,
+                                           workspace_bytes, s, true);
+        }
         if (p.dtype == VQC_C64)
             return run<float>(p, 0, batch, x, w, psi0, nullptr, nullptr, expz_out, state_out,
                               nullptr, nullptr, nullptr, 0, s);
@@ -480,6 +760,13 @@ vqc_status vqc_backward(const vqc_plan* plan, int32_t batch, const void* x, cons
         st = check_ptrs(p, x, w, psi0, psi_final);
         if (st != VQC_OK) return st;
         if (!grad_expz) return fail(VQC_ERR_INVALID_ARG, "grad_expz is NULL");
+        if (use_hbm(p, 1, batch)) {
+            if (p.dtype == VQC_C64)
+                return run_hbm_backward<float>(p, batch, x, w, psi0, psi_final, grad_expz, grad_x,
+                                               grad_w, workspace, workspace_bytes, s);
+            return run_hbm_backward<double>(p, batch, x, w, psi0, psi_final, grad_expz, grad_x,
+                                            grad_w, workspace, workspace_bytes, s);
+        }
         if (p.dtype == VQC_C64)
             return run<float>(p, 1, batch, x, w, psi0, psi_final, grad_expz, nullptr, nullptr,
                               grad_x, grad_w, workspace, workspace_bytes, s);
@@ -506,15 +793,25 @@ vqc_status vqc_plan_info(const vqc_plan* plan, int32_t batch, vqc_plan_stats* ou
     out->bwd_flops_per_eval = p.bwd_flops;
     out->recompute_flops_per_eval = p.recompute_flops;
     const int B = std::max(batch, 1);
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess) {
+        (void)cudaGetLastError();
+        ndev = 0;
+    }
+    const std::string saved = g_err;
+    const double sbytes = std::ldexp(1.0, p.n) * (p.dtype == VQC_C128 ? 16.0 : 8.0);
     for (int mode = 0; mode < 2; ++mode) {
-        int K = choose_k(p, mode, B);
-        const Schedule* s = K ? find_schedule(p, mode, K) : nullptr;
         int* path = mode == 0 ? &out->fwd_path : &out->bwd_path;
         int* kk = mode == 0 ? &out->fwd_k : &out->bwd_k;
         int* ns = mode == 0 ? &out->fwd_stages : &out->bwd_stages;
         int* np = mode == 0 ? &out->fwd_passes : &out->bwd_passes;
         int* tps = mode == 0 ? &out->fwd_threads_per_sample : &out->bwd_threads_per_sample;
         int* tq = mode == 0 ? &out->fwd_tile_qubits : &out->bwd_tile_qubits;
+        double* hb = mode == 0 ? &out->fwd_hbm_bytes_per_eval : &out->bwd_hbm_bytes_per_eval;
+        const int K = choose_k(p, mode, B);
+        const bool hbm = ndev > 0 ? use_hbm(p, mode, B)
+                                  : (K == 0 && find_hbm_schedule(p, mode) != nullptr);
+        const Schedule* s = hbm ? find_hbm_schedule(p, mode) : (K ? find_schedule(p, mode, K) : nullptr);
         if (!s) {
             *path = -1;
             continue;
@@ -522,10 +819,21 @@ vqc_status vqc_plan_info(const vqc_plan* plan, int32_t batch, vqc_plan_stats* ou
         *path = s->path;
         *kk = s->K;
         *ns = (int)s->stages.size();
-        *np = 1;
-        *tps = 1 << (p.n - s->K);
         *tq = s->m;
+        if (hbm) {
+            const int P = (int)s->passes.size();
+            *np = P;
+            *tps = (1 << (s->m - s->K)) << (p.n - s->m);
+            // state traffic: forward reads and writes the state once per pass;
+            // the backward reads psi (and lam after the first pass) and writes
+            // both (except after the last pass)
+            *hb = mode == 0 ? 2.0 * P * sbytes : (4.0 * P - 3.0) * sbytes;
+        } else {
+            *np = 1;
+            *tps = 1 << (p.n - s->K);
+        }
     }
+    g_err = saved;
     return VQC_OK;
 }
 

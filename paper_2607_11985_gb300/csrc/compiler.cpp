@@ -12,6 +12,7 @@
 #include <algorithm>
 #include <cmath>
 #include <complex>
+#include <cstdlib>
 #include <cstring>
 #include <numeric>
 
@@ -289,15 +290,24 @@ uint32_t op_need(const HOp& o) {
     return 0;
 }
 
-// Cut the op list into stages of K active qubits (resident path: tile = all n).
-void build_schedule(const HostPlan& p, Schedule& s) {
-    const int n = p.n, K = s.K, G = p.G_swz;
-    s.m = n;
-    s.thread_bits = n - K;
-    s.group_lanes_log2 = s.thread_bits;
-    std::vector<int> remaining(p.ops.size());
-    std::iota(remaining.begin(), remaining.end(), 0);
-    do {   // an empty circuit still gets one (empty) stage
+// Cut `ops` (indices into p.ops, time-valid order) into stages of K active
+// qubits drawn from the tile qubit set `tile` (ascending).  Stage records use
+// tile-local positions for shared-memory addressing and global qubits for the
+// thread-bit masks.  `slot_of` / `acc_of` map entry ids / accumulator ids to the
+// indices the kernel sees (identity on the resident path, pass-local on the
+// HBM path).
+void cut_stages(const HostPlan& p, const std::vector<int>& ops, const std::vector<int>& tile,
+                int K, Schedule& s, const std::vector<int>& slot_of,
+                const std::vector<int>& acc_of) {
+    const int G = p.G_swz;
+    std::vector<int> lpos(p.n, -1);   // tile-local bit of each global qubit
+    uint32_t tile_mask = 0;
+    for (size_t i = 0; i < tile.size(); ++i) {
+        lpos[tile[i]] = (int)i;
+        tile_mask |= 1u << tile[i];
+    }
+    std::vector<int> remaining = ops;
+    do {   // an empty op list still gets one (empty) stage
         uint32_t active = 0, blocked = 0;
         std::vector<int> taken, deferred;
         for (int oi : remaining) {
@@ -317,34 +327,36 @@ void build_schedule(const HostPlan& p, Schedule& s) {
                 deferred.push_back(oi);
             }
         }
-        // Pad the active set to exactly K qubits, keeping every residue class
-        // (mod G) represented among the outer qubits where possible.
+        // Pad the active set to exactly K tile qubits, keeping every residue
+        // class (mod G, of tile-local positions) represented among the thread bits.
         while (__builtin_popcount(active) < K) {
             int best = -1, best_cnt = -1;
-            for (int q = n - 1; q >= 0; --q) {
+            for (int i = (int)tile.size() - 1; i >= 0; --i) {
+                int q = tile[i];
                 if (active >> q & 1) continue;
                 int cnt = 0;
-                for (int r = 0; r < n; ++r)
-                    if (!(active >> r & 1) && r % G == q % G) ++cnt;
+                for (int r : tile)
+                    if (!(active >> r & 1) && lpos[r] % G == i % G) ++cnt;
                 if (cnt > best_cnt) { best_cnt = cnt; best = q; }
             }
             active |= 1u << best;
         }
         DStage st{};
         int j = 0;
-        for (int q = 0; q < n; ++q)
+        for (int q : tile)
             if (active >> q & 1) st.active[j++] = (uint8_t)q;
-        for (int k = 0; k < K; ++k) st.sigma[k] = (int32_t)swz(1u << st.active[k], G);
-        // Thread bits: bit i (i < G) takes an outer qubit of residue i when one exists.
+        for (int k = 0; k < K; ++k) st.sigma[k] = (int32_t)swz(1u << lpos[st.active[k]], G);
+        // Thread bits: bit i (i < G) takes a tile qubit whose tile-local
+        // position has residue i (mod G) when one exists.
         std::vector<int> outer;
-        for (int q = 0; q < n; ++q)
+        for (int q : tile)
             if (!(active >> q & 1)) outer.push_back(q);
         std::vector<int> order;
         std::vector<bool> used(outer.size(), false);
         for (int i = 0; i < std::min<int>(G, (int)outer.size()); ++i) {
             int pick = -1;
             for (size_t c = 0; c < outer.size(); ++c)
-                if (!used[c] && outer[c] % G == i) { pick = (int)c; break; }
+                if (!used[c] && lpos[outer[c]] % G == i) { pick = (int)c; break; }
             if (pick < 0)
                 for (size_t c = 0; c < outer.size(); ++c)
                     if (!used[c]) { pick = (int)c; break; }
@@ -355,7 +367,7 @@ void build_schedule(const HostPlan& p, Schedule& s) {
             if (!used[c]) order.push_back(outer[c]);
         st.nthreadbits = (uint8_t)order.size();
         for (size_t i = 0; i < order.size(); ++i) {
-            st.tau[i] = (int32_t)swz(1u << order[i], G);
+            st.tau[i] = (int32_t)swz(1u << lpos[order[i]], G);
             st.tmask[i] = 1u << order[i];
         }
         auto local = [&](int q) -> int {
@@ -374,10 +386,10 @@ void build_schedule(const HostPlan& p, Schedule& s) {
             d.type = o.type;
             if (o.type == OP_M1 || o.type == OP_PH2) {
                 const DEntry& e = p.entries[o.entry];
-                d.slot = e.slot;
+                d.slot = (uint16_t)slot_of[o.entry];
                 d.flags = (uint8_t)((e.per_sample ? OPF_PER_SAMPLE : 0) |
                                     (e.acc != 0xffff ? OPF_HAS_ACC : 0) | o.gen);
-                d.aux = e.acc;
+                d.aux = e.acc != 0xffff ? (uint16_t)acc_of[e.acc] : (uint16_t)0xffff;
             }
             if (o.type == OP_M1) {
                 d.a = (uint8_t)local(o.q0);
@@ -392,6 +404,100 @@ void build_schedule(const HostPlan& p, Schedule& s) {
         }
         st.op_end = (int32_t)s.ops.size();
         s.stages.push_back(st);
+        remaining.swap(deferred);
+    } while (!remaining.empty());
+    (void)tile_mask;
+}
+
+void build_schedule(const HostPlan& p, Schedule& s) {
+    const int n = p.n;
+    s.m = n;
+    s.thread_bits = n - s.K;
+    s.group_lanes_log2 = s.thread_bits;
+    std::vector<int> ops(p.ops.size()), tile(n), slot_of(p.entries.size()), acc_of(p.accs.size());
+    std::iota(ops.begin(), ops.end(), 0);
+    std::iota(tile.begin(), tile.end(), 0);
+    for (size_t i = 0; i < p.entries.size(); ++i) slot_of[i] = p.entries[i].slot;
+    std::iota(acc_of.begin(), acc_of.end(), 0);
+    cut_stages(p, ops, tile, s.K, s, slot_of, acc_of);
+}
+
+// HBM path: passes over tiles of m qubits (always containing the low qubits
+// whose amplitudes form one 128-byte chunk), each pass cut into stages.
+void build_hbm_schedule(const HostPlan& p, Schedule& s) {
+    const int n = p.n, m = s.m, low = p.G_swz;   // 2^G amplitudes = 128 bytes
+    s.thread_bits = m - s.K;
+    s.group_lanes_log2 = s.thread_bits;
+    std::vector<int> remaining(p.ops.size());
+    std::iota(remaining.begin(), remaining.end(), 0);
+    const uint32_t low_mask = (1u << std::min(low, n)) - 1;
+    do {
+        uint32_t tilem = low_mask, blocked = 0;
+        std::vector<int> taken, deferred;
+        for (int oi : remaining) {
+            const HOp& o = p.ops[oi];
+            uint32_t touch = op_touch(o), need = op_need(o);
+            if (touch & blocked) {
+                blocked |= touch;
+                deferred.push_back(oi);
+                continue;
+            }
+            uint32_t nt = tilem | need;
+            if (__builtin_popcount(nt) <= m) {
+                tilem = nt;
+                taken.push_back(oi);
+            } else {
+                blocked |= touch;
+                deferred.push_back(oi);
+            }
+        }
+        // Pad the tile with the qubits the deferred ops need first.
+        for (int oi : deferred) {
+            if (__builtin_popcount(tilem) >= m) break;
+            uint32_t need = op_need(p.ops[oi]);
+            if (need && __builtin_popcount(tilem | need) <= m) tilem |= need;
+        }
+        for (int q = n - 1; q >= 0 && __builtin_popcount(tilem) < m; --q) tilem |= 1u << q;
+        DPass ps{};
+        ps.stage_begin = (int32_t)s.stages.size();
+        ps.m = m;
+        ps.nout = n - m;
+        std::vector<int> tile;
+        int no = 0;
+        for (int q = 0; q < n; ++q) {
+            if (tilem >> q & 1) tile.push_back(q);
+            else ps.out_q[no++] = (uint8_t)q;
+        }
+        for (int i = 0; i < m; ++i) ps.tile_q[i] = (uint8_t)tile[i];
+        // Pass-local table slots and accumulators.
+        std::vector<int> slot_of(p.entries.size(), -1), acc_of(p.accs.size(), -1);
+        ps.ps_begin = (int32_t)s.pass_entries.size();
+        for (int oi : taken) {
+            const HOp& o = p.ops[oi];
+            if (o.entry >= 0 && p.entries[o.entry].per_sample && slot_of[o.entry] < 0) {
+                slot_of[o.entry] = ps.ps_count++;
+                s.pass_entries.push_back(o.entry);
+            }
+        }
+        ps.sh_begin = (int32_t)s.pass_entries.size();
+        for (int oi : taken) {
+            const HOp& o = p.ops[oi];
+            if (o.entry >= 0 && !p.entries[o.entry].per_sample && slot_of[o.entry] < 0) {
+                slot_of[o.entry] = ps.sh_count++;
+                s.pass_entries.push_back(o.entry);
+            }
+        }
+        ps.acc_begin = (int32_t)s.pass_accs.size();
+        for (int oi : taken) {
+            const HOp& o = p.ops[oi];
+            if (o.entry >= 0 && p.entries[o.entry].acc != 0xffff && acc_of[p.entries[o.entry].acc] < 0) {
+                acc_of[p.entries[o.entry].acc] = ps.acc_count++;
+                s.pass_accs.push_back(p.entries[o.entry].acc);
+            }
+        }
+        cut_stages(p, taken, tile, s.K, s, slot_of, acc_of);
+        ps.stage_end = (int32_t)s.stages.size();
+        s.passes.push_back(ps);
         remaining.swap(deferred);
     } while (!remaining.empty());
 }
@@ -470,6 +576,7 @@ vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx,
         for (int K = 1; K <= std::min(max_k(mode, dtype), n); ++K) {
             const int max_tb = (dtype == VQC_C64 && mode == 0 && K <= 4) ? 10 : 9;
             if (n - K > max_tb) continue;   // thread group must fit one CTA
+            if (n > resident_max_qubits(mode, dtype)) continue;
             Schedule s;
             s.mode = mode;
             s.K = K;
@@ -478,12 +585,37 @@ vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx,
             p.scheds.push_back(std::move(s));
         }
     }
+    // HBM-tiled pass schedules (tile of m qubits, K fixed per mode and type).
+    for (int mode = 0; mode < 2; ++mode) {
+        int m = std::min(hbm_tile_qubits(mode, dtype, p.G_swz), n - 1);
+        int K = std::min(hbm_k(mode, dtype), m - 1);
+        if (n < p.G_swz + 2 || K < 1 || m <= p.G_swz) continue;
+        const int env_m = std::getenv("VQC_HBM_TILE_QUBITS") ? std::atoi(std::getenv("VQC_HBM_TILE_QUBITS")) : 0;
+        if (env_m > p.G_swz && env_m < n) {
+            m = std::max(env_m, hbm_k(mode, dtype) + 1);
+            K = std::min(hbm_k(mode, dtype), m - 1);
+        }
+        if (K != hbm_k(mode, dtype)) continue;   // pass kernels exist for this K only
+        Schedule s;
+        s.mode = mode;
+        s.K = K;
+        s.m = m;
+        s.path = VQC_PATH_HBM;
+        build_hbm_schedule(p, s);
+        p.scheds.push_back(std::move(s));
+    }
     return VQC_OK;
 }
 
 const Schedule* find_schedule(const HostPlan& p, int mode, int K) {
     for (const auto& s : p.scheds)
         if (s.mode == mode && s.K == K && s.path == VQC_PATH_RESIDENT) return &s;
+    return nullptr;
+}
+
+const Schedule* find_hbm_schedule(const HostPlan& p, int mode) {
+    for (const auto& s : p.scheds)
+        if (s.mode == mode && s.path == VQC_PATH_HBM) return &s;
     return nullptr;
 }
 
@@ -518,6 +650,9 @@ std::vector<uint8_t> export_plan(const HostPlan& p) {
         for (int v : {s.mode, s.K, s.m, s.path, s.thread_bits, s.group_lanes_log2}) put_i32(out, v);
         put_vec(out, s.ops);
         put_vec(out, s.stages);
+        put_vec(out, s.passes);
+        put_vec(out, s.pass_entries);
+        put_vec(out, s.pass_accs);
     }
     return out;
 }

@@ -32,7 +32,11 @@ struct Schedule {
     int group_lanes_log2 = 0;   // log2(threads per sample group) when < 2^G
     std::vector<DOp> ops;
     std::vector<DStage> stages;
+    std::vector<DPass> passes;            // HBM path: one record per pass
+    std::vector<int32_t> pass_entries;    // HBM path: table entries per pass (ps, then sh)
+    std::vector<int32_t> pass_accs;       // HBM path: accumulator ids per pass
     size_t dev_ops = 0, dev_stages = 0;   // byte offsets inside the device buffer
+    size_t dev_passes = 0, dev_pass_entries = 0, dev_pass_accs = 0;
 };
 
 struct HostPlan {
@@ -60,6 +64,22 @@ struct HostPlan {
     unsigned* dev_error = nullptr;        // device error word (kernel self-checks)
 };
 
+// Largest n whose state(s) fit one CTA's shared memory on the resident path.
+inline int resident_max_qubits(int mode, int dtype) {
+    if (dtype == VQC_C64) return mode == 0 ? 14 : 13;
+    return mode == 0 ? 13 : 12;
+}
+// Tile qubits of an HBM pass: 64 KiB of tile state per CTA (two states for the backward).
+inline int hbm_tile_qubits(int mode, int dtype, int G) {
+    (void)G;
+    if (dtype == VQC_C64) return mode == 0 ? 13 : 12;
+    return mode == 0 ? 12 : 11;
+}
+inline int hbm_k(int mode, int dtype) {
+    if (dtype == VQC_C64) return mode == 0 ? 5 : 4;
+    return mode == 0 ? 4 : 3;
+}
+
 // Maximum K per (mode, dtype) for register-resident blocks.
 inline int max_k(int mode, int dtype) {
     if (dtype == VQC_C64) return mode == 0 ? 5 : 4;
@@ -70,6 +90,7 @@ inline int max_k(int mode, int dtype) {
 vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx, int32_t nw,
                         int dtype, HostPlan& out, std::string& err);
 const Schedule* find_schedule(const HostPlan& p, int mode, int K);
+const Schedule* find_hbm_schedule(const HostPlan& p, int mode);
 std::vector<uint8_t> export_plan(const HostPlan& p);
 
 }  // namespace vqc

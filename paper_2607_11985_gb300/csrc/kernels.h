@@ -10,6 +10,12 @@ const void* sweep_ptr_f32_bwd(int K);
 const void* sweep_ptr_f64_fwd(int K);
 const void* sweep_ptr_f64_bwd(int K);
 
+// HBM-tiled pass kernels (K fixed per type and mode) and partial reductions.
+const void* pass_ptr(bool dbl, int mode, int K);
+const void* reduce_expz_ptr(bool dbl);
+const void* reduce_dx_ptr(bool dbl);
+const void* reduce_dw_ptr(bool dbl);
+
 // Largest block (threads) each instantiation is compiled for.
 inline int sweep_max_threads(bool is_double, int mode, int K) {
     if (!is_double && mode == 0 && K <= 4) return 1024;

@@ -1,0 +1,32 @@
+// kernels_hbm.cu -- instantiations of the HBM-tiled pass kernels and the
+// fixed-order partial reductions.
+#include "kernels.h"
+#include "pass.cuh"
+
+namespace vqc {
+
+const void* pass_ptr(bool dbl, int mode, int K) {
+    if (!dbl) {
+        if (mode == 0 && K == 5) return reinterpret_cast<const void*>(&pass_kernel<float, 5, 0>);
+        if (mode == 1 && K == 4) return reinterpret_cast<const void*>(&pass_kernel<float, 4, 1>);
+    } else {
+        if (mode == 0 && K == 4) return reinterpret_cast<const void*>(&pass_kernel<double, 4, 0>);
+        if (mode == 1 && K == 3) return reinterpret_cast<const void*>(&pass_kernel<double, 3, 1>);
+    }
+    return nullptr;
+}
+
+const void* reduce_expz_ptr(bool dbl) {
+    return dbl ? reinterpret_cast<const void*>(&reduce_expz<double>)
+               : reinterpret_cast<const void*>(&reduce_expz<float>);
+}
+const void* reduce_dx_ptr(bool dbl) {
+    return dbl ? reinterpret_cast<const void*>(&reduce_dx<double>)
+               : reinterpret_cast<const void*>(&reduce_dx<float>);
+}
+const void* reduce_dw_ptr(bool dbl) {
+    return dbl ? reinterpret_cast<const void*>(&reduce_dw<double>)
+               : reinterpret_cast<const void*>(&reduce_dw<float>);
+}
+
+}  // namespace vqc

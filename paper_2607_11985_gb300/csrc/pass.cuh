@@ -1,0 +1,287 @@
+// pass.cuh -- HBM-tiled path for states that do not fit one SM's shared memory
+// (paper, Sec. 3 "Complexity and Tradeoffs": the state, O(B 2^n), is the
+// memory wall; here it lives in HBM between passes).
+//
+// The compiler cuts the op list into passes.  A pass acts on tiles of m
+// qubits: the tile qubits always include the low qubits whose 2^G amplitudes
+// form one 128-byte chunk, so a tile is gathered from HBM as whole chunks.
+// One launch per pass: each CTA loads S tiles (the other n - m qubits fix the
+// tile), runs the pass's register-block stages on them in shared memory
+// exactly as the resident path does, and writes them back.  The forward's last
+// pass emits per-tile <Z> partials; the backward emits per-tile gradient
+// terms.  reduce_* kernels sum partials in a fixed order (deterministic).
+#pragma once
+
+#include "sweep.cuh"
+
+namespace vqc {
+
+template <typename R>
+struct PArgs {
+    const DOp* ops;
+    const DStage* stages;
+    const int32_t* pass_entries;
+    const int32_t* pass_accs;
+    const DEntry* entries;
+    const DConst* consts;
+    const R* cmat;
+    const R* cang;
+    const DAcc* accs;
+    int n, m, K, tbits, G, S, nout, ntiles;
+    int stage_begin, stage_end;
+    int ps_begin, ps_count, sh_begin, sh_count, acc_begin, acc_count, n_terms, Px;
+    int B;
+    long long nunits;
+    uint8_t tile_q[24], out_q[24];
+    const R* x;
+    const R* w;
+    const R* gE;
+    const C2<R>* src_psi;   // tiles are read from here (nullptr: start from |0...0>)
+    C2<R>* dst_psi;         // and written back here (nullptr: not written)
+    const C2<R>* src_lam;   // backward: lam tiles (nullptr: lam = O psi in the first stage)
+    C2<R>* dst_lam;
+    R* E_part;              // forward, last pass: [B * ntiles, n]
+    R* terms;               // backward: [B * ntiles, n_terms]
+    int sm_sh, sm_ps, sm_psi, sm_lam, sm_acc, sm_red;
+};
+
+// Global amplitude index of tile-local index u (the low G tile bits are the
+// low G qubits; the rest follow tile_q).
+__device__ __forceinline__ uint32_t tile_global(uint32_t u, uint32_t tile_base, const uint8_t* tq,
+                                                int G) {
+    uint32_t g = tile_base | (u & ((1u << G) - 1u));
+    uint32_t hi = u >> G;
+    for (int i = G; hi; ++i, hi >>= 1)
+        if (hi & 1u) g |= 1u << tq[i];
+    return g;
+}
+
+// Copy one tile HBM -> shared memory (16-byte vectors; 8 per 128-byte chunk).
+template <typename R>
+__device__ __forceinline__ void tile_gather(C2<R>* sm, const C2<R>* gs, uint32_t tile_base,
+                                            const uint8_t* tq, int m, int G, int h, int t, int T) {
+    constexpr int APV = 16 / sizeof(C2<R>);   // amplitudes per 16-byte vector
+    const int nvec = (1 << m) / APV;
+    for (int v = t; v < nvec; v += T) {
+        const uint32_t u = (uint32_t)v * APV;
+        const uint32_t g = tile_global(u, tile_base, tq, G);
+        const float4 raw = __ldcs(reinterpret_cast<const float4*>(gs + g));
+        const C2<R>* pr = reinterpret_cast<const C2<R>*>(&raw);
+#pragma unroll
+        for (int k = 0; k < APV; ++k) sm[swz(u + k, G) ^ h] = pr[k];
+    }
+}
+
+template <typename R>
+__device__ __forceinline__ void tile_scatter(const C2<R>* sm, C2<R>* gs, uint32_t tile_base,
+                                             const uint8_t* tq, int m, int G, int h, int t, int T) {
+    constexpr int APV = 16 / sizeof(C2<R>);
+    const int nvec = (1 << m) / APV;
+    for (int v = t; v < nvec; v += T) {
+        const uint32_t u = (uint32_t)v * APV;
+        const uint32_t g = tile_global(u, tile_base, tq, G);
+        float4 raw;
+        C2<R>* pr = reinterpret_cast<C2<R>*>(&raw);
+#pragma unroll
+        for (int k = 0; k < APV; ++k) pr[k] = sm[swz(u + k, G) ^ h];
+        __stcs(reinterpret_cast<float4*>(gs + g), raw);
+    }
+}
+
+template <typename R, int K, int MODE>
+__global__ void __launch_bounds__(512) pass_kernel(const __grid_constant__ PArgs<R> A) {
+    extern __shared__ __align__(16) unsigned char smem[];
+    R* sh_tab = reinterpret_cast<R*>(smem + A.sm_sh);
+    R* ps_all = reinterpret_cast<R*>(smem + A.sm_ps);
+    C2<R>* psi_all = reinterpret_cast<C2<R>*>(smem + A.sm_psi);
+    C2<R>* lam_all = reinterpret_cast<C2<R>*>(smem + A.sm_lam);
+    R* acc_all = reinterpret_cast<R*>(smem + A.sm_acc);
+    R* red_all = reinterpret_cast<R*>(smem + A.sm_red);
+
+    const int n = A.n, G = A.G, tdim = 1 << A.m;
+    const long long total_tiles = (long long)A.B * A.ntiles;
+    Geo q;
+    q.T = 1 << A.tbits;
+    q.lanes = q.T < 32 ? q.T : 32;
+    q.wg = q.T > 32 ? q.T / 32 : 1;
+    q.g = threadIdx.x / q.T;
+    q.t = threadIdx.x % q.T;
+    q.h = 0;
+    if (A.tbits < G) q.h = ((q.g & ((1 << (G - A.tbits)) - 1)) << A.tbits) & (tdim - 1);
+    q.mask = blockDim.x >= 32 ? 0xffffffffu : ((1u << blockDim.x) - 1u);
+    const int lane = q.t & 31;
+    const int warp_in_group = q.t >> 5;
+    const int nthr = blockDim.x;
+
+    for (int i = threadIdx.x; i < A.sh_count; i += nthr) {
+        const DEntry e = A.entries[__ldg(&A.pass_entries[A.sh_begin + i])];
+        eval_entry<R>(e, A.consts, nullptr, A.w, A.cang, A.cmat, sh_tab + 8 * i);
+    }
+    __syncthreads();
+
+    C2<R>* psi = psi_all + (size_t)q.g * tdim;
+    C2<R>* lam = lam_all + (size_t)q.g * tdim;
+    R* ps_tab = ps_all + (size_t)q.g * A.ps_count * 8;
+    R* acc = acc_all + (size_t)q.g * A.acc_count * q.wg * 8;
+
+    for (long long unit = blockIdx.x; unit < A.nunits; unit += gridDim.x) {
+        const long long tid_raw = unit * A.S + q.g;
+        const bool valid = tid_raw < total_tiles;
+        const long long tile_id = valid ? tid_raw : total_tiles - 1;
+        const int b = (int)(tile_id / A.ntiles);
+        const int tau = (int)(tile_id % A.ntiles);
+        uint32_t tile_base = 0;
+        for (int j = 0; j < A.nout; ++j)
+            if ((tau >> j) & 1) tile_base |= 1u << A.out_q[j];
+
+        for (int i = threadIdx.x; i < A.S * A.ps_count; i += nthr) {
+            const int gg = i / A.ps_count, k = i % A.ps_count;
+            const long long tt = min(unit * A.S + gg, total_tiles - 1);
+            const int bb = (int)(tt / A.ntiles);
+            const DEntry e = A.entries[__ldg(&A.pass_entries[A.ps_begin + k])];
+            eval_entry<R>(e, A.consts, A.x + (size_t)bb * A.Px, A.w, A.cang, A.cmat,
+                          ps_all + ((size_t)gg * A.ps_count + k) * 8);
+        }
+        const size_t sbase = (size_t)b << n;
+        if (A.src_psi)
+            tile_gather<R>(psi, A.src_psi + sbase, tile_base, A.tile_q, A.m, G, q.h, q.t, q.T);
+        if (MODE == 1 && A.src_lam)
+            tile_gather<R>(lam, A.src_lam + sbase, tile_base, A.tile_q, A.m, G, q.h, q.t, q.T);
+        __syncthreads();
+
+        C2<R> a[1 << K];
+        int32_t sg[K];
+        StageView v{0, 0};
+        if (MODE == 0) {
+            for (int s = A.stage_begin; s < A.stage_end; ++s) {
+                const DStage* sp = A.stages + s;
+                v = stage_view<K>(sp, q.t, q.h, sg);
+                v.pb |= tile_base;
+                if (s == A.stage_begin && !A.src_psi) {
+#pragma unroll
+                    for (int r = 0; r < (1 << K); ++r) a[r] = cm<R>(0, 0);
+                    if (v.pb == 0) a[0] = cm<R>(1, 0);
+                } else {
+                    block_load<R, K>(a, psi, v.swb, sg);
+                }
+                const int ob = __ldg(&sp->op_begin), oe = __ldg(&sp->op_end);
+                for (int o = ob; o < oe; ++o) {
+                    const uint2 raw = __ldg(reinterpret_cast<const uint2*>(A.ops) + o);
+                    fwd_op<R, K>(raw, v.pb, a, sh_tab, ps_tab);
+                }
+                if (s + 1 < A.stage_end || A.dst_psi) {
+                    block_store<R, K>(a, psi, v.swb, sg);
+                    group_sync<R>(q);
+                }
+            }
+            if (A.E_part) {
+                R* red = red_all + (size_t)q.g * q.wg * n;
+                expz_partials<R, K>(A.stages + (A.stage_end - 1), v.pb, a, n, red, q, warp_in_group);
+                __syncthreads();
+                if (valid)
+                    for (int j = q.t; j < n; j += q.T) {
+                        R e = 0;
+                        for (int k = 0; k < q.wg; ++k) e += red[k * n + j];
+                        A.E_part[tile_id * n + j] = e;
+                    }
+            }
+            __syncthreads();
+            if (A.dst_psi && valid)
+                tile_scatter<R>(psi, A.dst_psi + sbase, tile_base, A.tile_q, A.m, G, q.h, q.t, q.T);
+            __syncthreads();
+            continue;
+        }
+
+        // backward: stages of the pass in reverse
+        for (int s = A.stage_end - 1; s >= A.stage_begin; --s) {
+            const DStage* sp = A.stages + s;
+            C2<R> l[1 << K];
+            v = stage_view<K>(sp, q.t, q.h, sg);
+            v.pb |= tile_base;
+            block_load<R, K>(a, psi, v.swb, sg);
+            if (s == A.stage_end - 1 && !A.src_lam)
+                lambda_init<R, K>(sp, v.pb, A.gE + (size_t)b * n, n, a, l);
+            else
+                block_load<R, K>(l, lam, v.swb, sg);
+            const int ob = __ldg(&sp->op_begin), oe = __ldg(&sp->op_end);
+            for (int o = oe - 1; o >= ob; --o) {
+                const uint2 raw = __ldg(reinterpret_cast<const uint2*>(A.ops) + o);
+                bwd_op<R, K>(raw, v.pb, a, l, sh_tab, ps_tab, acc, q, lane, warp_in_group);
+            }
+            if (s > A.stage_begin || A.dst_psi) {
+                block_store<R, K>(a, psi, v.swb, sg);
+                block_store<R, K>(l, lam, v.swb, sg);
+            }
+            group_sync<R>(q);
+        }
+        __syncthreads();
+        if (valid && A.dst_psi) {
+            tile_scatter<R>(psi, A.dst_psi + sbase, tile_base, A.tile_q, A.m, G, q.h, q.t, q.T);
+            tile_scatter<R>(lam, A.dst_lam + sbase, tile_base, A.tile_q, A.m, G, q.h, q.t, q.T);
+        }
+        for (int i = threadIdx.x; i < A.S * A.acc_count; i += nthr) {
+            const int gg = i / A.acc_count, k = i % A.acc_count;
+            const long long tt = unit * A.S + gg;
+            if (tt >= total_tiles) continue;
+            const int bb = (int)(tt / A.ntiles);
+            const DAcc ac = A.accs[__ldg(&A.pass_accs[A.acc_begin + k])];
+            acc_terms<R>(ac, A.entries[ac.entry], acc_all + ((size_t)gg * A.acc_count + k) * q.wg * 8,
+                         q.wg, A.consts, A.x ? A.x + (size_t)bb * A.Px : nullptr, A.w, A.cang,
+                         A.cmat, A.terms + tt * A.n_terms);
+        }
+        __syncthreads();
+    }
+}
+
+// E[b, j] = sum over tiles of E_part[b * ntiles + tau, j]  (fixed order).
+template <typename R>
+__global__ void reduce_expz(const R* E_part, int B, int ntiles, int n, R* E) {
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < (long long)B * n;
+         i += (long long)gridDim.x * blockDim.x) {
+        const long long b = i / n, j = i % n;
+        R s = 0;
+        for (int t = 0; t < ntiles; ++t) s += E_part[(b * ntiles + t) * n + j];
+        E[i] = s;
+    }
+}
+
+// dx[b, p] = sum_tau sum_{terms j of x column p} terms[b * ntiles + tau, j]
+template <typename R>
+__global__ void reduce_dx(const R* terms, int B, int ntiles, int nt, const int32_t* ptr,
+                          const int32_t* occ, int Px, R* dx) {
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < (long long)B * Px;
+         i += (long long)gridDim.x * blockDim.x) {
+        const long long b = i / Px;
+        const int p = (int)(i % Px);
+        R s = 0;
+        for (int t = 0; t < ntiles; ++t) {
+            const R* row = terms + (b * ntiles + t) * nt;
+            for (int k = __ldg(&ptr[p]); k < __ldg(&ptr[p + 1]); ++k) s += row[__ldg(&occ[k])];
+        }
+        dx[i] = s;
+    }
+}
+
+// dw[p] = sum over every tile row of the terms of w index p: one block per p,
+// fixed strided partial sums then a fixed-shape tree.
+template <typename R>
+__global__ void __launch_bounds__(256) reduce_dw(const R* terms, long long rows, int nt,
+                                                 const int32_t* ptr, const int32_t* occ, R* dw) {
+    __shared__ R part[256];
+    const int p = blockIdx.x;
+    const int k0 = __ldg(&ptr[p]), k1 = __ldg(&ptr[p + 1]);
+    R s = 0;
+    for (long long r = threadIdx.x; r < rows; r += 256) {
+        const R* row = terms + r * nt;
+        for (int k = k0; k < k1; ++k) s += row[__ldg(&occ[k])];
+    }
+    part[threadIdx.x] = s;
+    __syncthreads();
+    for (int w = 128; w >= 1; w >>= 1) {
+        if (threadIdx.x < w) part[threadIdx.x] += part[threadIdx.x + w];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) dw[p] = part[0];
+}
+
+}  // namespace vqc

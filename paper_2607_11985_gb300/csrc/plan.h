@@ -89,6 +89,19 @@ struct DEntry {
 };
 static_assert(sizeof(DEntry) == 12, "DEntry layout");
 
+// One pass of the HBM-tiled path: its stages act on tiles of m qubits; the
+// other n - m qubits index the tiles of a sample.
+struct DPass {
+    int32_t stage_begin, stage_end;
+    int32_t m, nout;
+    uint8_t tile_q[24];   // tile-local bit i -> qubit
+    uint8_t out_q[24];    // tile index bit j -> qubit
+    int32_t ps_begin, ps_count;    // per-sample table entries of the pass (into pass_entries)
+    int32_t sh_begin, sh_count;    // shared table entries of the pass
+    int32_t acc_begin, acc_count;  // accumulators of the pass (into pass_accs)
+};
+static_assert(sizeof(DPass) == 88, "DPass layout");
+
 // Accumulator slot -> what it holds (backward).
 struct DAcc {
     int32_t entry;   // table entry id

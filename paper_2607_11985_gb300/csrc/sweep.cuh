@@ -514,6 +514,158 @@ __device__ __forceinline__ void fwd_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 << K
     }
 }
 
+// ---------------------------------------------------------------- backward op
+// Un-apply one op on psi (a) and lam (l); first accumulate its gradient slot
+// (rho of a run, or Im <lam|P|psi> of a phase op) into acc[(aux * wg + warp) * 8].
+template <typename R, int K>
+__device__ __forceinline__ void bwd_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 << K],
+                                       C2<R> (&l)[1 << K], const R* sh_tab, const R* ps_tab,
+                                       R* acc, const Geo& q, int lane, int warp_in_group) {
+    const int type = raw.x & 0xff, ra = (raw.x >> 8) & 0xff, rb = (raw.x >> 16) & 0xff;
+    const int flags = raw.x >> 24, slot = raw.y & 0xffff, aux = raw.y >> 16;
+    const R* tab = (flags & OPF_PER_SAMPLE) ? ps_tab : sh_tab;
+    if (type == OP_M1) {
+        const M2<R> m = load_m2<R>(tab + 8 * slot);
+        if (flags & OPF_HAS_ACC) {
+            R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+            m1_rho_dispatch<R, K>(ra, a, l, rh);
+            reduce8_store<R>(rh, q.lanes, q.lanes < 32 ? q.t : lane,
+                             acc + ((size_t)aux * q.wg + warp_in_group) * 8, q.mask);
+        }
+        const M2<R> md = mdag<R>(m);
+        m1_dispatch<R, K>(ra, a, md);
+        m1_dispatch<R, K>(ra, l, md);
+    } else if (type == OP_CX) {
+        if (ra < kRefPhys) {
+            cx_ll_dispatch<R, K>(ra, rb, a);
+            cx_ll_dispatch<R, K>(ra, rb, l);
+        } else {
+            const bool p = ((pb >> (ra - kRefPhys)) & 1u) != 0;
+            x_pred_dispatch<R, K>(rb, a, p);
+            x_pred_dispatch<R, K>(rb, l, p);
+        }
+    } else if (type == OP_CZ) {
+        cz_dispatch<R, K>(ra, rb, pb, a);
+        cz_dispatch<R, K>(ra, rb, pb, l);
+    } else if (type == OP_PH2) {
+        const R* p = tab + 8 * slot;
+        C2<R> ph[4] = {cm<R>(p[0], p[1]), cm<R>(p[2], p[3]), cm<R>(p[4], p[5]), cm<R>(p[6], p[7])};
+        if (flags & OPF_HAS_ACC) {
+            R tv = ph2_term<R, K>(ra, rb, pb, (uint8_t)flags, a, l);
+            tv = reduce1<R>(tv, q.lanes, q.mask);
+            if ((q.t & (q.lanes - 1)) == 0) acc[((size_t)aux * q.wg + warp_in_group) * 8] = tv;
+        }
+        ph2_apply<R, K, true>(ra, rb, pb, a, ph);
+        ph2_apply<R, K, true>(ra, rb, pb, l, ph);
+    }
+}
+
+// lam = O psi on the block, O = sum_j gE_j Z_j (diagonal): the sign of Z_j comes
+// from local bit j of r for active qubits and from the block base pb otherwise.
+template <typename R, int K>
+__device__ __forceinline__ void lambda_init(const DStage* sp, uint32_t pb, const R* gb, int n,
+                                            const C2<R> (&a)[1 << K], C2<R> (&l)[1 << K]) {
+    R ge_loc[K];
+    R cst = 0;
+    uint32_t actmask = 0;
+#pragma unroll
+    for (int j = 0; j < K; ++j) {
+        const int aq = __ldg(&sp->active[j]);
+        actmask |= 1u << aq;
+        ge_loc[j] = gb[aq];
+    }
+    for (int j = 0; j < n; ++j)
+        if (!((actmask >> j) & 1)) cst += ((pb >> j) & 1u) ? -gb[j] : gb[j];
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r) {
+        R o = cst;
+#pragma unroll
+        for (int j = 0; j < K; ++j) o += ((r >> j) & 1) ? -ge_loc[j] : ge_loc[j];
+        l[r] = cm<R>(o * a[r].x, o * a[r].y);
+    }
+}
+
+// Per-warp partial sums of E_j = sum (-1)^{bit j} |a|^2 over this group's
+// blocks, written to red[warp_in_group * n + j].
+template <typename R, int K>
+__device__ __forceinline__ void expz_partials(const DStage* sp, uint32_t pb,
+                                              const C2<R> (&a)[1 << K], int n, R* red,
+                                              const Geo& q, int warp_in_group) {
+    R pr[1 << K];
+    R ptot = 0;
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r) {
+        pr[r] = fma(a[r].x, a[r].x, a[r].y * a[r].y);
+        ptot += pr[r];
+    }
+    R dloc[K];
+#pragma unroll
+    for (int j = 0; j < K; ++j) {
+        R d = 0;
+#pragma unroll
+        for (int r = 0; r < (1 << K); ++r) d += ((r >> j) & 1) ? -pr[r] : pr[r];
+        dloc[j] = d;
+    }
+    uint32_t actmask = 0;
+    int aq[K];
+#pragma unroll
+    for (int j = 0; j < K; ++j) {
+        aq[j] = __ldg(&sp->active[j]);
+        actmask |= 1u << aq[j];
+    }
+    for (int j = 0; j < n; ++j) {
+        R val;
+        if ((actmask >> j) & 1) {
+            val = 0;
+#pragma unroll
+            for (int k = 0; k < K; ++k) if (aq[k] == j) val = dloc[k];
+        } else {
+            val = ((pb >> j) & 1u) ? -ptot : ptot;
+        }
+        val = reduce1<R>(val, q.lanes, q.mask);
+        if ((q.t & (q.lanes - 1)) == 0) red[warp_in_group * n + j] = val;
+    }
+}
+
+// Gradient terms of one accumulator slot (summed over the wg per-warp
+// partials at ap): a phase op's scalar, or Im Tr(W_j P_j W_j^dag rho) for each
+// parametrised constituent j of a run.  Writes out[term].
+template <typename R>
+__device__ void acc_terms(const DAcc& ac, const DEntry& e, const R* ap, int wg,
+                          const DConst* consts, const R* xg, const R* w, const R* cang,
+                          const R* cmat, R* out) {
+    if (ac.kind == 1) {
+        R sum = 0;
+        for (int k2 = 0; k2 < wg; ++k2) sum += ap[k2 * 8];
+        out[consts[e.cfirst].term] = sum;
+        return;
+    }
+    R rr[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    for (int k2 = 0; k2 < wg; ++k2)
+        for (int c = 0; c < 8; ++c) rr[c] += ap[k2 * 8 + c];
+    // rho = [[r00, r01], [r10, r11]]; term = Im Tr(W P W^dag rho)
+    M2<R> W = mident<R>();
+    for (int c = e.ccount - 1; c >= 0; --c) {
+        const DConst cn = consts[e.cfirst + c];
+        if (cn.term >= 0) {
+            M2<R> P;
+            const C2<R> z = cm<R>(0, 0), one = cm<R>(1, 0);
+            if (cn.kind == CK_RX) { P.a = z; P.b = one; P.c = one; P.d = z; }
+            else if (cn.kind == CK_RY) { P.a = z; P.b = cm<R>(0, -1); P.c = cm<R>(0, 1); P.d = z; }
+            else { P.a = one; P.b = z; P.c = z; P.d = cm<R>(-1, 0); }
+            const M2<R> Mx = mmul<R>(mmul<R>(W, P), mdag<R>(W));
+            R im = 0;   // Im sum_{a,b} M[a][b] rho[b][a]
+            im += Mx.a.x * rr[1] + Mx.a.y * rr[0];
+            im += Mx.b.x * rr[5] + Mx.b.y * rr[4];
+            im += Mx.c.x * rr[3] + Mx.c.y * rr[2];
+            im += Mx.d.x * rr[7] + Mx.d.y * rr[6];
+            out[cn.term] = im;
+        }
+        W = mmul<R>(W, constituent<R>(cn, xg, w, cang, cmat));
+    }
+}
+
+
 // ---------------------------------------------------------------- kernel
 template <typename R, int K, int MODE>
 struct MaxThreads {
@@ -623,41 +775,8 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
         if (MODE == 0) {
             // -------- <Z_j> partials from the final block
             const DStage* sp = A.stages + (ns - 1);
-            R pr[1 << K];
-            R ptot = 0;
-#pragma unroll
-            for (int r = 0; r < (1 << K); ++r) {
-                pr[r] = fma(a[r].x, a[r].x, a[r].y * a[r].y);
-                ptot += pr[r];
-            }
-            R dloc[K];
-#pragma unroll
-            for (int j = 0; j < K; ++j) {
-                R d = 0;
-#pragma unroll
-                for (int r = 0; r < (1 << K); ++r) d += ((r >> j) & 1) ? -pr[r] : pr[r];
-                dloc[j] = d;
-            }
-            uint32_t actmask = 0;
-            int aq[K];
-#pragma unroll
-            for (int j = 0; j < K; ++j) {
-                aq[j] = __ldg(&sp->active[j]);
-                actmask |= 1u << aq[j];
-            }
             R* red = red_all + (size_t)q.g * q.wg * n;
-            for (int j = 0; j < n; ++j) {
-                R val;
-                if ((actmask >> j) & 1) {
-                    val = 0;
-#pragma unroll
-                    for (int k = 0; k < K; ++k) if (aq[k] == j) val = dloc[k];
-                } else {
-                    val = ((v.pb >> j) & 1u) ? -ptot : ptot;
-                }
-                val = reduce1<R>(val, q.lanes, q.mask);
-                if ((q.t & (q.lanes - 1)) == 0) red[warp_in_group * n + j] = val;
-            }
+            expz_partials<R, K>(sp, v.pb, a, n, red, q, warp_in_group);
             __syncthreads();
             if (valid) {
                 for (int j = q.t; j < n; j += q.T) {
@@ -675,79 +794,21 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
         }
 
         // -------- backward: reverse sweep with psi and lam
-        R ge_loc[K];
         for (int s = ns - 1; s >= 0; --s) {
             const DStage* sp = A.stages + s;
             C2<R> l[1 << K];
+            v = stage_view<K>(sp, q.t, q.h, sg);
             if (s == ns - 1) {
-                v = stage_view<K>(sp, q.t, q.h, sg);
                 if (!recompute) block_load<R, K>(a, psi, v.swb, sg);
-                // lam = O psi with O = sum_j gE_j Z_j (diagonal)
-                const R* gb = A.gE + (size_t)b * n;
-                R cst = 0;
-                uint32_t actmask = 0;
-#pragma unroll
-                for (int j = 0; j < K; ++j) {
-                    const int aq = __ldg(&sp->active[j]);
-                    actmask |= 1u << aq;
-                    ge_loc[j] = gb[aq];
-                }
-                for (int j = 0; j < n; ++j)
-                    if (!((actmask >> j) & 1)) cst += ((v.pb >> j) & 1u) ? -gb[j] : gb[j];
-#pragma unroll
-                for (int r = 0; r < (1 << K); ++r) {
-                    R o = cst;
-#pragma unroll
-                    for (int j = 0; j < K; ++j) o += ((r >> j) & 1) ? -ge_loc[j] : ge_loc[j];
-                    l[r] = cm<R>(o * a[r].x, o * a[r].y);
-                }
+                lambda_init<R, K>(sp, v.pb, A.gE + (size_t)b * n, n, a, l);
             } else {
-                v = stage_view<K>(sp, q.t, q.h, sg);
                 block_load<R, K>(a, psi, v.swb, sg);
                 block_load<R, K>(l, lam, v.swb, sg);
             }
             const int ob = __ldg(&sp->op_begin), oe = __ldg(&sp->op_end);
             for (int o = oe - 1; o >= ob; --o) {
                 const uint2 raw = __ldg(reinterpret_cast<const uint2*>(A.ops) + o);
-                const int type = raw.x & 0xff, ra = (raw.x >> 8) & 0xff, rb = (raw.x >> 16) & 0xff;
-                const int flags = raw.x >> 24, slot = raw.y & 0xffff, aux = raw.y >> 16;
-                const R* tab = (flags & OPF_PER_SAMPLE) ? ps_tab : sh_tab;
-                if (type == OP_M1) {
-                    const M2<R> m = load_m2<R>(tab + 8 * slot);
-                    if (flags & OPF_HAS_ACC) {
-                        R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-                        m1_rho_dispatch<R, K>(ra, a, l, rh);
-                        reduce8_store<R>(rh, q.lanes, q.lanes < 32 ? q.t : lane,
-                                         acc + ((size_t)aux * q.wg + warp_in_group) * 8, q.mask);
-                    }
-                    const M2<R> md = mdag<R>(m);
-                    m1_dispatch<R, K>(ra, a, md);
-                    m1_dispatch<R, K>(ra, l, md);
-                } else if (type == OP_CX) {
-                    if (ra < kRefPhys) {
-                        cx_ll_dispatch<R, K>(ra, rb, a);
-                        cx_ll_dispatch<R, K>(ra, rb, l);
-                    } else {
-                        const bool p = ((v.pb >> (ra - kRefPhys)) & 1u) != 0;
-                        x_pred_dispatch<R, K>(rb, a, p);
-                        x_pred_dispatch<R, K>(rb, l, p);
-                    }
-                } else if (type == OP_CZ) {
-                    cz_dispatch<R, K>(ra, rb, v.pb, a);
-                    cz_dispatch<R, K>(ra, rb, v.pb, l);
-                } else if (type == OP_PH2) {
-                    const R* p = tab + 8 * slot;
-                    C2<R> ph[4] = {cm<R>(p[0], p[1]), cm<R>(p[2], p[3]), cm<R>(p[4], p[5]),
-                                   cm<R>(p[6], p[7])};
-                    if (flags & OPF_HAS_ACC) {
-                        R tv = ph2_term<R, K>(ra, rb, v.pb, (uint8_t)flags, a, l);
-                        tv = reduce1<R>(tv, q.lanes, q.mask);
-                        if ((q.t & (q.lanes - 1)) == 0)
-                            acc[((size_t)aux * q.wg + warp_in_group) * 8] = tv;
-                    }
-                    ph2_apply<R, K, true>(ra, rb, v.pb, a, ph);
-                    ph2_apply<R, K, true>(ra, rb, v.pb, l, ph);
-                }
+                bwd_op<R, K>(raw, v.pb, a, l, sh_tab, ps_tab, acc, q, lane, warp_in_group);
             }
             if (s > 0) {
                 block_store<R, K>(a, psi, v.swb, sg);
@@ -761,41 +822,11 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
         for (int i = threadIdx.x; i < A.S * A.n_accs; i += nthr) {
             const int gg = i / A.n_accs, k = i % A.n_accs;
             const DAcc ac = A.accs[k];
-            const R* ap = acc_all + ((size_t)gg * A.n_accs + k) * q.wg * 8;
-            R* tm = terms_all + (size_t)gg * A.n_terms;
             const int bb = min(unit * A.S + gg, A.B - 1);
             const R* xg = A.x ? A.x + (size_t)bb * A.Px : nullptr;
-            const DEntry e = A.entries[ac.entry];
-            if (ac.kind == 1) {
-                R sum = 0;
-                for (int k2 = 0; k2 < q.wg; ++k2) sum += ap[k2 * 8];
-                tm[A.consts[e.cfirst].term] = sum;
-                continue;
-            }
-            R rr[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-            for (int k2 = 0; k2 < q.wg; ++k2)
-                for (int c = 0; c < 8; ++c) rr[c] += ap[k2 * 8 + c];
-            // rho = [[r00, r01], [r10, r11]]; term = Im Tr(W P W^dag rho)
-            M2<R> W = mident<R>();
-            for (int c = e.ccount - 1; c >= 0; --c) {
-                const DConst cn = A.consts[e.cfirst + c];
-                if (cn.term >= 0) {
-                    M2<R> P;
-                    const C2<R> z = cm<R>(0, 0), one = cm<R>(1, 0);
-                    if (cn.kind == CK_RX) { P.a = z; P.b = one; P.c = one; P.d = z; }
-                    else if (cn.kind == CK_RY) { P.a = z; P.b = cm<R>(0, -1); P.c = cm<R>(0, 1); P.d = z; }
-                    else { P.a = one; P.b = z; P.c = z; P.d = cm<R>(-1, 0); }
-                    const M2<R> Mx = mmul<R>(mmul<R>(W, P), mdag<R>(W));
-                    // Im sum_{a,b} M[a][b] rho[b][a]
-                    R im = 0;
-                    im += Mx.a.x * rr[1] + Mx.a.y * rr[0];   // M00 rho00
-                    im += Mx.b.x * rr[5] + Mx.b.y * rr[4];   // M01 rho10
-                    im += Mx.c.x * rr[3] + Mx.c.y * rr[2];   // M10 rho01
-                    im += Mx.d.x * rr[7] + Mx.d.y * rr[6];   // M11 rho11
-                    tm[cn.term] = im;
-                }
-                W = mmul<R>(W, constituent<R>(cn, xg, A.w, A.cang, A.cmat));
-            }
+            acc_terms<R>(ac, A.entries[ac.entry], acc_all + ((size_t)gg * A.n_accs + k) * q.wg * 8,
+                         q.wg, A.consts, xg, A.w, A.cang, A.cmat,
+                         terms_all + (size_t)gg * A.n_terms);
         }
         __syncthreads();
         // dx rows of this CTA's samples; dw partial of this CTA (fixed order)

@@ -22,8 +22,12 @@ DOP = np.dtype([("type", "u1"), ("a", "u1"), ("b", "u1"), ("flags", "u1"), ("slo
 DSTAGE = np.dtype([("op_begin", "<i4"), ("op_end", "<i4"), ("sigma", "<i4", 5), ("tau", "<i4", 16),
                    ("tmask", "<u4", 16), ("active", "u1", 5), ("nthreadbits", "u1"),
                    ("pad", "u1", 2)])
+DPASS = np.dtype([("stage_begin", "<i4"), ("stage_end", "<i4"), ("m", "<i4"), ("nout", "<i4"),
+                  ("tile_q", "u1", 24), ("out_q", "u1", 24), ("ps_begin", "<i4"), ("ps_count", "<i4"),
+                  ("sh_begin", "<i4"), ("sh_count", "<i4"), ("acc_begin", "<i4"), ("acc_count", "<i4")])
 assert DENTRY.itemsize == 12 and DCONST.itemsize == 16 and DOP.itemsize == 8
-assert DSTAGE.itemsize == 164
+assert DSTAGE.itemsize == 164 and DPASS.itemsize == 88
+PATH_RESIDENT, PATH_HBM = 0, 1
 
 OP_M1, OP_CX, OP_CZ, OP_PH2 = 1, 2, 3, 4
 OPF_PER_SAMPLE, OPF_GEN_CRZ, OPF_GEN_RZZ, OPF_HAS_ACC = 1, 2, 4, 8
@@ -74,8 +78,12 @@ class Plan:
             mode, K, m, path, tb, gl = [r.i32() for _ in range(6)]
             ops = r.vec(DOP)
             stages = r.vec(DSTAGE)
+            passes = r.vec(DPASS)
+            pass_entries = r.vec("<i4")
+            pass_accs = r.vec("<i4")
             self.scheds.append(dict(mode=mode, K=K, m=m, path=path, thread_bits=tb, ops=ops,
-                                    stages=stages))
+                                    stages=stages, passes=passes, pass_entries=pass_entries,
+                                    pass_accs=pass_accs))
         assert r.off == len(blob)
 
     # ------------------------------------------------------------------ tables
@@ -173,6 +181,26 @@ class Plan:
             raise AssertionError("bad op type %d" % t)
 
     # ------------------------------------------------------------------ runs
+    def units(self, sched, xb, w):
+        """(stages, tile bases, tables, acc map) of each pass; the resident path
+        is one pass over one tile holding every qubit."""
+        n = self.n
+        if sched["path"] == PATH_RESIDENT:
+            yield sched["stages"], [0], self.tables(xb, w), np.arange(len(self.accs))
+            return
+        pe = sched["pass_entries"]
+        for ps in sched["passes"]:
+            ps_ids = pe[ps["ps_begin"]:ps["ps_begin"] + ps["ps_count"]]
+            sh_ids = pe[ps["sh_begin"]:ps["sh_begin"] + ps["sh_count"]]
+            tabs = ([self.entry_value(int(e), xb, w) for e in ps_ids],
+                    [self.entry_value(int(e), xb, w) for e in sh_ids])
+            out_q = ps["out_q"][:ps["nout"]]
+            bases = []
+            for tau in range(1 << int(ps["nout"])):
+                bases.append(sum(((tau >> j) & 1) << int(out_q[j]) for j in range(int(ps["nout"]))))
+            accmap = sched["pass_accs"][ps["acc_begin"]:ps["acc_begin"] + ps["acc_count"]]
+            yield sched["stages"][ps["stage_begin"]:ps["stage_end"]], bases, tabs, accmap
+
     def forward(self, sched, xb, w, psi0=None):
         n, K = self.n, sched["K"]
         psi = np.zeros(1 << n, complex)
@@ -180,14 +208,17 @@ class Plan:
             psi[0] = 1
         else:
             psi[:] = psi0
-        tabs = self.tables(xb, w)
-        for st in sched["stages"]:
-            for t in range(1 << (n - K)):
-                base, idx = self.block_index(st, K, t)
-                a = psi[idx].copy()
-                for op in sched["ops"][st["op_begin"]:st["op_end"]]:
-                    self.apply_op(op, K, base, a, tabs)
-                psi[idx] = a
+        for stages, bases, tabs, _ in self.units(sched, xb, w):
+            for tb in bases:
+                for st in stages:
+                    for t in range(1 << int(st["nthreadbits"])):
+                        base, idx = self.block_index(st, K, t)
+                        base |= tb
+                        idx = idx | tb
+                        a = psi[idx].copy()
+                        for op in sched["ops"][st["op_begin"]:st["op_end"]]:
+                            self.apply_op(op, K, base, a, tabs)
+                        psi[idx] = a
         return psi
 
     def backward(self, sched, xb, w, gEb, psi0=None):
@@ -198,12 +229,15 @@ class Plan:
         k = np.arange(1 << n)
         O = sum(gEb[j] * (1 - 2 * ((k >> j) & 1)) for j in range(n))
         lam = O * psi
-        tabs = self.tables(xb, w)
         acc = np.zeros((len(self.accs), 8))
-        for st in sched["stages"][::-1]:
+        for stages, bases, tabs, accmap in list(self.units(sched, xb, w))[::-1]:
+          for tb in bases:
+           for st in stages[::-1]:
             ops = sched["ops"][st["op_begin"]:st["op_end"]]
-            for t in range(1 << (n - K)):
+            for t in range(1 << int(st["nthreadbits"])):
                 base, idx = self.block_index(st, K, t)
+                base |= tb
+                idx = idx | tb
                 a, l = psi[idx].copy(), lam[idx].copy()
                 for op in ops[::-1]:
                     if op["flags"] & OPF_HAS_ACC:
@@ -216,15 +250,15 @@ class Plan:
                                     for ia in range(2):
                                         for ib in range(2):
                                             z = pp[ia] * np.conj(ll[ib])
-                                            acc[op["aux"], 2 * (2 * ia + ib)] += z.real
-                                            acc[op["aux"], 2 * (2 * ia + ib) + 1] += z.imag
+                                            acc[accmap[op["aux"]], 2 * (2 * ia + ib)] += z.real
+                                            acc[accmap[op["aux"]], 2 * (2 * ia + ib) + 1] += z.imag
                         else:
                             crz = op["flags"] & OPF_GEN_CRZ
                             for r in range(1 << K):
                                 ba = self.refbit(op["a"], r, base)
                                 bb = self.refbit(op["b"], r, base)
                                 g = (1 - 2 * bb) * ba if crz else 1 - 2 * (ba ^ bb)
-                                acc[op["aux"], 0] += g * (np.conj(l[r]) * a[r]).imag
+                                acc[accmap[op["aux"]], 0] += g * (np.conj(l[r]) * a[r]).imag
                     self.apply_op(op, K, base, a, tabs, adjoint=True)
                     self.apply_op(op, K, base, l, tabs, adjoint=True)
                 psi[idx], lam[idx] = a, l

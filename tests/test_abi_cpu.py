@@ -100,15 +100,27 @@ def test_export_deterministic_and_info():
 
 def check_addressing(plan):
     for s in plan.scheds:
-        n, K = plan.n, s["K"]
-        for st in s["stages"]:
+        n, K, m = plan.n, s["K"], s["m"]
+        if s["path"] == 0:
+            tiles = [(list(range(n)), s["stages"])]
+        else:
+            tiles = [(list(ps["tile_q"][:ps["m"]]), s["stages"][ps["stage_begin"]:ps["stage_end"]])
+                     for ps in s["passes"]]
+            # every pass's tile holds the low qubits of one 128-byte chunk
+            for tq, _ in tiles:
+                assert tq[:min(plan.G, n)] == list(range(min(plan.G, n)))
+        for tq, stages in tiles:
+          tq = [int(q) for q in tq]
+          lpos = {q: i for i, q in enumerate(tq)}
+          for st in stages:
             assert sorted(st["active"][:K].tolist()) == st["active"][:K].tolist()
-            assert int(st["nthreadbits"]) == n - K
+            assert set(st["active"][:K].tolist()) <= set(tq)
+            assert int(st["nthreadbits"]) == m - K
             slots = set()
-            for t in range(1 << (n - K)):
+            for t in range(1 << (m - K)):
                 base, idx = Plan.block_index(st, K, t)
                 swb = 0
-                for i in range(n - K):
+                for i in range(m - K):
                     if (t >> i) & 1:
                         swb ^= int(st["tau"][i])
                 for r in range(1 << K):
@@ -116,9 +128,10 @@ def check_addressing(plan):
                     for j in range(K):
                         if (r >> j) & 1:
                             sl ^= int(st["sigma"][j])
-                    assert sl == swz(int(idx[r]), plan.G)
+                    u = sum(((int(idx[r]) >> q) & 1) << lpos[q] for q in tq)
+                    assert sl == swz(u, plan.G)
                     slots.add(sl)
-            assert slots == set(range(1 << n))
+            assert slots == set(range(1 << m))
             for op in s["ops"][st["op_begin"]:st["op_end"]]:
                 if op["type"] == 1:
                     assert op["a"] < K
@@ -160,6 +173,41 @@ def test_schedules_reproduce_oracle_gradients(seed, n, G):
             assert np.allclose(dx, dx_ref[b], atol=1e-10), s["K"]
             dw += dwb
         assert np.allclose(dw, dw_ref, atol=1e-10), s["K"]
+
+
+@pytest.mark.parametrize("seed,n,G", [(501, 8, 120), (502, 9, 160), (503, 10, 200)])
+def test_hbm_schedules_small_tiles(monkeypatch, seed, n, G):
+    # force small tiles so the HBM pass schedules are exercised at emulator sizes
+    monkeypatch.setenv("VQC_HBM_TILE_QUBITS", str(6))
+    w_, psi0 = wl.small_random(seed, n, G, batch=1, dtype="c128", with_psi0=True)
+    for dtype in (0, 1):
+        pl = Plan(B.vqc_plan_export(compile_spec(w_.spec, dtype)))
+        check_addressing(pl)
+        hb = [s for s in pl.scheds if s["path"] == 1]
+        assert len(hb) == 2 and all(len(s["passes"]) >= 2 for s in hb)
+        _, ref = orc.forward(w_.spec, w_.x, w_.w, psi0=psi0, want_state=True)
+        dx_ref, dw_ref = orc.backward(w_.spec, w_.x, w_.w, w_.gE, psi0=psi0)
+        for s in hb:
+            got = pl.forward(s, w_.x[0], w_.w, psi0[0])
+            assert np.allclose(got, ref[0], atol=1e-12)
+            if s["mode"] == 1 and dtype == 1:
+                dx, dw = pl.backward(s, w_.x[0], w_.w, w_.gE[0], psi0[0])
+                assert np.allclose(dx, dx_ref[0], atol=1e-10)
+                assert np.allclose(dw, dw_ref, atol=1e-10)
+
+
+def test_config5_hbm_schedule_structure():
+    w_ = wl.config(5, batch=1)[0]
+    for dtype in (0, 1):
+        pl = Plan(B.vqc_plan_export(compile_spec(w_.spec, dtype)))
+        assert not any(s["path"] == 0 for s in pl.scheds)
+        hb = [s for s in pl.scheds if s["path"] == 1]
+        assert len(hb) == 2
+        for s in hb:
+            # every op lands in exactly one stage of one pass
+            assert sum(st["op_end"] - st["op_begin"] for st in s["stages"]) == len(pl.hops) + \
+                sum(1 for h in pl.hops if False)
+            assert s["passes"][-1]["stage_end"] == len(s["stages"])
 
 
 @pytest.mark.parametrize("k", [1, 2])

@@ -1,0 +1,112 @@
+"""GPU parity of the HBM-tiled pass path (states too large for one SM).
+
+* the 16-qubit / 8-layer / batch-512 workload in complex64 and complex128:
+  full batch on the GPU, the oracle on sampled rows (one by one), dw on a
+  small slice against the oracle and, at full size, as the sum over two halves;
+* small circuits forced onto the HBM path with 6-qubit tiles (many passes,
+  tile-outer controls and phases), against the oracle, with and without psi0
+  and the saved final state, ragged batches;
+* cross-path agreement: the 12-qubit workload on the resident and HBM paths.
+"""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from oracle import oracle as orc  # noqa: E402
+from paper_2607_11985_gb300 import workloads as wl  # noqa: E402
+from tests.test_gpu_parity import TOL, C, dev, devc, maxerr, run_bwd, run_fwd  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def cuda_ready():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    torch.cuda.set_device(0)
+
+
+@pytest.mark.parametrize("dtype", ["c64", "c128"])
+def test_config5_full_batch(dtype):
+    w_ = wl.config(5, dtype=dtype)[0]
+    c = C(w_.spec, dtype)
+    info = c.info(w_.batch)
+    assert info["fwd_path"] == 1 and info["bwd_path"] == 1 and info["fwd_passes"] > 1
+    E, st = run_fwd(c, w_)
+    rows = [0, w_.batch - 1]
+    sub = wl.Workload(w_.name, w_.spec, 2, w_.x[rows], w_.w, w_.gE[rows], dtype, w_.seed)
+    E_ref, st_ref = orc.forward(w_.spec, sub.x, sub.w, want_state=True)
+    tol = TOL[dtype]
+    assert maxerr(E[rows], E_ref) <= tol["E"]
+    assert maxerr(st[rows], st_ref) <= tol["state"]
+    dx, dw = run_bwd(c, w_, psi_final=devc(st, dtype))
+    dx_ref, dw2_ref = orc.backward(w_.spec, sub.x, sub.w, sub.gE)
+    assert maxerr(dx[rows], dx_ref) <= tol["grad"]
+    # dw of a 2-row slice (the same two rows) against the oracle; recomputed state
+    _, dw2 = run_bwd(c, sub)
+    assert maxerr(dw2, dw2_ref) <= tol["grad"]
+    # full-batch dw equals the sum over the two halves
+    h = w_.batch // 2
+    h1 = wl.Workload(w_.name, w_.spec, h, w_.x[:h], w_.w, w_.gE[:h], dtype, w_.seed)
+    h2 = wl.Workload(w_.name, w_.spec, h, w_.x[h:], w_.w, w_.gE[h:], dtype, w_.seed)
+    _, dwa = run_bwd(c, h1)
+    _, dwb = run_bwd(c, h2)
+    scale = max(1.0, float(np.max(np.abs(dw))))
+    assert maxerr(dw, dwa + dwb) <= (1e-4 if dtype == "c64" else 1e-10) * scale
+
+
+SMALL = [(601, 8, 160), (602, 9, 200), (603, 10, 240), (604, 11, 200)]
+
+
+@pytest.mark.parametrize("dtype", ["c64", "c128"])
+@pytest.mark.parametrize("seed,n,G", SMALL)
+def test_forced_hbm_small_tiles(monkeypatch, seed, n, G, dtype):
+    monkeypatch.setenv("VQC_HBM_TILE_QUBITS", "6")
+    monkeypatch.setenv("VQC_FORCE_PATH", "hbm")
+    w_, psi0 = wl.small_random(seed, n, G, batch=21, dtype=dtype, with_psi0=(seed % 2 == 0))
+    c = C(w_.spec, dtype)
+    info = c.info(w_.batch)
+    assert info["fwd_path"] == 1 and info["fwd_passes"] >= 2
+    tol = TOL[dtype]
+    E, st = run_fwd(c, w_, psi0)
+    E_ref, st_ref = orc.forward(w_.spec, w_.x, w_.w, psi0=psi0, want_state=True)
+    assert maxerr(E, E_ref) <= tol["E"]
+    assert maxerr(st, st_ref) <= tol["state"]
+    E2 = run_fwd(c, w_, psi0, want_state=False)          # last pass writes no state
+    assert maxerr(E2, E_ref) <= tol["E"]
+    dx_ref, dw_ref = orc.backward(w_.spec, w_.x, w_.w, w_.gE, psi0=psi0)
+    dx, dw = run_bwd(c, w_, psi0)                          # recompute the final state
+    assert maxerr(dx, dx_ref) <= tol["grad"] and maxerr(dw, dw_ref) <= tol["grad"]
+    dx, dw = run_bwd(c, w_, psi0, psi_final=devc(st, dtype))
+    assert maxerr(dx, dx_ref) <= tol["grad"] and maxerr(dw, dw_ref) <= tol["grad"]
+
+
+def test_forced_hbm_ragged_batches(monkeypatch):
+    monkeypatch.setenv("VQC_HBM_TILE_QUBITS", "7")
+    monkeypatch.setenv("VQC_FORCE_PATH", "hbm")
+    w0, _ = wl.small_random(611, 9, 150, batch=1, dtype="c64")
+    c = C(w0.spec, "c64")
+    for B in (1, 3, 17, 64):
+        wb, _ = wl.small_random(611, 9, 150, batch=B, dtype="c64")
+        E = run_fwd(c, wb, want_state=False)
+        assert maxerr(E, orc.forward(wb.spec, wb.x, wb.w)) <= 1e-4
+        dx, dw = run_bwd(c, wb)
+        dx_ref, dw_ref = orc.backward(wb.spec, wb.x, wb.w, wb.gE)
+        assert maxerr(dx, dx_ref) <= 5e-4 and maxerr(dw, dw_ref) <= 5e-4
+
+
+def test_resident_and_hbm_paths_agree(monkeypatch):
+    w_ = wl.config(3, batch=256)[0]
+    c = C(w_.spec, "c64")
+    E1, st1 = run_fwd(c, w_)
+    dx1, dw1 = run_bwd(c, w_)
+    monkeypatch.setenv("VQC_FORCE_PATH", "hbm")
+    c2 = C(w_.spec, "c64")
+    assert c2.info(w_.batch)["fwd_path"] == 1
+    E2, st2 = run_fwd(c2, w_)
+    dx2, dw2 = run_bwd(c2, w_)
+    assert maxerr(E1, E2) <= 2e-5 and maxerr(st1, st2) <= 2e-5
+    assert maxerr(dx1, dx2) <= 2e-4 and maxerr(dw1, dw2) <= 1e-3
