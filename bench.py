@@ -152,11 +152,13 @@ def run_ours(args, rank, world, local_rank):
     dx = torch.empty_like(x)
     dw = torch.empty_like(w)
     ws, wsb = c.workspace(Bt, 1, stream)
+    wsf, wsfb = c.workspace(Bt, 0, stream)
+    wsf_ptr = wsf.data_ptr() if wsf is not None else None
     flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")   # > 129 MB L2
 
     def step():
         B.vqc_forward(c.plan, Bt, x.data_ptr(), w.data_ptr(), None, E.data_ptr(), st.data_ptr(),
-                      None, 0, sp)
+                      wsf_ptr, wsfb, sp)
         B.vqc_backward(c.plan, Bt, x.data_ptr(), w.data_ptr(), None, st.data_ptr(), gE.data_ptr(),
                        dx.data_ptr(), dw.data_ptr(), ws.data_ptr(), wsb, sp)
 
@@ -184,7 +186,7 @@ def run_ours(args, rank, world, local_rank):
         e0, e1, e2 = ev[i]
         e0.record(stream)
         B.vqc_forward(c.plan, Bt, x.data_ptr(), w.data_ptr(), None, E.data_ptr(), st.data_ptr(),
-                      None, 0, sp)
+                      wsf_ptr, wsfb, sp)
         e1.record(stream)
         B.vqc_backward(c.plan, Bt, x.data_ptr(), w.data_ptr(), None, st.data_ptr(), gE.data_ptr(),
                        dx.data_ptr(), dw.data_ptr(), ws.data_ptr(), wsb, sp)
@@ -249,13 +251,22 @@ def run_ours(args, rank, world, local_rank):
         return None
 
     pk, pk_kind = peaks()
-    peak = fp32_peak_tflops(pk.get("sm_max_mhz", SM_MAX_MHZ))
+    hbm_path = info["bwd_path"] == 1
     bwd_avg_s = statistics.mean(bwd_ms) / 1e3
     fwd_avg_s = statistics.mean(fwd_ms) / 1e3
-    bwd_flops = info["bwd_flops_per_eval"] * Bt
-    fwd_flops = info["fwd_flops_per_eval"] * Bt
-    ach_bwd = bwd_flops / bwd_avg_s / 1e12
-    ach_fwd = fwd_flops / fwd_avg_s / 1e12
+    if hbm_path:
+        # state bytes the passes move through HBM (vqc_plan_info), against copy bandwidth
+        peak = pk.get("hbm_gbs", 6800.0)
+        bwd_flops = info["bwd_hbm_bytes_per_eval"] * Bt
+        fwd_flops = info["fwd_hbm_bytes_per_eval"] * Bt
+        ach_bwd = bwd_flops / bwd_avg_s / 1e9
+        ach_fwd = fwd_flops / fwd_avg_s / 1e9
+    else:
+        peak = fp32_peak_tflops(pk.get("sm_max_mhz", SM_MAX_MHZ))
+        bwd_flops = info["bwd_flops_per_eval"] * Bt
+        fwd_flops = info["fwd_flops_per_eval"] * Bt
+        ach_bwd = bwd_flops / bwd_avg_s / 1e12
+        ach_fwd = fwd_flops / fwd_avg_s / 1e12
     traffic = None
     tpath = os.path.join(ROOT, "profiles", "traffic.txt")
     if os.path.exists(tpath):
@@ -278,21 +289,26 @@ def run_ours(args, rank, world, local_rank):
         "vs_baseline": None,
         "dtype": "c64 (fp32 arithmetic)",
         "data": "synthetic (seeded; RY(x) encoding + RX/RY/RZ layers + CZ ring)",
-        "config": {"workload": w_.name.split("_rank")[0], "qubits": w_.spec.n, "layers": 4,
+        "config": {"workload": w_.name.split("_rank")[0], "qubits": w_.spec.n,
                    "batch_per_gpu": Bt,
                    "gates": len(w_.spec.gates), "num_x": w_.spec.num_x, "num_w": w_.spec.num_w,
                    "parallelism": "dp%d (batch-sharded replicas, dw all-reduce)" % world,
                    "l2": "flushed between steps (256 MiB write) outside the per-step CUDA events",
                    "fwd_k": info["fwd_k"], "bwd_k": info["bwd_k"],
+                   "path": "hbm-tiled" if hbm_path else "resident",
                    "fwd_stages": info["fwd_stages"], "bwd_stages": info["bwd_stages"]},
         "fwd": {"value": world * Bt / fwd_avg_s, "unit": "circuit evals/s (fwd)",
-                "ms": fwd_avg_s * 1e3, "tflops": ach_fwd},
-        "roofline": {"kernel": "sweep_kernel<float,K=%d,bwd>" % info["bwd_k"], "bound": "alu",
-                     "achieved": ach_bwd, "peak": peak, "unit": "TFLOP/s",
+                "ms": fwd_avg_s * 1e3, "achieved": ach_fwd},
+        "roofline": {"kernel": ("pass_kernel<float,K=%d,bwd> x %d passes" % (info["bwd_k"], info["bwd_passes"]))
+                     if hbm_path else "sweep_kernel<float,K=%d,bwd>" % info["bwd_k"],
+                     "bound": "hbm" if hbm_path else "alu",
+                     "achieved": ach_bwd, "peak": peak, "unit": "GB/s" if hbm_path else "TFLOP/s",
                      "frac": ach_bwd / peak, "traffic": traffic,
-                     "peak_basis": "FP32 FFMA: 152 SMs x 128 lanes x 2 x %.0f MHz (%s sm_max_mhz)"
-                                   % (pk.get("sm_max_mhz", SM_MAX_MHZ), pk_kind),
-                     "flops_per_launch": bwd_flops, "launch_ms": bwd_avg_s * 1e3,
+                     "peak_basis": ("copy bandwidth, %s hbm_gbs" % pk_kind) if hbm_path else
+                     ("FP32 FFMA: 152 SMs x 128 lanes x 2 x %.0f MHz (%s sm_max_mhz)"
+                      % (pk.get("sm_max_mhz", SM_MAX_MHZ), pk_kind)),
+                     ("bytes_per_call" if hbm_path else "flops_per_launch"): bwd_flops,
+                     "launch_ms": bwd_avg_s * 1e3,
                      "fwd_frac": ach_fwd / peak},
         "e2e": {"value": e2e_value, "unit": "circuit evals/s (fwd+adjoint bwd, host buffers)",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": Ke},

@@ -74,10 +74,11 @@ size_t align256(size_t v) { return (v + 255) & ~size_t(255); }
 // Launch geometry of one call.
 struct Launch {
     const Schedule* s = nullptr;
-    int K = 0, T = 0, S = 0, block = 0, grid = 0, nunits = 0, wg = 1;
+    int K = 0, T = 0, S = 0, block = 0, grid = 0, nunits = 0, wg = 1, bpt = 1;
     size_t smem = 0;
     int sm_sh = 0, sm_ps = 0, sm_psi = 0, sm_lam = 0, sm_acc = 0, sm_terms = 0, sm_dw = 0,
-        sm_red = 0;
+        sm_red = 0, sm_plan = 0;
+    bool plan_smem = false;
     const void* fn = nullptr;
 };
 
@@ -117,7 +118,10 @@ vqc_status plan_launch(const HostPlan& p, int mode, int B, Launch& L) {
                                              std::to_string(p.n) + ")");
     const bool dbl = p.dtype == VQC_C128;
     const size_t rs = dbl ? 8 : 4, cs = 2 * rs;
-    L.T = 1 << (p.n - L.K);
+    // A sample needs 2^(n-K) register blocks; a group of at most 256 threads
+    // holds them, bpt blocks per thread.
+    L.T = std::min(1 << (p.n - L.K), sweep_max_threads(dbl, mode, L.K));
+    L.bpt = (1 << (p.n - L.K)) / L.T;
     L.wg = L.T > 32 ? L.T / 32 : 1;
     // Shared memory: a fixed part per CTA and a part per resident sample.
     const size_t dim = (size_t)1 << p.n;
@@ -157,6 +161,11 @@ vqc_status plan_launch(const HostPlan& p, int mode, int B, Launch& L) {
     L.sm_terms = take(mode == 1 ? (size_t)L.S * p.term_src.size() * rs : 0);
     L.sm_dw = take(mode == 1 ? (size_t)p.num_w * rs : 0);
     L.sm_red = take(mode == 0 ? (size_t)L.S * L.wg * p.n * rs : 0);
+    // the plan's table data and this schedule go to shared memory when they fit
+    const size_t plan_bytes = align16(p.dev_tab_end - p.dev_tab_begin) +
+                              (L.s->dev_region_end - L.s->dev_region_begin);
+    L.plan_smem = off + plan_bytes <= (size_t)di.smem_optin && env_int("VQC_PLAN_IN_SMEM", 1) != 0;
+    L.sm_plan = L.plan_smem ? take(plan_bytes) : 0;
     L.smem = off;
     if (L.smem > (size_t)di.smem_optin)
         return fail(VQC_ERR_UNSUPPORTED, "shared-memory layout exceeds the per-CTA limit");
@@ -194,6 +203,8 @@ void fill_plan_args(const HostPlan& p, const Launch& L, KArgs<R>& a) {
     a.tbits = p.n - L.K;
     a.G = p.G_swz;
     a.S = L.S;
+    a.tpg = L.T;
+    a.bpt = L.bpt;
     a.n_ps = p.n_ps;
     a.n_sh = p.n_sh;
     a.n_accs = (int)p.accs.size();
@@ -202,6 +213,13 @@ void fill_plan_args(const HostPlan& p, const Launch& L, KArgs<R>& a) {
     a.Pw = p.num_w;
     a.sm_sh = L.sm_sh; a.sm_ps = L.sm_ps; a.sm_psi = L.sm_psi; a.sm_lam = L.sm_lam;
     a.sm_acc = L.sm_acc; a.sm_terms = L.sm_terms; a.sm_dw = L.sm_dw; a.sm_red = L.sm_red;
+    a.plan = static_cast<const unsigned char*>(p.dbuf);
+    a.tab_off = (int)p.dev_tab_begin;
+    a.tab_bytes = (int)(p.dev_tab_end - p.dev_tab_begin);
+    a.sched_off = (int)L.s->dev_region_begin;
+    a.sched_bytes = (int)(L.s->dev_region_end - L.s->dev_region_begin);
+    a.sm_plan = L.sm_plan;
+    a.plan_smem = L.plan_smem ? 1 : 0;
 }
 
 // Device buffer layout of a plan (all sections 16-byte aligned).
@@ -231,12 +249,16 @@ vqc_status upload(HostPlan& p) {
     p.dev_xocc = put(p.xocc.data(), p.xocc.size() * 4);
     p.dev_wocc_ptr = put(p.wocc_ptr.data(), p.wocc_ptr.size() * 4);
     p.dev_wocc = put(p.wocc.data(), p.wocc.size() * 4);
+    p.dev_tab_begin = p.dev_entries;
+    p.dev_tab_end = blob.size();
     for (auto& s : p.scheds) {
+        s.dev_region_begin = blob.size();
         s.dev_ops = put(s.ops.data(), s.ops.size() * sizeof(DOp));
         s.dev_stages = put(s.stages.data(), s.stages.size() * sizeof(DStage));
         s.dev_passes = put(s.passes.data(), s.passes.size() * sizeof(DPass));
         s.dev_pass_entries = put(s.pass_entries.data(), s.pass_entries.size() * 4);
         s.dev_pass_accs = put(s.pass_accs.data(), s.pass_accs.size() * 4);
+        s.dev_region_end = blob.size();
     }
     size_t err_off = put(nullptr, 16);
     blob.resize(align256(blob.size()), 0);
@@ -310,7 +332,9 @@ struct PassGeo {
     int K = 0, T = 0, S = 0, block = 0, grid = 0, wg = 1, ntiles = 1;
     long long nunits = 0;
     size_t smem = 0;
-    int sm_sh = 0, sm_ps = 0, sm_psi = 0, sm_lam = 0, sm_acc = 0, sm_red = 0;
+    int sm_sh = 0, sm_ps = 0, sm_psi = 0, sm_lam = 0, sm_acc = 0, sm_red = 0, sm_plan = 0,
+        sm_koff = 0;
+    bool plan_smem = false;
     const void* fn = nullptr;
 };
 
@@ -336,7 +360,7 @@ vqc_status plan_hbm(const HostPlan& p, int mode, int B, PassGeo& L) {
         acc_max = std::max(acc_max, ps.acc_count);
     }
     const size_t tdim = (size_t)1 << m;
-    const size_t fixed = align16((size_t)sh_max * 8 * rs) + 8 * 16;
+    const size_t fixed = align16((size_t)sh_max * 8 * rs) + 8 * 16 + 1024;   // + tile-copy offsets
     const size_t per_tile = (size_t)ps_max * 8 * rs + tdim * cs * (mode == 1 ? 2 : 1) +
                             (mode == 1 ? (size_t)acc_max * L.wg * 8 * rs : (size_t)L.wg * p.n * rs);
     int S = std::max(1, 128 / L.T);
@@ -361,6 +385,14 @@ vqc_status plan_hbm(const HostPlan& p, int mode, int B, PassGeo& L) {
     L.sm_lam = take(mode == 1 ? (size_t)S * tdim * cs : 0);
     L.sm_acc = take(mode == 1 ? (size_t)S * acc_max * L.wg * 8 * rs : 0);
     L.sm_red = take(mode == 0 ? (size_t)S * L.wg * p.n * rs : 0);
+    {   // tile-copy offsets: one uint2 per vector round of a tile
+        const size_t apv = 16 / cs, nvec = tdim / apv;
+        L.sm_koff = take(((nvec + L.T - 1) / L.T) * 8);
+    }
+    const size_t plan_bytes = align16(p.dev_tab_end - p.dev_tab_begin) +
+                              (L.s->dev_region_end - L.s->dev_region_begin);
+    L.plan_smem = off + plan_bytes <= (size_t)di.smem_optin && plan_bytes <= 48 * 1024;
+    L.sm_plan = L.plan_smem ? take(plan_bytes) : 0;
     L.smem = off;
     L.fn = pass_ptr(dbl, mode, L.K);
     if (!L.fn) return fail(VQC_ERR_UNSUPPORTED, "pass kernel not instantiated for this K");
@@ -431,7 +463,14 @@ void fill_pass_args(const HostPlan& p, const PassGeo& L, const DPass& ps, PArgs<
         a.out_q[i] = ps.out_q[i];
     }
     a.sm_sh = L.sm_sh; a.sm_ps = L.sm_ps; a.sm_psi = L.sm_psi; a.sm_lam = L.sm_lam;
-    a.sm_acc = L.sm_acc; a.sm_red = L.sm_red;
+    a.sm_acc = L.sm_acc; a.sm_red = L.sm_red; a.sm_koff = L.sm_koff;
+    a.plan = static_cast<const unsigned char*>(p.dbuf);
+    a.tab_off = (int)p.dev_tab_begin;
+    a.tab_bytes = (int)(p.dev_tab_end - p.dev_tab_begin);
+    a.sched_off = (int)L.s->dev_region_begin;
+    a.sched_bytes = (int)(L.s->dev_region_end - L.s->dev_region_begin);
+    a.sm_plan = L.sm_plan;
+    a.plan_smem = L.plan_smem ? 1 : 0;
 }
 
 template <typename R>

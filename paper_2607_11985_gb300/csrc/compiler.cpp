@@ -383,7 +383,6 @@ void cut_stages(const HostPlan& p, const std::vector<int>& ops, const std::vecto
         for (int oi : taken) {
             const HOp& o = p.ops[oi];
             DOp d{};
-            d.type = o.type;
             if (o.type == OP_M1 || o.type == OP_PH2) {
                 const DEntry& e = p.entries[o.entry];
                 d.slot = (uint16_t)slot_of[o.entry];
@@ -393,12 +392,31 @@ void cut_stages(const HostPlan& p, const std::vector<int>& ops, const std::vecto
             }
             if (o.type == OP_M1) {
                 d.a = (uint8_t)local(o.q0);
+                d.code = (uint8_t)(DC_M1 + d.a);
             } else if (o.type == OP_CX) {
                 d.a = ref(o.q0);
                 d.b = (uint8_t)local(o.q1);
+                if (d.a < kRefPhys)
+                    d.code = (uint8_t)(DC_CX_LL + 4 * d.a + (d.b < d.a ? d.b : d.b - 1));
+                else
+                    d.code = (uint8_t)(DC_CX_PL + d.b);
+            } else if (o.type == OP_CZ) {
+                uint8_t ra = ref(o.q0), rb = ref(o.q1);
+                if (ra >= kRefPhys && rb >= kRefPhys) {
+                    d.code = DC_CZ_PP;
+                } else if (ra >= kRefPhys || rb >= kRefPhys) {
+                    if (ra >= kRefPhys) std::swap(ra, rb);   // local qubit first
+                    d.code = (uint8_t)(DC_CZ_PL + ra);
+                } else {
+                    if (ra > rb) std::swap(ra, rb);
+                    d.code = (uint8_t)(DC_CZ_LL + cz_pair_index(ra, rb));
+                }
+                d.a = ra;
+                d.b = rb;
             } else {
                 d.a = ref(o.q0);
                 d.b = ref(o.q1);
+                d.code = DC_PH2;
             }
             s.ops.push_back(d);
         }
@@ -574,8 +592,7 @@ vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx,
     // Stage schedules for every usable (mode, K) on the resident path.
     for (int mode = 0; mode < 2; ++mode) {
         for (int K = 1; K <= std::min(max_k(mode, dtype), n); ++K) {
-            const int max_tb = (dtype == VQC_C64 && mode == 0 && K <= 4) ? 10 : 9;
-            if (n - K > max_tb) continue;   // thread group must fit one CTA
+            if (n - K > 10) continue;   // at most 1024 register blocks per sample
             if (n > resident_max_qubits(mode, dtype)) continue;
             Schedule s;
             s.mode = mode;
@@ -592,7 +609,7 @@ vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx,
         if (n < p.G_swz + 2 || K < 1 || m <= p.G_swz) continue;
         const int env_m = std::getenv("VQC_HBM_TILE_QUBITS") ? std::atoi(std::getenv("VQC_HBM_TILE_QUBITS")) : 0;
         if (env_m > p.G_swz && env_m < n) {
-            m = std::max(env_m, hbm_k(mode, dtype) + 1);
+            m = std::min(std::max(env_m, hbm_k(mode, dtype) + 1), hbm_k(mode, dtype) + 8);
             K = std::min(hbm_k(mode, dtype), m - 1);
         }
         if (K != hbm_k(mode, dtype)) continue;   // pass kernels exist for this K only

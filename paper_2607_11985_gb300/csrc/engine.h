@@ -37,6 +37,7 @@ struct Schedule {
     std::vector<int32_t> pass_accs;       // HBM path: accumulator ids per pass
     size_t dev_ops = 0, dev_stages = 0;   // byte offsets inside the device buffer
     size_t dev_passes = 0, dev_pass_entries = 0, dev_pass_accs = 0;
+    size_t dev_region_begin = 0, dev_region_end = 0;   // [ops .. pass_accs] in the blob
 };
 
 struct HostPlan {
@@ -62,6 +63,7 @@ struct HostPlan {
     size_t dev_entries = 0, dev_ps_list = 0, dev_sh_list = 0, dev_consts = 0, dev_cmat = 0, dev_cang = 0;
     size_t dev_xocc_ptr = 0, dev_xocc = 0, dev_wocc_ptr = 0, dev_wocc = 0, dev_accs = 0;
     unsigned* dev_error = nullptr;        // device error word (kernel self-checks)
+    size_t dev_tab_begin = 0, dev_tab_end = 0;   // [entries .. wocc] in the blob
 };
 
 // Largest n whose state(s) fit one CTA's shared memory on the resident path.

@@ -43,6 +43,9 @@ struct PArgs {
     R* E_part;              // forward, last pass: [B * ntiles, n]
     R* terms;               // backward: [B * ntiles, n_terms]
     int sm_sh, sm_ps, sm_psi, sm_lam, sm_acc, sm_red;
+    const unsigned char* plan;   // plan regions copied to shared memory (see KArgs)
+    int tab_off, tab_bytes, sched_off, sched_bytes, sm_plan, plan_smem;
+    int sm_koff;                 // per-pass tile-copy offsets: [ceil(2^m / (APV * T))] uint2
 };
 
 // Global amplitude index of tile-local index u (the low G tile bits are the
@@ -56,40 +59,71 @@ __device__ __forceinline__ uint32_t tile_global(uint32_t u, uint32_t tile_base, 
     return g;
 }
 
-// Copy one tile HBM -> shared memory (16-byte vectors; 8 per 128-byte chunk).
+// 16-byte vectors of amplitudes, moved without taking register addresses.
+template <typename R> struct Vec16;
+template <> struct Vec16<float> {
+    float2 a[2];
+    __device__ __forceinline__ void ld(const float2* p) {
+        const float4 v = __ldcs(reinterpret_cast<const float4*>(p));
+        a[0] = make_float2(v.x, v.y);
+        a[1] = make_float2(v.z, v.w);
+    }
+    __device__ __forceinline__ void st(float2* p) const {
+        __stcs(reinterpret_cast<float4*>(p), make_float4(a[0].x, a[0].y, a[1].x, a[1].y));
+    }
+};
+template <> struct Vec16<double> {
+    double2 a[1];
+    __device__ __forceinline__ void ld(const double2* p) { a[0] = __ldcs(p); }
+    __device__ __forceinline__ void st(double2* p) const { __stcs(p, a[0]); }
+};
+
+// Tile copies between HBM and shared memory.  A CTA-thread t moves vectors
+// v = t + k*T; the tile-local index of v splits into disjoint bit fields of t
+// and of k, and both the index deposit into global qubits and the swizzle are
+// linear in those fields, so each is a per-thread part XOR a per-k part
+// (tabulated once per pass in shared memory: koff[k] = (global, slot)).
 template <typename R>
-__device__ __forceinline__ void tile_gather(C2<R>* sm, const C2<R>* gs, uint32_t tile_base,
-                                            const uint8_t* tq, int m, int G, int h, int t, int T) {
-    constexpr int APV = 16 / sizeof(C2<R>);   // amplitudes per 16-byte vector
-    const int nvec = (1 << m) / APV;
-    for (int v = t; v < nvec; v += T) {
-        const uint32_t u = (uint32_t)v * APV;
-        const uint32_t g = tile_global(u, tile_base, tq, G);
-        const float4 raw = __ldcs(reinterpret_cast<const float4*>(gs + g));
-        const C2<R>* pr = reinterpret_cast<const C2<R>*>(&raw);
+__device__ __forceinline__ void tile_gather(C2<R>* sm, const C2<R>* gs, uint32_t gt, uint32_t st,
+                                            const uint2* koff, int nk, int T, int t) {
+    constexpr int APV = 16 / sizeof(C2<R>);
+    constexpr int U = 8;
+    int k = 0;
+    for (; k + U <= nk; k += U) {
+        Vec16<R> v[U];
 #pragma unroll
-        for (int k = 0; k < APV; ++k) sm[swz(u + k, G) ^ h] = pr[k];
+        for (int j = 0; j < U; ++j) v[j].ld(gs + (gt | koff[k + j].x));
+#pragma unroll
+        for (int j = 0; j < U; ++j) {
+            const uint32_t sl = st ^ koff[k + j].y;
+#pragma unroll
+            for (int e = 0; e < APV; ++e) sm[sl ^ e] = v[j].a[e];
+        }
+    }
+    for (; k < nk; ++k) {
+        Vec16<R> v;
+        v.ld(gs + (gt | koff[k].x));
+        const uint32_t sl = st ^ koff[k].y;
+#pragma unroll
+        for (int e = 0; e < APV; ++e) sm[sl ^ e] = v.a[e];
     }
 }
 
 template <typename R>
-__device__ __forceinline__ void tile_scatter(const C2<R>* sm, C2<R>* gs, uint32_t tile_base,
-                                             const uint8_t* tq, int m, int G, int h, int t, int T) {
+__device__ __forceinline__ void tile_scatter(const C2<R>* sm, C2<R>* gs, uint32_t gt, uint32_t st,
+                                             const uint2* koff, int nk, int T, int t) {
     constexpr int APV = 16 / sizeof(C2<R>);
-    const int nvec = (1 << m) / APV;
-    for (int v = t; v < nvec; v += T) {
-        const uint32_t u = (uint32_t)v * APV;
-        const uint32_t g = tile_global(u, tile_base, tq, G);
-        float4 raw;
-        C2<R>* pr = reinterpret_cast<C2<R>*>(&raw);
+    for (int k = 0; k < nk; ++k) {
+        Vec16<R> v;
+        const uint32_t sl = st ^ koff[k].y;
 #pragma unroll
-        for (int k = 0; k < APV; ++k) pr[k] = sm[swz(u + k, G) ^ h];
-        __stcs(reinterpret_cast<float4*>(gs + g), raw);
+        for (int e = 0; e < APV; ++e) v.a[e] = sm[sl ^ e];
+        v.st(gs + (gt | koff[k].x));
     }
 }
 
 template <typename R, int K, int MODE>
-__global__ void __launch_bounds__(512) pass_kernel(const __grid_constant__ PArgs<R> A) {
+__global__ void __launch_bounds__(256) pass_kernel(const __grid_constant__ PArgs<R> A) {
     extern __shared__ __align__(16) unsigned char smem[];
     R* sh_tab = reinterpret_cast<R*>(smem + A.sm_sh);
     R* ps_all = reinterpret_cast<R*>(smem + A.sm_ps);
@@ -97,6 +131,29 @@ __global__ void __launch_bounds__(512) pass_kernel(const __grid_constant__ PArgs
     C2<R>* lam_all = reinterpret_cast<C2<R>*>(smem + A.sm_lam);
     R* acc_all = reinterpret_cast<R*>(smem + A.sm_acc);
     R* red_all = reinterpret_cast<R*>(smem + A.sm_red);
+
+    const unsigned char* smt = nullptr;
+    const unsigned char* sms = nullptr;
+    if (A.plan_smem) {
+        unsigned char* t = smem + A.sm_plan;
+        unsigned char* u = t + ((A.tab_bytes + 15) & ~15);
+        copy_region(t, A.plan + A.tab_off, A.tab_bytes);
+        copy_region(u, A.plan + A.sched_off, A.sched_bytes);
+        smt = t;
+        sms = u;
+    }
+    const DOp* P_ops = rebase(A.ops, A.plan, A.sched_off, sms);
+    const DStage* P_stages = rebase(A.stages, A.plan, A.sched_off, sms);
+    const int32_t* P_pass_entries = rebase(A.pass_entries, A.plan, A.sched_off, sms);
+    const int32_t* P_pass_accs = rebase(A.pass_accs, A.plan, A.sched_off, sms);
+    const DEntry* P_entries = rebase(A.entries, A.plan, A.tab_off, smt);
+    const DConst* P_consts = rebase(A.consts, A.plan, A.tab_off, smt);
+    const R* P_cmat = reinterpret_cast<const R*>(
+        rebase(reinterpret_cast<const unsigned char*>(A.cmat), A.plan, A.tab_off, smt));
+    const R* P_cang = reinterpret_cast<const R*>(
+        rebase(reinterpret_cast<const unsigned char*>(A.cang), A.plan, A.tab_off, smt));
+    const DAcc* P_accs = rebase(A.accs, A.plan, A.tab_off, smt);
+    if (A.plan_smem) __syncthreads();
 
     const int n = A.n, G = A.G, tdim = 1 << A.m;
     const long long total_tiles = (long long)A.B * A.ntiles;
@@ -113,9 +170,21 @@ __global__ void __launch_bounds__(512) pass_kernel(const __grid_constant__ PArgs
     const int warp_in_group = q.t >> 5;
     const int nthr = blockDim.x;
 
+    // Tile copy geometry: vectors v = t + k*T of APV amplitudes.
+    constexpr int APV = 16 / sizeof(C2<R>);
+    const int nvec = tdim / APV;
+    const int nk = (nvec + q.T - 1) / q.T;
+    uint2* koff = reinterpret_cast<uint2*>(smem + A.sm_koff);
+    for (int k = threadIdx.x; k < nk; k += nthr) {
+        const uint32_t u = (uint32_t)k * q.T * APV;
+        koff[k] = make_uint2(tile_global(u, 0, A.tile_q, G), swz(u, G));
+    }
+    const uint32_t u_t = (uint32_t)q.t * APV;
+    const uint32_t st_t = swz(u_t, G) ^ (uint32_t)q.h;
+
     for (int i = threadIdx.x; i < A.sh_count; i += nthr) {
-        const DEntry e = A.entries[__ldg(&A.pass_entries[A.sh_begin + i])];
-        eval_entry<R>(e, A.consts, nullptr, A.w, A.cang, A.cmat, sh_tab + 8 * i);
+        const DEntry e = P_entries[vqc_ld(&P_pass_entries[A.sh_begin + i])];
+        eval_entry<R>(e, P_consts, nullptr, A.w, P_cang, P_cmat, sh_tab + 8 * i);
     }
     __syncthreads();
 
@@ -138,15 +207,14 @@ __global__ void __launch_bounds__(512) pass_kernel(const __grid_constant__ PArgs
             const int gg = i / A.ps_count, k = i % A.ps_count;
             const long long tt = min(unit * A.S + gg, total_tiles - 1);
             const int bb = (int)(tt / A.ntiles);
-            const DEntry e = A.entries[__ldg(&A.pass_entries[A.ps_begin + k])];
-            eval_entry<R>(e, A.consts, A.x + (size_t)bb * A.Px, A.w, A.cang, A.cmat,
+            const DEntry e = P_entries[vqc_ld(&P_pass_entries[A.ps_begin + k])];
+            eval_entry<R>(e, P_consts, A.x + (size_t)bb * A.Px, A.w, P_cang, P_cmat,
                           ps_all + ((size_t)gg * A.ps_count + k) * 8);
         }
         const size_t sbase = (size_t)b << n;
-        if (A.src_psi)
-            tile_gather<R>(psi, A.src_psi + sbase, tile_base, A.tile_q, A.m, G, q.h, q.t, q.T);
-        if (MODE == 1 && A.src_lam)
-            tile_gather<R>(lam, A.src_lam + sbase, tile_base, A.tile_q, A.m, G, q.h, q.t, q.T);
+        const uint32_t gt = tile_global(u_t, tile_base, A.tile_q, G);
+        if (A.src_psi) tile_gather<R>(psi, A.src_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
+        if (MODE == 1 && A.src_lam) tile_gather<R>(lam, A.src_lam + sbase, gt, st_t, koff, nk, q.T, q.t);
         __syncthreads();
 
         C2<R> a[1 << K];
@@ -154,7 +222,7 @@ __global__ void __launch_bounds__(512) pass_kernel(const __grid_constant__ PArgs
         StageView v{0, 0};
         if (MODE == 0) {
             for (int s = A.stage_begin; s < A.stage_end; ++s) {
-                const DStage* sp = A.stages + s;
+                const DStage* sp = P_stages + s;
                 v = stage_view<K>(sp, q.t, q.h, sg);
                 v.pb |= tile_base;
                 if (s == A.stage_begin && !A.src_psi) {
@@ -164,11 +232,8 @@ __global__ void __launch_bounds__(512) pass_kernel(const __grid_constant__ PArgs
                 } else {
                     block_load<R, K>(a, psi, v.swb, sg);
                 }
-                const int ob = __ldg(&sp->op_begin), oe = __ldg(&sp->op_end);
-                for (int o = ob; o < oe; ++o) {
-                    const uint2 raw = __ldg(reinterpret_cast<const uint2*>(A.ops) + o);
-                    fwd_op<R, K>(raw, v.pb, a, sh_tab, ps_tab);
-                }
+                run_ops<R, K, 0>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
+                                 sh_tab, ps_tab, nullptr, q, lane, warp_in_group);
                 if (s + 1 < A.stage_end || A.dst_psi) {
                     block_store<R, K>(a, psi, v.swb, sg);
                     group_sync<R>(q);
@@ -176,7 +241,7 @@ __global__ void __launch_bounds__(512) pass_kernel(const __grid_constant__ PArgs
             }
             if (A.E_part) {
                 R* red = red_all + (size_t)q.g * q.wg * n;
-                expz_partials<R, K>(A.stages + (A.stage_end - 1), v.pb, a, n, red, q, warp_in_group);
+                expz_partials<R, K>(P_stages + (A.stage_end - 1), v.pb, a, n, red, q, warp_in_group);
                 __syncthreads();
                 if (valid)
                     for (int j = q.t; j < n; j += q.T) {
@@ -187,14 +252,14 @@ __global__ void __launch_bounds__(512) pass_kernel(const __grid_constant__ PArgs
             }
             __syncthreads();
             if (A.dst_psi && valid)
-                tile_scatter<R>(psi, A.dst_psi + sbase, tile_base, A.tile_q, A.m, G, q.h, q.t, q.T);
+                tile_scatter<R>(psi, A.dst_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
             __syncthreads();
             continue;
         }
 
         // backward: stages of the pass in reverse
         for (int s = A.stage_end - 1; s >= A.stage_begin; --s) {
-            const DStage* sp = A.stages + s;
+            const DStage* sp = P_stages + s;
             C2<R> l[1 << K];
             v = stage_view<K>(sp, q.t, q.h, sg);
             v.pb |= tile_base;
@@ -203,11 +268,8 @@ __global__ void __launch_bounds__(512) pass_kernel(const __grid_constant__ PArgs
                 lambda_init<R, K>(sp, v.pb, A.gE + (size_t)b * n, n, a, l);
             else
                 block_load<R, K>(l, lam, v.swb, sg);
-            const int ob = __ldg(&sp->op_begin), oe = __ldg(&sp->op_end);
-            for (int o = oe - 1; o >= ob; --o) {
-                const uint2 raw = __ldg(reinterpret_cast<const uint2*>(A.ops) + o);
-                bwd_op<R, K>(raw, v.pb, a, l, sh_tab, ps_tab, acc, q, lane, warp_in_group);
-            }
+            run_ops<R, K, 1>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l, sh_tab,
+                             ps_tab, acc, q, lane, warp_in_group);
             if (s > A.stage_begin || A.dst_psi) {
                 block_store<R, K>(a, psi, v.swb, sg);
                 block_store<R, K>(l, lam, v.swb, sg);
@@ -216,18 +278,18 @@ __global__ void __launch_bounds__(512) pass_kernel(const __grid_constant__ PArgs
         }
         __syncthreads();
         if (valid && A.dst_psi) {
-            tile_scatter<R>(psi, A.dst_psi + sbase, tile_base, A.tile_q, A.m, G, q.h, q.t, q.T);
-            tile_scatter<R>(lam, A.dst_lam + sbase, tile_base, A.tile_q, A.m, G, q.h, q.t, q.T);
+            tile_scatter<R>(psi, A.dst_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
+            tile_scatter<R>(lam, A.dst_lam + sbase, gt, st_t, koff, nk, q.T, q.t);
         }
         for (int i = threadIdx.x; i < A.S * A.acc_count; i += nthr) {
             const int gg = i / A.acc_count, k = i % A.acc_count;
             const long long tt = unit * A.S + gg;
             if (tt >= total_tiles) continue;
             const int bb = (int)(tt / A.ntiles);
-            const DAcc ac = A.accs[__ldg(&A.pass_accs[A.acc_begin + k])];
-            acc_terms<R>(ac, A.entries[ac.entry], acc_all + ((size_t)gg * A.acc_count + k) * q.wg * 8,
-                         q.wg, A.consts, A.x ? A.x + (size_t)bb * A.Px : nullptr, A.w, A.cang,
-                         A.cmat, A.terms + tt * A.n_terms);
+            const DAcc ac = P_accs[vqc_ld(&P_pass_accs[A.acc_begin + k])];
+            acc_terms<R>(ac, P_entries[ac.entry], acc_all + ((size_t)gg * A.acc_count + k) * q.wg * 8,
+                         q.wg, P_consts, A.x ? A.x + (size_t)bb * A.Px : nullptr, A.w, P_cang,
+                         P_cmat, A.terms + tt * A.n_terms);
         }
         __syncthreads();
     }
@@ -256,7 +318,7 @@ __global__ void reduce_dx(const R* terms, int B, int ntiles, int nt, const int32
         R s = 0;
         for (int t = 0; t < ntiles; ++t) {
             const R* row = terms + (b * ntiles + t) * nt;
-            for (int k = __ldg(&ptr[p]); k < __ldg(&ptr[p + 1]); ++k) s += row[__ldg(&occ[k])];
+            for (int k = vqc_ld(&ptr[p]); k < vqc_ld(&ptr[p + 1]); ++k) s += row[vqc_ld(&occ[k])];
         }
         dx[i] = s;
     }
@@ -269,11 +331,11 @@ __global__ void __launch_bounds__(256) reduce_dw(const R* terms, long long rows,
                                                  const int32_t* ptr, const int32_t* occ, R* dw) {
     __shared__ R part[256];
     const int p = blockIdx.x;
-    const int k0 = __ldg(&ptr[p]), k1 = __ldg(&ptr[p + 1]);
+    const int k0 = vqc_ld(&ptr[p]), k1 = vqc_ld(&ptr[p + 1]);
     R s = 0;
     for (long long r = threadIdx.x; r < rows; r += 256) {
         const R* row = terms + r * nt;
-        for (int k = k0; k < k1; ++k) s += row[__ldg(&occ[k])];
+        for (int k = k0; k < k1; ++k) s += row[vqc_ld(&occ[k])];
     }
     part[threadIdx.x] = s;
     __syncthreads();

@@ -44,8 +44,27 @@ enum OpFlags : uint8_t {
     OPF_HAS_ACC = 8       // op accumulates a gradient slot (aux) in the backward
 };
 
+// Dispatch code of a compiled op (DOp::code): the kernels take one jump-table
+// branch per op, each case specialised for fixed local positions.
+enum DispatchCode : uint8_t {
+    DC_M1 = 0,       // + t: 2x2 on local position t (0..4)
+    DC_CX_LL = 5,    // + 4c + (t < c ? t : t - 1): local control c, local target t
+    DC_CX_PL = 25,   // + t: control outside the block (ref a), local target t
+    DC_CZ_LL = 30,   // + cz_pair_index(lo, hi): both qubits local
+    DC_CZ_PL = 40,   // + l: local qubit l (ref a), other qubit outside the block (ref b)
+    DC_CZ_PP = 45,   // both qubits outside the block
+    DC_PH2 = 46,     // diagonal two-qubit phase, refs a and b (local or not)
+    DC_NUM = 47
+};
+// Index of the local pair (lo < hi < 5) in (0,1),(0,2),(0,3),(0,4),(1,2),...,(3,4).
+constexpr int cz_pair_index(int lo, int hi) {
+    return lo == 0 ? hi - 1 : lo == 1 ? 2 + hi : lo == 2 ? 4 + hi : 5 + hi;
+}
+
 struct DOp {
-    uint8_t type, a, b, flags;
+    uint8_t code;    // DispatchCode
+    uint8_t a, b;    // qubit refs (< kRefPhys: local position; else kRefPhys + qubit)
+    uint8_t flags;
     uint16_t slot;   // table entry index inside its table (per-sample or shared)
     uint16_t aux;    // accumulator slot for the backward (run or phase op id)
 };

@@ -74,6 +74,28 @@ __device__ __forceinline__ M2<R> mident() {
     return r;
 }
 
+// Plain load: plan arrays may live in shared memory (copied at kernel start)
+// or, when too large, in global memory.
+template <typename T>
+__device__ __forceinline__ T vqc_ld(const T* p) { return *p; }
+
+// Copy [src, src + bytes) (16-byte multiple) into shared memory; all loads are
+// independent, so a CTA pulls the whole plan in about one memory latency.
+__device__ __forceinline__ void copy_region(unsigned char* dst, const unsigned char* src, int bytes) {
+    const uint4* s = reinterpret_cast<const uint4*>(src);
+    uint4* d = reinterpret_cast<uint4*>(dst);
+    for (int i = threadIdx.x; i < bytes / 16; i += blockDim.x) d[i] = s[i];
+}
+
+// Pointer into the shared copy of a plan region (or the global one).
+template <typename T>
+__device__ __forceinline__ const T* rebase(const T* g, const unsigned char* plan, int region_off,
+                                           const unsigned char* sm_region) {
+    if (!sm_region) return g;
+    return reinterpret_cast<const T*>(sm_region +
+                                      (reinterpret_cast<const unsigned char*>(g) - plan - region_off));
+}
+
 __device__ __forceinline__ void sc(float t, float* s, float* c) { sincosf(t, s, c); }
 __device__ __forceinline__ void sc(double t, double* s, double* c) { sincos(t, s, c); }
 
@@ -97,6 +119,7 @@ struct KArgs {
     const int32_t* wocc;
     unsigned* err;
     int n, K, tbits, G, S;     // S = samples per CTA
+    int tpg, bpt;              // threads per sample group, register blocks per thread (tpg * bpt = 2^tbits)
     int n_ps, n_sh, n_accs, n_terms, Px, Pw;
     // batch
     int B, nunits;
@@ -113,6 +136,27 @@ struct KArgs {
     unsigned* counter;
     // shared-memory carve-up (byte offsets)
     int sm_sh, sm_ps, sm_psi, sm_lam, sm_acc, sm_terms, sm_dw, sm_red;
+    // plan regions copied to shared memory at sm_plan when plan_smem is set:
+    // table data [tab_off, tab_off + tab_bytes) and this schedule's
+    // [sched_off, sched_off + sched_bytes) of the plan's device blob.
+    const unsigned char* plan;
+    int tab_off, tab_bytes, sched_off, sched_bytes, sm_plan, plan_smem;
+};
+
+struct PlanPtrs {
+    const DOp* ops;
+    const DStage* stages;
+    const DEntry* entries;
+    const int32_t* ps_list;
+    const int32_t* sh_list;
+    const DConst* consts;
+    const void* cmat;
+    const void* cang;
+    const DAcc* accs;
+    const int32_t* xocc_ptr;
+    const int32_t* xocc;
+    const int32_t* wocc_ptr;
+    const int32_t* wocc;
 };
 
 // ---------------------------------------------------------------- tables
@@ -200,6 +244,34 @@ __device__ __forceinline__ void m1_apply(C2<R> (&a)[1 << K], const M2<R>& m) {
     }
 }
 
+// complex64: the same update with Blackwell's packed FP32 instructions on
+// (re, im) pairs.  With u~ = (u.im, u.re):
+//   m u = (Re m, Re m) * u + (-Im m, Im m) * u~
+// so a complex multiply-add is two FFMA2 and a pair update eight.
+template <int K, int T>
+__device__ __forceinline__ void m1_apply_f2(float2 (&a)[1 << K], const M2<float>& m) {
+    const float2 ar = make_float2(m.a.x, m.a.x), ai = make_float2(-m.a.y, m.a.y);
+    const float2 br = make_float2(m.b.x, m.b.x), bi = make_float2(-m.b.y, m.b.y);
+    const float2 cr = make_float2(m.c.x, m.c.x), ci = make_float2(-m.c.y, m.c.y);
+    const float2 dr = make_float2(m.d.x, m.d.x), di = make_float2(-m.d.y, m.d.y);
+#pragma unroll
+    for (int p = 0; p < (1 << (K - 1)); ++p) {
+        const int i0 = pair_lo<T>(p), i1 = i0 | (1 << T);
+        const float2 u = a[i0], v = a[i1];
+        const float2 us = make_float2(u.y, u.x), vs = make_float2(v.y, v.x);
+        float2 nu = __fmul2_rn(ar, u);
+        nu = __ffma2_rn(ai, us, nu);
+        nu = __ffma2_rn(br, v, nu);
+        nu = __ffma2_rn(bi, vs, nu);
+        float2 nv = __fmul2_rn(cr, u);
+        nv = __ffma2_rn(ci, us, nv);
+        nv = __ffma2_rn(dr, v, nv);
+        nv = __ffma2_rn(di, vs, nv);
+        a[i0] = nu;
+        a[i1] = nv;
+    }
+}
+
 // rho[a][b] += sum_pairs psi[a] conj(lam[b])  -> r[0..7] = (00, 01, 10, 11) re/im
 template <typename R, int K, int T>
 __device__ __forceinline__ void m1_rho(const C2<R> (&ps)[1 << K], const C2<R> (&la)[1 << K],
@@ -213,6 +285,42 @@ __device__ __forceinline__ void m1_rho(const C2<R> (&ps)[1 << K], const C2<R> (&
         r[4] = fma(v.x, q0.x, fma(v.y, q0.y, r[4])); r[5] = fma(v.y, q0.x, fma(-v.x, q0.y, r[5]));
         r[6] = fma(v.x, q1.x, fma(v.y, q1.y, r[6])); r[7] = fma(v.y, q1.x, fma(-v.x, q1.y, r[7]));
     }
+}
+
+// complex64 with packed FP32: psi conj(lam) = psi * (lam.re, lam.re) + psi~ * (lam.im, -lam.im)
+// with psi~ = (psi.im, psi.re); r is read as four float2 accumulators.
+template <int K, int T>
+__device__ __forceinline__ void m1_rho_f2(const float2 (&ps)[1 << K], const float2 (&la)[1 << K],
+                                          float (&r)[8]) {
+    float2 r00 = make_float2(r[0], r[1]), r01 = make_float2(r[2], r[3]);
+    float2 r10 = make_float2(r[4], r[5]), r11 = make_float2(r[6], r[7]);
+#pragma unroll
+    for (int p = 0; p < (1 << (K - 1)); ++p) {
+        const int i0 = pair_lo<T>(p), i1 = i0 | (1 << T);
+        const float2 u = ps[i0], v = ps[i1], q0 = la[i0], q1 = la[i1];
+        const float2 us = make_float2(u.y, u.x), vs = make_float2(v.y, v.x);
+        const float2 q0r = make_float2(q0.x, q0.x), q0i = make_float2(q0.y, -q0.y);
+        const float2 q1r = make_float2(q1.x, q1.x), q1i = make_float2(q1.y, -q1.y);
+        r00 = __ffma2_rn(u, q0r, r00); r00 = __ffma2_rn(us, q0i, r00);
+        r01 = __ffma2_rn(u, q1r, r01); r01 = __ffma2_rn(us, q1i, r01);
+        r10 = __ffma2_rn(v, q0r, r10); r10 = __ffma2_rn(vs, q0i, r10);
+        r11 = __ffma2_rn(v, q1r, r11); r11 = __ffma2_rn(vs, q1i, r11);
+    }
+    r[0] = r00.x; r[1] = r00.y; r[2] = r01.x; r[3] = r01.y;
+    r[4] = r10.x; r[5] = r10.y; r[6] = r11.x; r[7] = r11.y;
+}
+
+// Packed-FP32 variants for complex64, plain FMA for complex128.
+template <typename R, int K, int T>
+__device__ __forceinline__ void m1_go(C2<R> (&a)[1 << K], const M2<R>& m) {
+    if constexpr (sizeof(R) == 4) m1_apply_f2<K, T>(a, m);
+    else m1_apply<R, K, T>(a, m);
+}
+template <typename R, int K, int T>
+__device__ __forceinline__ void rho_go(const C2<R> (&ps)[1 << K], const C2<R> (&la)[1 << K],
+                                       R (&r)[8]) {
+    if constexpr (sizeof(R) == 4) m1_rho_f2<K, T>(ps, la, r);
+    else m1_rho<R, K, T>(ps, la, r);
 }
 
 template <typename R, int K>
@@ -383,7 +491,7 @@ __device__ __forceinline__ R shx(R v, int m, unsigned mask) { return __shfl_xor_
 // write the 8 sums to dst (reduce-scatter butterfly: 9 shuffles at 32 lanes).
 template <typename R>
 __device__ __forceinline__ void reduce8_store(R (&v)[8], int lanes, int lane, R* dst,
-                                              unsigned mask) {
+                                              unsigned mask, bool add) {
     int u0 = 0, u1 = 0, u2 = 0;
     if (lanes >= 2) {
         const int m = lanes >> 1;
@@ -412,14 +520,18 @@ __device__ __forceinline__ void reduce8_store(R (&v)[8], int lanes, int lane, R*
         R keep = u2 ? v[1] : v[0];
         v[0] = keep + shx<R>(send, m, mask);
         for (int mm = lanes >> 4; mm >= 1; mm >>= 1) v[0] += shx<R>(v[0], mm, mask);
-        if ((lane & ((lanes >> 3) - 1)) == 0) dst[4 * u0 + 2 * u1 + u2] = v[0];
+        if ((lane & ((lanes >> 3) - 1)) == 0) {
+            R* d = dst + 4 * u0 + 2 * u1 + u2;
+            *d = add ? *d + v[0] : v[0];
+        }
     } else if (lanes == 4) {
-        dst[4 * u0 + 2 * u1] = v[0];
-        dst[4 * u0 + 2 * u1 + 1] = v[1];
+        R* d = dst + 4 * u0 + 2 * u1;
+        d[0] = add ? d[0] + v[0] : v[0];
+        d[1] = add ? d[1] + v[1] : v[1];
     } else if (lanes == 2) {
-        for (int i = 0; i < 4; ++i) dst[4 * u0 + i] = v[i];
+        for (int i = 0; i < 4; ++i) dst[4 * u0 + i] = add ? dst[4 * u0 + i] + v[i] : v[i];
     } else {
-        for (int i = 0; i < 8; ++i) dst[i] = v[i];
+        for (int i = 0; i < 8; ++i) dst[i] = add ? dst[i] + v[i] : v[i];
     }
 }
 
@@ -467,13 +579,13 @@ struct StageView {
 template <int K>
 __device__ __forceinline__ StageView stage_view(const DStage* sp, int t, int h, int32_t (&sg)[K]) {
 #pragma unroll
-    for (int j = 0; j < K; ++j) sg[j] = __ldg(&sp->sigma[j]);
-    const int nb = __ldg(&sp->nthreadbits);   // uint8 load
+    for (int j = 0; j < K; ++j) sg[j] = vqc_ld(&sp->sigma[j]);
+    const int nb = vqc_ld(&sp->nthreadbits);   // uint8 load
     StageView v{(uint32_t)h, 0u};
     for (int i = 0; i < nb; ++i) {
         if ((t >> i) & 1) {
-            v.swb ^= (uint32_t)__ldg(&sp->tau[i]);
-            v.pb |= __ldg(&sp->tmask[i]);
+            v.swb ^= (uint32_t)vqc_ld(&sp->tau[i]);
+            v.pb |= vqc_ld(&sp->tmask[i]);
         }
     }
     return v;
@@ -485,78 +597,177 @@ __device__ __forceinline__ void block_load(C2<R> (&a)[1 << K], const C2<R>* st, 
 #pragma unroll
     for (int r = 0; r < (1 << K); ++r) a[r] = st[swb ^ block_off<K>(r, sg)];
 }
+// The store recomputes the 2^K slot offsets (an empty asm hides swb's value
+// from the compiler) instead of keeping the load's offsets live in registers
+// across the stage's ops.
 template <typename R, int K>
 __device__ __forceinline__ void block_store(const C2<R> (&a)[1 << K], C2<R>* st, uint32_t swb,
                                             const int32_t (&sg)[K]) {
+    asm volatile("" : "+r"(swb));
+    int32_t s2[K];
 #pragma unroll
-    for (int r = 0; r < (1 << K); ++r) st[swb ^ block_off<K>(r, sg)] = a[r];
+    for (int j = 0; j < K; ++j) {
+        s2[j] = sg[j];
+        asm volatile("" : "+r"(s2[j]));
+    }
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r) st[swb ^ block_off<K>(r, s2)] = a[r];
 }
 
-// ---------------------------------------------------------------- forward op
-template <typename R, int K>
-__device__ __forceinline__ void fwd_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 << K],
-                                       const R* sh_tab, const R* ps_tab) {
-    const int type = raw.x & 0xff, ra = (raw.x >> 8) & 0xff, rb = (raw.x >> 16) & 0xff;
-    const int flags = raw.x >> 24, slot = raw.y & 0xffff;
-    const R* tab = (flags & OPF_PER_SAMPLE) ? ps_tab : sh_tab;
-    if (type == OP_M1) {
-        const M2<R> m = load_m2<R>(tab + 8 * slot);
-        m1_dispatch<R, K>(ra, a, m);
-    } else if (type == OP_CX) {
-        if (ra < kRefPhys) cx_ll_dispatch<R, K>(ra, rb, a);
-        else x_pred_dispatch<R, K>(rb, a, ((pb >> (ra - kRefPhys)) & 1u) != 0);
-    } else if (type == OP_CZ) {
-        cz_dispatch<R, K>(ra, rb, pb, a);
-    } else if (type == OP_PH2) {
-        const R* p = tab + 8 * slot;
-        C2<R> ph[4] = {cm<R>(p[0], p[1]), cm<R>(p[2], p[3]), cm<R>(p[4], p[5]), cm<R>(p[6], p[7])};
-        ph2_apply<R, K, false>(ra, rb, pb, a, ph);
+// ---------------------------------------------------------------- op dispatch
+template <typename R> __device__ __forceinline__ M2<R> load_m2v(const R* p);
+template <> __device__ __forceinline__ M2<float> load_m2v<float>(const float* p) {
+    const float4 u = *reinterpret_cast<const float4*>(p);
+    const float4 v = *reinterpret_cast<const float4*>(p + 4);
+    M2<float> m;
+    m.a = make_float2(u.x, u.y); m.b = make_float2(u.z, u.w);
+    m.c = make_float2(v.x, v.y); m.d = make_float2(v.z, v.w);
+    return m;
+}
+template <> __device__ __forceinline__ M2<double> load_m2v<double>(const double* p) {
+    const double2* q = reinterpret_cast<const double2*>(p);
+    M2<double> m;
+    m.a = q[0]; m.b = q[1]; m.c = q[2]; m.d = q[3];
+    return m;
+}
+
+__device__ __forceinline__ bool physbit(uint32_t pb, int ref) {
+    return ((pb >> (ref - kRefPhys)) & 1u) != 0;
+}
+
+// Apply op `raw` to the block(s).  MODE 0: forward on a.  MODE 1: backward --
+// accumulate the op's gradient slot, then un-apply on a (psi) and l (lam).
+// One switch over the dispatch code; every case has fixed local positions.
+template <typename R, int K, int MODE>
+__device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 << K],
+                                         C2<R> (&l)[1 << K], const R* sh_tab, const R* ps_tab,
+                                         R* acc, const Geo& q, int lane, int warp_in_group,
+                                         bool acc_add) {
+    const int code = raw.x & 0xff, ra = (raw.x >> 8) & 0xff, rb = (raw.x >> 16) & 0xff;
+    const int flags = raw.x >> 24, slot = raw.y & 0xffff, aux = raw.y >> 16;
+    const R* tp = ((flags & OPF_PER_SAMPLE) ? ps_tab : sh_tab) + 8 * slot;
+    R* accp = acc + ((size_t)aux * q.wg + warp_in_group) * 8;
+    const int rlane = q.lanes < 32 ? q.t : lane;
+    switch (code) {
+#define VQC_M1(T_)                                                                   \
+    case DC_M1 + T_:                                                                 \
+        if constexpr (T_ < K) {                                                      \
+            const M2<R> m = load_m2v<R>(tp);                                         \
+            if (MODE == 0) {                                                         \
+                m1_go<R, K, T_>(a, m);                                               \
+            } else {                                                                 \
+                if (flags & OPF_HAS_ACC) {                                           \
+                    R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};                              \
+                    rho_go<R, K, T_>(a, l, rh);                                      \
+                    reduce8_store<R>(rh, q.lanes, rlane, accp, q.mask, acc_add);              \
+                }                                                                    \
+                const M2<R> md = mdag<R>(m);                                         \
+                m1_go<R, K, T_>(a, md);                                              \
+                m1_go<R, K, T_>(l, md);                                              \
+            }                                                                        \
+        }                                                                            \
+        break;
+        VQC_M1(0) VQC_M1(1) VQC_M1(2) VQC_M1(3) VQC_M1(4)
+#undef VQC_M1
+#define VQC_CXLL(C_, T_)                                                             \
+    case DC_CX_LL + 4 * C_ + (T_ < C_ ? T_ : T_ - 1):                                \
+        if constexpr (C_ < K && T_ < K) {                                            \
+            cx_ll<R, K, C_, T_>(a);                                                  \
+            if (MODE == 1) cx_ll<R, K, C_, T_>(l);                                   \
+        }                                                                            \
+        break;
+        VQC_CXLL(0, 1) VQC_CXLL(0, 2) VQC_CXLL(0, 3) VQC_CXLL(0, 4)
+        VQC_CXLL(1, 0) VQC_CXLL(1, 2) VQC_CXLL(1, 3) VQC_CXLL(1, 4)
+        VQC_CXLL(2, 0) VQC_CXLL(2, 1) VQC_CXLL(2, 3) VQC_CXLL(2, 4)
+        VQC_CXLL(3, 0) VQC_CXLL(3, 1) VQC_CXLL(3, 2) VQC_CXLL(3, 4)
+        VQC_CXLL(4, 0) VQC_CXLL(4, 1) VQC_CXLL(4, 2) VQC_CXLL(4, 3)
+#undef VQC_CXLL
+#define VQC_CXPL(T_)                                                                 \
+    case DC_CX_PL + T_:                                                              \
+        if constexpr (T_ < K) {                                                      \
+            const bool p_ = physbit(pb, ra);                                         \
+            x_pred<R, K, T_>(a, p_);                                                 \
+            if (MODE == 1) x_pred<R, K, T_>(l, p_);                                  \
+        }                                                                            \
+        break;
+        VQC_CXPL(0) VQC_CXPL(1) VQC_CXPL(2) VQC_CXPL(3) VQC_CXPL(4)
+#undef VQC_CXPL
+#define VQC_CZLL(A_, B_)                                                             \
+    case DC_CZ_LL + cz_pair_index(A_, B_):                                           \
+        if constexpr (A_ < K && B_ < K) {                                            \
+            z2_ll<R, K, A_, B_>(a);                                                  \
+            if (MODE == 1) z2_ll<R, K, A_, B_>(l);                                   \
+        }                                                                            \
+        break;
+        VQC_CZLL(0, 1) VQC_CZLL(0, 2) VQC_CZLL(0, 3) VQC_CZLL(0, 4)
+        VQC_CZLL(1, 2) VQC_CZLL(1, 3) VQC_CZLL(1, 4)
+        VQC_CZLL(2, 3) VQC_CZLL(2, 4) VQC_CZLL(3, 4)
+#undef VQC_CZLL
+#define VQC_CZPL(L_)                                                                 \
+    case DC_CZ_PL + L_:                                                              \
+        if constexpr (L_ < K) {                                                      \
+            const bool p_ = physbit(pb, rb);                                         \
+            z1_pred<R, K, L_>(a, p_);                                                \
+            if (MODE == 1) z1_pred<R, K, L_>(l, p_);                                 \
+        }                                                                            \
+        break;
+        VQC_CZPL(0) VQC_CZPL(1) VQC_CZPL(2) VQC_CZPL(3) VQC_CZPL(4)
+#undef VQC_CZPL
+    case DC_CZ_PP: {
+        const R sgn = (physbit(pb, ra) && physbit(pb, rb)) ? R(-1) : R(1);
+#pragma unroll
+        for (int r = 0; r < (1 << K); ++r) {
+            a[r] = cm<R>(sgn * a[r].x, sgn * a[r].y);
+            if (MODE == 1) l[r] = cm<R>(sgn * l[r].x, sgn * l[r].y);
+        }
+        break;
+    }
+    case DC_PH2: {
+        C2<R> ph[4] = {cm<R>(tp[0], tp[1]), cm<R>(tp[2], tp[3]), cm<R>(tp[4], tp[5]),
+                       cm<R>(tp[6], tp[7])};
+        if (MODE == 0) {
+            ph2_apply<R, K, false>(ra, rb, pb, a, ph);
+        } else {
+            if (flags & OPF_HAS_ACC) {
+                R tv = ph2_term<R, K>(ra, rb, pb, (uint8_t)flags, a, l);
+                tv = reduce1<R>(tv, q.lanes, q.mask);
+                if ((q.t & (q.lanes - 1)) == 0) accp[0] = acc_add ? accp[0] + tv : tv;
+            }
+            ph2_apply<R, K, true>(ra, rb, pb, a, ph);
+            ph2_apply<R, K, true>(ra, rb, pb, l, ph);
+        }
+        break;
+    }
+    default:
+        break;
     }
 }
 
-// ---------------------------------------------------------------- backward op
-// Un-apply one op on psi (a) and lam (l); first accumulate its gradient slot
-// (rho of a run, or Im <lam|P|psi> of a phase op) into acc[(aux * wg + warp) * 8].
-template <typename R, int K>
-__device__ __forceinline__ void bwd_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 << K],
-                                       C2<R> (&l)[1 << K], const R* sh_tab, const R* ps_tab,
-                                       R* acc, const Geo& q, int lane, int warp_in_group) {
-    const int type = raw.x & 0xff, ra = (raw.x >> 8) & 0xff, rb = (raw.x >> 16) & 0xff;
-    const int flags = raw.x >> 24, slot = raw.y & 0xffff, aux = raw.y >> 16;
-    const R* tab = (flags & OPF_PER_SAMPLE) ? ps_tab : sh_tab;
-    if (type == OP_M1) {
-        const M2<R> m = load_m2<R>(tab + 8 * slot);
-        if (flags & OPF_HAS_ACC) {
-            R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-            m1_rho_dispatch<R, K>(ra, a, l, rh);
-            reduce8_store<R>(rh, q.lanes, q.lanes < 32 ? q.t : lane,
-                             acc + ((size_t)aux * q.wg + warp_in_group) * 8, q.mask);
+// Run ops [ob, oe) of a stage (forward: in order; backward: reversed), with the
+// next op's descriptor fetched while the current one executes.
+template <typename R, int K, int MODE>
+__device__ __forceinline__ void run_ops(const DOp* ops, int ob, int oe, uint32_t pb,
+                                        C2<R> (&a)[1 << K], C2<R> (&l)[1 << K], const R* sh_tab,
+                                        const R* ps_tab, R* acc, const Geo& q, int lane,
+                                        int warp_in_group, bool acc_add = false) {
+    const uint2* op2 = reinterpret_cast<const uint2*>(ops);
+    if (ob >= oe) return;
+    if (MODE == 0) {
+        uint2 nxt = vqc_ld(op2 + ob);
+        for (int o = ob; o < oe; ++o) {
+            const uint2 raw = nxt;
+            if (o + 1 < oe) nxt = vqc_ld(op2 + o + 1);
+            apply_op<R, K, MODE>(raw, pb, a, l, sh_tab, ps_tab, acc, q, lane, warp_in_group,
+                                 acc_add);
         }
-        const M2<R> md = mdag<R>(m);
-        m1_dispatch<R, K>(ra, a, md);
-        m1_dispatch<R, K>(ra, l, md);
-    } else if (type == OP_CX) {
-        if (ra < kRefPhys) {
-            cx_ll_dispatch<R, K>(ra, rb, a);
-            cx_ll_dispatch<R, K>(ra, rb, l);
-        } else {
-            const bool p = ((pb >> (ra - kRefPhys)) & 1u) != 0;
-            x_pred_dispatch<R, K>(rb, a, p);
-            x_pred_dispatch<R, K>(rb, l, p);
+    } else {
+        uint2 nxt = vqc_ld(op2 + oe - 1);
+        for (int o = oe - 1; o >= ob; --o) {
+            const uint2 raw = nxt;
+            if (o > ob) nxt = vqc_ld(op2 + o - 1);
+            apply_op<R, K, MODE>(raw, pb, a, l, sh_tab, ps_tab, acc, q, lane, warp_in_group,
+                                 acc_add);
         }
-    } else if (type == OP_CZ) {
-        cz_dispatch<R, K>(ra, rb, pb, a);
-        cz_dispatch<R, K>(ra, rb, pb, l);
-    } else if (type == OP_PH2) {
-        const R* p = tab + 8 * slot;
-        C2<R> ph[4] = {cm<R>(p[0], p[1]), cm<R>(p[2], p[3]), cm<R>(p[4], p[5]), cm<R>(p[6], p[7])};
-        if (flags & OPF_HAS_ACC) {
-            R tv = ph2_term<R, K>(ra, rb, pb, (uint8_t)flags, a, l);
-            tv = reduce1<R>(tv, q.lanes, q.mask);
-            if ((q.t & (q.lanes - 1)) == 0) acc[((size_t)aux * q.wg + warp_in_group) * 8] = tv;
-        }
-        ph2_apply<R, K, true>(ra, rb, pb, a, ph);
-        ph2_apply<R, K, true>(ra, rb, pb, l, ph);
     }
 }
 
@@ -570,7 +781,7 @@ __device__ __forceinline__ void lambda_init(const DStage* sp, uint32_t pb, const
     uint32_t actmask = 0;
 #pragma unroll
     for (int j = 0; j < K; ++j) {
-        const int aq = __ldg(&sp->active[j]);
+        const int aq = vqc_ld(&sp->active[j]);
         actmask |= 1u << aq;
         ge_loc[j] = gb[aq];
     }
@@ -590,27 +801,23 @@ __device__ __forceinline__ void lambda_init(const DStage* sp, uint32_t pb, const
 template <typename R, int K>
 __device__ __forceinline__ void expz_partials(const DStage* sp, uint32_t pb,
                                               const C2<R> (&a)[1 << K], int n, R* red,
-                                              const Geo& q, int warp_in_group) {
-    R pr[1 << K];
+                                              const Geo& q, int warp_in_group, bool add = false) {
     R ptot = 0;
-#pragma unroll
-    for (int r = 0; r < (1 << K); ++r) {
-        pr[r] = fma(a[r].x, a[r].x, a[r].y * a[r].y);
-        ptot += pr[r];
-    }
     R dloc[K];
 #pragma unroll
-    for (int j = 0; j < K; ++j) {
-        R d = 0;
+    for (int j = 0; j < K; ++j) dloc[j] = 0;
 #pragma unroll
-        for (int r = 0; r < (1 << K); ++r) d += ((r >> j) & 1) ? -pr[r] : pr[r];
-        dloc[j] = d;
+    for (int r = 0; r < (1 << K); ++r) {
+        const R pr = fma(a[r].x, a[r].x, a[r].y * a[r].y);
+        ptot += pr;
+#pragma unroll
+        for (int j = 0; j < K; ++j) dloc[j] += ((r >> j) & 1) ? -pr : pr;
     }
     uint32_t actmask = 0;
     int aq[K];
 #pragma unroll
     for (int j = 0; j < K; ++j) {
-        aq[j] = __ldg(&sp->active[j]);
+        aq[j] = vqc_ld(&sp->active[j]);
         actmask |= 1u << aq[j];
     }
     for (int j = 0; j < n; ++j) {
@@ -623,7 +830,10 @@ __device__ __forceinline__ void expz_partials(const DStage* sp, uint32_t pb,
             val = ((pb >> j) & 1u) ? -ptot : ptot;
         }
         val = reduce1<R>(val, q.lanes, q.mask);
-        if ((q.t & (q.lanes - 1)) == 0) red[warp_in_group * n + j] = val;
+        if ((q.t & (q.lanes - 1)) == 0) {
+            R* d = red + warp_in_group * n + j;
+            *d = add ? *d + val : val;
+        }
     }
 }
 
@@ -667,15 +877,9 @@ __device__ void acc_terms(const DAcc& ac, const DEntry& e, const R* ap, int wg,
 
 
 // ---------------------------------------------------------------- kernel
-template <typename R, int K, int MODE>
-struct MaxThreads {
-    static constexpr int value = (sizeof(R) == 4 && MODE == 0 && K <= 4) ? 1024 : 512;
-};
-
 // MODE 0: forward, MODE 1: backward.
 template <typename R, int K, int MODE>
-__global__ void __launch_bounds__(MaxThreads<R, K, MODE>::value)
-sweep_kernel(const __grid_constant__ KArgs<R> A) {
+__global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArgs<R> A) {
     extern __shared__ __align__(16) unsigned char smem[];
     R* sh_tab = reinterpret_cast<R*>(smem + A.sm_sh);
     R* ps_all = reinterpret_cast<R*>(smem + A.sm_ps);
@@ -686,10 +890,38 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
     R* dw_cta = reinterpret_cast<R*>(smem + A.sm_dw);
     R* red_all = reinterpret_cast<R*>(smem + A.sm_red);
 
+    const unsigned char* smt = nullptr;
+    const unsigned char* sms = nullptr;
+    if (A.plan_smem) {
+        unsigned char* t = smem + A.sm_plan;
+        unsigned char* u = t + ((A.tab_bytes + 15) & ~15);
+        copy_region(t, A.plan + A.tab_off, A.tab_bytes);
+        copy_region(u, A.plan + A.sched_off, A.sched_bytes);
+        smt = t;
+        sms = u;
+    }
+    PlanPtrs P;
+    P.ops = rebase(A.ops, A.plan, A.sched_off, sms);
+    P.stages = rebase(A.stages, A.plan, A.sched_off, sms);
+    P.entries = rebase(A.entries, A.plan, A.tab_off, smt);
+    P.ps_list = rebase(A.ps_list, A.plan, A.tab_off, smt);
+    P.sh_list = rebase(A.sh_list, A.plan, A.tab_off, smt);
+    P.consts = rebase(A.consts, A.plan, A.tab_off, smt);
+    P.cmat = rebase(reinterpret_cast<const unsigned char*>(A.cmat), A.plan, A.tab_off, smt);
+    P.cang = rebase(reinterpret_cast<const unsigned char*>(A.cang), A.plan, A.tab_off, smt);
+    P.accs = rebase(A.accs, A.plan, A.tab_off, smt);
+    P.xocc_ptr = rebase(A.xocc_ptr, A.plan, A.tab_off, smt);
+    P.xocc = rebase(A.xocc, A.plan, A.tab_off, smt);
+    P.wocc_ptr = rebase(A.wocc_ptr, A.plan, A.tab_off, smt);
+    P.wocc = rebase(A.wocc, A.plan, A.tab_off, smt);
+    const R* Pcmat = reinterpret_cast<const R*>(P.cmat);
+    const R* Pcang = reinterpret_cast<const R*>(P.cang);
+    if (A.plan_smem) __syncthreads();
+
     const int n = A.n, G = A.G;
     const int dim = 1 << n;
     Geo q;
-    q.T = 1 << A.tbits;
+    q.T = A.tpg;
     q.lanes = q.T < 32 ? q.T : 32;
     q.wg = q.T > 32 ? q.T / 32 : 1;
     q.g = threadIdx.x / q.T;
@@ -703,9 +935,9 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
 
     // shared table (w and constants): once per CTA
     for (int i = threadIdx.x; i < A.n_sh; i += nthr) {
-        const int id = __ldg(&A.sh_list[i]);
-        const DEntry e = A.entries[id];
-        eval_entry<R>(e, A.consts, nullptr, A.w, A.cang, A.cmat, sh_tab + 8 * e.slot);
+        const int id = vqc_ld(&P.sh_list[i]);
+        const DEntry e = P.entries[id];
+        eval_entry<R>(e, P.consts, nullptr, A.w, Pcang, Pcmat, sh_tab + 8 * e.slot);
     }
     if (MODE == 1)
         for (int i = threadIdx.x; i < A.Pw; i += nthr) dw_cta[i] = 0;
@@ -727,9 +959,9 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
         for (int i = threadIdx.x; i < A.S * A.n_ps; i += nthr) {
             const int gg = i / A.n_ps, k = i % A.n_ps;
             const int bb = min(unit * A.S + gg, A.B - 1);
-            const int id = __ldg(&A.ps_list[k]);
-            const DEntry e = A.entries[id];
-            eval_entry<R>(e, A.consts, A.x + (size_t)bb * A.Px, A.w, A.cang, A.cmat,
+            const int id = vqc_ld(&P.ps_list[k]);
+            const DEntry e = P.entries[id];
+            eval_entry<R>(e, P.consts, A.x + (size_t)bb * A.Px, A.w, Pcang, Pcmat,
                           ps_all + ((size_t)gg * A.n_ps + e.slot) * 8);
         }
         // initial / final state from global memory (coalesced, into swizzled slots)
@@ -749,34 +981,32 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
         const int ns = A.nstages;
 
         // -------- forward sweep (forward mode, or backward recompute)
+        R* red = red_all + (size_t)q.g * q.wg * n;
         if (MODE == 0 || recompute) {
             for (int s = 0; s < ns; ++s) {
-                const DStage* sp = A.stages + s;
-                v = stage_view<K>(sp, q.t, q.h, sg);
-                if (s == 0 && !from_global) {
+                const DStage* sp = P.stages + s;
+                const bool last = s + 1 == ns;
+                const bool store = !last || (MODE == 0 && A.state_out) || (MODE == 1 && A.bpt > 1);
+                for (int bj = 0; bj < A.bpt; ++bj) {
+                    v = stage_view<K>(sp, q.t + bj * q.T, q.h, sg);
+                    if (s == 0 && !from_global) {
 #pragma unroll
-                    for (int r = 0; r < (1 << K); ++r) a[r] = cm<R>(0, 0);
-                    if (v.pb == 0) a[0] = cm<R>(1, 0);
-                } else {
-                    block_load<R, K>(a, psi, v.swb, sg);
+                        for (int r = 0; r < (1 << K); ++r) a[r] = cm<R>(0, 0);
+                        if (v.pb == 0) a[0] = cm<R>(1, 0);
+                    } else {
+                        block_load<R, K>(a, psi, v.swb, sg);
+                    }
+                    run_ops<R, K, 0>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
+                                     sh_tab, ps_tab, nullptr, q, lane, warp_in_group);
+                    if (MODE == 0 && last)   // <Z_j> partials from the final blocks
+                        expz_partials<R, K>(sp, v.pb, a, n, red, q, warp_in_group, bj > 0);
+                    if (store) block_store<R, K>(a, psi, v.swb, sg);
                 }
-                const int ob = __ldg(&sp->op_begin), oe = __ldg(&sp->op_end);
-                for (int o = ob; o < oe; ++o) {
-                    const uint2 raw = __ldg(reinterpret_cast<const uint2*>(A.ops) + o);
-                    fwd_op<R, K>(raw, v.pb, a, sh_tab, ps_tab);
-                }
-                if (s + 1 < ns || (MODE == 0 && A.state_out)) {
-                    block_store<R, K>(a, psi, v.swb, sg);
-                    group_sync<R>(q);
-                }
+                if (store) group_sync<R>(q);
             }
         }
 
         if (MODE == 0) {
-            // -------- <Z_j> partials from the final block
-            const DStage* sp = A.stages + (ns - 1);
-            R* red = red_all + (size_t)q.g * q.wg * n;
-            expz_partials<R, K>(sp, v.pb, a, n, red, q, warp_in_group);
             __syncthreads();
             if (valid) {
                 for (int j = q.t; j < n; j += q.T) {
@@ -795,24 +1025,23 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
 
         // -------- backward: reverse sweep with psi and lam
         for (int s = ns - 1; s >= 0; --s) {
-            const DStage* sp = A.stages + s;
-            C2<R> l[1 << K];
-            v = stage_view<K>(sp, q.t, q.h, sg);
-            if (s == ns - 1) {
-                if (!recompute) block_load<R, K>(a, psi, v.swb, sg);
-                lambda_init<R, K>(sp, v.pb, A.gE + (size_t)b * n, n, a, l);
-            } else {
-                block_load<R, K>(a, psi, v.swb, sg);
-                block_load<R, K>(l, lam, v.swb, sg);
-            }
-            const int ob = __ldg(&sp->op_begin), oe = __ldg(&sp->op_end);
-            for (int o = oe - 1; o >= ob; --o) {
-                const uint2 raw = __ldg(reinterpret_cast<const uint2*>(A.ops) + o);
-                bwd_op<R, K>(raw, v.pb, a, l, sh_tab, ps_tab, acc, q, lane, warp_in_group);
-            }
-            if (s > 0) {
-                block_store<R, K>(a, psi, v.swb, sg);
-                block_store<R, K>(l, lam, v.swb, sg);
+            const DStage* sp = P.stages + s;
+            for (int bj = 0; bj < A.bpt; ++bj) {
+                C2<R> l[1 << K];
+                v = stage_view<K>(sp, q.t + bj * q.T, q.h, sg);
+                if (s == ns - 1) {
+                    if (!recompute || A.bpt > 1) block_load<R, K>(a, psi, v.swb, sg);
+                    lambda_init<R, K>(sp, v.pb, A.gE + (size_t)b * n, n, a, l);
+                } else {
+                    block_load<R, K>(a, psi, v.swb, sg);
+                    block_load<R, K>(l, lam, v.swb, sg);
+                }
+                run_ops<R, K, 1>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l,
+                                 sh_tab, ps_tab, acc, q, lane, warp_in_group, bj > 0);
+                if (s > 0) {
+                    block_store<R, K>(a, psi, v.swb, sg);
+                    block_store<R, K>(l, lam, v.swb, sg);
+                }
             }
             group_sync<R>(q);
         }
@@ -821,11 +1050,11 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
         // -------- gradient terms from the accumulated rho / scalars
         for (int i = threadIdx.x; i < A.S * A.n_accs; i += nthr) {
             const int gg = i / A.n_accs, k = i % A.n_accs;
-            const DAcc ac = A.accs[k];
+            const DAcc ac = P.accs[k];
             const int bb = min(unit * A.S + gg, A.B - 1);
             const R* xg = A.x ? A.x + (size_t)bb * A.Px : nullptr;
-            acc_terms<R>(ac, A.entries[ac.entry], acc_all + ((size_t)gg * A.n_accs + k) * q.wg * 8,
-                         q.wg, A.consts, xg, A.w, A.cang, A.cmat,
+            acc_terms<R>(ac, P.entries[ac.entry], acc_all + ((size_t)gg * A.n_accs + k) * q.wg * 8,
+                         q.wg, P.consts, xg, A.w, Pcang, Pcmat,
                          terms_all + (size_t)gg * A.n_terms);
         }
         __syncthreads();
@@ -837,8 +1066,8 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
                 if (bb >= A.B) continue;
                 const R* tm = terms_all + (size_t)gg * A.n_terms;
                 R sum = 0;
-                for (int k = __ldg(&A.xocc_ptr[p]); k < __ldg(&A.xocc_ptr[p + 1]); ++k)
-                    sum += tm[__ldg(&A.xocc[k])];
+                for (int k = vqc_ld(&P.xocc_ptr[p]); k < vqc_ld(&P.xocc_ptr[p + 1]); ++k)
+                    sum += tm[vqc_ld(&P.xocc[k])];
                 A.dx[(size_t)bb * A.Px + p] = sum;
             }
         }
@@ -847,8 +1076,8 @@ sweep_kernel(const __grid_constant__ KArgs<R> A) {
             for (int gg = 0; gg < A.S; ++gg) {
                 if (unit * A.S + gg >= A.B) break;
                 const R* tm = terms_all + (size_t)gg * A.n_terms;
-                for (int k = __ldg(&A.wocc_ptr[p]); k < __ldg(&A.wocc_ptr[p + 1]); ++k)
-                    sum += tm[__ldg(&A.wocc[k])];
+                for (int k = vqc_ld(&P.wocc_ptr[p]); k < vqc_ld(&P.wocc_ptr[p + 1]); ++k)
+                    sum += tm[vqc_ld(&P.wocc[k])];
             }
             dw_cta[p] = sum;
         }

@@ -17,7 +17,7 @@ DENTRY = np.dtype([("cfirst", "<u2"), ("ccount", "<u2"), ("slot", "<u2"), ("per_
 DCONST = np.dtype([("kind", "u1"), ("src0", "u1"), ("src1", "u1"), ("pad", "u1"),
                    ("idx0", "<i4"), ("idx1", "<i4"), ("term", "<i4")])
 DACC = np.dtype([("entry", "<i4"), ("kind", "<i4")])
-DOP = np.dtype([("type", "u1"), ("a", "u1"), ("b", "u1"), ("flags", "u1"), ("slot", "<u2"),
+DOP = np.dtype([("code", "u1"), ("a", "u1"), ("b", "u1"), ("flags", "u1"), ("slot", "<u2"),
                 ("aux", "<u2")])
 DSTAGE = np.dtype([("op_begin", "<i4"), ("op_end", "<i4"), ("sigma", "<i4", 5), ("tau", "<i4", 16),
                    ("tmask", "<u4", 16), ("active", "u1", 5), ("nthreadbits", "u1"),
@@ -30,6 +30,37 @@ assert DSTAGE.itemsize == 164 and DPASS.itemsize == 88
 PATH_RESIDENT, PATH_HBM = 0, 1
 
 OP_M1, OP_CX, OP_CZ, OP_PH2 = 1, 2, 3, 4
+DC_M1, DC_CX_LL, DC_CX_PL, DC_CZ_LL, DC_CZ_PL, DC_CZ_PP, DC_PH2 = 0, 5, 25, 30, 40, 45, 46
+CZ_PAIRS = [(0, 1), (0, 2), (0, 3), (0, 4), (1, 2), (1, 3), (1, 4), (2, 3), (2, 4), (3, 4)]
+
+
+def op_type(op):
+    """Decode an op's dispatch code into (type, a, b), checking that the code
+    agrees with the refs it carries."""
+    c, a, b = int(op["code"]), int(op["a"]), int(op["b"])
+    if c < DC_CX_LL:
+        assert a == c - DC_M1
+        return OP_M1, a, b
+    if c < DC_CX_PL:
+        k = c - DC_CX_LL
+        cc, tt = k // 4, k % 4
+        tt = tt if tt < cc else tt + 1
+        assert (a, b) == (cc, tt)
+        return OP_CX, a, b
+    if c < DC_CZ_LL:
+        assert a >= REF_PHYS and b == c - DC_CX_PL
+        return OP_CX, a, b
+    if c < DC_CZ_PL:
+        assert (a, b) == CZ_PAIRS[c - DC_CZ_LL]
+        return OP_CZ, a, b
+    if c < DC_CZ_PP:
+        assert a == c - DC_CZ_PL and b >= REF_PHYS
+        return OP_CZ, a, b
+    if c == DC_CZ_PP:
+        assert a >= REF_PHYS and b >= REF_PHYS
+        return OP_CZ, a, b
+    assert c == DC_PH2
+    return OP_PH2, a, b
 OPF_PER_SAMPLE, OPF_GEN_CRZ, OPF_GEN_RZZ, OPF_HAS_ACC = 1, 2, 4, 8
 CK_CONST, CK_RX, CK_RY, CK_RZ, CK_GPHASE, CK_CRZ, CK_RZZ = 1, 2, 3, 4, 5, 6, 7
 SRC_CONST, SRC_X, SRC_W = 1, 2, 3
@@ -149,22 +180,22 @@ class Plan:
     def apply_op(self, op, K, base, a, tabs, adjoint=False):
         ps, sh = tabs
         tab = ps if op["flags"] & OPF_PER_SAMPLE else sh
-        t = op["type"]
+        t, oa, ob = op_type(op)
         if t == OP_M1:
             M = tab[op["slot"]]
             if adjoint:
                 M = M.conj().T
-            T = op["a"]
+            T = oa
             assert T < K
             for r in range(1 << K):
                 if not (r >> T) & 1:
                     u, v = a[r], a[r | (1 << T)]
                     a[r], a[r | (1 << T)] = M[0, 0] * u + M[0, 1] * v, M[1, 0] * u + M[1, 1] * v
         elif t == OP_CX:
-            T = op["b"]
+            T = ob
             assert T < K
             for r in range(1 << K):
-                if not (r >> T) & 1 and self.refbit(op["a"], r, base):
+                if not (r >> T) & 1 and self.refbit(oa, r, base):
                     a[r], a[r | (1 << T)] = a[r | (1 << T)], a[r]
         elif t == OP_CZ:
             for r in range(1 << K):
@@ -241,8 +272,8 @@ class Plan:
                 a, l = psi[idx].copy(), lam[idx].copy()
                 for op in ops[::-1]:
                     if op["flags"] & OPF_HAS_ACC:
-                        if op["type"] == OP_M1:
-                            T = op["a"]
+                        if op_type(op)[0] == OP_M1:
+                            T = int(op["a"])
                             for r in range(1 << K):
                                 if not (r >> T) & 1:
                                     pp = [a[r], a[r | (1 << T)]]

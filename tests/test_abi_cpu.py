@@ -18,7 +18,7 @@ import pytest
 from oracle import oracle as orc
 from paper_2607_11985_gb300 import binding as B
 from paper_2607_11985_gb300 import workloads as wl
-from tests.plan_emulator import Plan, swz
+from tests.plan_emulator import Plan, op_type, swz
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
@@ -133,10 +133,11 @@ def check_addressing(plan):
                     slots.add(sl)
             assert slots == set(range(1 << m))
             for op in s["ops"][st["op_begin"]:st["op_end"]]:
-                if op["type"] == 1:
-                    assert op["a"] < K
-                if op["type"] == 2:
-                    assert op["b"] < K
+                t, oa, ob = op_type(op)
+                if t == 1:
+                    assert oa < K
+                if t == 2:
+                    assert ob < K
 
 
 SMALL_CASES = [(s, n, g) for s, n, g in [(101, 1, 12), (102, 2, 30), (103, 3, 60), (104, 4, 80),
