@@ -7,6 +7,7 @@
 #include <algorithm>
 #include <cstdlib>
 #include <cstring>
+#include <map>
 #include <memory>
 #include <mutex>
 #include <new>
@@ -21,6 +22,24 @@
 struct vqc_plan {
     vqc::HostPlan hp;
 };
+
+namespace vqc {
+namespace {
+// Launch geometry depends only on (plan, mode, batch, device): cache it so a
+// call does not repeat the attribute and occupancy queries.
+struct GeoKey {
+    const void* plan;
+    int mode, batch, dev, hbm;
+    bool operator<(const GeoKey& o) const {
+        if (plan != o.plan) return plan < o.plan;
+        if (mode != o.mode) return mode < o.mode;
+        if (batch != o.batch) return batch < o.batch;
+        if (dev != o.dev) return dev < o.dev;
+        return hbm < o.hbm;
+    }
+};
+}  // namespace
+}  // namespace vqc
 
 namespace vqc {
 namespace {
@@ -77,7 +96,7 @@ struct Launch {
     int K = 0, T = 0, S = 0, block = 0, grid = 0, nunits = 0, wg = 1, bpt = 1;
     size_t smem = 0;
     int sm_sh = 0, sm_ps = 0, sm_psi = 0, sm_lam = 0, sm_acc = 0, sm_terms = 0, sm_dw = 0,
-        sm_red = 0, sm_plan = 0;
+        sm_red = 0, sm_plan = 0, sm_w = 0, sm_xg = 0;
     bool plan_smem = false;
     const void* fn = nullptr;
 };
@@ -105,7 +124,7 @@ int choose_k(const HostPlan& p, int mode, int B) {
     return K;
 }
 
-vqc_status plan_launch(const HostPlan& p, int mode, int B, Launch& L) {
+vqc_status plan_launch_uncached(const HostPlan& p, int mode, int B, Launch& L) {
     int dev = 0;
     VQC_CUDA(cudaGetDevice(&dev));
     DevInfo di;
@@ -125,8 +144,10 @@ vqc_status plan_launch(const HostPlan& p, int mode, int B, Launch& L) {
     L.wg = L.T > 32 ? L.T / 32 : 1;
     // Shared memory: a fixed part per CTA and a part per resident sample.
     const size_t dim = (size_t)1 << p.n;
-    const size_t fixed = align16((size_t)p.n_sh * 8 * rs) + align16(mode == 1 ? (size_t)p.num_w * rs : 0) + 8 * 16;
+    const size_t fixed = align16((size_t)p.n_sh * 8 * rs) + align16(mode == 1 ? (size_t)p.num_w * rs : 0) +
+                         align16((size_t)p.num_w * rs) + 10 * 16;
     const size_t per_sample = (size_t)p.n_ps * 8 * rs + dim * cs * (mode == 1 ? 2 : 1) +
+                              (size_t)(p.num_x + p.n) * rs +
                               (mode == 1 ? p.accs.size() * L.wg * 8 * rs + p.term_src.size() * rs
                                          : (size_t)L.wg * p.n * rs);
     int S = std::max(1, 128 / L.T);
@@ -161,6 +182,8 @@ vqc_status plan_launch(const HostPlan& p, int mode, int B, Launch& L) {
     L.sm_terms = take(mode == 1 ? (size_t)L.S * p.term_src.size() * rs : 0);
     L.sm_dw = take(mode == 1 ? (size_t)p.num_w * rs : 0);
     L.sm_red = take(mode == 0 ? (size_t)L.S * L.wg * p.n * rs : 0);
+    L.sm_w = take((size_t)p.num_w * rs);
+    L.sm_xg = take((size_t)L.S * (p.num_x + p.n) * rs);
     // the plan's table data and this schedule go to shared memory when they fit
     const size_t plan_bytes = align16(p.dev_tab_end - p.dev_tab_begin) +
                               (L.s->dev_region_end - L.s->dev_region_begin);
@@ -178,6 +201,36 @@ vqc_status plan_launch(const HostPlan& p, int mode, int B, Launch& L) {
     L.nunits = (B + L.S - 1) / L.S;
     L.grid = std::max(1, std::min(L.nunits, per_sm * di.sms));
     return VQC_OK;
+}
+
+std::mutex g_geo_mu;
+std::map<GeoKey, Launch> g_launch_cache;
+
+GeoKey geo_key(const HostPlan& p, int mode, int B, int hbm) {
+    int dev = -1;
+    cudaGetDevice(&dev);
+    // environment switches that change the geometry are part of the key
+    const int env = env_int("VQC_FORCE_K_FWD", 0) * 1000 + env_int("VQC_FORCE_K_BWD", 0) * 10 +
+                    (env_int("VQC_PLAN_IN_SMEM", 1) != 0 ? 1 : 0);
+    return GeoKey{&p, mode, B, dev, hbm * 100000 + env};
+}
+
+vqc_status plan_launch(const HostPlan& p, int mode, int B, Launch& L) {
+    const GeoKey k = geo_key(p, mode, B, 0);
+    {
+        std::lock_guard<std::mutex> lk(g_geo_mu);
+        auto it = g_launch_cache.find(k);
+        if (it != g_launch_cache.end()) {
+            L = it->second;
+            return VQC_OK;
+        }
+    }
+    vqc_status st = plan_launch_uncached(p, mode, B, L);
+    if (st == VQC_OK) {
+        std::lock_guard<std::mutex> lk(g_geo_mu);
+        g_launch_cache[k] = L;
+    }
+    return st;
 }
 
 template <typename R>
@@ -213,6 +266,7 @@ void fill_plan_args(const HostPlan& p, const Launch& L, KArgs<R>& a) {
     a.Pw = p.num_w;
     a.sm_sh = L.sm_sh; a.sm_ps = L.sm_ps; a.sm_psi = L.sm_psi; a.sm_lam = L.sm_lam;
     a.sm_acc = L.sm_acc; a.sm_terms = L.sm_terms; a.sm_dw = L.sm_dw; a.sm_red = L.sm_red;
+    a.sm_w = L.sm_w; a.sm_xg = L.sm_xg;
     a.plan = static_cast<const unsigned char*>(p.dbuf);
     a.tab_off = (int)p.dev_tab_begin;
     a.tab_bytes = (int)(p.dev_tab_end - p.dev_tab_begin);
@@ -322,6 +376,14 @@ vqc_status run(const HostPlan& p, int mode, int B, const void* x, const void* w,
     }
     void* args[] = {&a};
     VQC_CUDA(cudaLaunchKernel(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
+    if (mode == 1 && dw && p.num_w > 0) {
+        const R* part = a.dw_part;
+        int rows = L.grid, cols = p.num_w;
+        R* out = static_cast<R*>(dw);
+        void* rargs[] = {&part, &rows, &cols, &out};
+        VQC_CUDA(cudaLaunchKernel(reduce_cols_ptr(p.dtype == VQC_C128), dim3(cols), dim3(256), rargs,
+                                  0, stream));
+    }
     return VQC_OK;
 }
 
@@ -338,7 +400,7 @@ struct PassGeo {
     const void* fn = nullptr;
 };
 
-vqc_status plan_hbm(const HostPlan& p, int mode, int B, PassGeo& L) {
+vqc_status plan_hbm_uncached(const HostPlan& p, int mode, int B, PassGeo& L) {
     L.s = find_hbm_schedule(p, mode);
     if (!L.s) return fail(VQC_ERR_UNSUPPORTED, "no HBM-tiled schedule for this circuit");
     int dev = 0;
@@ -403,6 +465,34 @@ vqc_status plan_hbm(const HostPlan& p, int mode, int B, PassGeo& L) {
     L.nunits = ((long long)B * L.ntiles + S - 1) / S;
     L.grid = (int)std::max<long long>(1, std::min<long long>(L.nunits, (long long)per_sm * di.sms));
     return VQC_OK;
+}
+
+std::map<GeoKey, PassGeo> g_pass_cache;
+
+vqc_status plan_hbm(const HostPlan& p, int mode, int B, PassGeo& L) {
+    const GeoKey k = geo_key(p, mode, B, 1);
+    {
+        std::lock_guard<std::mutex> lk(g_geo_mu);
+        auto it = g_pass_cache.find(k);
+        if (it != g_pass_cache.end()) {
+            L = it->second;
+            return VQC_OK;
+        }
+    }
+    vqc_status st = plan_hbm_uncached(p, mode, B, L);
+    if (st == VQC_OK) {
+        std::lock_guard<std::mutex> lk(g_geo_mu);
+        g_pass_cache[k] = L;
+    }
+    return st;
+}
+
+void forget_plan(const HostPlan* p) {
+    std::lock_guard<std::mutex> lk(g_geo_mu);
+    for (auto it = g_launch_cache.begin(); it != g_launch_cache.end();)
+        it = it->first.plan == p ? g_launch_cache.erase(it) : std::next(it);
+    for (auto it = g_pass_cache.begin(); it != g_pass_cache.end();)
+        it = it->first.plan == p ? g_pass_cache.erase(it) : std::next(it);
 }
 
 // Workspace of the HBM path.  Forward: [control | working state | <Z> partials].
@@ -722,6 +812,7 @@ vqc_status vqc_compile(const vqc_gate* gates, int32_t num_gates, int32_t num_qub
 
 void vqc_free(vqc_plan* plan) {
     if (!plan) return;
+    forget_plan(&plan->hp);
     if (plan->hp.dbuf) {
         int cur = -1;
         cudaGetDevice(&cur);

@@ -15,6 +15,7 @@ const void* pass_ptr(bool dbl, int mode, int K);
 const void* reduce_expz_ptr(bool dbl);
 const void* reduce_dx_ptr(bool dbl);
 const void* reduce_dw_ptr(bool dbl);
+const void* reduce_cols_ptr(bool dbl);
 
 // Largest block (threads) each instantiation is compiled for.
 inline int sweep_max_threads(bool is_double, int mode, int K) {

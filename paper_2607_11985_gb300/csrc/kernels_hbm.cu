@@ -24,6 +24,10 @@ const void* reduce_dx_ptr(bool dbl) {
     return dbl ? reinterpret_cast<const void*>(&reduce_dx<double>)
                : reinterpret_cast<const void*>(&reduce_dx<float>);
 }
+const void* reduce_cols_ptr(bool dbl) {
+    return dbl ? reinterpret_cast<const void*>(&reduce_cols<double>)
+               : reinterpret_cast<const void*>(&reduce_cols<float>);
+}
 const void* reduce_dw_ptr(bool dbl) {
     return dbl ? reinterpret_cast<const void*>(&reduce_dw<double>)
                : reinterpret_cast<const void*>(&reduce_dw<float>);

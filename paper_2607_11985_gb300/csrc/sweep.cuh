@@ -136,6 +136,7 @@ struct KArgs {
     unsigned* counter;
     // shared-memory carve-up (byte offsets)
     int sm_sh, sm_ps, sm_psi, sm_lam, sm_acc, sm_terms, sm_dw, sm_red;
+    int sm_w, sm_xg;   // shared copies of w [Pw] and of the unit's x / gE rows [S][Px + n]
     // plan regions copied to shared memory at sm_plan when plan_smem is set:
     // table data [tab_off, tab_off + tab_bytes) and this schedule's
     // [sched_off, sched_off + sched_bytes) of the plan's device blob.
@@ -933,15 +934,20 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
     const int warp_in_group = q.t >> 5;
     const int nthr = blockDim.x;
 
-    // shared table (w and constants): once per CTA
+    // w to shared memory (one parallel copy), then the shared table (w and
+    // constants) once per CTA
+    R* w_sm = reinterpret_cast<R*>(smem + A.sm_w);
+    R* xg_all = reinterpret_cast<R*>(smem + A.sm_xg);
+    const int xgw = A.Px + n;   // row width of the x / gE staging area
+    for (int i = threadIdx.x; i < A.Pw; i += nthr) w_sm[i] = A.w[i];
+    __syncthreads();
     for (int i = threadIdx.x; i < A.n_sh; i += nthr) {
         const int id = vqc_ld(&P.sh_list[i]);
         const DEntry e = P.entries[id];
-        eval_entry<R>(e, P.consts, nullptr, A.w, Pcang, Pcmat, sh_tab + 8 * e.slot);
+        eval_entry<R>(e, P.consts, nullptr, w_sm, Pcang, Pcmat, sh_tab + 8 * e.slot);
     }
     if (MODE == 1)
         for (int i = threadIdx.x; i < A.Pw; i += nthr) dw_cta[i] = 0;
-    __syncthreads();
 
     C2<R>* psi = psi_all + (size_t)q.g * dim;
     C2<R>* lam = lam_all + (size_t)q.g * dim;
@@ -953,15 +959,25 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
         const int b_raw = unit * A.S + q.g;
         const bool valid = b_raw < A.B;
         const int b = valid ? b_raw : A.B - 1;
-        const R* xb = A.x ? A.x + (size_t)b * A.Px : nullptr;
+
+        // x (and, backward, gE) rows of this unit's samples to shared memory
+        for (int i = threadIdx.x; i < A.S * xgw; i += nthr) {
+            const int gg = i / xgw, c = i % xgw;
+            const int bb = min(unit * A.S + gg, A.B - 1);
+            R v = 0;
+            if (c < A.Px) v = A.x[(size_t)bb * A.Px + c];
+            else if (MODE == 1) v = A.gE[(size_t)bb * n + (c - A.Px)];
+            xg_all[i] = v;
+        }
+        __syncthreads();
+        const R* xrow = xg_all + (size_t)q.g * xgw;
 
         // per-sample table (x-dependent runs): threads of the CTA over (sample, entry)
         for (int i = threadIdx.x; i < A.S * A.n_ps; i += nthr) {
             const int gg = i / A.n_ps, k = i % A.n_ps;
-            const int bb = min(unit * A.S + gg, A.B - 1);
             const int id = vqc_ld(&P.ps_list[k]);
             const DEntry e = P.entries[id];
-            eval_entry<R>(e, P.consts, A.x + (size_t)bb * A.Px, A.w, Pcang, Pcmat,
+            eval_entry<R>(e, P.consts, xg_all + (size_t)gg * xgw, w_sm, Pcang, Pcmat,
                           ps_all + ((size_t)gg * A.n_ps + e.slot) * 8);
         }
         // initial / final state from global memory (coalesced, into swizzled slots)
@@ -1031,7 +1047,7 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                 v = stage_view<K>(sp, q.t + bj * q.T, q.h, sg);
                 if (s == ns - 1) {
                     if (!recompute || A.bpt > 1) block_load<R, K>(a, psi, v.swb, sg);
-                    lambda_init<R, K>(sp, v.pb, A.gE + (size_t)b * n, n, a, l);
+                    lambda_init<R, K>(sp, v.pb, xrow + A.Px, n, a, l);
                 } else {
                     block_load<R, K>(a, psi, v.swb, sg);
                     block_load<R, K>(l, lam, v.swb, sg);
@@ -1051,10 +1067,8 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
         for (int i = threadIdx.x; i < A.S * A.n_accs; i += nthr) {
             const int gg = i / A.n_accs, k = i % A.n_accs;
             const DAcc ac = P.accs[k];
-            const int bb = min(unit * A.S + gg, A.B - 1);
-            const R* xg = A.x ? A.x + (size_t)bb * A.Px : nullptr;
             acc_terms<R>(ac, P.entries[ac.entry], acc_all + ((size_t)gg * A.n_accs + k) * q.wg * 8,
-                         q.wg, P.consts, xg, A.w, Pcang, Pcmat,
+                         q.wg, P.consts, xg_all + (size_t)gg * xgw, w_sm, Pcang, Pcmat,
                          terms_all + (size_t)gg * A.n_terms);
         }
         __syncthreads();
@@ -1085,25 +1099,27 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
     }
 
     if (MODE == 1 && A.Pw > 0 && A.dw) {
-        // per-CTA partial, then the last CTA to finish sums all partials in
-        // block order (deterministic for a given grid).
+        // per-CTA partial of dw; reduce_cols sums the partials in CTA order
         for (int p = threadIdx.x; p < A.Pw; p += nthr)
             A.dw_part[(size_t)blockIdx.x * A.Pw + p] = dw_cta[p];
-        __threadfence();
-        __shared__ unsigned last;
-        __syncthreads();
-        if (threadIdx.x == 0) last = atomicInc(A.counter, gridDim.x - 1) == gridDim.x - 1;
-        __syncthreads();
-        if (last) {
-            __threadfence();
-            for (int p = threadIdx.x; p < A.Pw; p += nthr) {
-                R sum = 0;
-                for (int k = 0; k < (int)gridDim.x; ++k)
-                    sum += __ldcg(&A.dw_part[(size_t)k * A.Pw + p]);
-                A.dw[p] = sum;
-            }
-        }
     }
+}
+
+// out[c] = sum over rows r of part[r * cols + c]: one block per column,
+// fixed strided partial sums, then a fixed-shape tree (deterministic).
+template <typename R>
+__global__ void __launch_bounds__(256) reduce_cols(const R* part, int rows, int cols, R* out) {
+    __shared__ R buf[256];
+    const int c = blockIdx.x;
+    R s = 0;
+    for (int r = threadIdx.x; r < rows; r += 256) s += part[(size_t)r * cols + c];
+    buf[threadIdx.x] = s;
+    __syncthreads();
+    for (int w = 128; w >= 1; w >>= 1) {
+        if (threadIdx.x < w) buf[threadIdx.x] += buf[threadIdx.x + w];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) out[c] = buf[0];
 }
 
 }  // namespace vqc
