@@ -339,25 +339,36 @@ def info_digest():
 
 
 def extra_configs(torch, Circuit, B):
-    """Forward and fwd+bwd evaluations/s of the other workloads (quick, device-timed)."""
+    """Forward and fwd+bwd evaluations/s and roofline fractions of the other
+    workloads (device time, L2 flushed before each timed call)."""
     from paper_2607_11985_gb300 import workloads as wl
+    pk, _ = peaks()
+    fp32 = fp32_peak_tflops(pk.get("sm_max_mhz", SM_MAX_MHZ))
+    hbm = pk.get("hbm_gbs", 6800.0)
     res = {}
     flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
-    for k in (1, 3, 4):
+    cases = [("cfg1", 1, None), ("cfg3", 3, None), ("cfg4", 4, None), ("cfg5_c64", 5, "c64"),
+             ("cfg5_c128", 5, "c128")]
+    for key, k, dt in cases:
         try:
-            ws_ = wl.config(k)[:4] if k == 4 else wl.config(k)
-            tot_f, tot_b, evals, flops_f, flops_b = 0.0, 0.0, 0, 0.0, 0.0
+            ws_ = wl.config(k, dtype=dt)
+            tot_f = tot_b = 0.0
+            evals = 0
+            work_f = work_b = 0.0
+            path = None
             for w_ in ws_:
-                c = Circuit(w_.spec, "c64")
+                real = torch.float32 if w_.dtype == "c64" else torch.float64
+                c = Circuit(w_.spec, w_.dtype)
                 inf = c.info(w_.batch)
-                x = torch.tensor(w_.x, dtype=torch.float32, device="cuda")
-                w = torch.tensor(w_.w, dtype=torch.float32, device="cuda") if w_.spec.num_w else None
-                gE = torch.tensor(w_.gE, dtype=torch.float32, device="cuda")
+                path = "hbm-tiled" if inf["fwd_path"] == 1 else "resident"
+                x = torch.tensor(w_.x, dtype=real, device="cuda")
+                w = torch.tensor(w_.w, dtype=real, device="cuda") if w_.spec.num_w else None
+                gE = torch.tensor(w_.gE, dtype=real, device="cuda")
                 E, st = c.forward(x, w, want_state=True)
                 if w_.backward:
                     c.backward(x, w, gE, psi_final=st)
                 torch.cuda.synchronize()
-                n_rep = 5
+                n_rep = 3 if k == 5 else 5
                 for _ in range(n_rep):
                     flush.zero_()
                     a, b2, d = (torch.cuda.Event(enable_timing=True) for _ in range(3))
@@ -371,17 +382,30 @@ def extra_configs(torch, Circuit, B):
                     tot_f += a.elapsed_time(b2) / 1e3
                     tot_b += b2.elapsed_time(d) / 1e3
                 evals += n_rep * w_.batch
-                flops_f += n_rep * w_.batch * inf["fwd_flops_per_eval"]
-                if w_.backward:
-                    flops_b += n_rep * w_.batch * inf["bwd_flops_per_eval"]
+                if path == "hbm-tiled":
+                    work_f += n_rep * w_.batch * inf["fwd_hbm_bytes_per_eval"]
+                    work_b += n_rep * w_.batch * inf["bwd_hbm_bytes_per_eval"] if w_.backward else 0
+                else:
+                    work_f += n_rep * w_.batch * inf["fwd_flops_per_eval"]
+                    work_b += n_rep * w_.batch * inf["bwd_flops_per_eval"] if w_.backward else 0
                 del c
-            res["cfg%d" % k] = {"fwd_evals_per_s": evals / tot_f,
-                                "fwd_tflops": flops_f / tot_f / 1e12,
-                                "fwd_bwd_evals_per_s": (evals / (tot_f + tot_b)) if flops_b else None,
-                                "bwd_tflops": (flops_b / tot_b / 1e12) if flops_b else None,
-                                "circuits": len(ws_)}
+            r = {"path": path, "circuits": len(ws_), "batch": ws_[0].batch,
+                 "qubits": sorted({w_.spec.n for w_ in ws_}), "dtype": ws_[0].dtype,
+                 "fwd_evals_per_s": evals / tot_f,
+                 "fwd_bwd_evals_per_s": (evals / (tot_f + tot_b)) if work_b else None}
+            if path == "hbm-tiled":
+                r["fwd_gbs"] = work_f / tot_f / 1e9
+                r["bwd_gbs"] = work_b / tot_b / 1e9 if work_b else None
+                r["fwd_frac_hbm"] = r["fwd_gbs"] / hbm
+                r["bwd_frac_hbm"] = r["bwd_gbs"] / hbm if work_b else None
+            else:
+                r["fwd_tflops"] = work_f / tot_f / 1e12
+                r["bwd_tflops"] = work_b / tot_b / 1e12 if work_b else None
+                r["fwd_frac_fp32"] = r["fwd_tflops"] / fp32
+                r["bwd_frac_fp32"] = r["bwd_tflops"] / fp32 if work_b else None
+            res[key] = r
         except Exception as e:   # report, do not hide
-            res["cfg%d" % k] = {"error": str(e)[:200]}
+            res[key] = {"error": str(e)[:200]}
     return res
 
 
