@@ -106,6 +106,28 @@ int env_int(const char* name, int dflt) {
     return v && *v ? std::atoi(v) : dflt;
 }
 
+// Launch with programmatic stream serialisation: the kernel may be scheduled
+// while the previous kernel in the stream finishes, and waits for it (every
+// kernel calls grid_dep_wait() before touching caller memory), which hides most
+// of the launch gap between the back-to-back kernels of one call and between
+// consecutive calls.  VQC_PDL=0 turns it off (plain stream order).
+cudaError_t launch(const void* fn, dim3 grid, dim3 block, void** args, size_t smem,
+                   cudaStream_t stream) {
+    static const bool pdl = env_int("VQC_PDL", 1) != 0;
+    if (!pdl) return cudaLaunchKernel(fn, grid, block, args, smem, stream);
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelExC(&cfg, fn, args);
+}
+
 // Pick the register-block size: the largest K that still gives the batch
 // enough threads to cover every SM's schedulers (>= 152 * 4 warps), but not
 // below 3 (a block of 8 amplitudes) where the circuit allows it.
@@ -144,9 +166,10 @@ vqc_status plan_launch_uncached(const HostPlan& p, int mode, int B, Launch& L) {
     L.wg = L.T > 32 ? L.T / 32 : 1;
     // Shared memory: a fixed part per CTA and a part per resident sample.
     const size_t dim = (size_t)1 << p.n;
-    const size_t fixed = align16((size_t)p.n_sh * 8 * rs) + align16(mode == 1 ? (size_t)p.num_w * rs : 0) +
+    const size_t ew = dbl ? 8 : 32;   // reals per table entry
+    const size_t fixed = align16((size_t)p.n_sh * ew * rs) + align16(mode == 1 ? (size_t)p.num_w * rs : 0) +
                          align16((size_t)p.num_w * rs) + 10 * 16;
-    const size_t per_sample = (size_t)p.n_ps * 8 * rs + dim * cs * (mode == 1 ? 2 : 1) +
+    const size_t per_sample = (size_t)p.n_ps * ew * rs + dim * cs * (mode == 1 ? 2 : 1) +
                               (size_t)(p.num_x + p.n) * rs +
                               (mode == 1 ? p.accs.size() * L.wg * 8 * rs + p.term_src.size() * rs
                                          : (size_t)L.wg * p.n * rs);
@@ -174,8 +197,8 @@ vqc_status plan_launch_uncached(const HostPlan& p, int mode, int B, Launch& L) {
         off = align16(off + bytes);
         return (int)o;
     };
-    L.sm_sh = take((size_t)p.n_sh * 8 * rs);
-    L.sm_ps = take((size_t)L.S * p.n_ps * 8 * rs);
+    L.sm_sh = take((size_t)p.n_sh * ew * rs);
+    L.sm_ps = take((size_t)L.S * p.n_ps * ew * rs);
     L.sm_psi = take((size_t)L.S * dim * cs);
     L.sm_lam = take(mode == 1 ? (size_t)L.S * dim * cs : 0);
     L.sm_acc = take(mode == 1 ? (size_t)L.S * p.accs.size() * L.wg * 8 * rs : 0);
@@ -375,13 +398,13 @@ vqc_status run(const HostPlan& p, int mode, int B, const void* x, const void* w,
         a.dw_part = reinterpret_cast<R*>(static_cast<char*>(ws) + 256);
     }
     void* args[] = {&a};
-    VQC_CUDA(cudaLaunchKernel(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
+    VQC_CUDA(launch(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
     if (mode == 1 && dw && p.num_w > 0) {
         const R* part = a.dw_part;
         int rows = L.grid, cols = p.num_w;
         R* out = static_cast<R*>(dw);
         void* rargs[] = {&part, &rows, &cols, &out};
-        VQC_CUDA(cudaLaunchKernel(reduce_cols_ptr(p.dtype == VQC_C128), dim3(cols), dim3(256), rargs,
+        VQC_CUDA(launch(reduce_cols_ptr(p.dtype == VQC_C128), dim3(cols), dim3(256), rargs,
                                   0, stream));
     }
     return VQC_OK;
@@ -422,8 +445,9 @@ vqc_status plan_hbm_uncached(const HostPlan& p, int mode, int B, PassGeo& L) {
         acc_max = std::max(acc_max, ps.acc_count);
     }
     const size_t tdim = (size_t)1 << m;
-    const size_t fixed = align16((size_t)sh_max * 8 * rs) + 8 * 16 + 1024;   // + tile-copy offsets
-    const size_t per_tile = (size_t)ps_max * 8 * rs + tdim * cs * (mode == 1 ? 2 : 1) +
+    const size_t ew = dbl ? 8 : 32;   // reals per table entry
+    const size_t fixed = align16((size_t)sh_max * ew * rs) + 8 * 16 + 1024;   // + tile-copy offsets
+    const size_t per_tile = (size_t)ps_max * ew * rs + tdim * cs * (mode == 1 ? 2 : 1) +
                             (mode == 1 ? (size_t)acc_max * L.wg * 8 * rs : (size_t)L.wg * p.n * rs);
     int S = std::max(1, 128 / L.T);
     if ((size_t)di.smem_optin <= fixed + per_tile)
@@ -441,8 +465,8 @@ vqc_status plan_hbm_uncached(const HostPlan& p, int mode, int B, PassGeo& L) {
         off = align16(off + bytes);
         return (int)o;
     };
-    L.sm_sh = take((size_t)sh_max * 8 * rs);
-    L.sm_ps = take((size_t)S * ps_max * 8 * rs);
+    L.sm_sh = take((size_t)sh_max * ew * rs);
+    L.sm_ps = take((size_t)S * ps_max * ew * rs);
     L.sm_psi = take((size_t)S * tdim * cs);
     L.sm_lam = take(mode == 1 ? (size_t)S * tdim * cs : 0);
     L.sm_acc = take(mode == 1 ? (size_t)S * acc_max * L.wg * 8 * rs : 0);
@@ -590,7 +614,7 @@ vqc_status run_hbm_forward(const HostPlan& p, int B, const void* x, const void* 
         a.dst_psi = (last && want_E && !state_out) ? nullptr : W;
         a.E_part = (last && want_E) ? E_part : nullptr;
         void* args[] = {&a};
-        VQC_CUDA(cudaLaunchKernel(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
+        VQC_CUDA(launch(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
     }
     if (want_E) {
         const R* Ep = E_part;
@@ -598,7 +622,7 @@ vqc_status run_hbm_forward(const HostPlan& p, int B, const void* x, const void* 
         int Bi = B, nt = L.ntiles, n = p.n;
         void* args[] = {&Ep, &Bi, &nt, &n, &Eo};
         const int blocks = (int)std::min<long long>(4096, ((long long)B * n + 255) / 256);
-        VQC_CUDA(cudaLaunchKernel(reduce_expz_ptr(p.dtype == VQC_C128), dim3(std::max(blocks, 1)),
+        VQC_CUDA(launch(reduce_expz_ptr(p.dtype == VQC_C128), dim3(std::max(blocks, 1)),
                                   dim3(256), args, 0, stream));
     }
     return VQC_OK;
@@ -637,7 +661,7 @@ vqc_status run_hbm_backward(const HostPlan& p, int B, const void* x, const void*
             a.src_psi = i == 0 ? static_cast<const C*>(psi0) : Psi;
             a.dst_psi = Psi;
             void* args[] = {&a};
-            VQC_CUDA(cudaLaunchKernel(Lf.fn, dim3(Lf.grid), dim3(Lf.block), args, Lf.smem, stream));
+            VQC_CUDA(launch(Lf.fn, dim3(Lf.grid), dim3(Lf.block), args, Lf.smem, stream));
         }
         src0 = Psi;
     }
@@ -656,7 +680,7 @@ vqc_status run_hbm_backward(const HostPlan& p, int B, const void* x, const void*
         a.dst_lam = last ? nullptr : Lam;
         a.terms = terms;
         void* args[] = {&a};
-        VQC_CUDA(cudaLaunchKernel(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
+        VQC_CUDA(launch(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
     }
     const char* base = static_cast<const char*>(p.dbuf);
     const bool dbl = p.dtype == VQC_C128;
@@ -669,7 +693,7 @@ vqc_status run_hbm_backward(const HostPlan& p, int B, const void* x, const void*
         R* o = static_cast<R*>(dx);
         void* args[] = {&t, &Bi, &ntl, &nt, &ptr, &occ, &Px, &o};
         const int blocks = (int)std::min<long long>(4096, ((long long)B * Px + 255) / 256);
-        VQC_CUDA(cudaLaunchKernel(reduce_dx_ptr(dbl), dim3(std::max(blocks, 1)), dim3(256), args, 0,
+        VQC_CUDA(launch(reduce_dx_ptr(dbl), dim3(std::max(blocks, 1)), dim3(256), args, 0,
                                   stream));
     }
     if (dw && p.num_w > 0) {
@@ -679,7 +703,7 @@ vqc_status run_hbm_backward(const HostPlan& p, int B, const void* x, const void*
         const int32_t* occ = reinterpret_cast<const int32_t*>(base + p.dev_wocc);
         R* o = static_cast<R*>(dw);
         void* args[] = {&t, &rows, &nt, &ptr, &occ, &o};
-        VQC_CUDA(cudaLaunchKernel(reduce_dw_ptr(dbl), dim3(p.num_w), dim3(256), args, 0, stream));
+        VQC_CUDA(launch(reduce_dw_ptr(dbl), dim3(p.num_w), dim3(256), args, 0, stream));
     }
     return VQC_OK;
 }

@@ -298,7 +298,7 @@ uint32_t op_need(const HOp& o) {
 // HBM path).
 void cut_stages(const HostPlan& p, const std::vector<int>& ops, const std::vector<int>& tile,
                 int K, Schedule& s, const std::vector<int>& slot_of,
-                const std::vector<int>& acc_of) {
+                const std::vector<int>& acc_of, bool absorb) {
     const int G = p.G_swz;
     std::vector<int> lpos(p.n, -1);   // tile-local bit of each global qubit
     uint32_t tile_mask = 0;
@@ -307,13 +307,24 @@ void cut_stages(const HostPlan& p, const std::vector<int>& ops, const std::vecto
         tile_mask |= 1u << tile[i];
     }
     std::vector<int> remaining = ops;
+    bool last_perm = false;
     do {   // an empty op list still gets one (empty) stage
-        uint32_t active = 0, blocked = 0;
-        std::vector<int> taken, deferred;
+        uint32_t active = 0, blocked = 0, pend = 0;
+        std::vector<int> taken, deferred, perm;
         for (int oi : remaining) {
             const HOp& o = p.ops[oi];
             uint32_t touch = op_touch(o), need = op_need(o);
             if (touch & blocked) {
+                blocked |= touch;
+                deferred.push_back(oi);
+                continue;
+            }
+            if (absorb && o.type == OP_CX) {   // folded into this stage's store map
+                pend |= touch;
+                perm.push_back(oi);
+                continue;
+            }
+            if (touch & pend) {   // would have to run after an absorbed CX
                 blocked |= touch;
                 deferred.push_back(oi);
                 continue;
@@ -370,6 +381,34 @@ void cut_stages(const HostPlan& p, const std::vector<int>& ops, const std::vecto
             st.tau[i] = (int32_t)swz(1u << lpos[order[i]], G);
             st.tmask[i] = 1u << order[i];
         }
+        // Store map: the image of each basis index under the absorbed CX gates.
+        auto pi = [&](uint32_t v) {
+            for (int oi : perm) {
+                const HOp& o = p.ops[oi];
+                if ((v >> o.q0) & 1) v ^= 1u << o.q1;
+            }
+            return v;
+        };
+        auto tile_local = [&](uint32_t v) {
+            uint32_t u = 0;
+            for (size_t i = 0; i < tile.size(); ++i)
+                if ((v >> tile[i]) & 1) u |= 1u << i;
+            return u;
+        };
+        const size_t mb = s.store_masks.size();
+        s.store_masks.resize(mb + kMaxK + kMaxThreadBits, 0);
+        for (int k = 0; k < K; ++k) {
+            const uint32_t v = pi(1u << st.active[k]);
+            st.sigma_st[k] = (int32_t)swz(tile_local(v), G);
+            s.store_masks[mb + k] = v;
+        }
+        for (size_t i = 0; i < order.size(); ++i) {
+            const uint32_t v = pi(1u << order[i]);
+            st.tau_st[i] = (int32_t)swz(tile_local(v), G);
+            s.store_masks[mb + kMaxK + i] = v;
+        }
+        st.nperm = (uint8_t)std::min<size_t>(perm.size(), 255);
+        last_perm = !perm.empty();
         auto local = [&](int q) -> int {
             for (int k = 0; k < K; ++k)
                 if (st.active[k] == q) return k;
@@ -423,7 +462,9 @@ void cut_stages(const HostPlan& p, const std::vector<int>& ops, const std::vecto
         st.op_end = (int32_t)s.ops.size();
         s.stages.push_back(st);
         remaining.swap(deferred);
-    } while (!remaining.empty());
+        // The last stage computes <Z> / lambda from its registers, in the frame
+        // before its store map: a trailing permutation gets one more (empty) stage.
+    } while (!remaining.empty() || last_perm);
     (void)tile_mask;
 }
 
@@ -437,7 +478,7 @@ void build_schedule(const HostPlan& p, Schedule& s) {
     std::iota(tile.begin(), tile.end(), 0);
     for (size_t i = 0; i < p.entries.size(); ++i) slot_of[i] = p.entries[i].slot;
     std::iota(acc_of.begin(), acc_of.end(), 0);
-    cut_stages(p, ops, tile, s.K, s, slot_of, acc_of);
+    cut_stages(p, ops, tile, s.K, s, slot_of, acc_of, true);
 }
 
 // HBM path: passes over tiles of m qubits (always containing the low qubits
@@ -513,7 +554,7 @@ void build_hbm_schedule(const HostPlan& p, Schedule& s) {
                 s.pass_accs.push_back(p.entries[o.entry].acc);
             }
         }
-        cut_stages(p, taken, tile, s.K, s, slot_of, acc_of);
+        cut_stages(p, taken, tile, s.K, s, slot_of, acc_of, false);
         ps.stage_end = (int32_t)s.stages.size();
         s.passes.push_back(ps);
         remaining.swap(deferred);
@@ -638,7 +679,7 @@ const Schedule* find_hbm_schedule(const HostPlan& p, int mode) {
 
 std::vector<uint8_t> export_plan(const HostPlan& p) {
     std::vector<uint8_t> out = {'V', 'Q', 'C', 'P'};
-    put_i32(out, 1);
+    put_i32(out, 2);   // export format version
     for (int v : {p.n, p.num_x, p.num_w, p.dtype, p.num_gates_in, p.G_swz, p.n_ps, p.n_sh,
                   p.n_runs})
         put_i32(out, v);
@@ -670,6 +711,7 @@ std::vector<uint8_t> export_plan(const HostPlan& p) {
         put_vec(out, s.passes);
         put_vec(out, s.pass_entries);
         put_vec(out, s.pass_accs);
+        put_vec(out, s.store_masks);
     }
     return out;
 }

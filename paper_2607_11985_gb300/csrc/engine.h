@@ -35,6 +35,10 @@ struct Schedule {
     std::vector<DPass> passes;            // HBM path: one record per pass
     std::vector<int32_t> pass_entries;    // HBM path: table entries per pass (ps, then sh)
     std::vector<int32_t> pass_accs;       // HBM path: accumulator ids per pass
+    // Per stage, kMaxK + kMaxThreadBits physical-index masks: the image under
+    // the stage's absorbed permutation of each local bit, then of each thread
+    // bit (exported for tests; the kernels use the swizzled store map).
+    std::vector<uint32_t> store_masks;
     size_t dev_ops = 0, dev_stages = 0;   // byte offsets inside the device buffer
     size_t dev_passes = 0, dev_pass_entries = 0, dev_pass_accs = 0;
     size_t dev_region_begin = 0, dev_region_end = 0;   // [ops .. pass_accs] in the blob

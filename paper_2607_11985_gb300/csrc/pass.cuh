@@ -142,6 +142,8 @@ __global__ void __launch_bounds__(256) pass_kernel(const __grid_constant__ PArgs
         smt = t;
         sms = u;
     }
+    grid_dep_wait();
+    grid_dep_launch();
     const DOp* P_ops = rebase(A.ops, A.plan, A.sched_off, sms);
     const DStage* P_stages = rebase(A.stages, A.plan, A.sched_off, sms);
     const int32_t* P_pass_entries = rebase(A.pass_entries, A.plan, A.sched_off, sms);
@@ -184,13 +186,13 @@ __global__ void __launch_bounds__(256) pass_kernel(const __grid_constant__ PArgs
 
     for (int i = threadIdx.x; i < A.sh_count; i += nthr) {
         const DEntry e = P_entries[vqc_ld(&P_pass_entries[A.sh_begin + i])];
-        eval_entry<R>(e, P_consts, nullptr, A.w, P_cang, P_cmat, sh_tab + 8 * i);
+        eval_entry<R>(e, P_consts, nullptr, A.w, P_cang, P_cmat, sh_tab + EntryWords<R>::value * i);
     }
     __syncthreads();
 
     C2<R>* psi = psi_all + (size_t)q.g * tdim;
     C2<R>* lam = lam_all + (size_t)q.g * tdim;
-    R* ps_tab = ps_all + (size_t)q.g * A.ps_count * 8;
+    R* ps_tab = ps_all + (size_t)q.g * A.ps_count * EntryWords<R>::value;
     R* acc = acc_all + (size_t)q.g * A.acc_count * q.wg * 8;
 
     for (long long unit = blockIdx.x; unit < A.nunits; unit += gridDim.x) {
@@ -209,7 +211,7 @@ __global__ void __launch_bounds__(256) pass_kernel(const __grid_constant__ PArgs
             const int bb = (int)(tt / A.ntiles);
             const DEntry e = P_entries[vqc_ld(&P_pass_entries[A.ps_begin + k])];
             eval_entry<R>(e, P_consts, A.x + (size_t)bb * A.Px, A.w, P_cang, P_cmat,
-                          ps_all + ((size_t)gg * A.ps_count + k) * 8);
+                          ps_all + ((size_t)gg * A.ps_count + k) * EntryWords<R>::value);
         }
         const size_t sbase = (size_t)b << n;
         const uint32_t gt = tile_global(u_t, tile_base, A.tile_q, G);
@@ -232,7 +234,7 @@ __global__ void __launch_bounds__(256) pass_kernel(const __grid_constant__ PArgs
                 } else {
                     block_load<R, K>(a, psi, v.swb, sg);
                 }
-                run_ops<R, K, 0>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
+                run_ops<R, K, 0, true>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
                                  sh_tab, ps_tab, nullptr, q, lane, warp_in_group);
                 if (s + 1 < A.stage_end || A.dst_psi) {
                     block_store<R, K>(a, psi, v.swb, sg);
@@ -268,7 +270,7 @@ __global__ void __launch_bounds__(256) pass_kernel(const __grid_constant__ PArgs
                 lambda_init<R, K>(sp, v.pb, A.gE + (size_t)b * n, n, a, l);
             else
                 block_load<R, K>(l, lam, v.swb, sg);
-            run_ops<R, K, 1>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l, sh_tab,
+            run_ops<R, K, 1, true>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l, sh_tab,
                              ps_tab, acc, q, lane, warp_in_group);
             if (s > A.stage_begin || A.dst_psi) {
                 block_store<R, K>(a, psi, v.swb, sg);
@@ -298,6 +300,8 @@ __global__ void __launch_bounds__(256) pass_kernel(const __grid_constant__ PArgs
 // E[b, j] = sum over tiles of E_part[b * ntiles + tau, j]  (fixed order).
 template <typename R>
 __global__ void reduce_expz(const R* E_part, int B, int ntiles, int n, R* E) {
+    grid_dep_wait();
+    grid_dep_launch();
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < (long long)B * n;
          i += (long long)gridDim.x * blockDim.x) {
         const long long b = i / n, j = i % n;
@@ -311,6 +315,8 @@ __global__ void reduce_expz(const R* E_part, int B, int ntiles, int n, R* E) {
 template <typename R>
 __global__ void reduce_dx(const R* terms, int B, int ntiles, int nt, const int32_t* ptr,
                           const int32_t* occ, int Px, R* dx) {
+    grid_dep_wait();
+    grid_dep_launch();
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < (long long)B * Px;
          i += (long long)gridDim.x * blockDim.x) {
         const long long b = i / Px;
@@ -331,6 +337,8 @@ __global__ void __launch_bounds__(256) reduce_dw(const R* terms, long long rows,
                                                  const int32_t* ptr, const int32_t* occ, R* dw) {
     __shared__ R part[256];
     const int p = blockIdx.x;
+    grid_dep_wait();
+    grid_dep_launch();
     const int k0 = vqc_ld(&ptr[p]), k1 = vqc_ld(&ptr[p + 1]);
     R s = 0;
     for (long long r = threadIdx.x; r < rows; r += 256) {

@@ -71,15 +71,28 @@ struct DOp {
 static_assert(sizeof(DOp) == 8, "DOp layout");
 
 // ---- stages ----------------------------------------------------------------
+// A stage loads each block through its load map (sigma, tau), applies its ops
+// and stores the block through its store map (sigma_st, tau_st).  On the
+// resident path the compiler folds CX gates into the store map instead of
+// emitting them as ops: a CX is a permutation of basis states, linear over
+// GF(2) in the amplitude index, so storing amplitude k of the block at the slot
+// of pi(k) applies it at no arithmetic cost (pi = the stage's absorbed CX gates
+// in time order; every op of the stage that follows one of them in time acts on
+// other qubits, so it commutes with pi).  Without absorbed gates the two maps
+// are equal.
 struct DStage {
     int32_t op_begin, op_end;
-    int32_t sigma[kMaxK];             // swizzled slot offset of local bit j
-    int32_t tau[kMaxThreadBits];      // swizzled slot offset of thread bit i
+    int32_t sigma[kMaxK];             // load: swizzled slot offset of local bit j
+    int32_t tau[kMaxThreadBits];      // load: swizzled slot offset of thread bit i
     uint32_t tmask[kMaxThreadBits];   // physical-index bit of thread bit i
+    int32_t sigma_st[kMaxK];          // store: slot offset of pi(local bit j)
+    int32_t tau_st[kMaxThreadBits];   // store: slot offset of pi(thread bit i)
     uint8_t active[kMaxK];            // physical qubit of local bit j
     uint8_t nthreadbits;
-    uint8_t pad[2];
+    uint8_t nperm;                    // CX gates absorbed into the store map
+    uint8_t pad;
 };
+static_assert(sizeof(DStage) == 248, "DStage layout");
 
 // ---- table entries and their constituents ----------------------------------
 enum ConstKind : uint8_t {

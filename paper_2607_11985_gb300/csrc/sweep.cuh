@@ -87,6 +87,39 @@ __device__ __forceinline__ void copy_region(unsigned char* dst, const unsigned c
     for (int i = threadIdx.x; i < bytes / 16; i += blockDim.x) d[i] = s[i];
 }
 
+// Asynchronous global -> shared copies (cp.async, 4/8/16 bytes, both addresses
+// aligned to the size).  They hold no registers while in flight, so a thread
+// can issue all of a CTA's staging loads before the first wait; async_wait()
+// then blocks until this thread's copies have landed (a __syncthreads must
+// follow before other threads read them).
+template <int BYTES>
+__device__ __forceinline__ void async_copy(void* sdst, const void* gsrc) {
+    const unsigned sa = static_cast<unsigned>(__cvta_generic_to_shared(sdst));
+    asm volatile("cp.async.ca.shared.global [%0], [%1], %2;\n" ::"r"(sa), "l"(gsrc), "n"(BYTES)
+                 : "memory");
+}
+__device__ __forceinline__ void async_wait() { asm volatile("cp.async.wait_all;\n" ::: "memory"); }
+
+__device__ __forceinline__ void async_region(unsigned char* dst, const unsigned char* src, int bytes) {
+    for (int i = threadIdx.x; i < bytes / 16; i += blockDim.x) async_copy<16>(dst + 16 * i, src + 16 * i);
+}
+template <typename T>
+__device__ __forceinline__ void async_elem(T* sdst, const T* gsrc) {
+    async_copy<sizeof(T)>(sdst, gsrc);
+}
+
+// Programmatic dependent launch.  Every kernel of the library is launched so
+// that it may start while the previous kernel in the stream is finishing; it
+// reads and writes no caller memory (inputs, outputs, workspace) before
+// grid_dep_wait(), which returns once that kernel has completed and its writes
+// are visible (immediately when the launch had no such predecessor).  Only the
+// plan, which no kernel writes, is read before it.  grid_dep_launch() then lets
+// the next kernel in the stream begin its own prologue.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() {
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+}
+
 // Pointer into the shared copy of a plan region (or the global one).
 template <typename T>
 __device__ __forceinline__ const T* rebase(const T* g, const unsigned char* plan, int region_off,
@@ -161,6 +194,29 @@ struct PlanPtrs {
 };
 
 // ---------------------------------------------------------------- tables
+// Reals per table entry.  complex64 stores each 2x2 run matrix U twice in the
+// operand form of the packed-FP32 update (see m1_apply_f2): U at [0, 16) and
+// U^dag at [16, 32), each as (Re, Re), (-Im, Im) pairs of its four entries.
+// complex128 stores U once (8 reals).  Phase entries use the first 8 reals.
+template <typename R> struct EntryWords { static constexpr int value = sizeof(R) == 4 ? 32 : 8; };
+
+template <typename R>
+__device__ __forceinline__ void store_matrix(const M2<R>& m, R* out) {
+    if constexpr (sizeof(R) == 4) {
+        const C2<R> e[4] = {m.a, m.b, m.c, m.d};
+        const C2<R> d[4] = {cconj<R>(m.a), cconj<R>(m.c), cconj<R>(m.b), cconj<R>(m.d)};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            out[4 * k + 0] = e[k].x; out[4 * k + 1] = e[k].x;
+            out[4 * k + 2] = -e[k].y; out[4 * k + 3] = e[k].y;
+            out[16 + 4 * k + 0] = d[k].x; out[16 + 4 * k + 1] = d[k].x;
+            out[16 + 4 * k + 2] = -d[k].y; out[16 + 4 * k + 3] = d[k].y;
+        }
+    } else {
+        out[0] = m.a.x; out[1] = m.a.y; out[2] = m.b.x; out[3] = m.b.y;
+        out[4] = m.c.x; out[5] = m.c.y; out[6] = m.d.x; out[7] = m.d.y;
+    }
+}
 template <typename R>
 __device__ __forceinline__ R angle_of(uint8_t src, int32_t idx, const R* xb, const R* w,
                                       const R* cang) {
@@ -217,8 +273,7 @@ __device__ void eval_entry(const DEntry& e, const DConst* consts, const R* xb, c
         const DConst c = consts[e.cfirst + k];
         m = mmul<R>(constituent<R>(c, xb, w, cang, cmat), m);
     }
-    out[0] = m.a.x; out[1] = m.a.y; out[2] = m.b.x; out[3] = m.b.y;
-    out[4] = m.c.x; out[5] = m.c.y; out[6] = m.d.x; out[7] = m.d.y;
+    store_matrix<R>(m, out);
 }
 
 template <typename R>
@@ -309,6 +364,48 @@ __device__ __forceinline__ void m1_rho_f2(const float2 (&ps)[1 << K], const floa
     }
     r[0] = r00.x; r[1] = r00.y; r[2] = r01.x; r[3] = r01.y;
     r[4] = r10.x; r[5] = r10.y; r[6] = r11.x; r[7] = r11.y;
+}
+
+// complex64 2x2 update with the operand pairs read directly from a table entry
+// (w: 8 float2 = (Re a, Re a), (-Im a, Im a), (Re b, Re b), ... ).
+template <int K, int T>
+__device__ __forceinline__ void m1_apply_f2w(float2 (&a)[1 << K], const float* wp) {
+    const float4 w0 = *reinterpret_cast<const float4*>(wp);
+    const float4 w1 = *reinterpret_cast<const float4*>(wp + 4);
+    const float4 w2 = *reinterpret_cast<const float4*>(wp + 8);
+    const float4 w3 = *reinterpret_cast<const float4*>(wp + 12);
+    const float2 ar = make_float2(w0.x, w0.y), ai = make_float2(w0.z, w0.w);
+    const float2 br = make_float2(w1.x, w1.y), bi = make_float2(w1.z, w1.w);
+    const float2 cr = make_float2(w2.x, w2.y), ci = make_float2(w2.z, w2.w);
+    const float2 dr = make_float2(w3.x, w3.y), di = make_float2(w3.z, w3.w);
+#pragma unroll
+    for (int p = 0; p < (1 << (K - 1)); ++p) {
+        const int i0 = pair_lo<T>(p), i1 = i0 | (1 << T);
+        const float2 u = a[i0], v = a[i1];
+        const float2 us = make_float2(u.y, u.x), vs = make_float2(v.y, v.x);
+        float2 nu = __fmul2_rn(ar, u);
+        nu = __ffma2_rn(ai, us, nu);
+        nu = __ffma2_rn(br, v, nu);
+        nu = __ffma2_rn(bi, vs, nu);
+        float2 nv = __fmul2_rn(cr, u);
+        nv = __ffma2_rn(ci, us, nv);
+        nv = __ffma2_rn(dr, v, nv);
+        nv = __ffma2_rn(di, vs, nv);
+        a[i0] = nu;
+        a[i1] = nv;
+    }
+}
+
+// Apply the table entry at tp (forward: U; adjoint: U^dag).
+template <typename R, int K, int T, bool ADJ>
+__device__ __forceinline__ void m1_entry(C2<R> (&a)[1 << K], const R* tp) {
+    if constexpr (sizeof(R) == 4) {
+        m1_apply_f2w<K, T>(a, tp + (ADJ ? 16 : 0));
+    } else {
+        M2<R> m = load_m2<R>(tp);
+        if (ADJ) m = mdag<R>(m);
+        m1_apply<R, K, T>(a, m);
+    }
 }
 
 // Packed-FP32 variants for complex64, plain FMA for complex128.
@@ -592,6 +689,21 @@ __device__ __forceinline__ StageView stage_view(const DStage* sp, int t, int h, 
     return v;
 }
 
+// Slot base of thread t and the local offsets of a stage's load map (ST false)
+// or store map (ST true), read from the stage record.
+template <int K, bool ST>
+__device__ __forceinline__ uint32_t map_base(const DStage* sp, int t, int h, int32_t (&sg)[K]) {
+    const int32_t* sig = ST ? sp->sigma_st : sp->sigma;
+    const int32_t* ta = ST ? sp->tau_st : sp->tau;
+#pragma unroll
+    for (int j = 0; j < K; ++j) sg[j] = vqc_ld(&sig[j]);
+    const int nb = vqc_ld(&sp->nthreadbits);
+    uint32_t b = (uint32_t)h;
+    for (int i = 0; i < nb; ++i)
+        if ((t >> i) & 1) b ^= (uint32_t)vqc_ld(&ta[i]);
+    return b;
+}
+
 template <typename R, int K>
 __device__ __forceinline__ void block_load(C2<R> (&a)[1 << K], const C2<R>* st, uint32_t swb,
                                            const int32_t (&sg)[K]) {
@@ -639,32 +751,33 @@ __device__ __forceinline__ bool physbit(uint32_t pb, int ref) {
 // Apply op `raw` to the block(s).  MODE 0: forward on a.  MODE 1: backward --
 // accumulate the op's gradient slot, then un-apply on a (psi) and l (lam).
 // One switch over the dispatch code; every case has fixed local positions.
-template <typename R, int K, int MODE>
+// WITH_CX: the schedule may hold CX ops (HBM passes); resident schedules fold
+// every CX into stage store maps, and leaving those cases out of the switch
+// keeps the other cases' register allocation tight.
+template <typename R, int K, int MODE, bool WITH_CX>
 __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 << K],
                                          C2<R> (&l)[1 << K], const R* sh_tab, const R* ps_tab,
                                          R* acc, const Geo& q, int lane, int warp_in_group,
                                          bool acc_add) {
     const int code = raw.x & 0xff, ra = (raw.x >> 8) & 0xff, rb = (raw.x >> 16) & 0xff;
     const int flags = raw.x >> 24, slot = raw.y & 0xffff, aux = raw.y >> 16;
-    const R* tp = ((flags & OPF_PER_SAMPLE) ? ps_tab : sh_tab) + 8 * slot;
+    const R* tp = ((flags & OPF_PER_SAMPLE) ? ps_tab : sh_tab) + EntryWords<R>::value * slot;
     R* accp = acc + ((size_t)aux * q.wg + warp_in_group) * 8;
     const int rlane = q.lanes < 32 ? q.t : lane;
     switch (code) {
 #define VQC_M1(T_)                                                                   \
     case DC_M1 + T_:                                                                 \
         if constexpr (T_ < K) {                                                      \
-            const M2<R> m = load_m2v<R>(tp);                                         \
             if (MODE == 0) {                                                         \
-                m1_go<R, K, T_>(a, m);                                               \
+                m1_entry<R, K, T_, false>(a, tp);                                    \
             } else {                                                                 \
                 if (flags & OPF_HAS_ACC) {                                           \
                     R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};                              \
                     rho_go<R, K, T_>(a, l, rh);                                      \
-                    reduce8_store<R>(rh, q.lanes, rlane, accp, q.mask, acc_add);              \
+                    reduce8_store<R>(rh, q.lanes, rlane, accp, q.mask, acc_add);     \
                 }                                                                    \
-                const M2<R> md = mdag<R>(m);                                         \
-                m1_go<R, K, T_>(a, md);                                              \
-                m1_go<R, K, T_>(l, md);                                              \
+                m1_entry<R, K, T_, true>(a, tp);                                     \
+                m1_entry<R, K, T_, true>(l, tp);                                     \
             }                                                                        \
         }                                                                            \
         break;
@@ -672,7 +785,7 @@ __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 <<
 #undef VQC_M1
 #define VQC_CXLL(C_, T_)                                                             \
     case DC_CX_LL + 4 * C_ + (T_ < C_ ? T_ : T_ - 1):                                \
-        if constexpr (C_ < K && T_ < K) {                                            \
+        if constexpr (WITH_CX && C_ < K && T_ < K) {                                 \
             cx_ll<R, K, C_, T_>(a);                                                  \
             if (MODE == 1) cx_ll<R, K, C_, T_>(l);                                   \
         }                                                                            \
@@ -685,7 +798,7 @@ __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 <<
 #undef VQC_CXLL
 #define VQC_CXPL(T_)                                                                 \
     case DC_CX_PL + T_:                                                              \
-        if constexpr (T_ < K) {                                                      \
+        if constexpr (WITH_CX && T_ < K) {                                           \
             const bool p_ = physbit(pb, ra);                                         \
             x_pred<R, K, T_>(a, p_);                                                 \
             if (MODE == 1) x_pred<R, K, T_>(l, p_);                                  \
@@ -744,31 +857,23 @@ __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 <<
     }
 }
 
-// Run ops [ob, oe) of a stage (forward: in order; backward: reversed), with the
-// next op's descriptor fetched while the current one executes.
-template <typename R, int K, int MODE>
+// Run ops [ob, oe) of a stage (forward: in order; backward: reversed).  The
+// descriptor is read when the op starts: keeping a prefetched one live across
+// the dispatch switch costs more registers than the load latency it hides.
+template <typename R, int K, int MODE, bool WITH_CX>
 __device__ __forceinline__ void run_ops(const DOp* ops, int ob, int oe, uint32_t pb,
                                         C2<R> (&a)[1 << K], C2<R> (&l)[1 << K], const R* sh_tab,
                                         const R* ps_tab, R* acc, const Geo& q, int lane,
                                         int warp_in_group, bool acc_add = false) {
     const uint2* op2 = reinterpret_cast<const uint2*>(ops);
-    if (ob >= oe) return;
     if (MODE == 0) {
-        uint2 nxt = vqc_ld(op2 + ob);
-        for (int o = ob; o < oe; ++o) {
-            const uint2 raw = nxt;
-            if (o + 1 < oe) nxt = vqc_ld(op2 + o + 1);
-            apply_op<R, K, MODE>(raw, pb, a, l, sh_tab, ps_tab, acc, q, lane, warp_in_group,
-                                 acc_add);
-        }
+        for (int o = ob; o < oe; ++o)
+            apply_op<R, K, MODE, WITH_CX>(vqc_ld(op2 + o), pb, a, l, sh_tab, ps_tab, acc, q, lane,
+                                          warp_in_group, acc_add);
     } else {
-        uint2 nxt = vqc_ld(op2 + oe - 1);
-        for (int o = oe - 1; o >= ob; --o) {
-            const uint2 raw = nxt;
-            if (o > ob) nxt = vqc_ld(op2 + o - 1);
-            apply_op<R, K, MODE>(raw, pb, a, l, sh_tab, ps_tab, acc, q, lane, warp_in_group,
-                                 acc_add);
-        }
+        for (int o = oe - 1; o >= ob; --o)
+            apply_op<R, K, MODE, WITH_CX>(vqc_ld(op2 + o), pb, a, l, sh_tab, ps_tab, acc, q, lane,
+                                          warp_in_group, acc_add);
     }
 }
 
@@ -891,16 +996,67 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
     R* dw_cta = reinterpret_cast<R*>(smem + A.sm_dw);
     R* red_all = reinterpret_cast<R*>(smem + A.sm_red);
 
+    const int n = A.n, G = A.G;
+    const int dim = 1 << n;
+    Geo q;
+    q.T = A.tpg;
+    q.lanes = q.T < 32 ? q.T : 32;
+    q.wg = q.T > 32 ? q.T / 32 : 1;
+    q.g = threadIdx.x / q.T;
+    q.t = threadIdx.x % q.T;
+    q.h = 0;
+    if (A.tbits < G) q.h = ((q.g & ((1 << (G - A.tbits)) - 1)) << A.tbits) & (dim - 1);
+    q.mask = blockDim.x >= 32 ? 0xffffffffu : ((1u << blockDim.x) - 1u);
+    const int lane = q.t & 31;
+    const int warp_in_group = q.t >> 5;
+    const int nthr = blockDim.x;
+
+    R* w_sm = reinterpret_cast<R*>(smem + A.sm_w);
+    R* xg_all = reinterpret_cast<R*>(smem + A.sm_xg);
+    const int xgw = A.Px + n;   // row width of the x / gE staging area
+    C2<R>* psi = psi_all + (size_t)q.g * dim;
+    C2<R>* lam = lam_all + (size_t)q.g * dim;
+
+    // initial (forward) or final (backward) state source; null: |0...0>
+    const C2<R>* src = MODE == 1 ? A.psi_final : A.psi0;
+    if (MODE == 1 && !src) src = A.psi0;
+    const bool from_global = src != nullptr;
+
+    // One unit's inputs to shared memory, asynchronously: x (and, backward,
+    // gE) rows of its samples and each sample's initial / final state
+    // (coalesced reads, swizzled slots).
+    auto stage_unit = [&](int unit) {
+        for (int i = threadIdx.x; i < A.S * xgw; i += nthr) {
+            const int gg = i / xgw, c = i % xgw;
+            const int bb = min(unit * A.S + gg, A.B - 1);
+            if (c < A.Px) async_elem<R>(xg_all + i, A.x + (size_t)bb * A.Px + c);
+            else if (MODE == 1) async_elem<R>(xg_all + i, A.gE + (size_t)bb * n + (c - A.Px));
+        }
+        if (from_global) {
+            const int b = min(unit * A.S + q.g, A.B - 1);
+            const C2<R>* gs = src + (size_t)b * dim;
+            for (int u = q.t; u < dim; u += q.T) async_elem<C2<R>>(psi + (swz(u, G) ^ q.h), gs + u);
+        }
+    };
+
+    // Prologue: the plan regions, w and the first unit's inputs all in flight
+    // at once, one wait.
     const unsigned char* smt = nullptr;
     const unsigned char* sms = nullptr;
     if (A.plan_smem) {
         unsigned char* t = smem + A.sm_plan;
         unsigned char* u = t + ((A.tab_bytes + 15) & ~15);
-        copy_region(t, A.plan + A.tab_off, A.tab_bytes);
-        copy_region(u, A.plan + A.sched_off, A.sched_bytes);
+        async_region(t, A.plan + A.tab_off, A.tab_bytes);
+        async_region(u, A.plan + A.sched_off, A.sched_bytes);
         smt = t;
         sms = u;
     }
+    grid_dep_wait();
+    grid_dep_launch();
+    for (int i = threadIdx.x; i < A.Pw; i += nthr) async_elem<R>(w_sm + i, A.w + i);
+    if ((int)blockIdx.x < A.nunits) stage_unit(blockIdx.x);
+    if (MODE == 1)
+        for (int i = threadIdx.x; i < A.Pw; i += nthr) dw_cta[i] = 0;
     PlanPtrs P;
     P.ops = rebase(A.ops, A.plan, A.sched_off, sms);
     P.stages = rebase(A.stages, A.plan, A.sched_off, sms);
@@ -917,41 +1073,18 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
     P.wocc = rebase(A.wocc, A.plan, A.tab_off, smt);
     const R* Pcmat = reinterpret_cast<const R*>(P.cmat);
     const R* Pcang = reinterpret_cast<const R*>(P.cang);
-    if (A.plan_smem) __syncthreads();
-
-    const int n = A.n, G = A.G;
-    const int dim = 1 << n;
-    Geo q;
-    q.T = A.tpg;
-    q.lanes = q.T < 32 ? q.T : 32;
-    q.wg = q.T > 32 ? q.T / 32 : 1;
-    q.g = threadIdx.x / q.T;
-    q.t = threadIdx.x % q.T;
-    q.h = 0;
-    if (A.tbits < G) q.h = ((q.g & ((1 << (G - A.tbits)) - 1)) << A.tbits) & (dim - 1);
-    q.mask = blockDim.x >= 32 ? 0xffffffffu : ((1u << blockDim.x) - 1u);
-    const int lane = q.t & 31;
-    const int warp_in_group = q.t >> 5;
-    const int nthr = blockDim.x;
-
-    // w to shared memory (one parallel copy), then the shared table (w and
-    // constants) once per CTA
-    R* w_sm = reinterpret_cast<R*>(smem + A.sm_w);
-    R* xg_all = reinterpret_cast<R*>(smem + A.sm_xg);
-    const int xgw = A.Px + n;   // row width of the x / gE staging area
-    for (int i = threadIdx.x; i < A.Pw; i += nthr) w_sm[i] = A.w[i];
+    async_wait();
     __syncthreads();
-    for (int i = threadIdx.x; i < A.n_sh; i += nthr) {
+
+    // shared table (w and constants) once per CTA, on the CTA's last threads
+    // so that it runs beside the first unit's per-sample table
+    for (int i = nthr - 1 - threadIdx.x; i < A.n_sh; i += nthr) {
         const int id = vqc_ld(&P.sh_list[i]);
         const DEntry e = P.entries[id];
-        eval_entry<R>(e, P.consts, nullptr, w_sm, Pcang, Pcmat, sh_tab + 8 * e.slot);
+        eval_entry<R>(e, P.consts, nullptr, w_sm, Pcang, Pcmat, sh_tab + EntryWords<R>::value * e.slot);
     }
-    if (MODE == 1)
-        for (int i = threadIdx.x; i < A.Pw; i += nthr) dw_cta[i] = 0;
 
-    C2<R>* psi = psi_all + (size_t)q.g * dim;
-    C2<R>* lam = lam_all + (size_t)q.g * dim;
-    R* ps_tab = ps_all + (size_t)q.g * A.n_ps * 8;
+    R* ps_tab = ps_all + (size_t)q.g * A.n_ps * EntryWords<R>::value;
     R* acc = acc_all + (size_t)q.g * A.n_accs * q.wg * 8;
     R* terms = terms_all + (size_t)q.g * A.n_terms;
 
@@ -959,17 +1092,11 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
         const int b_raw = unit * A.S + q.g;
         const bool valid = b_raw < A.B;
         const int b = valid ? b_raw : A.B - 1;
-
-        // x (and, backward, gE) rows of this unit's samples to shared memory
-        for (int i = threadIdx.x; i < A.S * xgw; i += nthr) {
-            const int gg = i / xgw, c = i % xgw;
-            const int bb = min(unit * A.S + gg, A.B - 1);
-            R v = 0;
-            if (c < A.Px) v = A.x[(size_t)bb * A.Px + c];
-            else if (MODE == 1) v = A.gE[(size_t)bb * n + (c - A.Px)];
-            xg_all[i] = v;
+        if (unit != (int)blockIdx.x) {
+            stage_unit(unit);
+            async_wait();
+            __syncthreads();
         }
-        __syncthreads();
         const R* xrow = xg_all + (size_t)q.g * xgw;
 
         // per-sample table (x-dependent runs): threads of the CTA over (sample, entry)
@@ -978,15 +1105,7 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
             const int id = vqc_ld(&P.ps_list[k]);
             const DEntry e = P.entries[id];
             eval_entry<R>(e, P.consts, xg_all + (size_t)gg * xgw, w_sm, Pcang, Pcmat,
-                          ps_all + ((size_t)gg * A.n_ps + e.slot) * 8);
-        }
-        // initial / final state from global memory (coalesced, into swizzled slots)
-        const C2<R>* src = MODE == 1 ? A.psi_final : A.psi0;
-        if (MODE == 1 && !src) src = A.psi0;
-        const bool from_global = src != nullptr;
-        if (from_global) {
-            const C2<R>* gs = src + (size_t)b * dim;
-            for (int u = q.t; u < dim; u += q.T) psi[swz(u, G) ^ q.h] = gs[u];
+                          ps_all + ((size_t)gg * A.n_ps + e.slot) * EntryWords<R>::value);
         }
         __syncthreads();
 
@@ -1012,11 +1131,15 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                     } else {
                         block_load<R, K>(a, psi, v.swb, sg);
                     }
-                    run_ops<R, K, 0>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
+                    run_ops<R, K, 0, false>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
                                      sh_tab, ps_tab, nullptr, q, lane, warp_in_group);
                     if (MODE == 0 && last)   // <Z_j> partials from the final blocks
                         expz_partials<R, K>(sp, v.pb, a, n, red, q, warp_in_group, bj > 0);
-                    if (store) block_store<R, K>(a, psi, v.swb, sg);
+                    if (store) {   // through the store map (absorbed CX gates)
+                        int32_t s2[K];
+                        const uint32_t b2 = map_base<K, true>(sp, q.t + bj * q.T, q.h, s2);
+                        block_store<R, K>(a, psi, b2, s2);
+                    }
                 }
                 if (store) group_sync<R>(q);
             }
@@ -1048,15 +1171,19 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                 if (s == ns - 1) {
                     if (!recompute || A.bpt > 1) block_load<R, K>(a, psi, v.swb, sg);
                     lambda_init<R, K>(sp, v.pb, xrow + A.Px, n, a, l);
-                } else {
-                    block_load<R, K>(a, psi, v.swb, sg);
-                    block_load<R, K>(l, lam, v.swb, sg);
+                } else {   // the forward left this stage's output in its store map
+                    int32_t s2[K];
+                    const uint32_t b2 = map_base<K, true>(sp, q.t + bj * q.T, q.h, s2);
+                    block_load<R, K>(a, psi, b2, s2);
+                    block_load<R, K>(l, lam, b2, s2);
                 }
-                run_ops<R, K, 1>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l,
+                run_ops<R, K, 1, false>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l,
                                  sh_tab, ps_tab, acc, q, lane, warp_in_group, bj > 0);
-                if (s > 0) {
-                    block_store<R, K>(a, psi, v.swb, sg);
-                    block_store<R, K>(l, lam, v.swb, sg);
+                if (s > 0) {   // back to the stage's input layout (load map)
+                    int32_t s2[K];
+                    const uint32_t b2 = map_base<K, false>(sp, q.t + bj * q.T, q.h, s2);
+                    block_store<R, K>(a, psi, b2, s2);
+                    block_store<R, K>(l, lam, b2, s2);
                 }
             }
             group_sync<R>(q);
@@ -1111,6 +1238,8 @@ template <typename R>
 __global__ void __launch_bounds__(256) reduce_cols(const R* part, int rows, int cols, R* out) {
     __shared__ R buf[256];
     const int c = blockIdx.x;
+    grid_dep_wait();
+    grid_dep_launch();
     R s = 0;
     for (int r = threadIdx.x; r < rows; r += 256) s += part[(size_t)r * cols + c];
     buf[threadIdx.x] = s;

@@ -20,13 +20,13 @@ DACC = np.dtype([("entry", "<i4"), ("kind", "<i4")])
 DOP = np.dtype([("code", "u1"), ("a", "u1"), ("b", "u1"), ("flags", "u1"), ("slot", "<u2"),
                 ("aux", "<u2")])
 DSTAGE = np.dtype([("op_begin", "<i4"), ("op_end", "<i4"), ("sigma", "<i4", 5), ("tau", "<i4", 16),
-                   ("tmask", "<u4", 16), ("active", "u1", 5), ("nthreadbits", "u1"),
-                   ("pad", "u1", 2)])
+                   ("tmask", "<u4", 16), ("sigma_st", "<i4", 5), ("tau_st", "<i4", 16),
+                   ("active", "u1", 5), ("nthreadbits", "u1"), ("nperm", "u1"), ("pad", "u1")])
 DPASS = np.dtype([("stage_begin", "<i4"), ("stage_end", "<i4"), ("m", "<i4"), ("nout", "<i4"),
                   ("tile_q", "u1", 24), ("out_q", "u1", 24), ("ps_begin", "<i4"), ("ps_count", "<i4"),
                   ("sh_begin", "<i4"), ("sh_count", "<i4"), ("acc_begin", "<i4"), ("acc_count", "<i4")])
 assert DENTRY.itemsize == 12 and DCONST.itemsize == 16 and DOP.itemsize == 8
-assert DSTAGE.itemsize == 164 and DPASS.itemsize == 88
+assert DSTAGE.itemsize == 248 and DPASS.itemsize == 88
 PATH_RESIDENT, PATH_HBM = 0, 1
 
 OP_M1, OP_CX, OP_CZ, OP_PH2 = 1, 2, 3, 4
@@ -89,7 +89,7 @@ class Plan:
         assert blob[:4] == b"VQCP"
         r = Reader(blob)
         r.off = 4
-        assert r.i32() == 1
+        assert r.i32() == 2
         (self.n, self.num_x, self.num_w, self.dtype, self.num_gates_in, self.G, self.n_ps,
          self.n_sh, self.n_runs) = [r.i32() for _ in range(9)]
         self.hops = r.vec("<i4").reshape(-1, 5)
@@ -112,9 +112,10 @@ class Plan:
             passes = r.vec(DPASS)
             pass_entries = r.vec("<i4")
             pass_accs = r.vec("<i4")
+            store_masks = r.vec("<u4").reshape(len(stages), 5 + 16)
             self.scheds.append(dict(mode=mode, K=K, m=m, path=path, thread_bits=tb, ops=ops,
                                     stages=stages, passes=passes, pass_entries=pass_entries,
-                                    pass_accs=pass_accs))
+                                    pass_accs=pass_accs, store_masks=store_masks))
         assert r.off == len(blob)
 
     # ------------------------------------------------------------------ tables
@@ -173,6 +174,23 @@ class Plan:
         return base, idx
 
     @staticmethod
+    def store_index(masks, K, nthreadbits, t):
+        """Physical indices the block of thread t is stored to: the images of
+        its indices under the stage's absorbed permutation (XOR-linear)."""
+        base = 0
+        for i in range(int(nthreadbits)):
+            if (t >> i) & 1:
+                base ^= int(masks[5 + i])
+        idx = []
+        for r in range(1 << K):
+            v = base
+            for j in range(K):
+                if (r >> j) & 1:
+                    v ^= int(masks[j])
+            idx.append(v)
+        return np.array(idx)
+
+    @staticmethod
     def refbit(ref, r, base):
         ref, r, base = int(ref), int(r), int(base)
         return (base >> (ref - REF_PHYS)) & 1 if ref >= REF_PHYS else (r >> ref) & 1
@@ -217,7 +235,8 @@ class Plan:
         is one pass over one tile holding every qubit."""
         n = self.n
         if sched["path"] == PATH_RESIDENT:
-            yield sched["stages"], [0], self.tables(xb, w), np.arange(len(self.accs))
+            yield (sched["stages"], [0], self.tables(xb, w), np.arange(len(self.accs)),
+                   sched["store_masks"])
             return
         pe = sched["pass_entries"]
         for ps in sched["passes"]:
@@ -230,7 +249,8 @@ class Plan:
             for tau in range(1 << int(ps["nout"])):
                 bases.append(sum(((tau >> j) & 1) << int(out_q[j]) for j in range(int(ps["nout"]))))
             accmap = sched["pass_accs"][ps["acc_begin"]:ps["acc_begin"] + ps["acc_count"]]
-            yield sched["stages"][ps["stage_begin"]:ps["stage_end"]], bases, tabs, accmap
+            yield (sched["stages"][ps["stage_begin"]:ps["stage_end"]], bases, tabs, accmap,
+                   sched["store_masks"][ps["stage_begin"]:ps["stage_end"]])
 
     def forward(self, sched, xb, w, psi0=None):
         n, K = self.n, sched["K"]
@@ -239,9 +259,10 @@ class Plan:
             psi[0] = 1
         else:
             psi[:] = psi0
-        for stages, bases, tabs, _ in self.units(sched, xb, w):
+        for stages, bases, tabs, _, smasks in self.units(sched, xb, w):
             for tb in bases:
-                for st in stages:
+                for st, sm in zip(stages, smasks):
+                    new = psi.copy()
                     for t in range(1 << int(st["nthreadbits"])):
                         base, idx = self.block_index(st, K, t)
                         base |= tb
@@ -249,7 +270,8 @@ class Plan:
                         a = psi[idx].copy()
                         for op in sched["ops"][st["op_begin"]:st["op_end"]]:
                             self.apply_op(op, K, base, a, tabs)
-                        psi[idx] = a
+                        new[self.store_index(sm, K, st["nthreadbits"], t) | tb] = a
+                    psi = new
         return psi
 
     def backward(self, sched, xb, w, gEb, psi0=None):
@@ -261,15 +283,17 @@ class Plan:
         O = sum(gEb[j] * (1 - 2 * ((k >> j) & 1)) for j in range(n))
         lam = O * psi
         acc = np.zeros((len(self.accs), 8))
-        for stages, bases, tabs, accmap in list(self.units(sched, xb, w))[::-1]:
+        for stages, bases, tabs, accmap, smasks in list(self.units(sched, xb, w))[::-1]:
           for tb in bases:
-           for st in stages[::-1]:
+           for st, sm in list(zip(stages, smasks))[::-1]:
             ops = sched["ops"][st["op_begin"]:st["op_end"]]
+            npsi, nlam = psi.copy(), lam.copy()
             for t in range(1 << int(st["nthreadbits"])):
                 base, idx = self.block_index(st, K, t)
                 base |= tb
                 idx = idx | tb
-                a, l = psi[idx].copy(), lam[idx].copy()
+                sidx = self.store_index(sm, K, st["nthreadbits"], t) | tb
+                a, l = psi[sidx].copy(), lam[sidx].copy()
                 for op in ops[::-1]:
                     if op["flags"] & OPF_HAS_ACC:
                         if op_type(op)[0] == OP_M1:
@@ -292,7 +316,8 @@ class Plan:
                                 acc[accmap[op["aux"]], 0] += g * (np.conj(l[r]) * a[r]).imag
                     self.apply_op(op, K, base, a, tabs, adjoint=True)
                     self.apply_op(op, K, base, l, tabs, adjoint=True)
-                psi[idx], lam[idx] = a, l
+                npsi[idx], nlam[idx] = a, l
+            psi, lam = npsi, nlam
         terms = np.zeros(len(self.term_src))
         P = {CK_RX: np.array([[0, 1], [1, 0]], complex),
              CK_RY: np.array([[0, -1j], [1j, 0]]),

@@ -98,46 +98,64 @@ def test_export_deterministic_and_info():
         B.vqc_free(p2)
 
 
+def slot_of(st, K, t, r, sig, tau):
+    sl = 0
+    for i in range(int(st["nthreadbits"])):
+        if (t >> i) & 1:
+            sl ^= int(st[tau][i])
+    for j in range(K):
+        if (r >> j) & 1:
+            sl ^= int(st[sig][j])
+    return sl
+
+
 def check_addressing(plan):
+    """Load and store maps of every stage agree with the swizzle of the
+    indices the emulator assigns to each (thread, register) and are
+    bijections onto the tile's slots."""
     for s in plan.scheds:
         n, K, m = plan.n, s["K"], s["m"]
         if s["path"] == 0:
-            tiles = [(list(range(n)), s["stages"])]
+            tiles = [(list(range(n)), range(len(s["stages"])))]
         else:
-            tiles = [(list(ps["tile_q"][:ps["m"]]), s["stages"][ps["stage_begin"]:ps["stage_end"]])
+            tiles = [(list(ps["tile_q"][:ps["m"]]), range(ps["stage_begin"], ps["stage_end"]))
                      for ps in s["passes"]]
             # every pass's tile holds the low qubits of one 128-byte chunk
             for tq, _ in tiles:
                 assert tq[:min(plan.G, n)] == list(range(min(plan.G, n)))
-        for tq, stages in tiles:
-          tq = [int(q) for q in tq]
-          lpos = {q: i for i, q in enumerate(tq)}
-          for st in stages:
-            assert sorted(st["active"][:K].tolist()) == st["active"][:K].tolist()
-            assert set(st["active"][:K].tolist()) <= set(tq)
-            assert int(st["nthreadbits"]) == m - K
-            slots = set()
-            for t in range(1 << (m - K)):
-                base, idx = Plan.block_index(st, K, t)
-                swb = 0
-                for i in range(m - K):
-                    if (t >> i) & 1:
-                        swb ^= int(st["tau"][i])
-                for r in range(1 << K):
-                    sl = swb
-                    for j in range(K):
-                        if (r >> j) & 1:
-                            sl ^= int(st["sigma"][j])
-                    u = sum(((int(idx[r]) >> q) & 1) << lpos[q] for q in tq)
-                    assert sl == swz(u, plan.G)
-                    slots.add(sl)
-            assert slots == set(range(1 << m))
-            for op in s["ops"][st["op_begin"]:st["op_end"]]:
-                t, oa, ob = op_type(op)
-                if t == 1:
-                    assert oa < K
-                if t == 2:
-                    assert ob < K
+        for tq, srange in tiles:
+            tq = [int(q) for q in tq]
+            lpos = {q: i for i, q in enumerate(tq)}
+            local = lambda v: sum(((int(v) >> q) & 1) << lpos[q] for q in tq)
+            for si in srange:
+                st, sm = s["stages"][si], s["store_masks"][si]
+                assert sorted(st["active"][:K].tolist()) == st["active"][:K].tolist()
+                assert set(st["active"][:K].tolist()) <= set(tq)
+                assert int(st["nthreadbits"]) == m - K
+                slots, slots_st = set(), set()
+                for t in range(1 << (m - K)):
+                    _, idx = Plan.block_index(st, K, t)
+                    sidx = Plan.store_index(sm, K, st["nthreadbits"], t)
+                    for r in range(1 << K):
+                        sl = slot_of(st, K, t, r, "sigma", "tau")
+                        assert sl == swz(local(idx[r]), plan.G)
+                        slots.add(sl)
+                        sl = slot_of(st, K, t, r, "sigma_st", "tau_st")
+                        assert sl == swz(local(sidx[r]), plan.G)
+                        slots_st.add(sl)
+                assert slots == set(range(1 << m)) and slots_st == slots
+                if int(st["nperm"]) == 0:
+                    assert list(st["sigma_st"][:K]) == list(st["sigma"][:K])
+                    assert list(st["tau_st"]) == list(st["tau"])
+                for op in s["ops"][st["op_begin"]:st["op_end"]]:
+                    t, oa, ob = op_type(op)
+                    if t == 1:
+                        assert oa < K
+                    if t == 2:
+                        assert ob < K
+                        assert s["path"] == 1   # resident schedules fold every CX
+            if s["path"] == 0:   # <Z> / lambda come from the last stage's registers
+                assert int(s["stages"][-1]["nperm"]) == 0
 
 
 SMALL_CASES = [(s, n, g) for s, n, g in [(101, 1, 12), (102, 2, 30), (103, 3, 60), (104, 4, 80),
