@@ -129,7 +129,33 @@ __device__ __forceinline__ const T* rebase(const T* g, const unsigned char* plan
                                       (reinterpret_cast<const unsigned char*>(g) - plan - region_off));
 }
 
-__device__ __forceinline__ void sc(float t, float* s, float* c) { sincosf(t, s, c); }
+// sin and cos for complex64 table entries, written out so that the half-angle
+// evaluation is a short chain of FMAs: Cody-Waite reduction t = k pi/2 + r
+// with pi/2 split in three parts (the head has 8 significant bits, so k *
+// head is exact for |k| < 2^16), |r| <= pi/4, then the Taylor polynomials of
+// sin (through r^9) and cos (through r^10), whose truncation errors on
+// [-pi/4, pi/4] are below 2e-9, and the quadrant of k.  complex128 uses the
+// library routine.
+__device__ __forceinline__ void sc(float t, float* s, float* c) {
+    const float k = rintf(t * 0.636619772367581343f);   // t / (pi/2)
+    float r = fmaf(-k, 1.5703125f, t);
+    r = fmaf(-k, 4.838267923332751e-4f, r);
+    r = fmaf(-k, 2.5633440682570896e-12f, r);
+    const float r2 = r * r;
+    float ps = fmaf(r2, 2.75573192239858907e-6f, -1.98412698412698413e-4f);   // 1/9!, -1/7!
+    ps = fmaf(r2, ps, 8.33333333333333333e-3f);                               // 1/5!
+    ps = fmaf(r2, ps, -1.66666666666666667e-1f);                              // -1/3!
+    const float sr = fmaf(r * r2, ps, r);
+    float pc = fmaf(r2, -2.75573192239858907e-7f, 2.48015873015873016e-5f);   // -1/10!, 1/8!
+    pc = fmaf(r2, pc, -1.38888888888888889e-3f);                              // -1/6!
+    pc = fmaf(r2, pc, 4.16666666666666667e-2f);                               // 1/4!
+    pc = fmaf(r2, pc, -0.5f);                                                 // -1/2!
+    const float cr = fmaf(r2, pc, 1.0f);
+    const int q = (int)k & 3;
+    const float sv = (q & 1) ? cr : sr, cv = (q & 1) ? sr : cr;
+    *s = (q & 2) ? -sv : sv;
+    *c = ((q + 1) & 2) ? -cv : cv;
+}
 __device__ __forceinline__ void sc(double t, double* s, double* c) { sincos(t, s, c); }
 
 // ---------------------------------------------------------------- kernel args
@@ -202,15 +228,14 @@ template <typename R> struct EntryWords { static constexpr int value = sizeof(R)
 
 template <typename R>
 __device__ __forceinline__ void store_matrix(const M2<R>& m, R* out) {
-    if constexpr (sizeof(R) == 4) {
+    if constexpr (sizeof(R) == 4) {   // 16-byte stores (entries are 128-byte aligned)
         const C2<R> e[4] = {m.a, m.b, m.c, m.d};
         const C2<R> d[4] = {cconj<R>(m.a), cconj<R>(m.c), cconj<R>(m.b), cconj<R>(m.d)};
+        float4* o4 = reinterpret_cast<float4*>(out);
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-            out[4 * k + 0] = e[k].x; out[4 * k + 1] = e[k].x;
-            out[4 * k + 2] = -e[k].y; out[4 * k + 3] = e[k].y;
-            out[16 + 4 * k + 0] = d[k].x; out[16 + 4 * k + 1] = d[k].x;
-            out[16 + 4 * k + 2] = -d[k].y; out[16 + 4 * k + 3] = d[k].y;
+            o4[k] = make_float4(e[k].x, e[k].x, -e[k].y, e[k].y);
+            o4[4 + k] = make_float4(d[k].x, d[k].x, -d[k].y, d[k].y);
         }
     } else {
         out[0] = m.a.x; out[1] = m.a.y; out[2] = m.b.x; out[3] = m.b.y;
@@ -227,7 +252,7 @@ __device__ __forceinline__ R angle_of(uint8_t src, int32_t idx, const R* xb, con
 
 // Matrix of one constituent of a run.
 template <typename R>
-__device__ M2<R> constituent(const DConst& c, const R* xb, const R* w, const R* cang,
+__device__ __forceinline__ M2<R> constituent(const DConst& c, const R* xb, const R* w, const R* cang,
                              const R* cmat) {
     M2<R> u;
     if (c.kind == CK_CONST) {
@@ -252,7 +277,7 @@ __device__ M2<R> constituent(const DConst& c, const R* xb, const R* w, const R* 
 
 // Evaluate one table entry (8 reals) for sample row xb.
 template <typename R>
-__device__ void eval_entry(const DEntry& e, const DConst* consts, const R* xb, const R* w,
+__device__ __forceinline__ void eval_entry(const DEntry& e, const DConst* consts, const R* xb, const R* w,
                            const R* cang, const R* cmat, R* out) {
     if (e.phase) {
         const DConst c = consts[e.cfirst];
