@@ -927,6 +927,64 @@ __device__ __forceinline__ void lambda_init(const DStage* sp, uint32_t pb, const
     }
 }
 
+// Adds this block's contributions to E_j = sum (-1)^{bit j} |a|^2 for qubits
+// j < NV into ez[j] (a qubit outside the block contributes +-(block norm) by
+// its bit in pb; entries j >= n stay untouched and are never read).
+template <typename R, int K, int NV>
+__device__ __forceinline__ void expz_accum(const DStage* sp, uint32_t pb, const C2<R> (&a)[1 << K],
+                                           R (&ez)[NV]) {
+    R ptot = 0;
+    R dloc[K];
+#pragma unroll
+    for (int j = 0; j < K; ++j) dloc[j] = 0;
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r) {
+        const R pr = fma(a[r].x, a[r].x, a[r].y * a[r].y);
+        ptot += pr;
+#pragma unroll
+        for (int j = 0; j < K; ++j) dloc[j] += ((r >> j) & 1) ? -pr : pr;
+    }
+    uint32_t actmask = 0;
+    int aq[K];
+#pragma unroll
+    for (int j = 0; j < K; ++j) {
+        aq[j] = vqc_ld(&sp->active[j]);
+        actmask |= 1u << aq[j];
+    }
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+        R val = ((pb >> j) & 1u) ? -ptot : ptot;
+#pragma unroll
+        for (int k = 0; k < K; ++k) val = aq[k] == j ? dloc[k] : val;
+        ez[j] += val;
+    }
+}
+
+// Sum NV values over the 32 lanes of a warp (reduce-scatter butterfly, NV - 1
+// + log2(32 / NV) shuffles).  Returns the value index this lane ends up with;
+// v[0] then holds that value's warp sum in every lane whose bits below the
+// scatter bits are zero (and in their partners).
+template <typename R, int NV>
+__device__ __forceinline__ int warp_reduce_scatter(R (&v)[NV], int lane) {
+    int idx = 0;
+    int m = 16;
+#pragma unroll
+    for (int w = NV; w > 1; w >>= 1, m >>= 1) {
+        const int u = (lane & m) ? 1 : 0;
+        const int h = w >> 1;
+#pragma unroll
+        for (int i = 0; i < h; ++i) {
+            const R send = u ? v[i] : v[i + h];
+            const R keep = u ? v[i + h] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, m);
+        }
+        idx = 2 * idx + u;
+    }
+#pragma unroll
+    for (; m >= 1; m >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], m);
+    return idx;
+}
+
 // Per-warp partial sums of E_j = sum (-1)^{bit j} |a|^2 over this group's
 // blocks, written to red[warp_in_group * n + j].
 template <typename R, int K>
@@ -1147,6 +1205,8 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                 const DStage* sp = P.stages + s;
                 const bool last = s + 1 == ns;
                 const bool store = !last || (MODE == 0 && A.state_out) || (MODE == 1 && A.bpt > 1);
+                R eacc = 0;   // full-warp groups: this lane's share of the warp's <Z> sums
+                int eidx = 0;
                 for (int bj = 0; bj < A.bpt; ++bj) {
                     v = stage_view<K>(sp, q.t + bj * q.T, q.h, sg);
                     if (s == 0 && !from_global) {
@@ -1158,12 +1218,42 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                     }
                     run_ops<R, K, 0, false>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
                                      sh_tab, ps_tab, nullptr, q, lane, warp_in_group);
-                    if (MODE == 0 && last)   // <Z_j> partials from the final blocks
-                        expz_partials<R, K>(sp, v.pb, a, n, red, q, warp_in_group, bj > 0);
+                    if (MODE == 0 && last) {   // <Z_j> partials from the final blocks
+                        if (q.lanes == 32) {   // butterfly over the warp (n <= 16 here)
+                            if (n <= 8) {
+                                R ez[8];
+#pragma unroll
+                                for (int j = 0; j < 8; ++j) ez[j] = 0;
+                                expz_accum<R, K, 8>(sp, v.pb, a, ez);
+                                eidx = warp_reduce_scatter<R, 8>(ez, lane);
+                                eacc += ez[0];
+                            } else {
+                                R ez[16];
+#pragma unroll
+                                for (int j = 0; j < 16; ++j) ez[j] = 0;
+                                expz_accum<R, K, 16>(sp, v.pb, a, ez);
+                                eidx = warp_reduce_scatter<R, 16>(ez, lane);
+                                eacc += ez[0];
+                            }
+                        } else {
+                            expz_partials<R, K>(sp, v.pb, a, n, red, q, warp_in_group, bj > 0);
+                        }
+                    }
                     if (store) {   // through the store map (absorbed CX gates)
                         int32_t s2[K];
                         const uint32_t b2 = map_base<K, true>(sp, q.t + bj * q.T, q.h, s2);
                         block_store<R, K>(a, psi, b2, s2);
+                    }
+                }
+                if (MODE == 0 && last && q.lanes == 32) {
+                    // a single-warp group writes E itself
+                    const int low = n <= 8 ? 3 : 1;   // lane bits below the scatter bits
+                    if ((lane & low) == 0 && eidx < n) {
+                        if (q.wg == 1) {
+                            if (valid) A.E[(size_t)b * n + eidx] = eacc;
+                        } else {
+                            red[warp_in_group * n + eidx] = eacc;
+                        }
                     }
                 }
                 if (store) group_sync<R>(q);
@@ -1171,19 +1261,24 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
         }
 
         if (MODE == 0) {
-            __syncthreads();
-            if (valid) {
-                for (int j = q.t; j < n; j += q.T) {
-                    R e = 0;
-                    for (int k = 0; k < q.wg; ++k) e += red[k * n + j];
-                    A.E[(size_t)b * n + j] = e;
-                }
-                if (A.state_out) {
-                    C2<R>* go = A.state_out + (size_t)b * dim;
-                    for (int u = q.t; u < dim; u += q.T) go[u] = psi[swz(u, G) ^ q.h];
+            const bool direct = q.lanes == 32 && q.wg == 1;   // E already written
+            if (!direct || A.state_out) {
+                __syncthreads();
+                if (valid) {
+                    if (!direct) {
+                        for (int j = q.t; j < n; j += q.T) {
+                            R e = 0;
+                            for (int k = 0; k < q.wg; ++k) e += red[k * n + j];
+                            A.E[(size_t)b * n + j] = e;
+                        }
+                    }
+                    if (A.state_out) {
+                        C2<R>* go = A.state_out + (size_t)b * dim;
+                        for (int u = q.t; u < dim; u += q.T) go[u] = psi[swz(u, G) ^ q.h];
+                    }
                 }
             }
-            __syncthreads();
+            if (unit + (int)gridDim.x < A.nunits) __syncthreads();
             continue;
         }
 
