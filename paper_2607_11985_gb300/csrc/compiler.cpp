@@ -319,7 +319,8 @@ void cut_stages(const HostPlan& p, const std::vector<int>& ops, const std::vecto
                 deferred.push_back(oi);
                 continue;
             }
-            if (absorb && o.type == OP_CX) {   // folded into this stage's store map
+            if (absorb && o.type == OP_CX && lpos[o.q0] >= 0 && lpos[o.q1] >= 0) {
+                // folded into this stage's store map (both qubits in the tile)
                 pend |= touch;
                 perm.push_back(oi);
                 continue;
@@ -554,7 +555,7 @@ void build_hbm_schedule(const HostPlan& p, Schedule& s) {
                 s.pass_accs.push_back(p.entries[o.entry].acc);
             }
         }
-        cut_stages(p, taken, tile, s.K, s, slot_of, acc_of, false);
+        cut_stages(p, taken, tile, s.K, s, slot_of, acc_of, true);
         ps.stage_end = (int32_t)s.stages.size();
         s.passes.push_back(ps);
         remaining.swap(deferred);

@@ -236,8 +236,10 @@ __global__ void __launch_bounds__(256) pass_kernel(const __grid_constant__ PArgs
                 }
                 run_ops<R, K, 0, true>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
                                  sh_tab, ps_tab, nullptr, q, lane, warp_in_group);
-                if (s + 1 < A.stage_end || A.dst_psi) {
-                    block_store<R, K>(a, psi, v.swb, sg);
+                if (s + 1 < A.stage_end || A.dst_psi) {   // store map: absorbed CX gates
+                    int32_t s2[K];
+                    const uint32_t b2 = map_base<K, true>(sp, q.t, q.h, s2);
+                    block_store<R, K>(a, psi, b2, s2);
                     group_sync<R>(q);
                 }
             }
@@ -265,16 +267,22 @@ __global__ void __launch_bounds__(256) pass_kernel(const __grid_constant__ PArgs
             C2<R> l[1 << K];
             v = stage_view<K>(sp, q.t, q.h, sg);
             v.pb |= tile_base;
-            block_load<R, K>(a, psi, v.swb, sg);
-            if (s == A.stage_end - 1 && !A.src_lam)
-                lambda_init<R, K>(sp, v.pb, A.gE + (size_t)b * n, n, a, l);
-            else
-                block_load<R, K>(l, lam, v.swb, sg);
+            {   // the forward left this stage's output in its store map
+                int32_t s2[K];
+                const uint32_t b2 = map_base<K, true>(sp, q.t, q.h, s2);
+                block_load<R, K>(a, psi, b2, s2);
+                if (s == A.stage_end - 1 && !A.src_lam)
+                    lambda_init<R, K>(sp, v.pb, A.gE + (size_t)b * n, n, a, l);
+                else
+                    block_load<R, K>(l, lam, b2, s2);
+            }
             run_ops<R, K, 1, true>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l, sh_tab,
                              ps_tab, acc, q, lane, warp_in_group);
-            if (s > A.stage_begin || A.dst_psi) {
-                block_store<R, K>(a, psi, v.swb, sg);
-                block_store<R, K>(l, lam, v.swb, sg);
+            if (s > A.stage_begin || A.dst_psi) {   // back to the stage's load map
+                int32_t s2[K];
+                const uint32_t b2 = map_base<K, false>(sp, q.t, q.h, s2);
+                block_store<R, K>(a, psi, b2, s2);
+                block_store<R, K>(l, lam, b2, s2);
             }
             group_sync<R>(q);
         }

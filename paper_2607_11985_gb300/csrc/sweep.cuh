@@ -658,6 +658,37 @@ __device__ __forceinline__ void reduce8_store(R (&v)[8], int lanes, int lane, R*
     }
 }
 
+// reduce8_store for a full warp, branch-free: 4 + 2 + 1 scatter shuffles and
+// 2 plain ones; lanes with (lane & 3) == 0 write their sum.
+template <typename R>
+__device__ __forceinline__ void reduce8_full(R (&v)[8], int lane, R* dst, bool add) {
+    const unsigned full = 0xffffffffu;
+    const int u0 = (lane >> 4) & 1, u1 = (lane >> 3) & 1, u2 = (lane >> 2) & 1;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const R send = u0 ? v[i] : v[i + 4];
+        const R keep = u0 ? v[i + 4] : v[i];
+        v[i] = keep + __shfl_xor_sync(full, send, 16);
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        const R send = u1 ? v[i] : v[i + 2];
+        const R keep = u1 ? v[i + 2] : v[i];
+        v[i] = keep + __shfl_xor_sync(full, send, 8);
+    }
+    {
+        const R send = u2 ? v[0] : v[1];
+        const R keep = u2 ? v[1] : v[0];
+        v[0] = keep + __shfl_xor_sync(full, send, 4);
+    }
+    v[0] += __shfl_xor_sync(full, v[0], 2);
+    v[0] += __shfl_xor_sync(full, v[0], 1);
+    if ((lane & 3) == 0) {
+        R* d = dst + 4 * u0 + 2 * u1 + u2;
+        *d = add ? *d + v[0] : v[0];
+    }
+}
+
 template <typename R>
 __device__ __forceinline__ R reduce1(R v, int lanes, unsigned mask) {
     for (int m = lanes >> 1; m >= 1; m >>= 1) v += shx<R>(v, m, mask);
@@ -796,13 +827,23 @@ __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 <<
             if (MODE == 0) {                                                         \
                 m1_entry<R, K, T_, false>(a, tp);                                    \
             } else {                                                                 \
-                if (flags & OPF_HAS_ACC) {                                           \
+                if ((flags & OPF_HAS_ACC) && q.lanes == 32) {                        \
+                    /* one basic block: the butterfly's shuffles can overlap  */     \
+                    /* the adjoint arithmetic                                 */     \
                     R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};                              \
                     rho_go<R, K, T_>(a, l, rh);                                      \
-                    reduce8_store<R>(rh, q.lanes, rlane, accp, q.mask, acc_add);     \
+                    m1_entry<R, K, T_, true>(a, tp);                                 \
+                    m1_entry<R, K, T_, true>(l, tp);                                 \
+                    reduce8_full<R>(rh, lane, accp, acc_add);                        \
+                } else {                                                             \
+                    if (flags & OPF_HAS_ACC) {                                       \
+                        R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};                          \
+                        rho_go<R, K, T_>(a, l, rh);                                  \
+                        reduce8_store<R>(rh, q.lanes, rlane, accp, q.mask, acc_add); \
+                    }                                                                \
+                    m1_entry<R, K, T_, true>(a, tp);                                 \
+                    m1_entry<R, K, T_, true>(l, tp);                                 \
                 }                                                                    \
-                m1_entry<R, K, T_, true>(a, tp);                                     \
-                m1_entry<R, K, T_, true>(l, tp);                                     \
             }                                                                        \
         }                                                                            \
         break;
