@@ -730,18 +730,28 @@ struct StageView {
     uint32_t swb, pb;
 };
 
+// XOR of the entries of v[0 .. 16) selected by the set bits of t, with all
+// loads independent (no loop-carried branch): a thread's slot base.  Entries
+// past the stage's thread bits are zero in the record, and t has no bits there.
+__device__ __forceinline__ uint32_t xor_select(const int32_t* v, int nb, int t) {
+    uint32_t b = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) b ^= ((t >> i) & 1) ? (uint32_t)vqc_ld(&v[i]) : 0u;
+    if (nb > 8) {
+#pragma unroll
+        for (int i = 8; i < kMaxThreadBits; ++i) b ^= ((t >> i) & 1) ? (uint32_t)vqc_ld(&v[i]) : 0u;
+    }
+    return b;
+}
+
 template <int K>
 __device__ __forceinline__ StageView stage_view(const DStage* sp, int t, int h, int32_t (&sg)[K]) {
 #pragma unroll
     for (int j = 0; j < K; ++j) sg[j] = vqc_ld(&sp->sigma[j]);
     const int nb = vqc_ld(&sp->nthreadbits);   // uint8 load
-    StageView v{(uint32_t)h, 0u};
-    for (int i = 0; i < nb; ++i) {
-        if ((t >> i) & 1) {
-            v.swb ^= (uint32_t)vqc_ld(&sp->tau[i]);
-            v.pb |= vqc_ld(&sp->tmask[i]);
-        }
-    }
+    StageView v;
+    v.swb = (uint32_t)h ^ xor_select(sp->tau, nb, t);
+    v.pb = xor_select(reinterpret_cast<const int32_t*>(sp->tmask), nb, t);   // disjoint bits
     return v;
 }
 
@@ -750,14 +760,10 @@ __device__ __forceinline__ StageView stage_view(const DStage* sp, int t, int h, 
 template <int K, bool ST>
 __device__ __forceinline__ uint32_t map_base(const DStage* sp, int t, int h, int32_t (&sg)[K]) {
     const int32_t* sig = ST ? sp->sigma_st : sp->sigma;
-    const int32_t* ta = ST ? sp->tau_st : sp->tau;
 #pragma unroll
     for (int j = 0; j < K; ++j) sg[j] = vqc_ld(&sig[j]);
     const int nb = vqc_ld(&sp->nthreadbits);
-    uint32_t b = (uint32_t)h;
-    for (int i = 0; i < nb; ++i)
-        if ((t >> i) & 1) b ^= (uint32_t)vqc_ld(&ta[i]);
-    return b;
+    return (uint32_t)h ^ xor_select(ST ? sp->tau_st : sp->tau, nb, t);
 }
 
 template <typename R, int K>
