@@ -1089,25 +1089,25 @@ __device__ void acc_terms(const DAcc& ac, const DEntry& e, const R* ap, int wg,
     R rr[8] = {0, 0, 0, 0, 0, 0, 0, 0};
     for (int k2 = 0; k2 < wg; ++k2)
         for (int c = 0; c < 8; ++c) rr[c] += ap[k2 * 8 + c];
-    // rho = [[r00, r01], [r10, r11]]; term = Im Tr(W P W^dag rho)
-    M2<R> W = mident<R>();
+    // rho = [[r00, r01], [r10, r11]] (pairs rr[0..1], rr[2..3], rr[4..5],
+    // rr[6..7]).  term_j = Im Tr(W_j P_j W_j^dag rho) = Im Tr(P_j rho_j) with
+    // rho_j = W_j^dag rho W_j, carried from the last constituent backwards:
+    // rho <- U^dag rho U after each one.
+    M2<R> rho;
+    rho.a = cm<R>(rr[0], rr[1]); rho.b = cm<R>(rr[2], rr[3]);
+    rho.c = cm<R>(rr[4], rr[5]); rho.d = cm<R>(rr[6], rr[7]);
     for (int c = e.ccount - 1; c >= 0; --c) {
         const DConst cn = consts[e.cfirst + c];
         if (cn.term >= 0) {
-            M2<R> P;
-            const C2<R> z = cm<R>(0, 0), one = cm<R>(1, 0);
-            if (cn.kind == CK_RX) { P.a = z; P.b = one; P.c = one; P.d = z; }
-            else if (cn.kind == CK_RY) { P.a = z; P.b = cm<R>(0, -1); P.c = cm<R>(0, 1); P.d = z; }
-            else { P.a = one; P.b = z; P.c = z; P.d = cm<R>(-1, 0); }
-            const M2<R> Mx = mmul<R>(mmul<R>(W, P), mdag<R>(W));
-            R im = 0;   // Im sum_{a,b} M[a][b] rho[b][a]
-            im += Mx.a.x * rr[1] + Mx.a.y * rr[0];
-            im += Mx.b.x * rr[5] + Mx.b.y * rr[4];
-            im += Mx.c.x * rr[3] + Mx.c.y * rr[2];
-            im += Mx.d.x * rr[7] + Mx.d.y * rr[6];
-            out[cn.term] = im;
+            // Im Tr(X rho) = Im r01 + Im r10, Im Tr(Y rho) = Re r01 - Re r10,
+            // Im Tr(Z rho) = Im r00 - Im r11
+            const R tx = rho.b.y + rho.c.y, ty = rho.b.x - rho.c.x, tz = rho.a.y - rho.d.y;
+            out[cn.term] = cn.kind == CK_RX ? tx : cn.kind == CK_RY ? ty : tz;
         }
-        W = mmul<R>(W, constituent<R>(cn, xg, w, cang, cmat));
+        if (c > 0) {
+            const M2<R> u = constituent<R>(cn, xg, w, cang, cmat);
+            rho = mmul<R>(mdag<R>(u), mmul<R>(rho, u));
+        }
     }
 }
 
