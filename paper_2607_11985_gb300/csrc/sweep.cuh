@@ -1373,19 +1373,25 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                 const int bb = unit * A.S + gg;
                 if (bb >= A.B) continue;
                 const R* tm = terms_all + (size_t)gg * A.n_terms;
+                const int k0 = vqc_ld(&P.xocc_ptr[p]), k1 = vqc_ld(&P.xocc_ptr[p + 1]);
                 R sum = 0;
-                for (int k = vqc_ld(&P.xocc_ptr[p]); k < vqc_ld(&P.xocc_ptr[p + 1]); ++k)
-                    sum += tm[vqc_ld(&P.xocc[k])];
+                for (int k = k0; k < k1; ++k) sum += tm[vqc_ld(&P.xocc[k])];
                 A.dx[(size_t)bb * A.Px + p] = sum;
             }
         }
+        const int nvalid = min(A.S, A.B - unit * A.S);
         for (int p = threadIdx.x; p < A.Pw; p += nthr) {
+            // samples in order, each sample's occurrences in order
+            const int k0 = vqc_ld(&P.wocc_ptr[p]), k1 = vqc_ld(&P.wocc_ptr[p + 1]);
             R sum = dw_cta[p];
-            for (int gg = 0; gg < A.S; ++gg) {
-                if (unit * A.S + gg >= A.B) break;
-                const R* tm = terms_all + (size_t)gg * A.n_terms;
-                for (int k = vqc_ld(&P.wocc_ptr[p]); k < vqc_ld(&P.wocc_ptr[p + 1]); ++k)
-                    sum += tm[vqc_ld(&P.wocc[k])];
+            if (k1 - k0 == 1) {   // the common case: independent loads
+                const int j = vqc_ld(&P.wocc[k0]);
+                for (int gg = 0; gg < nvalid; ++gg) sum += terms_all[(size_t)gg * A.n_terms + j];
+            } else {
+                for (int gg = 0; gg < nvalid; ++gg) {
+                    const R* tm = terms_all + (size_t)gg * A.n_terms;
+                    for (int k = k0; k < k1; ++k) sum += tm[vqc_ld(&P.wocc[k])];
+                }
             }
             dw_cta[p] = sum;
         }
