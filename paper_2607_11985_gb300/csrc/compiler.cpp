@@ -456,7 +456,13 @@ void cut_stages(const HostPlan& p, const std::vector<int>& ops, const std::vecto
             } else {
                 d.a = ref(o.q0);
                 d.b = ref(o.q1);
-                d.code = DC_PH2;
+                const bool la = d.a < kRefPhys, lb = d.b < kRefPhys;
+                if (la && lb)
+                    d.code = (uint8_t)(DC_PH2_LL + cz_pair_index(std::min(d.a, d.b), std::max(d.a, d.b)));
+                else if (la || lb)
+                    d.code = (uint8_t)(DC_PH2_PL + (la ? d.a : d.b));
+                else
+                    d.code = DC_PH2_PP;
             }
             s.ops.push_back(d);
         }

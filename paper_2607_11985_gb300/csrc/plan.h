@@ -53,8 +53,10 @@ enum DispatchCode : uint8_t {
     DC_CZ_LL = 30,   // + cz_pair_index(lo, hi): both qubits local
     DC_CZ_PL = 40,   // + l: local qubit l (ref a), other qubit outside the block (ref b)
     DC_CZ_PP = 45,   // both qubits outside the block
-    DC_PH2 = 46,     // diagonal two-qubit phase, refs a and b (local or not)
-    DC_NUM = 47
+    DC_PH2_LL = 46,  // + cz_pair_index(lo, hi): diagonal two-qubit phase, both qubits local
+    DC_PH2_PL = 56,  // + l: diagonal phase, one qubit local (position l), the other outside
+    DC_PH2_PP = 61,  // diagonal phase, both qubits outside the block
+    DC_NUM = 62
 };
 // Index of the local pair (lo < hi < 5) in (0,1),(0,2),(0,3),(0,4),(1,2),...,(3,4).
 constexpr int cz_pair_index(int lo, int hi) {

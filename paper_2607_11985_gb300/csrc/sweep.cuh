@@ -577,35 +577,6 @@ __device__ __forceinline__ int refbit(int ref, int r, uint32_t pb) {
     return ref >= kRefPhys ? (int)((pb >> (ref - kRefPhys)) & 1u) : ((r >> ref) & 1);
 }
 
-// Diagonal two-qubit phase: a[r] *= ph[bit a + 2 bit b]  (conj when ADJ).
-template <typename R, int K, bool ADJ>
-__device__ __forceinline__ void ph2_apply(int ra, int rb, uint32_t pb, C2<R> (&a)[1 << K],
-                                          const C2<R> (&ph)[4]) {
-#pragma unroll
-    for (int r = 0; r < (1 << K); ++r) {
-        const int s = refbit(ra, r, pb) + 2 * refbit(rb, r, pb);
-        C2<R> f = s == 0 ? ph[0] : s == 1 ? ph[1] : s == 2 ? ph[2] : ph[3];
-        if (ADJ) f.y = -f.y;
-        a[r] = cmul<R>(a[r], f);
-    }
-}
-
-// Im <lam|P|psi> over the block for the phase op's generator.
-template <typename R, int K>
-__device__ __forceinline__ R ph2_term(int ra, int rb, uint32_t pb, uint8_t flags,
-                                      const C2<R> (&ps)[1 << K], const C2<R> (&la)[1 << K]) {
-    R acc = 0;
-#pragma unroll
-    for (int r = 0; r < (1 << K); ++r) {
-        const int ba = refbit(ra, r, pb), bb = refbit(rb, r, pb);
-        R g;
-        if (flags & OPF_GEN_CRZ) g = ba ? (bb ? R(-1) : R(1)) : R(0);
-        else g = (ba ^ bb) ? R(-1) : R(1);
-        acc = fma(g, la[r].x * ps[r].y - la[r].y * ps[r].x, acc);
-    }
-    return acc;
-}
-
 // ---------------------------------------------------------------- reductions
 template <typename R>
 __device__ __forceinline__ R shx(R v, int m, unsigned mask) { return __shfl_xor_sync(mask, v, m); }
@@ -789,6 +760,107 @@ __device__ __forceinline__ void block_store(const C2<R> (&a)[1 << K], C2<R>* st,
     for (int r = 0; r < (1 << K); ++r) st[swb ^ block_off<K>(r, s2)] = a[r];
 }
 
+// Diagonal two-qubit phase (CRZ, RZZ): amplitude r is multiplied by ph[s],
+// s = bit a + 2 bit b (a, b = the gate's first and second qubit), conjugated in
+// the backward, where the gradient term Im <lam|P|psi> = sum_r g[s] Im(conj(lam_r)
+// psi_r) is taken first (g = the generator's diagonal: CRZ (0, 1, 0, -1), RZZ
+// (1, -1, -1, 1)).  Three forms by where a and b live; each resolves s per
+// amplitude at compile time except for one per-op selection.
+template <typename R>
+__device__ __forceinline__ void ph2_gen(uint8_t flags, R (&g)[4]) {
+    if (flags & OPF_GEN_CRZ) { g[0] = 0; g[1] = 1; g[2] = 0; g[3] = -1; }
+    else { g[0] = 1; g[1] = -1; g[2] = -1; g[3] = 1; }
+}
+template <typename R>
+__device__ __forceinline__ R gen_at(uint8_t flags, int s) {   // g[s] for a runtime s
+    if (flags & OPF_GEN_CRZ) return s == 1 ? R(1) : s == 3 ? R(-1) : R(0);
+    return (s == 0 || s == 3) ? R(1) : R(-1);
+}
+template <typename R>
+__device__ __forceinline__ R im_conj_mul(const C2<R>& la, const C2<R>& ps) {
+    return la.x * ps.y - la.y * ps.x;
+}
+template <typename R>
+__device__ __forceinline__ void ph2_term_store(R tv, const Geo& q, R* accp, bool acc_add) {
+    tv = reduce1<R>(tv, q.lanes, q.mask);
+    if ((q.t & (q.lanes - 1)) == 0) accp[0] = acc_add ? accp[0] + tv : tv;
+}
+template <typename R, int K, int MODE, int LO, int HI>
+__device__ __forceinline__ void ph2_ll(bool swapped, const R* tp, uint8_t flags,
+                                       C2<R> (&a)[1 << K], C2<R> (&l)[1 << K], const Geo& q,
+                                       R* accp, bool acc_add) {
+    // index by (bit LO) + 2 (bit HI): swap entries 1 and 2 when a is the higher position
+    C2<R> ph[4] = {cm<R>(tp[0], tp[1]), cm<R>(tp[2], tp[3]), cm<R>(tp[4], tp[5]), cm<R>(tp[6], tp[7])};
+    R g[4];
+    ph2_gen<R>(flags, g);
+    if (swapped) {
+        const C2<R> t = ph[1]; ph[1] = ph[2]; ph[2] = t;
+        const R u = g[1]; g[1] = g[2]; g[2] = u;
+    }
+    if (MODE == 1) {
+#pragma unroll
+        for (int s = 0; s < 4; ++s) ph[s].y = -ph[s].y;
+        if (flags & OPF_HAS_ACC) {
+            R tv = 0;
+#pragma unroll
+            for (int r = 0; r < (1 << K); ++r)
+                tv = fma(g[((r >> LO) & 1) + 2 * ((r >> HI) & 1)], im_conj_mul<R>(l[r], a[r]), tv);
+            ph2_term_store<R>(tv, q, accp, acc_add);
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r) {
+        const int s = ((r >> LO) & 1) + 2 * ((r >> HI) & 1);
+        a[r] = cmul<R>(a[r], ph[s]);
+        if (MODE == 1) l[r] = cmul<R>(l[r], ph[s]);
+    }
+}
+template <typename R, int K, int MODE, int L>
+__device__ __forceinline__ void ph2_pl(bool a_local, bool p, const R* tp, uint8_t flags,
+                                       C2<R> (&a)[1 << K], C2<R> (&l)[1 << K], const Geo& q,
+                                       R* accp, bool acc_add) {
+    // s = bit L + 2 p (a local) or p + 2 bit L (b local)
+    const int s0 = a_local ? 2 * (int)p : (int)p, s1 = a_local ? 1 + 2 * (int)p : (int)p + 2;
+    C2<R> f0 = cm<R>(tp[2 * s0], tp[2 * s0 + 1]), f1 = cm<R>(tp[2 * s1], tp[2 * s1 + 1]);
+    const R g0 = gen_at<R>(flags, s0), g1 = gen_at<R>(flags, s1);
+    if (MODE == 1) {
+        f0.y = -f0.y;
+        f1.y = -f1.y;
+        if (flags & OPF_HAS_ACC) {
+            R tv = 0;
+#pragma unroll
+            for (int r = 0; r < (1 << K); ++r)
+                tv = fma(((r >> L) & 1) ? g1 : g0, im_conj_mul<R>(l[r], a[r]), tv);
+            ph2_term_store<R>(tv, q, accp, acc_add);
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r) {
+        const C2<R> f = ((r >> L) & 1) ? f1 : f0;
+        a[r] = cmul<R>(a[r], f);
+        if (MODE == 1) l[r] = cmul<R>(l[r], f);
+    }
+}
+template <typename R, int K, int MODE>
+__device__ __forceinline__ void ph2_pp(int s, const R* tp, uint8_t flags, C2<R> (&a)[1 << K],
+                                       C2<R> (&l)[1 << K], const Geo& q, R* accp, bool acc_add) {
+    C2<R> f = cm<R>(tp[2 * s], tp[2 * s + 1]);
+    if (MODE == 1) {
+        f.y = -f.y;
+        if (flags & OPF_HAS_ACC) {
+            R tv = 0;
+#pragma unroll
+            for (int r = 0; r < (1 << K); ++r) tv += im_conj_mul<R>(l[r], a[r]);
+            ph2_term_store<R>(gen_at<R>(flags, s) * tv, q, accp, acc_add);
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r) {
+        a[r] = cmul<R>(a[r], f);
+        if (MODE == 1) l[r] = cmul<R>(l[r], f);
+    }
+}
+
 // ---------------------------------------------------------------- op dispatch
 template <typename R> __device__ __forceinline__ M2<R> load_m2v(const R* p);
 template <> __device__ __forceinline__ M2<float> load_m2v<float>(const float* p) {
@@ -908,22 +980,24 @@ __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 <<
         }
         break;
     }
-    case DC_PH2: {
-        C2<R> ph[4] = {cm<R>(tp[0], tp[1]), cm<R>(tp[2], tp[3]), cm<R>(tp[4], tp[5]),
-                       cm<R>(tp[6], tp[7])};
-        if (MODE == 0) {
-            ph2_apply<R, K, false>(ra, rb, pb, a, ph);
-        } else {
-            if (flags & OPF_HAS_ACC) {
-                R tv = ph2_term<R, K>(ra, rb, pb, (uint8_t)flags, a, l);
-                tv = reduce1<R>(tv, q.lanes, q.mask);
-                if ((q.t & (q.lanes - 1)) == 0) accp[0] = acc_add ? accp[0] + tv : tv;
-            }
-            ph2_apply<R, K, true>(ra, rb, pb, a, ph);
-            ph2_apply<R, K, true>(ra, rb, pb, l, ph);
-        }
+#define VQC_PH2LL(LO_, HI_)                                                          \
+    case DC_PH2_LL + cz_pair_index(LO_, HI_):                                        \
+        if constexpr (LO_ < K && HI_ < K) ph2_ll<R, K, MODE, LO_, HI_>(ra > rb, tp, flags, a, l, q, accp, acc_add); \
         break;
-    }
+        VQC_PH2LL(0, 1) VQC_PH2LL(0, 2) VQC_PH2LL(0, 3) VQC_PH2LL(0, 4)
+        VQC_PH2LL(1, 2) VQC_PH2LL(1, 3) VQC_PH2LL(1, 4)
+        VQC_PH2LL(2, 3) VQC_PH2LL(2, 4) VQC_PH2LL(3, 4)
+#undef VQC_PH2LL
+#define VQC_PH2PL(L_)                                                                \
+    case DC_PH2_PL + L_:                                                             \
+        if constexpr (L_ < K) ph2_pl<R, K, MODE, L_>(ra < kRefPhys, physbit(pb, ra < kRefPhys ? rb : ra), tp, flags, a, l, q, accp, acc_add); \
+        break;
+        VQC_PH2PL(0) VQC_PH2PL(1) VQC_PH2PL(2) VQC_PH2PL(3) VQC_PH2PL(4)
+#undef VQC_PH2PL
+    case DC_PH2_PP:
+        ph2_pp<R, K, MODE>((int)physbit(pb, ra) + 2 * (int)physbit(pb, rb), tp, flags, a, l, q, accp,
+                           acc_add);
+        break;
     default:
         break;
     }

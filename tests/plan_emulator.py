@@ -30,7 +30,8 @@ assert DSTAGE.itemsize == 248 and DPASS.itemsize == 88
 PATH_RESIDENT, PATH_HBM = 0, 1
 
 OP_M1, OP_CX, OP_CZ, OP_PH2 = 1, 2, 3, 4
-DC_M1, DC_CX_LL, DC_CX_PL, DC_CZ_LL, DC_CZ_PL, DC_CZ_PP, DC_PH2 = 0, 5, 25, 30, 40, 45, 46
+DC_M1, DC_CX_LL, DC_CX_PL, DC_CZ_LL, DC_CZ_PL, DC_CZ_PP = 0, 5, 25, 30, 40, 45
+DC_PH2_LL, DC_PH2_PL, DC_PH2_PP, DC_NUM = 46, 56, 61, 62
 CZ_PAIRS = [(0, 1), (0, 2), (0, 3), (0, 4), (1, 2), (1, 3), (1, 4), (2, 3), (2, 4), (3, 4)]
 
 
@@ -59,7 +60,13 @@ def op_type(op):
     if c == DC_CZ_PP:
         assert a >= REF_PHYS and b >= REF_PHYS
         return OP_CZ, a, b
-    assert c == DC_PH2
+    if c < DC_PH2_PL:
+        lo, hi = CZ_PAIRS[c - DC_PH2_LL]
+        assert a < REF_PHYS and b < REF_PHYS and (min(a, b), max(a, b)) == (lo, hi)
+    elif c < DC_PH2_PP:
+        assert (a < REF_PHYS) != (b < REF_PHYS) and min(a, b) == c - DC_PH2_PL
+    else:
+        assert c == DC_PH2_PP and a >= REF_PHYS and b >= REF_PHYS
     return OP_PH2, a, b
 OPF_PER_SAMPLE, OPF_GEN_CRZ, OPF_GEN_RZZ, OPF_HAS_ACC = 1, 2, 4, 8
 CK_CONST, CK_RX, CK_RY, CK_RZ, CK_GPHASE, CK_CRZ, CK_RZZ = 1, 2, 3, 4, 5, 6, 7
