@@ -485,6 +485,8 @@ void build_schedule(const HostPlan& p, Schedule& s) {
     std::iota(tile.begin(), tile.end(), 0);
     for (size_t i = 0; i < p.entries.size(); ++i) slot_of[i] = p.entries[i].slot;
     std::iota(acc_of.begin(), acc_of.end(), 0);
+    // Resident schedules have one register block per thread (n - K <= 9, see
+    // the schedule list), so every CX can be folded into a store map.
     cut_stages(p, ops, tile, s.K, s, slot_of, acc_of, true);
 }
 
@@ -640,7 +642,10 @@ vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx,
     // Stage schedules for every usable (mode, K) on the resident path.
     for (int mode = 0; mode < 2; ++mode) {
         for (int K = 1; K <= std::min(max_k(mode, dtype), n); ++K) {
-            if (n - K > 10) continue;   // at most 1024 register blocks per sample
+            // at most 512 register blocks per sample: one block per thread, which
+            // the folded CX gates need (a thread holding two blocks would store
+            // one before loading the other)
+            if (n - K > 9) continue;
             if (n > resident_max_qubits(mode, dtype)) continue;
             Schedule s;
             s.mode = mode;

@@ -123,7 +123,7 @@ __device__ __forceinline__ void tile_scatter(const C2<R>* sm, C2<R>* gs, uint32_
 }
 
 template <typename R, int K, int MODE>
-__global__ void __launch_bounds__(256) pass_kernel(const __grid_constant__ PArgs<R> A) {
+__global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PArgs<R> A) {
     extern __shared__ __align__(16) unsigned char smem[];
     R* sh_tab = reinterpret_cast<R*>(smem + A.sm_sh);
     R* ps_all = reinterpret_cast<R*>(smem + A.sm_ps);
@@ -237,6 +237,7 @@ __global__ void __launch_bounds__(256) pass_kernel(const __grid_constant__ PArgs
                 run_ops<R, K, 0, true>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
                                  sh_tab, ps_tab, nullptr, q, lane, warp_in_group);
                 if (s + 1 < A.stage_end || A.dst_psi) {   // store map: absorbed CX gates
+                    if (vqc_ld(&sp->nperm)) group_sync<R>(q);   // all loads of the stage first
                     int32_t s2[K];
                     const uint32_t b2 = map_base<K, true>(sp, q.t, q.h, s2);
                     block_store<R, K>(a, psi, b2, s2);
@@ -279,6 +280,7 @@ __global__ void __launch_bounds__(256) pass_kernel(const __grid_constant__ PArgs
             run_ops<R, K, 1, true>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l, sh_tab,
                              ps_tab, acc, q, lane, warp_in_group);
             if (s > A.stage_begin || A.dst_psi) {   // back to the stage's load map
+                if (vqc_ld(&sp->nperm)) group_sync<R>(q);   // all loads of the stage first
                 int32_t s2[K];
                 const uint32_t b2 = map_base<K, false>(sp, q.t, q.h, s2);
                 block_store<R, K>(a, psi, b2, s2);

@@ -1361,6 +1361,9 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                         }
                     }
                     if (store) {   // through the store map (absorbed CX gates)
+                        // a permuting store writes slots other threads load in this
+                        // stage: every load of the group must be done first
+                        if (vqc_ld(&sp->nperm)) group_sync<R>(q);
                         int32_t s2[K];
                         const uint32_t b2 = map_base<K, true>(sp, q.t + bj * q.T, q.h, s2);
                         block_store<R, K>(a, psi, b2, s2);
@@ -1421,6 +1424,7 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                 run_ops<R, K, 1, false>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l,
                                  sh_tab, ps_tab, acc, q, lane, warp_in_group, bj > 0);
                 if (s > 0) {   // back to the stage's input layout (load map)
+                    if (vqc_ld(&sp->nperm)) group_sync<R>(q);   // see the forward's store
                     int32_t s2[K];
                     const uint32_t b2 = map_base<K, false>(sp, q.t + bj * q.T, q.h, s2);
                     block_store<R, K>(a, psi, b2, s2);

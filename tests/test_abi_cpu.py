@@ -144,6 +144,8 @@ def check_addressing(plan):
                         assert sl == swz(local(sidx[r]), plan.G)
                         slots_st.add(sl)
                 assert slots == set(range(1 << m)) and slots_st == slots
+                if s["path"] == 0:   # one register block per thread (<= 512 threads)
+                    assert n - K <= 9
                 if int(st["nperm"]) == 0:
                     assert list(st["sigma_st"][:K]) == list(st["sigma"][:K])
                     assert list(st["tau_st"]) == list(st["tau"])

@@ -263,3 +263,56 @@ def test_deterministic_dw():
     _, dw1 = run_bwd(c, w_)
     _, dw2 = run_bwd(c, w_)
     assert np.array_equal(dw1, dw2)
+
+
+# ------------------------------------------------------------------ folded CX, multi-warp groups
+@pytest.mark.parametrize("n", [11, 12, 13])
+def test_folded_cx_multiwarp_groups(n):
+    """CX rings folded into stage store maps while a sample is spread over
+    several warps (2^(n-K) >= 64 threads): a permuting store writes slots other
+    warps load in the same stage, so the kernels order every load of the stage
+    before the stores.  Repeated calls against the oracle, forward and
+    backward."""
+    spec = wl.layered(n, 3, ("RX", "RY"), "CX", ring_range=lambda l: l + 1)
+    rng = np.random.default_rng(900 + n)
+    B = 24
+    x = wl._round(rng.uniform(-np.pi, np.pi, (B, n)), "c64")
+    w = wl._round(rng.uniform(-np.pi, np.pi, spec.num_w), "c64")
+    gE = wl._round(rng.standard_normal((B, n)), "c64")
+    w_ = wl.Workload("cx_ring_n%d" % n, spec, B, x, w, gE, "c64", 900 + n)
+    c = C(spec, "c64")
+    info = c.info(B)
+    assert info["fwd_path"] == 0 and info["fwd_threads_per_sample"] >= 64
+    E_ref, st_ref = orc.forward(spec, x, w, want_state=True)
+    dx_ref, dw_ref = orc.backward(spec, x, w, gE)
+    for _ in range(3):
+        E, st = run_fwd(c, w_)
+        assert maxerr(E, E_ref) <= TOL["c64"]["E"] and maxerr(st, st_ref) <= TOL["c64"]["state"]
+        dx, dw = run_bwd(c, w_)                       # recomputed forward inside the backward
+        assert maxerr(dx, dx_ref) <= 5e-4 and maxerr(dw, dw_ref) <= 1e-3
+        dx, dw = run_bwd(c, w_, psi_final=devc(st, "c64"))
+        assert maxerr(dx, dx_ref) <= 5e-4 and maxerr(dw, dw_ref) <= 1e-3
+
+
+def test_largest_resident_forward_n14():
+    """14 qubits at batch 3: the largest resident forward (register blocks of 32
+    amplitudes, 512 threads per sample, folded CX rings); the backward runs
+    HBM-tiled passes."""
+    n = 14
+    spec = wl.layered(n, 2, ("RY", "RZ"), "CX")
+    rng = np.random.default_rng(914)
+    B = 3
+    x = wl._round(rng.uniform(-np.pi, np.pi, (B, n)), "c64")
+    w = wl._round(rng.uniform(-np.pi, np.pi, spec.num_w), "c64")
+    gE = wl._round(rng.standard_normal((B, n)), "c64")
+    w_ = wl.Workload("cx_ring_n14", spec, B, x, w, gE, "c64", 914)
+    c = C(spec, "c64")
+    info = c.info(B)
+    assert info["fwd_path"] == 0 and info["fwd_threads_per_sample"] == 512
+    E_ref, st_ref = orc.forward(spec, x, w, want_state=True)
+    dx_ref, dw_ref = orc.backward(spec, x, w, gE)
+    E, st = run_fwd(c, w_)
+    assert maxerr(E, E_ref) <= TOL["c64"]["E"] and maxerr(st, st_ref) <= TOL["c64"]["state"]
+    for psi_final in (None, devc(st, "c64")):
+        dx, dw = run_bwd(c, w_, psi_final=psi_final)
+        assert maxerr(dx, dx_ref) <= 5e-4 and maxerr(dw, dw_ref) <= 5e-4
