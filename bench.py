@@ -128,6 +128,33 @@ def oracle_rate(w_, seconds=12.0, chunk=16, backward=True):
     return done / dt, done, dt
 
 
+def oracle_rate_parallel(w_, seconds=12.0, chunk=16, workers=None, backward=True):
+    """The same oracle on all host cores: one thread per core, each cycling its
+    own rows (the oracle runs in C; ctypes releases the GIL during each call)."""
+    import concurrent.futures as cf
+    from oracle import oracle as orc
+    workers = workers or os.cpu_count() or 1
+    orc.forward(w_.spec, w_.x[:1], w_.w)    # load the library before the threads start
+    t0 = time.perf_counter()
+
+    def work(k):
+        done, row = 0, k * chunk
+        while time.perf_counter() - t0 < seconds:
+            rows = [(row + i) % w_.batch for i in range(chunk)]
+            x = w_.x[rows]
+            orc.forward(w_.spec, x, w_.w)
+            if backward:
+                orc.backward(w_.spec, x, w_.w, w_.gE[rows])
+            done += chunk
+            row += chunk * workers
+        return done
+
+    with cf.ThreadPoolExecutor(max_workers=workers) as ex:
+        done = sum(ex.map(work, range(workers)))
+    dt = time.perf_counter() - t0
+    return done / dt, done, dt, workers
+
+
 # ------------------------------------------------------------------ our engine
 def run_ours(args, rank, world, local_rank):
     import torch
@@ -344,6 +371,11 @@ def run_ours(args, rank, world, local_rank):
                                "cores": 1, "kind": "oracle",
                                "sample": "%d rows of the workload (cycled), fwd+bwd, %.1f s"
                                          % (done, dt)}
+        prate, pdone, pdt, nw = oracle_rate_parallel(w_, seconds=args.cpu_seconds)
+        out["cpu_baseline_all_cores"] = {
+            "value": prate, "unit": "circuit evals/s (fwd+adjoint bwd)", "cores": nw,
+            "kind": "oracle, batch-parallel threads",
+            "sample": "%d rows of the workload (cycled), fwd+bwd, %.1f s" % (pdone, pdt)}
     if args.extra:
         out["configs"] = extra_configs(torch, Circuit, B)
     return out
