@@ -378,6 +378,10 @@ def run_ours(args, rank, world, local_rank):
             "sample": "%d rows of the workload (cycled), fwd+bwd, %.1f s" % (pdone, pdt)}
     if args.extra:
         out["configs"] = extra_configs(torch, Circuit, B)
+    if args.ablation:
+        out["ablation"] = ablation(torch, Circuit, w_)
+    if args.regime:
+        out["regime_map"] = regime_map(torch, Circuit)
     return out
 
 
@@ -390,6 +394,120 @@ def info_digest():
         from paper_2607_11985_gb300 import build
         _DIGEST = build._sources_digest()[:16]
     return _DIGEST
+
+
+def ablation(torch, Circuit, w_):
+    """Internal ablation on this engine (the paper's Table 5 design choices),
+    8-qubit workload: compile once vs compile per call; one batched launch vs a
+    loop over samples; adjoint gradients vs central finite differences (the
+    same forward kernel, 2 calls per parameter).  Device and host time."""
+    import numpy as np
+    real = torch.float32
+    x = torch.tensor(w_.x, dtype=real, device="cuda")
+    w = torch.tensor(w_.w, dtype=real, device="cuda")
+    gE = torch.tensor(w_.gE, dtype=real, device="cuda")
+    Bt = w_.batch
+
+    def wall(fn, reps):
+        fn()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(reps):
+            fn()
+        torch.cuda.synchronize()
+        return (time.perf_counter() - t0) / reps
+
+    c = Circuit(w_.spec, "c64")
+    E = c.forward(x, w)
+    out = {"workload": w_.name, "batch": Bt}
+    t_once = wall(lambda: c.forward(x, w, out=E), 50)
+    t_recompile = wall(lambda: Circuit(w_.spec, "c64").forward(x, w, out=E), 20)
+    out["compile_once_fwd_s"] = t_once
+    out["compile_per_call_fwd_s"] = t_recompile
+    out["compile_per_call_slowdown"] = t_recompile / t_once
+    rows = min(Bt, 128)
+    xs = [x[i:i + 1] for i in range(rows)]
+    t_loop = wall(lambda: [c.forward(xi, w) for xi in xs], 3) * Bt / rows
+    out["batched_fwd_s"] = t_once
+    out["per_sample_loop_fwd_s"] = t_loop
+    out["per_sample_loop_slowdown"] = t_loop / t_once
+    st = c.forward(x, w, want_state=True)[1]
+    t_adj = wall(lambda: c.backward(x, w, gE, psi_final=st), 20)
+    h = 1e-2   # central differences in fp32 arithmetic: h balances truncation and rounding
+
+    def fd():
+        gx = torch.empty_like(x)
+        gw = torch.empty_like(w)
+        for j in range(x.shape[1]):
+            xp, xm = x.clone(), x.clone()
+            xp[:, j] += h
+            xm[:, j] -= h
+            gx[:, j] = ((c.forward(xp, w) - c.forward(xm, w)) * gE).sum(1) / (2 * h)
+        for j in range(w.shape[0]):
+            wp, wm = w.clone(), w.clone()
+            wp[j] += h
+            wm[j] -= h
+            gw[j] = ((c.forward(x, wp) - c.forward(x, wm)) * gE).sum() / (2 * h)
+        return gx, gw
+
+    t_fd = wall(fd, 3)
+    gx_fd, gw_fd = fd()
+    dx, dw = c.backward(x, w, gE, psi_final=st)
+    torch.cuda.synchronize()
+    out["adjoint_bwd_s"] = t_adj
+    out["central_fd_grad_s"] = t_fd
+    out["central_fd_slowdown"] = t_fd / t_adj
+    out["fd_minus_adjoint_max_abs"] = {"dx": float((gx_fd - dx).abs().max()),
+                                       "dw": float((gw_fd - dw).abs().max())}
+    return out
+
+
+def regime_map(torch, Circuit, qubits=(4, 8, 12, 16, 18, 20), batches=(1, 8, 32, 128), layers=4):
+    """Qubits x batch sweep (the paper's regime map, Sec. 4.4): RY(x) encoding,
+    `layers` x (RX RY RZ per qubit + CX ring), complex64.  Per point: path, passes,
+    device workspace bytes of the backward (the memory the caller must provide
+    beyond inputs and outputs), forward and fwd+bwd device time (L2 flushed)."""
+    import numpy as np
+    from paper_2607_11985_gb300 import binding as Bd
+    from paper_2607_11985_gb300 import workloads as wl
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    pts = []
+    for n in qubits:
+        spec = wl.layered(n, layers, ("RX", "RY", "RZ"), "CX")
+        c = Circuit(spec, "c64")
+        rng = np.random.default_rng(7000 + n)
+        for Bt in batches:
+            x = torch.tensor(rng.uniform(-np.pi, np.pi, (Bt, n)), dtype=torch.float32, device="cuda")
+            w = torch.tensor(rng.uniform(-np.pi, np.pi, spec.num_w), dtype=torch.float32, device="cuda")
+            gE = torch.tensor(rng.standard_normal((Bt, n)), dtype=torch.float32, device="cuda")
+            inf = c.info(Bt)
+            E, st = c.forward(x, w, want_state=True)
+            c.backward(x, w, gE, psi_final=st)
+            torch.cuda.synchronize()
+            reps = 5 if n <= 16 else 2
+            tf = tb = 0.0
+            for _ in range(reps):
+                flush.zero_()
+                a, b2, d = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+                a.record()
+                c.forward(x, w, out=E, state_out=st)
+                b2.record()
+                c.backward(x, w, gE, psi_final=st)
+                d.record()
+                torch.cuda.synchronize()
+                tf += a.elapsed_time(b2) / reps
+                tb += b2.elapsed_time(d) / reps
+            pts.append({"qubits": n, "batch": Bt,
+                        "path": "hbm-tiled" if inf["bwd_path"] == 1 else "resident",
+                        "passes_fwd_bwd": [inf["fwd_passes"], inf["bwd_passes"]],
+                        "state_bytes": Bt * (8 << n),
+                        "bwd_workspace_bytes": int(Bd.vqc_workspace_bytes(c.plan, Bt, 1)),
+                        "fwd_ms": tf, "fwd_bwd_ms": tf + tb,
+                        "fwd_bwd_evals_per_s": Bt / ((tf + tb) / 1e3)})
+            del x, w, gE, E, st
+        del c
+        torch.cuda.empty_cache()
+    return pts
 
 
 def extra_configs(torch, Circuit, B):
@@ -507,7 +625,11 @@ def main():
     ap.add_argument("--config", type=int, default=2)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--extra", action="store_true", help="also time configs 1, 3, 4")
+    ap.add_argument("--extra", action="store_true", help="also time configs 1, 3, 4 and 5")
+    ap.add_argument("--regime", action="store_true",
+                    help="qubits x batch sweep to 20 qubits (HBM-tiled beyond one SM's state)")
+    ap.add_argument("--ablation", action="store_true",
+                    help="compile-once / batching / adjoint-vs-FD ablation on the bench workload")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))

@@ -110,3 +110,25 @@ def test_resident_and_hbm_paths_agree(monkeypatch):
     dx2, dw2 = run_bwd(c2, w_)
     assert maxerr(E1, E2) <= 2e-5 and maxerr(st1, st2) <= 2e-5
     assert maxerr(dx1, dx2) <= 2e-4 and maxerr(dw1, dw2) <= 1e-3
+
+
+def test_hbm_18_qubits_sampled():
+    """18 qubits (2 MB complex64 state per sample, 32 tiles per sample per pass):
+    E and dx of two rows against the oracle, dw of the whole batch of 3."""
+    n = 18
+    spec = wl.layered(n, 2, ("RX", "RY", "RZ"), "CX")
+    rng = np.random.default_rng(1800)
+    B = 3
+    x = wl._round(rng.uniform(-np.pi, np.pi, (B, n)), "c64")
+    w = wl._round(rng.uniform(-np.pi, np.pi, spec.num_w), "c64")
+    gE = wl._round(rng.standard_normal((B, n)), "c64")
+    w_ = wl.Workload("layered_n18", spec, B, x, w, gE, "c64", 1800)
+    c = C(spec, "c64")
+    info = c.info(B)
+    assert info["fwd_path"] == 1 and info["bwd_path"] == 1
+    E = run_fwd(c, w_, want_state=False)
+    E_ref = orc.forward(spec, x, w)
+    assert maxerr(E, E_ref) <= 1e-4
+    dx, dw = run_bwd(c, w_)
+    dx_ref, dw_ref = orc.backward(spec, x, w, gE)
+    assert maxerr(dx, dx_ref) <= 5e-4 and maxerr(dw, dw_ref) <= 5e-4
