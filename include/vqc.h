@@ -140,12 +140,40 @@ typedef struct {
 vqc_status vqc_compile(const vqc_gate* gates, int32_t num_gates, int32_t num_qubits,
                        int32_t num_x, int32_t num_w, vqc_dtype dtype, vqc_plan** out_plan);
 
+/* OpenQASM 2 front end (paper, Sec. 3 "Static Circuit Scope" and Fig. 2: the
+ * circuit is given as normalised OpenQASM and parsed once).  Accepted:
+ * "OPENQASM 2.0;", include "qelib1.inc", qreg / creg declarations (quantum
+ * registers are numbered in declaration order, qubit 0 first), the gate set
+ * under its qelib1 names -- h x y z s t sx rx ry rz u3 (also u, U) cx (CX) cz
+ * swap crz rzz -- and the exact U3 special cases u1 / p, u2, sdg, tdg, id;
+ * `barrier` and `measure` are accepted and ignored (the engine returns <Z>).
+ * Whole-register operands broadcast over equal-sized registers.  An angle is a
+ * constant expression (numbers, pi, + - * / ^, unary minus, parentheses, sin
+ * cos tan exp ln sqrt) or, as the variational extension, exactly one parameter
+ * reference: x[i] (per-sample column i) or w[j] (shared weight j).  Gate
+ * definitions, opaque, if and reset are rejected (VQC_ERR_UNSUPPORTED_GATE),
+ * as are gates outside the set; errors name the source line.
+ *
+ * vqc_parse_qasm lowers `source` to vqc_gate records: *inout_num_gates is the
+ * capacity of `gates` on entry and the program's gate count on return; pass
+ * gates = NULL to query the count.  num_qubits, num_x (largest x index + 1) and
+ * num_w (largest w index + 1) are written on success.  Host only. */
+vqc_status vqc_parse_qasm(const char* source, vqc_gate* gates, int32_t* inout_num_gates,
+                          int32_t* num_qubits, int32_t* num_x, int32_t* num_w);
+
+/* vqc_parse_qasm followed by vqc_compile.  num_x / num_w < 0 take the counts
+ * the program implies; given counts must cover every referenced index
+ * (VQC_ERR_PARAM_RANGE otherwise).  Other errors as vqc_compile. */
+vqc_status vqc_compile_qasm(const char* source, int32_t num_x, int32_t num_w, vqc_dtype dtype,
+                            vqc_plan** out_plan);
+
 /* Release a plan (NULL-safe).  The caller must make sure no enqueued call
  * still uses it (synchronise the streams first). */
 void vqc_free(vqc_plan* plan);
 
-/* Bytes of device workspace a call needs: mode 0 = vqc_forward, 1 = vqc_backward.
- * Returns 0 when no workspace is needed; (size_t)-1 for a NULL plan. */
+/* Bytes of device workspace a call needs: mode 0 = vqc_forward, 1 = vqc_backward,
+ * 2 = vqc_probabilities.  Returns 0 when no workspace is needed; (size_t)-1 for
+ * a NULL plan. */
 size_t vqc_workspace_bytes(const vqc_plan* plan, int32_t batch, int32_t mode);
 
 /* Zero a workspace's control block on `stream` (enqueued memset).  A freshly
@@ -183,6 +211,18 @@ vqc_status vqc_backward(const vqc_plan* plan, int32_t batch, const void* x, cons
                         const void* psi0, const void* psi_final, const void* grad_expz,
                         void* grad_x, void* grad_w, void* workspace, size_t workspace_bytes,
                         void* stream);
+
+/* Measurement probabilities |psi_b[k]|^2 of the final states (paper, Sec. 3:
+ * the engine's outputs are the statevector or its probabilities, and <Z>):
+ * probs_out [B, 2^n] real (float / double), logical amplitude order.  Runs the
+ * forward sweep into the workspace (vqc_workspace_bytes mode 2: the forward's
+ * own workspace, then the states and <Z> of the batch; 256-byte aligned, the
+ * first 256 bytes cleared once by vqc_workspace_init), then one elementwise
+ * kernel.  Inputs as vqc_forward.  Errors as vqc_forward, VQC_ERR_WORKSPACE for
+ * a missing, short or misaligned workspace. */
+vqc_status vqc_probabilities(const vqc_plan* plan, int32_t batch, const void* x, const void* w,
+                             const void* psi0, void* probs_out, void* workspace,
+                             size_t workspace_bytes, void* stream);
 
 /* Bytes of device scratch built into the library for vqc_backward_noalloc
  * (one array per GPU that loads the library, held until the process exits). */

@@ -74,6 +74,10 @@ SIGNATURES = [
     ("vqc_sync_check", _I, [_P]),
     ("vqc_last_error", ctypes.c_char_p, []),
     ("vqc_abi_version", _I, []),
+    ("vqc_probabilities", _I, [_P, _I, _P, _P, _P, _P, _P, _S, _P]),
+    ("vqc_parse_qasm", _I, [ctypes.c_char_p, ctypes.POINTER(vqc_gate), ctypes.POINTER(_I),
+                            ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_I)]),
+    ("vqc_compile_qasm", _I, [ctypes.c_char_p, _I, _I, _I, ctypes.POINTER(_P)]),
 ]
 
 
@@ -121,6 +125,25 @@ def vqc_compile(gates, num_gates, num_qubits, num_x, num_w, dtype):
     return plan.value
 
 
+def vqc_parse_qasm(source):
+    """(gates array, num_gates, num_qubits, num_x, num_w) of an OpenQASM 2 program."""
+    src = source.encode() if isinstance(source, str) else source
+    n, nq, nx, nw = _I(0), _I(0), _I(0), _I(0)
+    _check(lib().vqc_parse_qasm(src, None, ctypes.byref(n), ctypes.byref(nq), ctypes.byref(nx),
+                                ctypes.byref(nw)))
+    arr = (vqc_gate * max(n.value, 1))()
+    _check(lib().vqc_parse_qasm(src, arr, ctypes.byref(n), ctypes.byref(nq), ctypes.byref(nx),
+                                ctypes.byref(nw)))
+    return arr, n.value, nq.value, nx.value, nw.value
+
+
+def vqc_compile_qasm(source, num_x=-1, num_w=-1, dtype=0):
+    src = source.encode() if isinstance(source, str) else source
+    plan = ctypes.c_void_p()
+    _check(lib().vqc_compile_qasm(src, num_x, num_w, dtype, ctypes.byref(plan)))
+    return plan.value
+
+
 def vqc_free(plan):
     lib().vqc_free(plan)
 
@@ -136,6 +159,11 @@ def vqc_workspace_init(workspace, nbytes, stream):
 def vqc_forward(plan, batch, x, w, psi0, expz_out, state_out, workspace, workspace_bytes, stream):
     _check(lib().vqc_forward(plan, batch, x, w, psi0, expz_out, state_out, workspace,
                              workspace_bytes, stream))
+
+
+def vqc_probabilities(plan, batch, x, w, psi0, probs_out, workspace, workspace_bytes, stream):
+    _check(lib().vqc_probabilities(plan, batch, x, w, psi0, probs_out, workspace, workspace_bytes,
+                                   stream))
 
 
 def vqc_backward(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x, grad_w, workspace,

@@ -35,6 +35,23 @@ class Circuit:
                                   self.code)
         self._ws = {}
 
+    @classmethod
+    def from_qasm(cls, source: str, dtype: str = "c64", num_x: int = -1, num_w: int = -1):
+        """Compile an OpenQASM 2 program (gate set, parameter references x[i] /
+        w[j]: see vqc_compile_qasm in include/vqc.h)."""
+        if dtype not in _DT:
+            raise ValueError("dtype must be 'c64' or 'c128'")
+        self = cls.__new__(cls)
+        self.spec = None
+        self.dtype = dtype
+        self.code, self.real, self.cplx = _DT[dtype]
+        self._gates = None
+        self.plan = B.vqc_compile_qasm(source, num_x, num_w, self.code)
+        info = B.vqc_plan_info(self.plan, 1)
+        self.n, self.num_x, self.num_w = info["num_qubits"], info["num_x"], info["num_w"]
+        self._ws = {}
+        return self
+
     def __del__(self):
         plan = getattr(self, "plan", None)
         if plan:
@@ -89,6 +106,19 @@ class Circuit:
         B.vqc_forward(self.plan, batch, _ptr(x), _ptr(w), _ptr(psi0), _ptr(E), _ptr(st),
                       _ptr(ws), wsb, stream.cuda_stream)
         return (E, st) if want_state else E
+
+    def probabilities(self, x, w, psi0=None, out=None):
+        """|psi_b[k]|^2 of the final states, [B, 2^n] real."""
+        batch = x.shape[0] if x is not None and x.dim() == 2 else (psi0.shape[0] if psi0 is not None else 1)
+        x = self._check(x, self.real, (batch, self.num_x), "x") if self.num_x else None
+        w = self._check(w, self.real, (self.num_w,), "w") if self.num_w else None
+        psi0 = self._check(psi0, self.cplx, (batch, 1 << self.n), "psi0")
+        P = out if out is not None else torch.empty(batch, 1 << self.n, dtype=self.real, device="cuda")
+        stream = torch.cuda.current_stream()
+        ws, wsb = self.workspace(batch, 2, stream)
+        B.vqc_probabilities(self.plan, batch, _ptr(x), _ptr(w), _ptr(psi0), _ptr(P), _ptr(ws), wsb,
+                            stream.cuda_stream)
+        return P
 
     def backward(self, x, w, grad_expz, psi0=None, psi_final=None, need_x=True, need_w=True,
                  grad_x=None, grad_w=None):

@@ -849,6 +849,12 @@ void vqc_free(vqc_plan* plan) {
 
 size_t vqc_workspace_bytes(const vqc_plan* plan, int32_t batch, int32_t mode) {
     if (!plan) return (size_t)-1;
+    if (mode == 2 && batch > 0) {   // vqc_probabilities: forward workspace + state + E
+        const HostPlan& p = plan->hp;
+        const size_t rs = p.dtype == VQC_C128 ? 8 : 4;
+        return align256(vqc_workspace_bytes(plan, batch, 0)) +
+               align256(((size_t)batch << p.n) * 2 * rs) + align256((size_t)batch * p.n * rs);
+    }
     if ((mode != 0 && mode != 1) || batch <= 0) return 0;
     const HostPlan& p = plan->hp;
     if (use_hbm(p, mode, batch)) {
@@ -860,6 +866,40 @@ size_t vqc_workspace_bytes(const vqc_plan* plan, int32_t batch, int32_t mode) {
     Launch L;
     if (plan_launch(p, 1, batch, L) != VQC_OK) return 0;
     return bwd_workspace(p, L);
+}
+
+vqc_status vqc_probabilities(const vqc_plan* plan, int32_t batch, const void* x, const void* w,
+                             const void* psi0, void* probs_out, void* workspace,
+                             size_t workspace_bytes, void* stream) {
+    try {
+        vqc_status st = check_common(plan, batch);
+        if (st != VQC_OK) return st;
+        if (batch == 0) return VQC_OK;
+        const HostPlan& p = plan->hp;
+        if (!probs_out) return fail(VQC_ERR_INVALID_ARG, "probs_out is NULL");
+        const bool dbl = p.dtype == VQC_C128;
+        const size_t rs = dbl ? 8 : 4;
+        const size_t fws = vqc_workspace_bytes(plan, batch, 0);
+        const size_t need = vqc_workspace_bytes(plan, batch, 2);
+        if (!workspace || workspace_bytes < need || misaligned(workspace, 256))
+            return fail(VQC_ERR_WORKSPACE, "probabilities workspace must be >= " + std::to_string(need) +
+                                               " bytes and 256-byte aligned");
+        char* base = static_cast<char*>(workspace);
+        void* state = base + align256(fws);
+        void* E = base + align256(fws) + align256(((size_t)batch << p.n) * 2 * rs);
+        st = vqc_forward(plan, batch, x, w, psi0, E, state, fws ? workspace : nullptr, fws, stream);
+        if (st != VQC_OK) return st;
+        cudaStream_t s = static_cast<cudaStream_t>(stream);
+        long long count = (long long)batch << p.n;
+        int blocks = (int)std::min<long long>((count + 255) / 256, 152LL * 16);
+        const void* src = state;
+        void* dst = probs_out;
+        void* args[] = {&src, &count, &dst};
+        VQC_CUDA(launch(abs2_ptr(dbl), dim3(std::max(blocks, 1)), dim3(256), args, 0, s));
+        return VQC_OK;
+    } catch (...) {
+        return fail(VQC_ERR_INVALID_ARG, "internal error in vqc_probabilities");
+    }
 }
 
 vqc_status vqc_workspace_init(void* workspace, size_t workspace_bytes, void* stream) {

@@ -16,6 +16,7 @@ const void* reduce_expz_ptr(bool dbl);
 const void* reduce_dx_ptr(bool dbl);
 const void* reduce_dw_ptr(bool dbl);
 const void* reduce_cols_ptr(bool dbl);
+const void* abs2_ptr(bool dbl);   // |psi|^2, elementwise
 
 // Largest block (threads) each instantiation is compiled for.
 inline int sweep_max_threads(bool is_double, int mode, int K) {

@@ -28,6 +28,10 @@ const void* reduce_cols_ptr(bool dbl) {
     return dbl ? reinterpret_cast<const void*>(&reduce_cols<double>)
                : reinterpret_cast<const void*>(&reduce_cols<float>);
 }
+const void* abs2_ptr(bool dbl) {
+    return dbl ? reinterpret_cast<const void*>(&abs2_kernel<double>)
+               : reinterpret_cast<const void*>(&abs2_kernel<float>);
+}
 const void* reduce_dw_ptr(bool dbl) {
     return dbl ? reinterpret_cast<const void*>(&reduce_dw<double>)
                : reinterpret_cast<const void*>(&reduce_dw<float>);

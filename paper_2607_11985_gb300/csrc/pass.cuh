@@ -364,4 +364,16 @@ __global__ void __launch_bounds__(256) reduce_dw(const R* terms, long long rows,
     if (threadIdx.x == 0) dw[p] = part[0];
 }
 
+// probs[i] = |psi[i]|^2 over count amplitudes (the probabilities output).
+template <typename R>
+__global__ void __launch_bounds__(256) abs2_kernel(const C2<R>* psi, long long count, R* probs) {
+    grid_dep_wait();
+    grid_dep_launch();
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < count;
+         i += (long long)gridDim.x * blockDim.x) {
+        const C2<R> v = psi[i];
+        probs[i] = fma(v.x, v.x, v.y * v.y);
+    }
+}
+
 }  // namespace vqc
