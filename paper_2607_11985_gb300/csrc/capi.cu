@@ -82,9 +82,13 @@ vqc_status device_info(int dev, DevInfo& out) {
     return VQC_OK;
 }
 
-const void* kernel_ptr(int dtype, int mode, int K) {
-    if (dtype == VQC_C64) return mode == 0 ? sweep_ptr_f32_fwd(K) : sweep_ptr_f32_bwd(K);
-    return mode == 0 ? sweep_ptr_f64_fwd(K) : sweep_ptr_f64_bwd(K);
+const void* kernel_ptr(int dtype, int mode, int K, bool full) {
+    if (full) {
+        if (dtype == VQC_C64) return mode == 0 ? sweep_ptr_f32_fwd(K) : sweep_ptr_f32_bwd(K);
+        return mode == 0 ? sweep_ptr_f64_fwd(K) : sweep_ptr_f64_bwd(K);
+    }
+    if (dtype == VQC_C64) return mode == 0 ? sweep_ptr_f32_fwd_small(K) : sweep_ptr_f32_bwd_small(K);
+    return mode == 0 ? sweep_ptr_f64_fwd_small(K) : sweep_ptr_f64_bwd_small(K);
 }
 
 size_t align16(size_t v) { return (v + 15) & ~size_t(15); }
@@ -215,7 +219,7 @@ vqc_status plan_launch_uncached(const HostPlan& p, int mode, int B, Launch& L) {
     L.smem = off;
     if (L.smem > (size_t)di.smem_optin)
         return fail(VQC_ERR_UNSUPPORTED, "shared-memory layout exceeds the per-CTA limit");
-    L.fn = kernel_ptr(p.dtype, mode, L.K);
+    L.fn = kernel_ptr(p.dtype, mode, L.K, L.T >= 32);
     if (!L.fn) return fail(VQC_ERR_UNSUPPORTED, "kernel not instantiated for this K");
     VQC_CUDA(cudaFuncSetAttribute(L.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem));
     int per_sm = 0;
@@ -480,7 +484,7 @@ vqc_status plan_hbm_uncached(const HostPlan& p, int mode, int B, PassGeo& L) {
     L.plan_smem = off + plan_bytes <= (size_t)di.smem_optin && plan_bytes <= 48 * 1024;
     L.sm_plan = L.plan_smem ? take(plan_bytes) : 0;
     L.smem = off;
-    L.fn = pass_ptr(dbl, mode, L.K);
+    L.fn = pass_ptr(dbl, mode, L.K, L.T >= 32);
     if (!L.fn) return fail(VQC_ERR_UNSUPPORTED, "pass kernel not instantiated for this K");
     VQC_CUDA(cudaFuncSetAttribute(L.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem));
     int per_sm = 0;

@@ -5,13 +5,17 @@
 
 namespace vqc {
 
-const void* sweep_ptr_f32_fwd(int K);
+const void* sweep_ptr_f32_fwd(int K);          // sample groups of >= 32 threads
 const void* sweep_ptr_f32_bwd(int K);
 const void* sweep_ptr_f64_fwd(int K);
 const void* sweep_ptr_f64_bwd(int K);
+const void* sweep_ptr_f32_fwd_small(int K);    // sample groups of < 32 threads
+const void* sweep_ptr_f32_bwd_small(int K);
+const void* sweep_ptr_f64_fwd_small(int K);
+const void* sweep_ptr_f64_bwd_small(int K);
 
 // HBM-tiled pass kernels (K fixed per type and mode) and partial reductions.
-const void* pass_ptr(bool dbl, int mode, int K);
+const void* pass_ptr(bool dbl, int mode, int K, bool full);   // full: tile groups >= 32 threads
 const void* reduce_expz_ptr(bool dbl);
 const void* reduce_dx_ptr(bool dbl);
 const void* reduce_dw_ptr(bool dbl);

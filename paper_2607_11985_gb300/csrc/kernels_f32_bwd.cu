@@ -1,4 +1,5 @@
-// kernels_f32_bwd.cu -- instantiations of the sweep kernel for float, mode 1.
+// kernels_f32_bwd.cu -- instantiations of the sweep kernel for float, mode 1, sample
+// groups of at least one warp (full-warp reductions).
 #include "kernels.h"
 #include "sweep.cuh"
 
@@ -6,10 +7,10 @@ namespace vqc {
 
 const void* sweep_ptr_f32_bwd(int K) {
     switch (K) {
-    case 1: return reinterpret_cast<const void*>(&sweep_kernel<float, 1, 1>);
-    case 2: return reinterpret_cast<const void*>(&sweep_kernel<float, 2, 1>);
-    case 3: return reinterpret_cast<const void*>(&sweep_kernel<float, 3, 1>);
-    case 4: return reinterpret_cast<const void*>(&sweep_kernel<float, 4, 1>);
+    case 1: return reinterpret_cast<const void*>(&sweep_kernel<float, 1, 1, true>);
+    case 2: return reinterpret_cast<const void*>(&sweep_kernel<float, 2, 1, true>);
+    case 3: return reinterpret_cast<const void*>(&sweep_kernel<float, 3, 1, true>);
+    case 4: return reinterpret_cast<const void*>(&sweep_kernel<float, 4, 1, true>);
     default: return nullptr;
     }
 }

@@ -1,4 +1,5 @@
-// kernels_f64_bwd.cu -- instantiations of the sweep kernel for double, mode 1.
+// kernels_f64_bwd.cu -- instantiations of the sweep kernel for double, mode 1, sample
+// groups of at least one warp (full-warp reductions).
 #include "kernels.h"
 #include "sweep.cuh"
 
@@ -6,9 +7,9 @@ namespace vqc {
 
 const void* sweep_ptr_f64_bwd(int K) {
     switch (K) {
-    case 1: return reinterpret_cast<const void*>(&sweep_kernel<double, 1, 1>);
-    case 2: return reinterpret_cast<const void*>(&sweep_kernel<double, 2, 1>);
-    case 3: return reinterpret_cast<const void*>(&sweep_kernel<double, 3, 1>);
+    case 1: return reinterpret_cast<const void*>(&sweep_kernel<double, 1, 1, true>);
+    case 2: return reinterpret_cast<const void*>(&sweep_kernel<double, 2, 1, true>);
+    case 3: return reinterpret_cast<const void*>(&sweep_kernel<double, 3, 1, true>);
     default: return nullptr;
     }
 }

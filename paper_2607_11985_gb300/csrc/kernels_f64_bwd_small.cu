@@ -1,0 +1,17 @@
+// kernels_f64_bwd_small.cu -- instantiations of the sweep kernel for double, mode 1, sample
+// groups of fewer than 32 threads (small circuits or large blocks).
+#include "kernels.h"
+#include "sweep.cuh"
+
+namespace vqc {
+
+const void* sweep_ptr_f64_bwd_small(int K) {
+    switch (K) {
+    case 1: return reinterpret_cast<const void*>(&sweep_kernel<double, 1, 1, false>);
+    case 2: return reinterpret_cast<const void*>(&sweep_kernel<double, 2, 1, false>);
+    case 3: return reinterpret_cast<const void*>(&sweep_kernel<double, 3, 1, false>);
+    default: return nullptr;
+    }
+}
+
+}  // namespace vqc

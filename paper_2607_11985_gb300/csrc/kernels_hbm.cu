@@ -5,13 +5,17 @@
 
 namespace vqc {
 
-const void* pass_ptr(bool dbl, int mode, int K) {
+const void* pass_ptr(bool dbl, int mode, int K, bool full) {
     if (!dbl) {
-        if (mode == 0 && K == 5) return reinterpret_cast<const void*>(&pass_kernel<float, 5, 0>);
-        if (mode == 1 && K == 4) return reinterpret_cast<const void*>(&pass_kernel<float, 4, 1>);
+        if (mode == 0 && K == 5) return full ? reinterpret_cast<const void*>(&pass_kernel<float, 5, 0, true>)
+                                             : reinterpret_cast<const void*>(&pass_kernel<float, 5, 0, false>);
+        if (mode == 1 && K == 4) return full ? reinterpret_cast<const void*>(&pass_kernel<float, 4, 1, true>)
+                                             : reinterpret_cast<const void*>(&pass_kernel<float, 4, 1, false>);
     } else {
-        if (mode == 0 && K == 4) return reinterpret_cast<const void*>(&pass_kernel<double, 4, 0>);
-        if (mode == 1 && K == 3) return reinterpret_cast<const void*>(&pass_kernel<double, 3, 1>);
+        if (mode == 0 && K == 4) return full ? reinterpret_cast<const void*>(&pass_kernel<double, 4, 0, true>)
+                                             : reinterpret_cast<const void*>(&pass_kernel<double, 4, 0, false>);
+        if (mode == 1 && K == 3) return full ? reinterpret_cast<const void*>(&pass_kernel<double, 3, 1, true>)
+                                             : reinterpret_cast<const void*>(&pass_kernel<double, 3, 1, false>);
     }
     return nullptr;
 }

@@ -122,7 +122,9 @@ __device__ __forceinline__ void tile_scatter(const C2<R>* sm, C2<R>* gs, uint32_
     }
 }
 
-template <typename R, int K, int MODE>
+// FULL: tile groups span whole warps (2^(m-K) >= 32 threads; every production
+// tile), see sweep_kernel.
+template <typename R, int K, int MODE, bool FULL>
 __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PArgs<R> A) {
     extern __shared__ __align__(16) unsigned char smem[];
     R* sh_tab = reinterpret_cast<R*>(smem + A.sm_sh);
@@ -234,7 +236,7 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
                 } else {
                     block_load<R, K>(a, psi, v.swb, sg);
                 }
-                run_ops<R, K, 0, true>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
+                run_ops<R, K, 0, true, FULL>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
                                  sh_tab, ps_tab, nullptr, q, lane, warp_in_group);
                 if (s + 1 < A.stage_end || A.dst_psi) {   // store map: absorbed CX gates
                     if (vqc_ld(&sp->nperm)) group_sync<R>(q);   // all loads of the stage first
@@ -277,7 +279,7 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
                 else
                     block_load<R, K>(l, lam, b2, s2);
             }
-            run_ops<R, K, 1, true>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l, sh_tab,
+            run_ops<R, K, 1, true, FULL>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l, sh_tab,
                              ps_tab, acc, q, lane, warp_in_group);
             if (s > A.stage_begin || A.dst_psi) {   // back to the stage's load map
                 if (vqc_ld(&sp->nperm)) group_sync<R>(q);   // all loads of the stage first

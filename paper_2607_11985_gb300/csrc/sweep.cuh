@@ -780,12 +780,17 @@ template <typename R>
 __device__ __forceinline__ R im_conj_mul(const C2<R>& la, const C2<R>& ps) {
     return la.x * ps.y - la.y * ps.x;
 }
-template <typename R>
+template <typename R, bool FULL>
 __device__ __forceinline__ void ph2_term_store(R tv, const Geo& q, R* accp, bool acc_add) {
-    tv = reduce1<R>(tv, q.lanes, q.mask);
+    if (FULL) {
+#pragma unroll
+        for (int m = 16; m >= 1; m >>= 1) tv += __shfl_xor_sync(0xffffffffu, tv, m);
+    } else {
+        tv = reduce1<R>(tv, q.lanes, q.mask);
+    }
     if ((q.t & (q.lanes - 1)) == 0) accp[0] = acc_add ? accp[0] + tv : tv;
 }
-template <typename R, int K, int MODE, int LO, int HI>
+template <typename R, int K, int MODE, bool FULL, int LO, int HI>
 __device__ __forceinline__ void ph2_ll(bool swapped, const R* tp, uint8_t flags,
                                        C2<R> (&a)[1 << K], C2<R> (&l)[1 << K], const Geo& q,
                                        R* accp, bool acc_add) {
@@ -805,7 +810,7 @@ __device__ __forceinline__ void ph2_ll(bool swapped, const R* tp, uint8_t flags,
 #pragma unroll
             for (int r = 0; r < (1 << K); ++r)
                 tv = fma(g[((r >> LO) & 1) + 2 * ((r >> HI) & 1)], im_conj_mul<R>(l[r], a[r]), tv);
-            ph2_term_store<R>(tv, q, accp, acc_add);
+            ph2_term_store<R, FULL>(tv, q, accp, acc_add);
         }
     }
 #pragma unroll
@@ -815,7 +820,7 @@ __device__ __forceinline__ void ph2_ll(bool swapped, const R* tp, uint8_t flags,
         if (MODE == 1) l[r] = cmul<R>(l[r], ph[s]);
     }
 }
-template <typename R, int K, int MODE, int L>
+template <typename R, int K, int MODE, bool FULL, int L>
 __device__ __forceinline__ void ph2_pl(bool a_local, bool p, const R* tp, uint8_t flags,
                                        C2<R> (&a)[1 << K], C2<R> (&l)[1 << K], const Geo& q,
                                        R* accp, bool acc_add) {
@@ -831,7 +836,7 @@ __device__ __forceinline__ void ph2_pl(bool a_local, bool p, const R* tp, uint8_
 #pragma unroll
             for (int r = 0; r < (1 << K); ++r)
                 tv = fma(((r >> L) & 1) ? g1 : g0, im_conj_mul<R>(l[r], a[r]), tv);
-            ph2_term_store<R>(tv, q, accp, acc_add);
+            ph2_term_store<R, FULL>(tv, q, accp, acc_add);
         }
     }
 #pragma unroll
@@ -841,7 +846,7 @@ __device__ __forceinline__ void ph2_pl(bool a_local, bool p, const R* tp, uint8_
         if (MODE == 1) l[r] = cmul<R>(l[r], f);
     }
 }
-template <typename R, int K, int MODE>
+template <typename R, int K, int MODE, bool FULL>
 __device__ __forceinline__ void ph2_pp(int s, const R* tp, uint8_t flags, C2<R> (&a)[1 << K],
                                        C2<R> (&l)[1 << K], const Geo& q, R* accp, bool acc_add) {
     C2<R> f = cm<R>(tp[2 * s], tp[2 * s + 1]);
@@ -851,7 +856,7 @@ __device__ __forceinline__ void ph2_pp(int s, const R* tp, uint8_t flags, C2<R> 
             R tv = 0;
 #pragma unroll
             for (int r = 0; r < (1 << K); ++r) tv += im_conj_mul<R>(l[r], a[r]);
-            ph2_term_store<R>(gen_at<R>(flags, s) * tv, q, accp, acc_add);
+            ph2_term_store<R, FULL>(gen_at<R>(flags, s) * tv, q, accp, acc_add);
         }
     }
 #pragma unroll
@@ -888,7 +893,7 @@ __device__ __forceinline__ bool physbit(uint32_t pb, int ref) {
 // WITH_CX: the schedule may hold CX ops (HBM passes); resident schedules fold
 // every CX into stage store maps, and leaving those cases out of the switch
 // keeps the other cases' register allocation tight.
-template <typename R, int K, int MODE, bool WITH_CX>
+template <typename R, int K, int MODE, bool WITH_CX, bool FULL>
 __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 << K],
                                          C2<R> (&l)[1 << K], const R* sh_tab, const R* ps_tab,
                                          R* acc, const Geo& q, int lane, int warp_in_group,
@@ -897,7 +902,7 @@ __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 <<
     const int flags = raw.x >> 24, slot = raw.y & 0xffff, aux = raw.y >> 16;
     const R* tp = ((flags & OPF_PER_SAMPLE) ? ps_tab : sh_tab) + EntryWords<R>::value * slot;
     R* accp = acc + ((size_t)aux * q.wg + warp_in_group) * 8;
-    const int rlane = q.lanes < 32 ? q.t : lane;
+    const int rlane = FULL ? lane : q.t;
     switch (code) {
 #define VQC_M1(T_)                                                                   \
     case DC_M1 + T_:                                                                 \
@@ -905,14 +910,19 @@ __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 <<
             if (MODE == 0) {                                                         \
                 m1_entry<R, K, T_, false>(a, tp);                                    \
             } else {                                                                 \
-                if ((flags & OPF_HAS_ACC) && q.lanes == 32) {                        \
+                if constexpr (FULL) {                                                \
                     /* one basic block: the butterfly's shuffles can overlap  */     \
                     /* the adjoint arithmetic                                 */     \
-                    R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};                              \
-                    rho_go<R, K, T_>(a, l, rh);                                      \
-                    m1_entry<R, K, T_, true>(a, tp);                                 \
-                    m1_entry<R, K, T_, true>(l, tp);                                 \
-                    reduce8_full<R>(rh, lane, accp, acc_add);                        \
+                    if (flags & OPF_HAS_ACC) {                                       \
+                        R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};                          \
+                        rho_go<R, K, T_>(a, l, rh);                                  \
+                        m1_entry<R, K, T_, true>(a, tp);                             \
+                        m1_entry<R, K, T_, true>(l, tp);                             \
+                        reduce8_full<R>(rh, lane, accp, acc_add);                    \
+                    } else {                                                         \
+                        m1_entry<R, K, T_, true>(a, tp);                             \
+                        m1_entry<R, K, T_, true>(l, tp);                             \
+                    }                                                                \
                 } else {                                                             \
                     if (flags & OPF_HAS_ACC) {                                       \
                         R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};                          \
@@ -982,7 +992,7 @@ __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 <<
     }
 #define VQC_PH2LL(LO_, HI_)                                                          \
     case DC_PH2_LL + cz_pair_index(LO_, HI_):                                        \
-        if constexpr (LO_ < K && HI_ < K) ph2_ll<R, K, MODE, LO_, HI_>(ra > rb, tp, flags, a, l, q, accp, acc_add); \
+        if constexpr (LO_ < K && HI_ < K) ph2_ll<R, K, MODE, FULL, LO_, HI_>(ra > rb, tp, flags, a, l, q, accp, acc_add); \
         break;
         VQC_PH2LL(0, 1) VQC_PH2LL(0, 2) VQC_PH2LL(0, 3) VQC_PH2LL(0, 4)
         VQC_PH2LL(1, 2) VQC_PH2LL(1, 3) VQC_PH2LL(1, 4)
@@ -990,12 +1000,12 @@ __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 <<
 #undef VQC_PH2LL
 #define VQC_PH2PL(L_)                                                                \
     case DC_PH2_PL + L_:                                                             \
-        if constexpr (L_ < K) ph2_pl<R, K, MODE, L_>(ra < kRefPhys, physbit(pb, ra < kRefPhys ? rb : ra), tp, flags, a, l, q, accp, acc_add); \
+        if constexpr (L_ < K) ph2_pl<R, K, MODE, FULL, L_>(ra < kRefPhys, physbit(pb, ra < kRefPhys ? rb : ra), tp, flags, a, l, q, accp, acc_add); \
         break;
         VQC_PH2PL(0) VQC_PH2PL(1) VQC_PH2PL(2) VQC_PH2PL(3) VQC_PH2PL(4)
 #undef VQC_PH2PL
     case DC_PH2_PP:
-        ph2_pp<R, K, MODE>((int)physbit(pb, ra) + 2 * (int)physbit(pb, rb), tp, flags, a, l, q, accp,
+        ph2_pp<R, K, MODE, FULL>((int)physbit(pb, ra) + 2 * (int)physbit(pb, rb), tp, flags, a, l, q, accp,
                            acc_add);
         break;
     default:
@@ -1006,7 +1016,7 @@ __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 <<
 // Run ops [ob, oe) of a stage (forward: in order; backward: reversed).  The
 // descriptor is read when the op starts: keeping a prefetched one live across
 // the dispatch switch costs more registers than the load latency it hides.
-template <typename R, int K, int MODE, bool WITH_CX>
+template <typename R, int K, int MODE, bool WITH_CX, bool FULL>
 __device__ __forceinline__ void run_ops(const DOp* ops, int ob, int oe, uint32_t pb,
                                         C2<R> (&a)[1 << K], C2<R> (&l)[1 << K], const R* sh_tab,
                                         const R* ps_tab, R* acc, const Geo& q, int lane,
@@ -1014,11 +1024,11 @@ __device__ __forceinline__ void run_ops(const DOp* ops, int ob, int oe, uint32_t
     const uint2* op2 = reinterpret_cast<const uint2*>(ops);
     if (MODE == 0) {
         for (int o = ob; o < oe; ++o)
-            apply_op<R, K, MODE, WITH_CX>(vqc_ld(op2 + o), pb, a, l, sh_tab, ps_tab, acc, q, lane,
+            apply_op<R, K, MODE, WITH_CX, FULL>(vqc_ld(op2 + o), pb, a, l, sh_tab, ps_tab, acc, q, lane,
                                           warp_in_group, acc_add);
     } else {
         for (int o = oe - 1; o >= ob; --o)
-            apply_op<R, K, MODE, WITH_CX>(vqc_ld(op2 + o), pb, a, l, sh_tab, ps_tab, acc, q, lane,
+            apply_op<R, K, MODE, WITH_CX, FULL>(vqc_ld(op2 + o), pb, a, l, sh_tab, ps_tab, acc, q, lane,
                                           warp_in_group, acc_add);
     }
 }
@@ -1188,7 +1198,9 @@ __device__ void acc_terms(const DAcc& ac, const DEntry& e, const R* ap, int wg,
 
 // ---------------------------------------------------------------- kernel
 // MODE 0: forward, MODE 1: backward.
-template <typename R, int K, int MODE>
+// FULL: every sample group spans whole warps (2^(n-K) >= 32 threads), so warp
+// reductions are fixed full-warp butterflies; the launch picks the variant.
+template <typename R, int K, int MODE, bool FULL>
 __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArgs<R> A) {
     extern __shared__ __align__(16) unsigned char smem[];
     R* sh_tab = reinterpret_cast<R*>(smem + A.sm_sh);
@@ -1337,10 +1349,10 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                     } else {
                         block_load<R, K>(a, psi, v.swb, sg);
                     }
-                    run_ops<R, K, 0, false>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
+                    run_ops<R, K, 0, false, FULL>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
                                      sh_tab, ps_tab, nullptr, q, lane, warp_in_group);
                     if (MODE == 0 && last) {   // <Z_j> partials from the final blocks
-                        if (q.lanes == 32) {   // butterfly over the warp (n <= 16 here)
+                        if constexpr (FULL) {   // butterfly over the warp (n <= 16 here)
                             if (n <= 8) {
                                 R ez[8];
 #pragma unroll
@@ -1369,7 +1381,7 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                         block_store<R, K>(a, psi, b2, s2);
                     }
                 }
-                if (MODE == 0 && last && q.lanes == 32) {
+                if (MODE == 0 && last && FULL) {
                     // a single-warp group writes E itself
                     const int low = n <= 8 ? 3 : 1;   // lane bits below the scatter bits
                     if ((lane & low) == 0 && eidx < n) {
@@ -1385,7 +1397,7 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
         }
 
         if (MODE == 0) {
-            const bool direct = q.lanes == 32 && q.wg == 1;   // E already written
+            const bool direct = FULL && q.wg == 1;   // E already written
             if (!direct || A.state_out) {
                 __syncthreads();
                 if (valid) {
@@ -1421,7 +1433,7 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                     block_load<R, K>(a, psi, b2, s2);
                     block_load<R, K>(l, lam, b2, s2);
                 }
-                run_ops<R, K, 1, false>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l,
+                run_ops<R, K, 1, false, FULL>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l,
                                  sh_tab, ps_tab, acc, q, lane, warp_in_group, bj > 0);
                 if (s > 0) {   // back to the stage's input layout (load map)
                     if (vqc_ld(&sp->nperm)) group_sync<R>(q);   // see the forward's store
