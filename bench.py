@@ -298,7 +298,7 @@ def run_ours(args, rank, world, local_rank):
     # fixed-order dw sum; HBM-tiled: one launch per pass plus the partial sums
     # (E; dx and dw), the backward starting from the saved final state
     nw, nx = w_.spec.num_w > 0, w_.spec.num_x > 0
-    launches_fwd = 1 if info["fwd_path"] == 0 else info["fwd_passes"] + 1
+    launches_fwd = info["fwd_passes"] + 1 if info["fwd_path"] == 1 else 1
     launches_bwd = (1 + int(nw)) if not hbm_path else info["bwd_passes"] + int(nx) + int(nw)
     launches_per_step = launches_fwd + launches_bwd
     bwd_avg_s = statistics.mean(bwd_ms) / 1e3
@@ -532,7 +532,7 @@ def extra_configs(torch, Circuit, B):
                 real = torch.float32 if w_.dtype == "c64" else torch.float64
                 c = Circuit(w_.spec, w_.dtype)
                 inf = c.info(w_.batch)
-                path = "hbm-tiled" if inf["fwd_path"] == 1 else "resident"
+                path = {0: "resident", 1: "hbm-tiled", 2: "cluster"}[inf["fwd_path"]]
                 x = torch.tensor(w_.x, dtype=real, device="cuda")
                 w = torch.tensor(w_.w, dtype=real, device="cuda") if w_.spec.num_w else None
                 gE = torch.tensor(w_.gE, dtype=real, device="cuda")

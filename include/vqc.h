@@ -104,7 +104,11 @@ typedef struct {
 /* Execution paths a plan can take. */
 typedef enum {
     VQC_PATH_RESIDENT = 0,  /* each sample's state stays in one CTA's shared memory */
-    VQC_PATH_HBM = 1        /* state in HBM, swept in shared-memory tiles, one launch per pass */
+    VQC_PATH_HBM = 1,       /* state in HBM, swept in shared-memory tiles, one launch per pass */
+    VQC_PATH_CLUSTER = 2    /* forward: each sample's state spread over the shared memory of a
+                               thread-block cluster (2..8 CTAs), one launch; taken only when the
+                               environment sets VQC_FORCE_PATH=cluster (otherwise such states
+                               go through VQC_PATH_HBM, measured faster) */
 } vqc_path;
 
 typedef struct {

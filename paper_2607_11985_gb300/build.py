@@ -24,7 +24,7 @@ NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2",
 UNITS = ["compiler.cpp", "qasm.cpp", "capi.cu", "noalloc.cu",
          "kernels_f32_fwd.cu", "kernels_f32_bwd.cu", "kernels_f64_fwd.cu", "kernels_f64_bwd.cu",
          "kernels_f32_fwd_small.cu", "kernels_f32_bwd_small.cu", "kernels_f64_fwd_small.cu",
-         "kernels_f64_bwd_small.cu", "kernels_hbm.cu"]
+         "kernels_f64_bwd_small.cu", "kernels_hbm.cu", "kernels_cluster.cu"]
 
 
 def nvcc() -> str:

@@ -101,6 +101,7 @@ struct Launch {
     size_t smem = 0;
     int sm_sh = 0, sm_ps = 0, sm_psi = 0, sm_lam = 0, sm_acc = 0, sm_terms = 0, sm_dw = 0,
         sm_red = 0, sm_plan = 0, sm_w = 0, sm_xg = 0;
+    int cl = 0, sm_ecl = 0;   // cluster path: log2 CTAs per sample, <Z> gather area
     bool plan_smem = false;
     const void* fn = nullptr;
 };
@@ -130,6 +131,11 @@ cudaError_t launch(const void* fn, dim3 grid, dim3 block, void** args, size_t sm
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cudaLaunchKernelExC(&cfg, fn, args);
+}
+
+int cta_threads() {
+    const int t = env_int("VQC_CTA_THREADS", 128);
+    return t >= 32 && t <= 512 ? t : 128;
 }
 
 // Pick the register-block size: the largest K that still gives the batch
@@ -177,7 +183,8 @@ vqc_status plan_launch_uncached(const HostPlan& p, int mode, int B, Launch& L) {
                               (size_t)(p.num_x + p.n) * rs +
                               (mode == 1 ? p.accs.size() * L.wg * 8 * rs + p.term_src.size() * rs
                                          : (size_t)L.wg * p.n * rs);
-    int S = std::max(1, 128 / L.T);
+    // samples per CTA: groups up to VQC_CTA_THREADS (default 128) threads
+    int S = std::max(1, cta_threads() / L.T);
     if ((size_t)di.smem_optin > fixed) {
         size_t fit = ((size_t)di.smem_optin - fixed) / per_sample;
         S = (int)std::min<size_t>((size_t)S, fit);
@@ -232,13 +239,14 @@ vqc_status plan_launch_uncached(const HostPlan& p, int mode, int B, Launch& L) {
 
 std::mutex g_geo_mu;
 std::map<GeoKey, Launch> g_launch_cache;
+std::map<GeoKey, Launch> g_cluster_cache;   // cluster-path geometry (forget_plan clears it too)
 
 GeoKey geo_key(const HostPlan& p, int mode, int B, int hbm) {
     int dev = -1;
     cudaGetDevice(&dev);
     // environment switches that change the geometry are part of the key
     const int env = env_int("VQC_FORCE_K_FWD", 0) * 1000 + env_int("VQC_FORCE_K_BWD", 0) * 10 +
-                    (env_int("VQC_PLAN_IN_SMEM", 1) != 0 ? 1 : 0);
+                    (env_int("VQC_PLAN_IN_SMEM", 1) != 0 ? 1 : 0) + cta_threads() * 1000000;
     return GeoKey{&p, mode, B, dev, hbm * 100000 + env};
 }
 
@@ -301,6 +309,8 @@ void fill_plan_args(const HostPlan& p, const Launch& L, KArgs<R>& a) {
     a.sched_bytes = (int)(L.s->dev_region_end - L.s->dev_region_begin);
     a.sm_plan = L.sm_plan;
     a.plan_smem = L.plan_smem ? 1 : 0;
+    a.cl = L.cl;
+    a.sm_ecl = L.sm_ecl;
 }
 
 // Device buffer layout of a plan (all sections 16-byte aligned).
@@ -415,6 +425,122 @@ vqc_status run(const HostPlan& p, int mode, int B, const void* x, const void* w,
 }
 
 
+// ---------------------------------------------------------------- cluster path
+
+vqc_status plan_cluster(const HostPlan& p, int B, Launch& L) {
+    const GeoKey k = geo_key(p, 0, B, 2);
+    {
+        std::lock_guard<std::mutex> lk(g_geo_mu);
+        auto it = g_cluster_cache.find(k);
+        if (it != g_cluster_cache.end()) {
+            L = it->second;
+            return VQC_OK;
+        }
+    }
+    L = Launch();
+    L.s = find_cluster_schedule(p, 0);
+    if (!L.s) return fail(VQC_ERR_UNSUPPORTED, "no cluster schedule for this circuit");
+    int dev = 0;
+    VQC_CUDA(cudaGetDevice(&dev));
+    DevInfo di;
+    vqc_status st = device_info(dev, di);
+    if (st != VQC_OK) return st;
+    const bool dbl = p.dtype == VQC_C128;
+    const size_t rs = dbl ? 8 : 4, cs = 2 * rs, ew = dbl ? 8 : 32;
+    L.K = L.s->K;
+    L.cl = p.n - L.K - 9;
+    L.T = 1 << (p.n - L.K);           // threads of a sample group, over the whole cluster
+    L.block = L.T >> L.cl;            // 512
+    L.S = 1;
+    L.bpt = 1;
+    L.wg = L.block / 32;
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        size_t o = off;
+        off = align16(off + bytes);
+        return (int)o;
+    };
+    L.sm_sh = take((size_t)p.n_sh * ew * rs);
+    L.sm_ps = take((size_t)p.n_ps * ew * rs);
+    L.sm_psi = take(((size_t)1 << (p.n - L.cl)) * cs);
+    L.sm_red = take((size_t)L.wg * p.n * rs);
+    L.sm_ecl = take(((size_t)1 << L.cl) * p.n * rs);
+    L.sm_w = take((size_t)p.num_w * rs);
+    L.sm_xg = take((size_t)p.num_x * rs);
+    const size_t plan_bytes = align16(p.dev_tab_end - p.dev_tab_begin) +
+                              (L.s->dev_region_end - L.s->dev_region_begin);
+    L.plan_smem = off + plan_bytes <= (size_t)di.smem_optin && env_int("VQC_PLAN_IN_SMEM", 1) != 0;
+    L.sm_plan = L.plan_smem ? take(plan_bytes) : 0;
+    L.smem = off;
+    if (L.smem > (size_t)di.smem_optin)
+        return fail(VQC_ERR_UNSUPPORTED, "cluster slice does not fit in shared memory");
+    L.fn = cluster_ptr(dbl);
+    VQC_CUDA(cudaFuncSetAttribute(L.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem));
+    cudaLaunchConfig_t cfg{};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1u << L.cl;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(1u << L.cl);
+    cfg.blockDim = dim3(L.block);
+    cfg.dynamicSmemBytes = L.smem;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int nclusters = 0;
+    VQC_CUDA(cudaOccupancyMaxActiveClusters(&nclusters, L.fn, &cfg));
+    if (nclusters < 1) return fail(VQC_ERR_UNSUPPORTED, "cluster kernel cannot be resident");
+    L.nunits = B;
+    L.grid = std::min(B, nclusters) << L.cl;
+    std::lock_guard<std::mutex> lk(g_geo_mu);
+    g_cluster_cache[k] = L;
+    return VQC_OK;
+}
+
+// The cluster forward only when VQC_FORCE_PATH=cluster asks for it: on the
+// 16-qubit, 8-layer workload it measures below the HBM-tiled passes (one sample
+// per cluster leaves too few warps per SM to hide the per-stage cluster barriers).
+bool use_cluster(const HostPlan& p, int mode) {
+    if (mode != 0 || !find_cluster_schedule(p, 0)) return false;
+    const char* f = std::getenv("VQC_FORCE_PATH");
+    return f && std::string(f) == "cluster";
+}
+
+template <typename R>
+vqc_status run_cluster_forward(const HostPlan& p, int B, const void* x, const void* w,
+                               const void* psi0, void* E, void* state_out, cudaStream_t stream) {
+    using C = C2<R>;
+    Launch L;
+    vqc_status st = plan_cluster(p, B, L);
+    if (st != VQC_OK) return st;
+    KArgs<R> a{};
+    fill_plan_args<R>(p, L, a);
+    a.B = B;
+    a.nunits = B;
+    a.x = static_cast<const R*>(x);
+    a.w = static_cast<const R*>(w);
+    a.psi0 = static_cast<const C*>(psi0);
+    a.E = static_cast<R*>(E);
+    a.state_out = static_cast<C*>(state_out);
+    void* args[] = {&a};
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1u << L.cl;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(L.grid);
+    cfg.blockDim = dim3(L.block);
+    cfg.dynamicSmemBytes = L.smem;
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = env_int("VQC_PDL", 1) != 0 ? 2 : 1;
+    VQC_CUDA(cudaLaunchKernelExC(&cfg, L.fn, args));
+    return VQC_OK;
+}
+
 // ---------------------------------------------------------------- HBM path
 struct PassGeo {
     const Schedule* s = nullptr;
@@ -521,6 +647,8 @@ void forget_plan(const HostPlan* p) {
         it = it->first.plan == p ? g_launch_cache.erase(it) : std::next(it);
     for (auto it = g_pass_cache.begin(); it != g_pass_cache.end();)
         it = it->first.plan == p ? g_pass_cache.erase(it) : std::next(it);
+    for (auto it = g_cluster_cache.begin(); it != g_cluster_cache.end();)
+        it = it->first.plan == p ? g_cluster_cache.erase(it) : std::next(it);
 }
 
 // Workspace of the HBM path.  Forward: [control | working state | <Z> partials].
@@ -861,6 +989,7 @@ size_t vqc_workspace_bytes(const vqc_plan* plan, int32_t batch, int32_t mode) {
     }
     if ((mode != 0 && mode != 1) || batch <= 0) return 0;
     const HostPlan& p = plan->hp;
+    if (use_cluster(p, mode)) return 0;
     if (use_hbm(p, mode, batch)) {
         PassGeo L;
         if (plan_hbm(p, mode, batch, L) != VQC_OK) return 0;
@@ -924,6 +1053,11 @@ vqc_status vqc_forward(const vqc_plan* plan, int32_t batch, const void* x, const
         if (st != VQC_OK) return st;
         if (!expz_out) return fail(VQC_ERR_INVALID_ARG, "expz_out is NULL");
         cudaStream_t s = static_cast<cudaStream_t>(stream);
+        if (use_cluster(p, 0)) {
+            if (p.dtype == VQC_C64)
+                return run_cluster_forward<float>(p, batch, x, w, psi0, expz_out, state_out, s);
+            return run_cluster_forward<double>(p, batch, x, w, psi0, expz_out, state_out, s);
+        }
         if (use_hbm(p, 0, batch)) {
             if (p.dtype == VQC_C64)
                 return run_hbm_forward<float>(p, batch, x, w, psi0, expz_out, state_out, workspace,
@@ -1007,9 +1141,11 @@ vqc_status vqc_plan_info(const vqc_plan* plan, int32_t batch, vqc_plan_stats* ou
         int* tq = mode == 0 ? &out->fwd_tile_qubits : &out->bwd_tile_qubits;
         double* hb = mode == 0 ? &out->fwd_hbm_bytes_per_eval : &out->bwd_hbm_bytes_per_eval;
         const int K = choose_k(p, mode, B);
-        const bool hbm = ndev > 0 ? use_hbm(p, mode, B)
-                                  : (K == 0 && find_hbm_schedule(p, mode) != nullptr);
-        const Schedule* s = hbm ? find_hbm_schedule(p, mode) : (K ? find_schedule(p, mode, K) : nullptr);
+        const bool clu = use_cluster(p, mode);
+        const bool hbm = !clu && (ndev > 0 ? use_hbm(p, mode, B)
+                                           : (K == 0 && find_hbm_schedule(p, mode) != nullptr));
+        const Schedule* s = clu ? find_cluster_schedule(p, mode)
+                          : hbm ? find_hbm_schedule(p, mode) : (K ? find_schedule(p, mode, K) : nullptr);
         if (!s) {
             *path = -1;
             continue;

@@ -1,0 +1,239 @@
+// cluster.cuh -- forward sweep with a sample's state spread over a thread-block
+// cluster (distributed shared memory), for states larger than one SM's shared
+// memory but small enough for 2..8 SMs (complex64: 15-17 qubits, complex128:
+// 14-16 qubits).
+//
+// Same stage program as the resident path (sweep.cuh): the stage maps give
+// every register amplitude a slot in [0, 2^n); slot s lives in the shared memory
+// of cluster rank s >> (n - CL) at local position s & (2^(n-CL) - 1).  The
+// swizzle only XORs the lowest G index bits, so a CTA holds exactly the
+// amplitudes whose top CL qubits equal its rank.  Loads and stores go through
+// the cluster window (mapa + ld/st.shared::cluster); a cluster barrier replaces
+// the group barrier between stages.  A stage whose maps keep every block inside
+// its thread's own CTA (the compiler's cl_local flags) uses plain shared loads
+// and stores and, when no data crosses CTAs at its end, the CTA barrier.  One sample per cluster at a time; the
+// 2^(n-K) threads of its group are spread over the cluster's CTAs in rank
+// order.  The <Z> sums go from each CTA to rank 0, which writes E.
+#pragma once
+
+#include "sweep.cuh"
+
+namespace vqc {
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+// Every thread of every CTA of the cluster arrives; memory operations before
+// it (including shared::cluster stores) are visible to all of them after it.
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n"
+                 "barrier.cluster.wait.acquire.aligned;\n" ::: "memory");
+}
+// Address of local shared address `sa` in the shared memory of cluster rank r.
+__device__ __forceinline__ uint32_t cluster_map(uint32_t sa, uint32_t r) {
+    uint32_t d;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(sa), "r"(r));
+    return d;
+}
+__device__ __forceinline__ float2 dsm_load(uint32_t a, float2*) {
+    float2 v;
+    asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a) : "memory");
+    return v;
+}
+__device__ __forceinline__ double2 dsm_load(uint32_t a, double2*) {
+    double2 v;
+    asm volatile("ld.shared::cluster.v2.f64 {%0, %1}, [%2];" : "=d"(v.x), "=d"(v.y) : "r"(a) : "memory");
+    return v;
+}
+__device__ __forceinline__ void dsm_store(uint32_t a, float2 v) {
+    asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(a), "f"(v.x), "f"(v.y) : "memory");
+}
+__device__ __forceinline__ void dsm_store(uint32_t a, double2 v) {
+    asm volatile("st.shared::cluster.v2.f64 [%0], {%1, %2};" ::"r"(a), "d"(v.x), "d"(v.y) : "memory");
+}
+__device__ __forceinline__ void dsm_store(uint32_t a, float v) {
+    asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(a), "f"(v) : "memory");
+}
+__device__ __forceinline__ void dsm_store(uint32_t a, double v) {
+    asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(a), "d"(v) : "memory");
+}
+
+// Cluster address of slot s of the distributed state (psi_sa: this CTA's local
+// shared address of its slice; slices are 2^slice amplitudes).
+template <typename R>
+__device__ __forceinline__ uint32_t slot_addr(uint32_t psi_sa, uint32_t s, int slice) {
+    const uint32_t owner = s >> slice, off = s & ((1u << slice) - 1u);
+    return cluster_map(psi_sa + off * (uint32_t)sizeof(C2<R>), owner);
+}
+
+template <typename R, int K>
+__device__ __forceinline__ void cl_block_load(C2<R> (&a)[1 << K], uint32_t psi_sa, int slice,
+                                              uint32_t swb, const int32_t (&sg)[K]) {
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r)
+        a[r] = dsm_load(slot_addr<R>(psi_sa, swb ^ block_off<K>(r, sg), slice), (C2<R>*)nullptr);
+}
+template <typename R, int K>
+__device__ __forceinline__ void cl_block_store(const C2<R> (&a)[1 << K], uint32_t psi_sa, int slice,
+                                               uint32_t swb, const int32_t (&sg)[K]) {
+#pragma unroll
+    for (int r = 0; r < (1 << K); ++r) dsm_store(slot_addr<R>(psi_sa, swb ^ block_off<K>(r, sg), slice), a[r]);
+}
+
+// KArgs fields used: the plan, n, K, G, tpg (= 2^(n-K), threads per sample over
+// the cluster), nunits (= B), x, w, psi0, E, state_out, the shared-memory
+// carve-up (sm_psi holds this CTA's slice of 2^(n - cl) amplitudes, sm_red the
+// per-warp <Z> sums, sm_ecl rank 0's [2^cl][n] gather of per-CTA sums), cl.
+template <typename R, int K>
+__global__ void __launch_bounds__(512) cluster_fwd_kernel(const __grid_constant__ KArgs<R> A) {
+    extern __shared__ __align__(16) unsigned char smem[];
+    R* sh_tab = reinterpret_cast<R*>(smem + A.sm_sh);
+    R* ps_tab = reinterpret_cast<R*>(smem + A.sm_ps);
+    C2<R>* psi = reinterpret_cast<C2<R>*>(smem + A.sm_psi);
+    R* red = reinterpret_cast<R*>(smem + A.sm_red);
+    R* ecl = reinterpret_cast<R*>(smem + A.sm_ecl);
+    R* w_sm = reinterpret_cast<R*>(smem + A.sm_w);
+    R* xrow = reinterpret_cast<R*>(smem + A.sm_xg);
+
+    const int n = A.n, G = A.G, CL = A.cl;
+    const int slice = n - CL;
+    const uint32_t smask = (1u << slice) - 1u;
+    const uint32_t rank = cluster_rank();
+    const int cid = (int)(blockIdx.x >> CL), ncl = (int)(gridDim.x >> CL);
+    const int nthr = blockDim.x;
+    const int tg = (int)rank * nthr + (int)threadIdx.x;   // thread index in the sample group
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = nthr >> 5;
+    Geo q;
+    q.T = A.tpg;
+    q.lanes = 32;
+    q.wg = nwarps;
+    q.g = 0;
+    q.t = tg;
+    q.h = 0;
+    q.mask = 0xffffffffu;
+    const uint32_t psi_sa = static_cast<uint32_t>(__cvta_generic_to_shared(psi));
+    const uint32_t ecl_sa = static_cast<uint32_t>(__cvta_generic_to_shared(ecl));
+
+    // plan regions (immutable) before the dependency wait; then caller memory
+    const unsigned char* smt = nullptr;
+    const unsigned char* sms = nullptr;
+    if (A.plan_smem) {
+        unsigned char* t = smem + A.sm_plan;
+        unsigned char* u = t + ((A.tab_bytes + 15) & ~15);
+        async_region(t, A.plan + A.tab_off, A.tab_bytes);
+        async_region(u, A.plan + A.sched_off, A.sched_bytes);
+        smt = t;
+        sms = u;
+    }
+    grid_dep_wait();
+    grid_dep_launch();
+    for (int i = threadIdx.x; i < A.Pw; i += nthr) async_elem<R>(w_sm + i, A.w + i);
+    async_wait();
+    PlanPtrs P;
+    P.ops = rebase(A.ops, A.plan, A.sched_off, sms);
+    P.stages = rebase(A.stages, A.plan, A.sched_off, sms);
+    P.entries = rebase(A.entries, A.plan, A.tab_off, smt);
+    P.ps_list = rebase(A.ps_list, A.plan, A.tab_off, smt);
+    P.sh_list = rebase(A.sh_list, A.plan, A.tab_off, smt);
+    P.consts = rebase(A.consts, A.plan, A.tab_off, smt);
+    P.cmat = rebase(reinterpret_cast<const unsigned char*>(A.cmat), A.plan, A.tab_off, smt);
+    P.cang = rebase(reinterpret_cast<const unsigned char*>(A.cang), A.plan, A.tab_off, smt);
+    const R* Pcmat = reinterpret_cast<const R*>(P.cmat);
+    const R* Pcang = reinterpret_cast<const R*>(P.cang);
+    __syncthreads();
+    for (int i = threadIdx.x; i < A.n_sh; i += nthr) {
+        const DEntry e = P.entries[vqc_ld(&P.sh_list[i])];
+        eval_entry<R>(e, P.consts, nullptr, w_sm, Pcang, Pcmat, sh_tab + EntryWords<R>::value * e.slot);
+    }
+
+    const int ns = A.nstages;
+    for (int b = cid; b < A.nunits; b += ncl) {
+        // this sample's x row, per-sample table and (given psi0) this CTA's slice
+        for (int i = threadIdx.x; i < A.Px; i += nthr) xrow[i] = A.x[(size_t)b * A.Px + i];
+        if (A.psi0) {
+            const C2<R>* gs = A.psi0 + ((size_t)b << n) + ((size_t)rank << slice);
+            const uint32_t u0 = rank << slice;
+            for (uint32_t v = threadIdx.x; v < (1u << slice); v += nthr)
+                psi[swz(u0 + v, G) & ((1u << slice) - 1u)] = gs[v];
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < A.n_ps; i += nthr) {
+            const DEntry e = P.entries[vqc_ld(&P.ps_list[i])];
+            eval_entry<R>(e, P.consts, xrow, w_sm, Pcang, Pcmat, ps_tab + EntryWords<R>::value * e.slot);
+        }
+        cluster_sync();   // tables ready here, every slice loaded cluster-wide
+
+        C2<R> a[1 << K];
+        int32_t sg[K];
+        R eacc = 0;
+        int eidx = 0;
+        for (int s = 0; s < ns; ++s) {
+            const DStage* sp = P.stages + s;
+            const bool last = s + 1 == ns;
+            const StageView v = stage_view<K>(sp, tg, 0, sg);
+            const int loc = vqc_ld(&sp->cl_local);
+            const int loc_next = last ? 1 : vqc_ld(&sp[1].cl_local);
+            if (s == 0 && !A.psi0) {
+#pragma unroll
+                for (int r = 0; r < (1 << K); ++r) a[r] = cm<R>(0, 0);
+                if (v.pb == 0) a[0] = cm<R>(1, 0);
+            } else if (loc & 1) {   // every block in this CTA: plain shared loads
+                block_load<R, K>(a, psi, v.swb & smask, sg);
+            } else {
+                cl_block_load<R, K>(a, psi_sa, slice, v.swb, sg);
+            }
+            run_ops<R, K, 0, false, true>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
+                                         sh_tab, ps_tab, nullptr, q, lane, warp);
+            if (last) {   // <Z_j> partials: one butterfly per warp (n <= 16 here)
+                R ez[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) ez[j] = 0;
+                expz_accum<R, K, 16>(sp, v.pb, a, ez);
+                eidx = warp_reduce_scatter<R, 16>(ez, lane);
+                eacc = ez[0];
+            }
+            if (!last || A.state_out) {
+                // Permuting store: every load that reads a slot it overwrites first
+                // (only this CTA's threads read this CTA's slice when the loads are local).
+                if (vqc_ld(&sp->nperm)) {
+                    if (loc == 3) __syncthreads();
+                    else cluster_sync();
+                }
+                int32_t s2[K];
+                const uint32_t b2 = map_base<K, true>(sp, tg, 0, s2);
+                if (loc & 2) block_store<R, K>(a, psi, b2 & smask, s2);
+                else cl_block_store<R, K>(a, psi_sa, slice, b2, s2);
+                // Data crosses CTAs only through a remote store here or a remote
+                // load next; otherwise the CTA's own barrier orders the stages.
+                if ((loc & 2) && (loc_next & 1)) __syncthreads();
+                else cluster_sync();
+            }
+        }
+        // E: warps -> CTA -> rank 0, summed in fixed order
+        if ((lane & 1) == 0 && eidx < n) red[warp * n + eidx] = eacc;
+        __syncthreads();
+        for (int j = threadIdx.x; j < n; j += nthr) {
+            R e = 0;
+            for (int k = 0; k < nwarps; ++k) e += red[k * n + j];
+            dsm_store(cluster_map(ecl_sa + (uint32_t)((rank * n + j) * sizeof(R)), 0), e);
+        }
+        cluster_sync();
+        if (rank == 0)
+            for (int j = threadIdx.x; j < n; j += nthr) {
+                R e = 0;
+                for (int r = 0; r < (1 << CL); ++r) e += ecl[r * n + j];
+                A.E[(size_t)b * n + j] = e;
+            }
+        if (A.state_out) {   // this CTA's slice, logical order
+            C2<R>* go = A.state_out + ((size_t)b << n) + ((size_t)rank << slice);
+            const uint32_t u0 = rank << slice;
+            for (uint32_t v = threadIdx.x; v < (1u << slice); v += nthr)
+                go[v] = psi[swz(u0 + v, G) & ((1u << slice) - 1u)];
+        }
+        cluster_sync();   // slices and rank 0's gather area are reused by the next sample
+    }
+}
+
+}  // namespace vqc

@@ -655,6 +655,42 @@ vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx,
             p.scheds.push_back(std::move(s));
         }
     }
+    // Cluster schedules (forward): states up to 16 qubits over 2..8 CTAs of a
+    // thread-block cluster, one register block per thread (2^(n-K) threads, at
+    // most 512 per CTA) and at most 128 KiB of state per CTA.
+    {
+        const int K = max_k(0, dtype);
+        const int cl = n - K - 9;
+        const size_t cs = dtype == VQC_C128 ? 16 : 8;
+        if (n > resident_max_qubits(0, dtype) && n <= 16 && cl >= 1 && cl <= 3 &&
+            (((size_t)1 << (n - cl)) * cs) <= 128 * 1024) {
+            Schedule s;
+            s.mode = 0;
+            s.K = K;
+            s.path = VQC_PATH_CLUSTER;
+            build_schedule(p, s);
+            // A map keeps every block in its thread's own CTA when no local offset
+            // reaches the top cl slot bits (those index the CTA) and the top cl
+            // thread bits (the thread's rank) map onto them identically.
+            const int slice = n - cl;
+            for (DStage& st : s.stages) {
+                const int nb = st.nthreadbits;
+                auto local = [&](const int32_t* sig, const int32_t* tau) {
+                    for (int j = 0; j < K; ++j)
+                        if ((uint32_t)sig[j] >> slice) return false;
+                    for (int i = 0; i < nb; ++i) {
+                        const uint32_t top = (uint32_t)tau[i] >> slice;
+                        const uint32_t want = i >= nb - cl ? 1u << (i - (nb - cl)) : 0u;
+                        if (top != want) return false;
+                    }
+                    return true;
+                };
+                st.cl_local = (uint8_t)((local(st.sigma, st.tau) ? 1 : 0) |
+                                        (local(st.sigma_st, st.tau_st) ? 2 : 0));
+            }
+            p.scheds.push_back(std::move(s));
+        }
+    }
     // HBM-tiled pass schedules (tile of m qubits, K fixed per mode and type).
     for (int mode = 0; mode < 2; ++mode) {
         int m = std::min(hbm_tile_qubits(mode, dtype, p.G_swz), n - 1);
@@ -680,6 +716,12 @@ vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx,
 const Schedule* find_schedule(const HostPlan& p, int mode, int K) {
     for (const auto& s : p.scheds)
         if (s.mode == mode && s.K == K && s.path == VQC_PATH_RESIDENT) return &s;
+    return nullptr;
+}
+
+const Schedule* find_cluster_schedule(const HostPlan& p, int mode) {
+    for (const auto& s : p.scheds)
+        if (s.mode == mode && s.path == VQC_PATH_CLUSTER) return &s;
     return nullptr;
 }
 

@@ -97,6 +97,7 @@ vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx,
                         int dtype, HostPlan& out, std::string& err);
 const Schedule* find_schedule(const HostPlan& p, int mode, int K);
 const Schedule* find_hbm_schedule(const HostPlan& p, int mode);
+const Schedule* find_cluster_schedule(const HostPlan& p, int mode);
 std::vector<uint8_t> export_plan(const HostPlan& p);
 
 }  // namespace vqc

@@ -21,6 +21,7 @@ const void* reduce_dx_ptr(bool dbl);
 const void* reduce_dw_ptr(bool dbl);
 const void* reduce_cols_ptr(bool dbl);
 const void* abs2_ptr(bool dbl);   // |psi|^2, elementwise
+const void* cluster_ptr(bool dbl);   // cluster-path forward (K = 5 / 4 for complex64 / 128)
 
 // Largest block (threads) each instantiation is compiled for.
 inline int sweep_max_threads(bool is_double, int mode, int K) {

@@ -92,7 +92,8 @@ struct DStage {
     uint8_t active[kMaxK];            // physical qubit of local bit j
     uint8_t nthreadbits;
     uint8_t nperm;                    // CX gates absorbed into the store map
-    uint8_t pad;
+    uint8_t cl_local;                 // cluster path: bit 0 loads, bit 1 stores stay in the
+                                      // thread's own CTA (its rank = top thread bits)
 };
 static_assert(sizeof(DStage) == 248, "DStage layout");
 

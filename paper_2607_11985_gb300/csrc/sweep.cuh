@@ -201,6 +201,8 @@ struct KArgs {
     // [sched_off, sched_off + sched_bytes) of the plan's device blob.
     const unsigned char* plan;
     int tab_off, tab_bytes, sched_off, sched_bytes, sm_plan, plan_smem;
+    // cluster path only (cluster.cuh): log2 CTAs per sample, rank 0's <Z> gather area
+    int cl, sm_ecl;
 };
 
 struct PlanPtrs {

@@ -21,13 +21,13 @@ DOP = np.dtype([("code", "u1"), ("a", "u1"), ("b", "u1"), ("flags", "u1"), ("slo
                 ("aux", "<u2")])
 DSTAGE = np.dtype([("op_begin", "<i4"), ("op_end", "<i4"), ("sigma", "<i4", 5), ("tau", "<i4", 16),
                    ("tmask", "<u4", 16), ("sigma_st", "<i4", 5), ("tau_st", "<i4", 16),
-                   ("active", "u1", 5), ("nthreadbits", "u1"), ("nperm", "u1"), ("pad", "u1")])
+                   ("active", "u1", 5), ("nthreadbits", "u1"), ("nperm", "u1"), ("cl_local", "u1")])
 DPASS = np.dtype([("stage_begin", "<i4"), ("stage_end", "<i4"), ("m", "<i4"), ("nout", "<i4"),
                   ("tile_q", "u1", 24), ("out_q", "u1", 24), ("ps_begin", "<i4"), ("ps_count", "<i4"),
                   ("sh_begin", "<i4"), ("sh_count", "<i4"), ("acc_begin", "<i4"), ("acc_count", "<i4")])
 assert DENTRY.itemsize == 12 and DCONST.itemsize == 16 and DOP.itemsize == 8
 assert DSTAGE.itemsize == 248 and DPASS.itemsize == 88
-PATH_RESIDENT, PATH_HBM = 0, 1
+PATH_RESIDENT, PATH_HBM, PATH_CLUSTER = 0, 1, 2
 
 OP_M1, OP_CX, OP_CZ, OP_PH2 = 1, 2, 3, 4
 DC_M1, DC_CX_LL, DC_CX_PL, DC_CZ_LL, DC_CZ_PL, DC_CZ_PP = 0, 5, 25, 30, 40, 45
@@ -241,7 +241,7 @@ class Plan:
         """(stages, tile bases, tables, acc map) of each pass; the resident path
         is one pass over one tile holding every qubit."""
         n = self.n
-        if sched["path"] == PATH_RESIDENT:
+        if sched["path"] in (PATH_RESIDENT, PATH_CLUSTER):
             yield (sched["stages"], [0], self.tables(xb, w), np.arange(len(self.accs)),
                    sched["store_masks"])
             return

@@ -115,7 +115,7 @@ def check_addressing(plan):
     bijections onto the tile's slots."""
     for s in plan.scheds:
         n, K, m = plan.n, s["K"], s["m"]
-        if s["path"] == 0:
+        if s["path"] in (0, 2):   # resident / cluster: one tile holding every qubit
             tiles = [(list(range(n)), range(len(s["stages"])))]
         else:
             tiles = [(list(ps["tile_q"][:ps["m"]]), range(ps["stage_begin"], ps["stage_end"]))
@@ -155,7 +155,7 @@ def check_addressing(plan):
                         assert oa < K
                     if t == 2:
                         assert ob < K
-                        assert s["path"] == 1   # resident schedules fold every CX
+                        assert s["path"] == 1   # resident and cluster schedules fold every CX
             # <Z> / lambda come from the last stage's registers (of each pass)
             assert int(s["stages"][srange[-1]]["nperm"]) == 0
 
@@ -231,6 +231,47 @@ def test_config5_hbm_schedule_structure():
                 int(s["stages"]["nperm"].sum()) == len(pl.hops)
             assert int(s["stages"]["nperm"].sum()) > 0
             assert s["passes"][-1]["stage_end"] == len(s["stages"])
+
+
+def slots_all(st, K, sig, tau):
+    """slot_of for every (thread, register) pair at once: [threads, 2^K]."""
+    nb = int(st["nthreadbits"])
+    t = np.arange(1 << nb)
+    base = np.zeros(1 << nb, np.int64)
+    for i in range(nb):
+        base ^= np.where((t >> i) & 1, int(st[tau][i]), 0)
+    r = np.arange(1 << K)
+    off = np.zeros(1 << K, np.int64)
+    for j in range(K):
+        off ^= np.where((r >> j) & 1, int(st[sig][j]), 0)
+    return base[:, None] ^ off[None, :]
+
+
+def test_cluster_locality_flags():
+    """Cluster schedules (512 threads per CTA, 2^(n-K-9) CTAs): a stage's
+    cl_local bit 0 / bit 1 is set exactly when every slot its load / store map
+    gives a thread lies in the slice of that thread's own CTA."""
+    w_ = wl.config(5, batch=1)[0]
+    seen = 0
+    for dtype in (0, 1):
+        pl = Plan(B.vqc_plan_export(compile_spec(w_.spec, dtype)))
+        for s in (s for s in pl.scheds if s["path"] == 2):
+            n, K = pl.n, s["K"]
+            slice_ = K + 9
+            rank = (np.arange(1 << (n - K)) >> 9)[:, None]
+            flags = []
+            for st in s["stages"]:
+                ld = bool(((slots_all(st, K, "sigma", "tau") >> slice_) == rank).all())
+                sto = bool(((slots_all(st, K, "sigma_st", "tau_st") >> slice_) == rank).all())
+                assert int(st["cl_local"]) == (ld | (sto << 1))
+                flags.append(int(st["cl_local"]))
+            # a non-permuting stage stores where it loads
+            for st in s["stages"]:
+                if int(st["nperm"]) == 0:
+                    assert int(st["cl_local"]) in (0, 3)
+            assert 3 in flags
+            seen += 1
+    assert seen >= 1
 
 
 @pytest.mark.parametrize("k", [1, 2])

@@ -6,7 +6,9 @@
 * small circuits forced onto the HBM path with 6-qubit tiles (many passes,
   tile-outer controls and phases), against the oracle, with and without psi0
   and the saved final state, ragged batches;
-* cross-path agreement: the 12-qubit workload on the resident and HBM paths.
+* cross-path agreement: the 12-qubit workload on the resident and HBM paths;
+* the thread-block-cluster forward (VQC_FORCE_PATH=cluster) at 14-16 qubits
+  against the oracle and against the HBM passes, and on the 16-qubit workload.
 """
 import numpy as np
 import pytest
@@ -34,7 +36,8 @@ def test_config5_full_batch(dtype):
     w_ = wl.config(5, dtype=dtype)[0]
     c = C(w_.spec, dtype)
     info = c.info(w_.batch)
-    assert info["fwd_path"] == 1 and info["bwd_path"] == 1 and info["fwd_passes"] > 1
+    # 16 qubits: forward and backward in HBM-tiled passes
+    assert info["fwd_path"] == 1 and info["bwd_path"] == 1 and info["bwd_passes"] > 1
     E, st = run_fwd(c, w_)
     rows = [0, w_.batch - 1]
     sub = wl.Workload(w_.name, w_.spec, 2, w_.x[rows], w_.w, w_.gE[rows], dtype, w_.seed)
@@ -132,3 +135,52 @@ def test_hbm_18_qubits_sampled():
     dx, dw = run_bwd(c, w_)
     dx_ref, dw_ref = orc.backward(spec, x, w, gE)
     assert maxerr(dx, dx_ref) <= 5e-4 and maxerr(dw, dw_ref) <= 5e-4
+
+
+@pytest.mark.parametrize("dtype,n", [("c64", 15), ("c64", 16), ("c128", 14), ("c128", 15), ("c128", 16)])
+def test_cluster_forward(monkeypatch, dtype, n):
+    """Forward with the state spread over a thread-block cluster (2, 4 or 8 CTAs):
+    E and the final states against the oracle, from |0...0> and from a given
+    psi0, with and without the state output; the same batch through the
+    HBM-tiled passes agrees."""
+    spec = wl.layered(n, 2, ("RX", "RY", "RZ"), "CX", ring_range=lambda l: 2 * l + 1)
+    rng = np.random.default_rng(1500 + n)
+    B = 3
+    x = wl._round(rng.uniform(-np.pi, np.pi, (B, n)), dtype)
+    w = wl._round(rng.uniform(-np.pi, np.pi, spec.num_w), dtype)
+    gE = wl._round(rng.standard_normal((B, n)), dtype)
+    z = rng.standard_normal((B, 1 << n)) + 1j * rng.standard_normal((B, 1 << n))
+    z /= np.linalg.norm(z, axis=1, keepdims=True)
+    if dtype == "c64":
+        z = z.astype(np.complex64).astype(np.complex128)
+    w_ = wl.Workload("cluster_n%d" % n, spec, B, x, w, gE, dtype, 1500 + n)
+    c = C(spec, dtype)
+    assert c.info(B)["fwd_path"] == 1   # the HBM passes unless asked for the cluster
+    monkeypatch.setenv("VQC_FORCE_PATH", "cluster")
+    assert c.info(B)["fwd_path"] == 2
+    tol = TOL[dtype]
+    for psi0 in (None, z):
+        E_ref, st_ref = orc.forward(spec, x, w, psi0=psi0, want_state=True)
+        E, st = run_fwd(c, w_, psi0)
+        assert maxerr(E, E_ref) <= tol["E"] and maxerr(st, st_ref) <= tol["state"]
+        E2 = run_fwd(c, w_, psi0, want_state=False)
+        assert maxerr(E2, E_ref) <= tol["E"]
+        monkeypatch.setenv("VQC_FORCE_PATH", "hbm")
+        E3, st3 = run_fwd(c, w_, psi0)
+        monkeypatch.setenv("VQC_FORCE_PATH", "cluster")
+        assert maxerr(E3, E) <= tol["E"] and maxerr(st3, st) <= tol["state"]
+
+
+@pytest.mark.parametrize("dtype", ["c64", "c128"])
+def test_config5_cluster_forward(monkeypatch, dtype):
+    """The 16-qubit, 8-layer batch through the cluster forward: sampled rows
+    against the oracle."""
+    monkeypatch.setenv("VQC_FORCE_PATH", "cluster")
+    w_ = wl.config(5, dtype=dtype)[0]
+    c = C(w_.spec, dtype)
+    assert c.info(w_.batch)["fwd_path"] == 2
+    E, st = run_fwd(c, w_)
+    rows = [0, 257, w_.batch - 1]
+    E_ref, st_ref = orc.forward(w_.spec, w_.x[rows], w_.w, want_state=True)
+    assert maxerr(E[rows], E_ref) <= TOL[dtype]["E"]
+    assert maxerr(st[rows], st_ref) <= TOL[dtype]["state"]
