@@ -355,42 +355,35 @@ __device__ __forceinline__ void m1_apply_f2(float2 (&a)[1 << K], const M2<float>
     }
 }
 
-// rho[a][b] += sum_pairs psi[a] conj(lam[b])  -> r[0..7] = (00, 01, 10, 11) re/im
+// Gradient accumulator of a fused run.  With rho = sum_pairs psi conj(lam)^T
+// (2x2, rho[a][b] = psi_a conj(lam_b)), every term the run needs is
+// Im Tr(P rho') for a Pauli P and rho' = W^dag rho W, i.e. it depends only on
+// the traceless anti-Hermitian part of rho, (i/2)(tx X + ty Y + tz Z), and that
+// part stays traceless anti-Hermitian under W^dag . W.  So three reals per
+// thread are summed instead of rho's eight:
+//   tx = Im(rho01 + rho10), ty = Re(rho01 - rho10), tz = Im(rho00 - rho11).
+// Two partial sums per component keep the FMA chains short.
 template <typename R, int K, int T>
-__device__ __forceinline__ void m1_rho(const C2<R> (&ps)[1 << K], const C2<R> (&la)[1 << K],
-                                       R (&r)[8]) {
+__device__ __forceinline__ void m1_t3(const C2<R> (&ps)[1 << K], const C2<R> (&la)[1 << K],
+                                      R (&v)[4]) {
+    R x0 = 0, x1 = 0, y0 = 0, y1 = 0, z0 = 0, z1 = 0;
 #pragma unroll
     for (int p = 0; p < (1 << (K - 1)); ++p) {
         const int i0 = pair_lo<T>(p), i1 = i0 | (1 << T);
-        const C2<R> u = ps[i0], v = ps[i1], q0 = la[i0], q1 = la[i1];
-        r[0] = fma(u.x, q0.x, fma(u.y, q0.y, r[0])); r[1] = fma(u.y, q0.x, fma(-u.x, q0.y, r[1]));
-        r[2] = fma(u.x, q1.x, fma(u.y, q1.y, r[2])); r[3] = fma(u.y, q1.x, fma(-u.x, q1.y, r[3]));
-        r[4] = fma(v.x, q0.x, fma(v.y, q0.y, r[4])); r[5] = fma(v.y, q0.x, fma(-v.x, q0.y, r[5]));
-        r[6] = fma(v.x, q1.x, fma(v.y, q1.y, r[6])); r[7] = fma(v.y, q1.x, fma(-v.x, q1.y, r[7]));
+        const C2<R> u = ps[i0], w = ps[i1], q0 = la[i0], q1 = la[i1];
+        R& xa = (p & 1) ? x1 : x0;
+        R& ya = (p & 1) ? y1 : y0;
+        R& za = (p & 1) ? z1 : z0;
+        // Im(u conj q1) + Im(w conj q0)
+        xa = fma(u.y, q1.x, fma(-u.x, q1.y, fma(w.y, q0.x, fma(-w.x, q0.y, xa))));
+        // Re(u conj q1) - Re(w conj q0)
+        ya = fma(u.x, q1.x, fma(u.y, q1.y, fma(-w.x, q0.x, fma(-w.y, q0.y, ya))));
+        // Im(u conj q0) - Im(w conj q1)
+        za = fma(u.y, q0.x, fma(-u.x, q0.y, fma(-w.y, q1.x, fma(w.x, q1.y, za))));
     }
-}
-
-// complex64 with packed FP32: psi conj(lam) = psi * (lam.re, lam.re) + psi~ * (lam.im, -lam.im)
-// with psi~ = (psi.im, psi.re); r is read as four float2 accumulators.
-template <int K, int T>
-__device__ __forceinline__ void m1_rho_f2(const float2 (&ps)[1 << K], const float2 (&la)[1 << K],
-                                          float (&r)[8]) {
-    float2 r00 = make_float2(r[0], r[1]), r01 = make_float2(r[2], r[3]);
-    float2 r10 = make_float2(r[4], r[5]), r11 = make_float2(r[6], r[7]);
-#pragma unroll
-    for (int p = 0; p < (1 << (K - 1)); ++p) {
-        const int i0 = pair_lo<T>(p), i1 = i0 | (1 << T);
-        const float2 u = ps[i0], v = ps[i1], q0 = la[i0], q1 = la[i1];
-        const float2 us = make_float2(u.y, u.x), vs = make_float2(v.y, v.x);
-        const float2 q0r = make_float2(q0.x, q0.x), q0i = make_float2(q0.y, -q0.y);
-        const float2 q1r = make_float2(q1.x, q1.x), q1i = make_float2(q1.y, -q1.y);
-        r00 = __ffma2_rn(u, q0r, r00); r00 = __ffma2_rn(us, q0i, r00);
-        r01 = __ffma2_rn(u, q1r, r01); r01 = __ffma2_rn(us, q1i, r01);
-        r10 = __ffma2_rn(v, q0r, r10); r10 = __ffma2_rn(vs, q0i, r10);
-        r11 = __ffma2_rn(v, q1r, r11); r11 = __ffma2_rn(vs, q1i, r11);
-    }
-    r[0] = r00.x; r[1] = r00.y; r[2] = r01.x; r[3] = r01.y;
-    r[4] = r10.x; r[5] = r10.y; r[6] = r11.x; r[7] = r11.y;
+    v[0] += x0 + x1;
+    v[1] += y0 + y1;
+    v[2] += z0 + z1;
 }
 
 // complex64 2x2 update with the operand pairs read directly from a table entry
@@ -441,37 +434,7 @@ __device__ __forceinline__ void m1_go(C2<R> (&a)[1 << K], const M2<R>& m) {
     if constexpr (sizeof(R) == 4) m1_apply_f2<K, T>(a, m);
     else m1_apply<R, K, T>(a, m);
 }
-template <typename R, int K, int T>
-__device__ __forceinline__ void rho_go(const C2<R> (&ps)[1 << K], const C2<R> (&la)[1 << K],
-                                       R (&r)[8]) {
-    if constexpr (sizeof(R) == 4) m1_rho_f2<K, T>(ps, la, r);
-    else m1_rho<R, K, T>(ps, la, r);
-}
 
-template <typename R, int K>
-__device__ __forceinline__ void m1_dispatch(int t, C2<R> (&a)[1 << K], const M2<R>& m) {
-    switch (t) {
-    case 0: m1_apply<R, K, 0>(a, m); break;
-    case 1: if constexpr (K > 1) m1_apply<R, K, 1>(a, m); break;
-    case 2: if constexpr (K > 2) m1_apply<R, K, 2>(a, m); break;
-    case 3: if constexpr (K > 3) m1_apply<R, K, 3>(a, m); break;
-    case 4: if constexpr (K > 4) m1_apply<R, K, 4>(a, m); break;
-    default: break;
-    }
-}
-
-template <typename R, int K>
-__device__ __forceinline__ void m1_rho_dispatch(int t, const C2<R> (&ps)[1 << K],
-                                                const C2<R> (&la)[1 << K], R (&r)[8]) {
-    switch (t) {
-    case 0: m1_rho<R, K, 0>(ps, la, r); break;
-    case 1: if constexpr (K > 1) m1_rho<R, K, 1>(ps, la, r); break;
-    case 2: if constexpr (K > 2) m1_rho<R, K, 2>(ps, la, r); break;
-    case 3: if constexpr (K > 3) m1_rho<R, K, 3>(ps, la, r); break;
-    case 4: if constexpr (K > 4) m1_rho<R, K, 4>(ps, la, r); break;
-    default: break;
-    }
-}
 
 // CX with local control C and local target T: swap (r, r^T) for r with C set, T clear.
 template <typename R, int K, int Cc, int T>
@@ -583,81 +546,62 @@ __device__ __forceinline__ int refbit(int ref, int r, uint32_t pb) {
 template <typename R>
 __device__ __forceinline__ R shx(R v, int m, unsigned mask) { return __shfl_xor_sync(mask, v, m); }
 
-// Reduce 8 values over a group of `lanes` lanes (power of two <= 32) and
-// write the 8 sums to dst (reduce-scatter butterfly: 9 shuffles at 32 lanes).
+// Reduce 4 values over a group of `lanes` lanes (power of two <= 32) and write
+// the 4 sums to dst[0..3] (reduce-scatter: 2 + 1 exchanges, then plain steps).
 template <typename R>
-__device__ __forceinline__ void reduce8_store(R (&v)[8], int lanes, int lane, R* dst,
+__device__ __forceinline__ void reduce4_store(R (&v)[4], int lanes, int lane, R* dst,
                                               unsigned mask, bool add) {
-    int u0 = 0, u1 = 0, u2 = 0;
+    int u0 = 0, u1 = 0;
     if (lanes >= 2) {
         const int m = lanes >> 1;
         u0 = (lane & m) ? 1 : 0;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            R send = u0 ? v[i] : v[i + 4];
-            R keep = u0 ? v[i + 4] : v[i];
+        for (int i = 0; i < 2; ++i) {
+            R send = u0 ? v[i] : v[i + 2];
+            R keep = u0 ? v[i + 2] : v[i];
             v[i] = keep + shx<R>(send, m, mask);
         }
     }
     if (lanes >= 4) {
         const int m = lanes >> 2;
         u1 = (lane & m) ? 1 : 0;
-#pragma unroll
-        for (int i = 0; i < 2; ++i) {
-            R send = u1 ? v[i] : v[i + 2];
-            R keep = u1 ? v[i + 2] : v[i];
-            v[i] = keep + shx<R>(send, m, mask);
-        }
-    }
-    if (lanes >= 8) {
-        const int m = lanes >> 3;
-        u2 = (lane & m) ? 1 : 0;
-        R send = u2 ? v[0] : v[1];
-        R keep = u2 ? v[1] : v[0];
+        R send = u1 ? v[0] : v[1];
+        R keep = u1 ? v[1] : v[0];
         v[0] = keep + shx<R>(send, m, mask);
-        for (int mm = lanes >> 4; mm >= 1; mm >>= 1) v[0] += shx<R>(v[0], mm, mask);
-        if ((lane & ((lanes >> 3) - 1)) == 0) {
-            R* d = dst + 4 * u0 + 2 * u1 + u2;
+        for (int mm = lanes >> 3; mm >= 1; mm >>= 1) v[0] += shx<R>(v[0], mm, mask);
+        if ((lane & ((lanes >> 2) - 1)) == 0) {
+            R* d = dst + 2 * u0 + u1;
             *d = add ? *d + v[0] : v[0];
         }
-    } else if (lanes == 4) {
-        R* d = dst + 4 * u0 + 2 * u1;
-        d[0] = add ? d[0] + v[0] : v[0];
-        d[1] = add ? d[1] + v[1] : v[1];
     } else if (lanes == 2) {
-        for (int i = 0; i < 4; ++i) dst[4 * u0 + i] = add ? dst[4 * u0 + i] + v[i] : v[i];
+        for (int i = 0; i < 2; ++i) dst[2 * u0 + i] = add ? dst[2 * u0 + i] + v[i] : v[i];
     } else {
-        for (int i = 0; i < 8; ++i) dst[i] = add ? dst[i] + v[i] : v[i];
+        for (int i = 0; i < 4; ++i) dst[i] = add ? dst[i] + v[i] : v[i];
     }
 }
 
-// reduce8_store for a full warp, branch-free: 4 + 2 + 1 scatter shuffles and
-// 2 plain ones; lanes with (lane & 3) == 0 write their sum.
+// reduce4_store for a full warp, branch-free: 2 + 1 scatter shuffles and 3
+// plain ones; lanes with (lane & 7) == 0 write their sum.
 template <typename R>
-__device__ __forceinline__ void reduce8_full(R (&v)[8], int lane, R* dst, bool add) {
+__device__ __forceinline__ void reduce4_full(R (&v)[4], int lane, R* dst, bool add) {
     const unsigned full = 0xffffffffu;
-    const int u0 = (lane >> 4) & 1, u1 = (lane >> 3) & 1, u2 = (lane >> 2) & 1;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const R send = u0 ? v[i] : v[i + 4];
-        const R keep = u0 ? v[i + 4] : v[i];
-        v[i] = keep + __shfl_xor_sync(full, send, 16);
-    }
+    const int u0 = (lane >> 4) & 1, u1 = (lane >> 3) & 1;
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
-        const R send = u1 ? v[i] : v[i + 2];
-        const R keep = u1 ? v[i + 2] : v[i];
-        v[i] = keep + __shfl_xor_sync(full, send, 8);
+        const R send = u0 ? v[i] : v[i + 2];
+        const R keep = u0 ? v[i + 2] : v[i];
+        v[i] = keep + __shfl_xor_sync(full, send, 16);
     }
     {
-        const R send = u2 ? v[0] : v[1];
-        const R keep = u2 ? v[1] : v[0];
-        v[0] = keep + __shfl_xor_sync(full, send, 4);
+        const R send = u1 ? v[0] : v[1];
+        const R keep = u1 ? v[1] : v[0];
+        v[0] = keep + __shfl_xor_sync(full, send, 8);
     }
+    v[0] += __shfl_xor_sync(full, v[0], 4);
     v[0] += __shfl_xor_sync(full, v[0], 2);
     v[0] += __shfl_xor_sync(full, v[0], 1);
-    if ((lane & 3) == 0) {
-        R* d = dst + 4 * u0 + 2 * u1 + u2;
+    if ((lane & 7) == 0) {
+        R* d = dst + 2 * u0 + u1;
         *d = add ? *d + v[0] : v[0];
     }
 }
@@ -916,20 +860,20 @@ __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 <<
                     /* one basic block: the butterfly's shuffles can overlap  */     \
                     /* the adjoint arithmetic                                 */     \
                     if (flags & OPF_HAS_ACC) {                                       \
-                        R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};                          \
-                        rho_go<R, K, T_>(a, l, rh);                                  \
+                        R rh[4] = {0, 0, 0, 0};                                      \
+                        m1_t3<R, K, T_>(a, l, rh);                                   \
                         m1_entry<R, K, T_, true>(a, tp);                             \
                         m1_entry<R, K, T_, true>(l, tp);                             \
-                        reduce8_full<R>(rh, lane, accp, acc_add);                    \
+                        reduce4_full<R>(rh, lane, accp, acc_add);                    \
                     } else {                                                         \
                         m1_entry<R, K, T_, true>(a, tp);                             \
                         m1_entry<R, K, T_, true>(l, tp);                             \
                     }                                                                \
                 } else {                                                             \
                     if (flags & OPF_HAS_ACC) {                                       \
-                        R rh[8] = {0, 0, 0, 0, 0, 0, 0, 0};                          \
-                        rho_go<R, K, T_>(a, l, rh);                                  \
-                        reduce8_store<R>(rh, q.lanes, rlane, accp, q.mask, acc_add); \
+                        R rh[4] = {0, 0, 0, 0};                                      \
+                        m1_t3<R, K, T_>(a, l, rh);                                   \
+                        reduce4_store<R>(rh, q.lanes, rlane, accp, q.mask, acc_add); \
                     }                                                                \
                     m1_entry<R, K, T_, true>(a, tp);                                 \
                     m1_entry<R, K, T_, true>(l, tp);                                 \
@@ -1172,16 +1116,17 @@ __device__ void acc_terms(const DAcc& ac, const DEntry& e, const R* ap, int wg,
         out[consts[e.cfirst].term] = sum;
         return;
     }
-    R rr[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    R t[3] = {0, 0, 0};
     for (int k2 = 0; k2 < wg; ++k2)
-        for (int c = 0; c < 8; ++c) rr[c] += ap[k2 * 8 + c];
-    // rho = [[r00, r01], [r10, r11]] (pairs rr[0..1], rr[2..3], rr[4..5],
-    // rr[6..7]).  term_j = Im Tr(W_j P_j W_j^dag rho) = Im Tr(P_j rho_j) with
-    // rho_j = W_j^dag rho W_j, carried from the last constituent backwards:
-    // rho <- U^dag rho U after each one.
+        for (int c = 0; c < 3; ++c) t[c] += ap[k2 * 8 + c];
+    // The accumulator holds (tx, ty, tz) of rho's traceless anti-Hermitian part
+    // rho' = (i/2)(tx X + ty Y + tz Z).  term_j = Im Tr(W_j P_j W_j^dag rho) =
+    // Im Tr(P_j rho_j) with rho_j = W_j^dag rho' W_j, carried from the last
+    // constituent backwards: rho <- U^dag rho U after each one.
+    const R h = R(0.5);
     M2<R> rho;
-    rho.a = cm<R>(rr[0], rr[1]); rho.b = cm<R>(rr[2], rr[3]);
-    rho.c = cm<R>(rr[4], rr[5]); rho.d = cm<R>(rr[6], rr[7]);
+    rho.a = cm<R>(0, h * t[2]); rho.b = cm<R>(h * t[1], h * t[0]);
+    rho.c = cm<R>(-h * t[1], h * t[0]); rho.d = cm<R>(0, -h * t[2]);
     for (int c = e.ccount - 1; c >= 0; --c) {
         const DConst cn = consts[e.cfirst + c];
         if (cn.term >= 0) {
