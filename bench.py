@@ -251,28 +251,23 @@ def run_ours(args, rank, world, local_rank):
     ms_per_step = total_ms / K
     value = world * Bt * K / (total_ms / 1e3)
 
-    # ---- end to end through the public API: pinned host inputs in, results out
-    xh = torch.tensor(w_.x, dtype=torch.float32).pin_memory()
-    wh = torch.tensor(w_.w, dtype=torch.float32).pin_memory()
-    gh = torch.tensor(w_.gE, dtype=torch.float32).pin_memory()
-    Eh = torch.empty(Bt, w_.spec.n, dtype=torch.float32).pin_memory()
-    dxh = torch.empty_like(xh).pin_memory()
-    dwh = torch.empty_like(wh).pin_memory()
-    h2d = xh.numel() * 4 + wh.numel() * 4 + gh.numel() * 4
-    d2h = Eh.numel() * 4 + dxh.numel() * 4 + dwh.numel() * 4
+    # ---- end to end through the C ABI with HOST buffers (vqc_evaluate_host):
+    # every step copies x, w, gE in and E, dx, dw out (one packed copy each way)
+    xh = np.ascontiguousarray(w_.x, dtype=np.float32)
+    wh = np.ascontiguousarray(w_.w, dtype=np.float32)
+    gh = np.ascontiguousarray(w_.gE, dtype=np.float32)
+    Eh = np.empty((Bt, w_.spec.n), np.float32)
+    dxh = np.empty_like(xh)
+    dwh = np.empty_like(wh)
+    h2d = xh.nbytes + wh.nbytes + gh.nbytes
+    d2h = Eh.nbytes + dxh.nbytes + dwh.nbytes
 
     def e2e_step():
-        xd = xh.to("cuda", non_blocking=True)
-        wd = wh.to("cuda", non_blocking=True)
-        gd = gh.to("cuda", non_blocking=True)
-        Ed, sd = c.forward(xd, wd, want_state=True)
-        dxd, dwd = c.backward(xd, wd, gd, psi_final=sd)
-        if world > 1:
-            dist.all_reduce(dwd)
-        Eh.copy_(Ed, non_blocking=True)
-        dxh.copy_(dxd, non_blocking=True)
-        dwh.copy_(dwd, non_blocking=True)
-        torch.cuda.current_stream().synchronize()
+        c.evaluate_host(xh, wh, gh, out=(Eh, dxh, dwh), stream=sp)
+        if world > 1:   # the data-parallel dw sum of the step
+            t = torch.from_numpy(dwh).to("cuda")
+            dist.all_reduce(t)
+            dwh[:] = t.cpu().numpy()
 
     for _ in range(max(3, args.warmup // 4)):
         e2e_step()
@@ -286,8 +281,8 @@ def run_ours(args, rank, world, local_rank):
     if world > 1:
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
     e2e_value = world * Bt * Ke / float(t.item())
-    E_check = float(np.max(np.abs(Eh.numpy()))) if Eh.numel() else 0.0
-    assert np.isfinite(E_check)
+    E_check = float(np.max(np.abs(Eh))) if Eh.size else 0.0
+    assert np.isfinite(E_check) and np.all(np.isfinite(dwh))
 
     if rank != 0:
         return None
@@ -360,6 +355,7 @@ def run_ours(args, rank, world, local_rank):
                      "launch_ms": bwd_avg_s * 1e3,
                      "fwd_frac": ach_fwd / peak},
         "e2e": {"value": e2e_value, "unit": "circuit evals/s (fwd+adjoint bwd, host buffers)",
+                "call": "vqc_evaluate_host (pageable numpy in/out; one packed copy each way)",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": Ke},
         "gpu_launches": launches_per_step * K,
         "clocks": clocks,

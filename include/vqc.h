@@ -251,6 +251,30 @@ vqc_status vqc_backward_noalloc(const vqc_plan* plan, int32_t batch, const void*
                                 const void* w, const void* psi0, const void* psi_final,
                                 const void* grad_expz, void* grad_x, void* grad_w, void* stream);
 
+/* One evaluation with inputs and outputs in HOST memory (pageable or pinned):
+ * the forward sweep and, when grad_expz is given, the adjoint backward from the
+ * forward's final states (paper, Alg. 1 execute phase and Sec. 3 gradients;
+ * the loss is L = sum gE * E with gE known before the call, e.g. fixed
+ * observable weights).  For callers whose data live on the host: the inputs
+ * are packed into a pinned staging area and moved in ONE host-to-device copy,
+ * the outputs come back in ONE device-to-host copy.
+ *   x         host [B, num_x] real (NULL when num_x == 0).
+ *   w         host [num_w] real (NULL when num_w == 0).
+ *   grad_expz host [B, n] real gE, or NULL for the forward only.
+ *   expz_out  host [B, n] real: E (required).
+ *   grad_x    host [B, num_x] real dL/dx, or NULL (ignored without grad_expz).
+ *   grad_w    host [num_w] real dL/dw summed over the batch, or NULL.
+ *   stream    cudaStream_t the work is enqueued on.
+ * Initial states are |0...0>.  The plan owns a device arena (packed inputs and
+ * outputs, final states, both workspaces) and a pinned host mirror, sized for
+ * the largest batch seen on the current device and released by vqc_free; calls
+ * on one plan are serialised by the plan.  Blocking: returns after `stream`
+ * has finished the call's work.  Errors as vqc_forward / vqc_backward, plus
+ * VQC_ERR_OUT_OF_MEMORY when the arena or the staging area cannot be allocated. */
+vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, const void* x, const void* w,
+                             const void* grad_expz, void* expz_out, void* grad_x, void* grad_w,
+                             void* stream);
+
 /* Plan statistics (paths, stage counts, algorithmic flop and byte counts per
  * evaluation) for a batch of `batch` samples. */
 vqc_status vqc_plan_info(const vqc_plan* plan, int32_t batch, vqc_plan_stats* out);

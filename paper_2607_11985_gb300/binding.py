@@ -78,6 +78,7 @@ SIGNATURES = [
     ("vqc_parse_qasm", _I, [ctypes.c_char_p, ctypes.POINTER(vqc_gate), ctypes.POINTER(_I),
                             ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_I)]),
     ("vqc_compile_qasm", _I, [ctypes.c_char_p, _I, _I, _I, ctypes.POINTER(_P)]),
+    ("vqc_evaluate_host", _I, [_P, _I, _P, _P, _P, _P, _P, _P, _P]),
 ]
 
 
@@ -175,6 +176,12 @@ def vqc_backward(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x, grad_w, 
 def vqc_backward_noalloc(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x, grad_w, stream):
     _check(lib().vqc_backward_noalloc(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x,
                                       grad_w, stream))
+
+
+def vqc_evaluate_host(plan, batch, x, w, grad_expz, expz_out, grad_x, grad_w, stream):
+    """Host-memory evaluation: x, w, grad_expz, expz_out, grad_x, grad_w are
+    host addresses (e.g. ``ndarray.ctypes.data``) or None."""
+    _check(lib().vqc_evaluate_host(plan, batch, x, w, grad_expz, expz_out, grad_x, grad_w, stream))
 
 
 def vqc_plan_info(plan, batch):

@@ -21,7 +21,7 @@ BUILD = os.path.join(HERE, "_build")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2",
               "--expt-relaxed-constexpr", "-I" + os.path.join(ROOT, "include")]
-UNITS = ["compiler.cpp", "qasm.cpp", "capi.cu", "noalloc.cu",
+UNITS = ["compiler.cpp", "qasm.cpp", "capi.cu", "noalloc.cu", "host_eval.cu",
          "kernels_f32_fwd.cu", "kernels_f32_bwd.cu", "kernels_f64_fwd.cu", "kernels_f64_bwd.cu",
          "kernels_f32_fwd_small.cu", "kernels_f32_bwd_small.cu", "kernels_f64_fwd_small.cu",
          "kernels_f64_bwd_small.cu", "kernels_hbm.cu", "kernels_cluster.cu"]

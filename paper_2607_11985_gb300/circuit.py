@@ -141,6 +141,43 @@ class Circuit:
                        _ptr(gE), _ptr(dx), _ptr(dw), _ptr(ws), wsb, stream.cuda_stream)
         return dx, dw
 
+    def evaluate_host(self, x, w, grad_expz=None, out=None, stream=None):
+        """One evaluation from and to host memory (numpy arrays): E [B, n] and,
+        given grad_expz [B, n], (dL/dx [B, num_x], dL/dw [num_w]) for
+        L = sum(grad_expz * E).  One copy in, one copy out (vqc_evaluate_host).
+        ``out`` = (E, dx, dw) preallocated host arrays to fill."""
+        import numpy as np
+        rdt = np.float32 if self.dtype == "c64" else np.float64
+
+        def arr(a, shape, name):
+            if a is None:
+                return None
+            if not isinstance(a, np.ndarray) or a.dtype != rdt or a.shape != tuple(shape) \
+                    or not a.flags.c_contiguous:
+                raise ValueError("%s must be a C-contiguous %s array of shape %s"
+                                 % (name, np.dtype(rdt).name, tuple(shape)))
+            return a
+
+        batch = x.shape[0] if x is not None and self.num_x else \
+            (grad_expz.shape[0] if grad_expz is not None else 1)
+        x = arr(x, (batch, self.num_x), "x") if self.num_x else None
+        w = arr(w, (self.num_w,), "w") if self.num_w else None
+        gE = arr(grad_expz, (batch, self.n), "grad_expz")
+        if out is None:
+            E = np.empty((batch, self.n), rdt)
+            dx = np.empty((batch, self.num_x), rdt) if gE is not None and self.num_x else None
+            dw = np.empty((self.num_w,), rdt) if gE is not None and self.num_w else None
+        else:
+            E, dx, dw = out
+            E = arr(E, (batch, self.n), "E")
+            dx = arr(dx, (batch, self.num_x), "dx")
+            dw = arr(dw, (self.num_w,), "dw")
+        hp = lambda a: None if a is None else a.ctypes.data   # noqa: E731
+        if stream is None:
+            stream = torch.cuda.current_stream().cuda_stream
+        B.vqc_evaluate_host(self.plan, batch, hp(x), hp(w), hp(gE), hp(E), hp(dx), hp(dw), stream)
+        return E if gE is None else (E, dx, dw)
+
     def __call__(self, x, w, psi0=None):
         return VQCFunction.apply(x, w, self, psi0)
 

@@ -19,10 +19,6 @@
 #include "pass.cuh"
 #include "sweep.cuh"
 
-struct vqc_plan {
-    vqc::HostPlan hp;
-};
-
 namespace vqc {
 namespace {
 // Launch geometry depends only on (plan, mode, batch, device): cache it so a
@@ -889,6 +885,9 @@ vqc_status check_ptrs(const HostPlan& p, const void* x, const void* w, const voi
 
 vqc_status set_error(vqc_status s, const std::string& msg) { return fail(s, msg); }
 
+// host_eval.cu: the per-plan arena of vqc_evaluate_host.
+void release_host_arena(const vqc_plan* plan);
+
 // The backward with an explicit scratch buffer, for vqc_backward_noalloc: the
 // scratch must hold the same layout as a vqc_backward workspace; with
 // clear_control the control block is zeroed on `stream` before the launch.
@@ -969,6 +968,7 @@ vqc_status vqc_compile(const vqc_gate* gates, int32_t num_gates, int32_t num_qub
 void vqc_free(vqc_plan* plan) {
     if (!plan) return;
     forget_plan(&plan->hp);
+    release_host_arena(plan);
     if (plan->hp.dbuf) {
         int cur = -1;
         cudaGetDevice(&cur);

@@ -101,3 +101,8 @@ const Schedule* find_cluster_schedule(const HostPlan& p, int mode);
 std::vector<uint8_t> export_plan(const HostPlan& p);
 
 }  // namespace vqc
+
+// The opaque handle of the C ABI: a compiled host plan (and its device copy).
+struct vqc_plan {
+    vqc::HostPlan hp;
+};
