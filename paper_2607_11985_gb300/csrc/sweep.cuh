@@ -1116,28 +1116,47 @@ __device__ void acc_terms(const DAcc& ac, const DEntry& e, const R* ap, int wg,
         out[consts[e.cfirst].term] = sum;
         return;
     }
-    R t[3] = {0, 0, 0};
-    for (int k2 = 0; k2 < wg; ++k2)
-        for (int c = 0; c < 3; ++c) t[c] += ap[k2 * 8 + c];
+    R vx = 0, vy = 0, vz = 0;
+    for (int k2 = 0; k2 < wg; ++k2) {
+        vx += ap[k2 * 8 + 0];
+        vy += ap[k2 * 8 + 1];
+        vz += ap[k2 * 8 + 2];
+    }
     // The accumulator holds (tx, ty, tz) of rho's traceless anti-Hermitian part
     // rho' = (i/2)(tx X + ty Y + tz Z).  term_j = Im Tr(W_j P_j W_j^dag rho) =
-    // Im Tr(P_j rho_j) with rho_j = W_j^dag rho' W_j, carried from the last
-    // constituent backwards: rho <- U^dag rho U after each one.
-    const R h = R(0.5);
-    M2<R> rho;
-    rho.a = cm<R>(0, h * t[2]); rho.b = cm<R>(h * t[1], h * t[0]);
-    rho.c = cm<R>(-h * t[1], h * t[0]); rho.d = cm<R>(0, -h * t[2]);
+    // Im Tr(P_j rho_j) = the P_j component of rho_j = W_j^dag rho' W_j, carried
+    // from the last constituent backwards: rho' <- U^dag rho' U after each one.
+    // For U = exp(-i t P / 2) that turns (tx, ty, tz) by the full angle t about
+    // P's axis; a scalar phase leaves it; a constant 2x2 goes through its matrix.
     for (int c = e.ccount - 1; c >= 0; --c) {
         const DConst cn = consts[e.cfirst + c];
-        if (cn.term >= 0) {
-            // Im Tr(X rho) = Im r01 + Im r10, Im Tr(Y rho) = Re r01 - Re r10,
-            // Im Tr(Z rho) = Im r00 - Im r11
-            const R tx = rho.b.y + rho.c.y, ty = rho.b.x - rho.c.x, tz = rho.a.y - rho.d.y;
-            out[cn.term] = cn.kind == CK_RX ? tx : cn.kind == CK_RY ? ty : tz;
-        }
-        if (c > 0) {
+        if (cn.term >= 0) out[cn.term] = cn.kind == CK_RX ? vx : cn.kind == CK_RY ? vy : vz;
+        if (c == 0) break;
+        if (cn.kind == CK_RX || cn.kind == CK_RY || cn.kind == CK_RZ) {
+            R sn, co;
+            sc(angle_of<R>(cn.src0, cn.idx0, xg, w, cang), &sn, &co);
+            if (cn.kind == CK_RX) {
+                const R y2 = vy * co + vz * sn, z2 = vz * co - vy * sn;
+                vy = y2; vz = z2;
+            } else if (cn.kind == CK_RY) {
+                const R x2 = vx * co - vz * sn, z2 = vz * co + vx * sn;
+                vx = x2; vz = z2;
+            } else {
+                const R x2 = vx * co + vy * sn, y2 = vy * co - vx * sn;
+                vx = x2; vy = y2;
+            }
+        } else if (cn.kind == CK_CONST) {
+            const R h = R(0.5);
+            M2<R> rho;
+            rho.a = cm<R>(0, h * vz); rho.b = cm<R>(h * vy, h * vx);
+            rho.c = cm<R>(-h * vy, h * vx); rho.d = cm<R>(0, -h * vz);
             const M2<R> u = constituent<R>(cn, xg, w, cang, cmat);
             rho = mmul<R>(mdag<R>(u), mmul<R>(rho, u));
+            // Im Tr(X rho) = Im r01 + Im r10, Im Tr(Y rho) = Re r01 - Re r10,
+            // Im Tr(Z rho) = Im r00 - Im r11
+            vx = rho.b.y + rho.c.y;
+            vy = rho.b.x - rho.c.x;
+            vz = rho.a.y - rho.d.y;
         }
     }
 }
