@@ -41,7 +41,8 @@ def _sources_digest() -> str:
             h.update(name.encode() + f.read())
     with open(os.path.join(ROOT, "include", "vqc.h"), "rb") as f:
         h.update(f.read())
-    h.update(" ".join(ARCH + NVCC_FLAGS).encode())
+    # flags without the include path, so that a checkout anywhere hashes alike
+    h.update(" ".join(ARCH + [f for f in NVCC_FLAGS if not f.startswith("-I")]).encode())
     return h.hexdigest()
 
 
