@@ -355,7 +355,9 @@ def run_ours(args, rank, world, local_rank):
                      "launch_ms": bwd_avg_s * 1e3,
                      "fwd_frac": ach_fwd / peak},
         "e2e": {"value": e2e_value, "unit": "circuit evals/s (fwd+adjoint bwd, host buffers)",
-                "call": "vqc_evaluate_host (pageable numpy in/out; one packed copy each way)",
+                "call": "vqc_evaluate_host (pageable numpy in/out; %s)" % (
+                    "kernels access the host arrays in place over NVLink-C2C"
+                    if B.vqc_host_direct(local_rank) else "one packed copy each way"),
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": Ke},
         "gpu_launches": launches_per_step * K,
         "clocks": clocks,

@@ -255,9 +255,12 @@ vqc_status vqc_backward_noalloc(const vqc_plan* plan, int32_t batch, const void*
  * the forward sweep and, when grad_expz is given, the adjoint backward from the
  * forward's final states (paper, Alg. 1 execute phase and Sec. 3 gradients;
  * the loss is L = sum gE * E with gE known before the call, e.g. fixed
- * observable weights).  For callers whose data live on the host: the inputs
- * are packed into a pinned staging area and moved in ONE host-to-device copy,
- * the outputs come back in ONE device-to-host copy.
+ * observable weights).  For callers whose data live on the host.  Where the
+ * device accesses pageable host memory coherently (vqc_host_direct() == 1,
+ * e.g. Grace-Blackwell over NVLink-C2C) the kernels read and write the
+ * caller's arrays in place and no copy is made; otherwise the inputs are packed
+ * into a pinned staging area and moved in ONE host-to-device copy and the
+ * outputs come back in ONE device-to-host copy.
  *   x         host [B, num_x] real (NULL when num_x == 0).
  *   w         host [num_w] real (NULL when num_w == 0).
  *   grad_expz host [B, n] real gE, or NULL for the forward only.
@@ -274,6 +277,11 @@ vqc_status vqc_backward_noalloc(const vqc_plan* plan, int32_t batch, const void*
 vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, const void* x, const void* w,
                              const void* grad_expz, void* expz_out, void* grad_x, void* grad_w,
                              void* stream);
+
+/* 1 when vqc_evaluate_host on `device` lets the kernels access host arrays in
+ * place (cudaDevAttrPageableMemoryAccess is set and the environment does not
+ * set VQC_HOST_DIRECT=0), else 0 (staged copies). */
+int32_t vqc_host_direct(int32_t device);
 
 /* Plan statistics (paths, stage counts, algorithmic flop and byte counts per
  * evaluation) for a batch of `batch` samples. */

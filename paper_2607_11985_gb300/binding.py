@@ -79,6 +79,7 @@ SIGNATURES = [
                             ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_I)]),
     ("vqc_compile_qasm", _I, [ctypes.c_char_p, _I, _I, _I, ctypes.POINTER(_P)]),
     ("vqc_evaluate_host", _I, [_P, _I, _P, _P, _P, _P, _P, _P, _P]),
+    ("vqc_host_direct", _I, [_I]),
 ]
 
 
@@ -182,6 +183,10 @@ def vqc_evaluate_host(plan, batch, x, w, grad_expz, expz_out, grad_x, grad_w, st
     """Host-memory evaluation: x, w, grad_expz, expz_out, grad_x, grad_w are
     host addresses (e.g. ``ndarray.ctypes.data``) or None."""
     _check(lib().vqc_evaluate_host(plan, batch, x, w, grad_expz, expz_out, grad_x, grad_w, stream))
+
+
+def vqc_host_direct(device):
+    return int(lib().vqc_host_direct(device))
 
 
 def vqc_plan_info(plan, batch):

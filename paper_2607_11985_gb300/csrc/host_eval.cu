@@ -10,9 +10,14 @@
 //   host x, w, gE  --memcpy-->  pinned [x | w | gE]  --1 copy-->  device
 //   vqc_forward (E, final states) ; vqc_backward (dx, dw) from those states
 //   device [E | dx | dw]  --1 copy-->  pinned  --memcpy-->  host E, dx, dw
-// and the call returns after the stream has finished.  From the second call
-// with the same batch and outputs on, the device part is one CUDA graph launch
-// (captured once on a private stream; VQC_HOST_GRAPH=0 turns this off).  The arena is released
+// and the call returns after the stream has finished.  Where the device can
+// access pageable host memory coherently (cudaDevAttrPageableMemoryAccess, e.g.
+// a Grace-Blackwell node over NVLink-C2C) there is no staging at all: the
+// kernels read x, w, gE from and write E, dx, dw to the caller's arrays
+// (VQC_HOST_DIRECT=0 forces the staged copies).  From the second call with the
+// same batch and outputs (and, direct, the same arrays) on, the device part is
+// one CUDA graph launch (captured once on a private stream; VQC_HOST_GRAPH=0
+// turns this off).  The arena is released
 // by vqc_free.
 #include <cuda_runtime.h>
 
@@ -56,6 +61,7 @@ struct Arena {
     cudaStream_t cap = nullptr;
     cudaGraphExec_t exec = nullptr;
     int shape_batch = -1, shape_flags = -1;   // shape of the previous call
+    const void* shape_ptrs[6] = {};           // its host arrays (direct access: part of the shape)
     bool graph_failed = false;
     void drop_graph() {
         if (exec) cudaGraphExecDestroy(exec);
@@ -109,6 +115,30 @@ vqc_status cuda_err(cudaError_t e, const char* what) {
 bool env_flag(const char* name, bool dflt) {
     const char* v = std::getenv(name);
     return v ? std::atoi(v) != 0 : dflt;
+}
+
+// Whether kernels on `dev` may read and write pageable host memory directly
+// (cudaDevAttrPageableMemoryAccess: coherent access through the host's page
+// tables, as on Grace-Blackwell's NVLink-C2C).  Queried once per device.
+bool host_direct(int dev) {
+    static std::mutex mu;
+    static int known[64];
+    static bool init = false;
+    if (dev < 0 || dev >= 64) return false;
+    std::lock_guard<std::mutex> lk(mu);
+    if (!init) {
+        for (int& k : known) k = -1;
+        init = true;
+    }
+    if (known[dev] < 0) {
+        int v = 0;
+        if (cudaDeviceGetAttribute(&v, cudaDevAttrPageableMemoryAccess, dev) != cudaSuccess) {
+            (void)cudaGetLastError();
+            v = 0;
+        }
+        known[dev] = v ? 1 : 0;
+    }
+    return known[dev] == 1;
 }
 
 // Capture enqueue() on the arena's private stream into an executable graph.
@@ -197,8 +227,14 @@ extern "C" vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, con
                                                            std::to_string(A->device) + ", current device is " +
                                                            std::to_string(dev));
         const Layout L = layout_for(plan, batch, bwd);
-        const int flags = (bwd ? 1 : 0) | (bwd && grad_x ? 2 : 0) | (bwd && grad_w ? 4 : 0);
-        if (A->shape_batch != batch || A->shape_flags != flags) A->drop_graph();
+        const bool direct = env_flag("VQC_HOST_DIRECT", true) && host_direct(dev);
+        const int flags = (bwd ? 1 : 0) | (bwd && grad_x ? 2 : 0) | (bwd && grad_w ? 4 : 0) |
+                          (direct ? 8 : 0);
+        const void* ptrs[6] = {x, w, grad_expz, expz_out, grad_x, grad_w};
+        bool same_shape = A->shape_batch == batch && A->shape_flags == flags;
+        if (direct)
+            for (int i = 0; i < 6; ++i) same_shape = same_shape && A->shape_ptrs[i] == ptrs[i];
+        if (!same_shape) A->drop_graph();
         if (L.dev_bytes > A->dev_cap) {
             A->drop_graph();
             if (A->dev) {
@@ -218,7 +254,7 @@ extern "C" vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, con
             A->device = dev;
             A->have_last = false;
         }
-        const size_t pin_need = L.in_bytes + L.out_bytes;
+        const size_t pin_need = direct ? 0 : L.in_bytes + L.out_bytes;
         if (pin_need > A->pin_cap) {
             if (A->pin) cudaFreeHost(A->pin);
             A->pin = nullptr;
@@ -246,13 +282,30 @@ extern "C" vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, con
             A->have_last = true;
         }
 
+        // Direct access: the kernels read x, w, gE and write E, dx, dw in the
+        // caller's host arrays themselves; only states and workspaces are in
+        // the arena.
+        auto enqueue_direct = [&](cudaStream_t q) -> vqc_status {
+            const void* xh = p.num_x > 0 ? x : nullptr;
+            const void* wh = p.num_w > 0 ? w : nullptr;
+            vqc_status r = vqc_forward(plan, batch, xh, wh, nullptr, expz_out, bwd ? D + L.state : nullptr,
+                                       L.ws0_bytes ? D + L.ws0 : nullptr, L.ws0_bytes, q);
+            if (r != VQC_OK || !bwd) return r;
+            return vqc_backward(plan, batch, xh, wh, nullptr, D + L.state, grad_expz,
+                                (flags & 2) && p.num_x > 0 ? grad_x : nullptr,
+                                (flags & 4) && p.num_w > 0 ? grad_w : nullptr,
+                                L.ws1_bytes ? D + L.ws1 : nullptr, L.ws1_bytes, q);
+        };
+
         // inputs: caller memory -> pinned mirror (one copy to the device below)
-        if (p.num_x > 0) std::memcpy(H + L.x, x, (size_t)batch * p.num_x * rs);
-        if (p.num_w > 0) std::memcpy(H + L.w, w, (size_t)p.num_w * rs);
-        if (bwd) std::memcpy(H + L.g, grad_expz, (size_t)batch * p.n * rs);
+        if (!direct) {
+            if (p.num_x > 0) std::memcpy(H + L.x, x, (size_t)batch * p.num_x * rs);
+            if (p.num_w > 0) std::memcpy(H + L.w, w, (size_t)p.num_w * rs);
+            if (bwd) std::memcpy(H + L.g, grad_expz, (size_t)batch * p.n * rs);
+        }
 
         // The device work: input copy, forward, backward, output copy.
-        auto enqueue = [&](cudaStream_t q) -> vqc_status {
+        auto enqueue_staged = [&](cudaStream_t q) -> vqc_status {
             cudaError_t ce = cudaMemcpyAsync(D, H, L.in_bytes, cudaMemcpyHostToDevice, q);
             if (ce != cudaSuccess) return cuda_err(ce, "cudaMemcpyAsync(inputs)");
             const void* xd = p.num_x > 0 ? D + L.x : nullptr;
@@ -272,11 +325,14 @@ extern "C" vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, con
             if (ce != cudaSuccess) return cuda_err(ce, "cudaMemcpyAsync(outputs)");
             return VQC_OK;
         };
+        auto enqueue = [&](cudaStream_t q) -> vqc_status {
+            return direct ? enqueue_direct(q) : enqueue_staged(q);
+        };
         const bool graphs = !A->graph_failed && env_flag("VQC_HOST_GRAPH", true);
-        const bool same_shape = A->shape_batch == batch && A->shape_flags == flags;
         if (graphs && same_shape && !A->exec) A->exec = capture(A, enqueue);
         A->shape_batch = batch;
         A->shape_flags = flags;
+        for (int i = 0; i < 6; ++i) A->shape_ptrs[i] = ptrs[i];
         if (A->exec) {
             e = cudaGraphLaunch(A->exec, s);
             if (e != cudaSuccess) return cuda_err(e, "cudaGraphLaunch");
@@ -286,6 +342,7 @@ extern "C" vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, con
         }
         e = cudaStreamSynchronize(s);
         if (e != cudaSuccess) return cuda_err(e, "cudaStreamSynchronize");
+        if (direct) return VQC_OK;
 
         const unsigned char* HO = H + L.in_bytes;
         std::memcpy(expz_out, HO + L.E, (size_t)batch * p.n * rs);
@@ -297,4 +354,8 @@ extern "C" vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, con
     } catch (...) {
         return vqc::set_error(VQC_ERR_INVALID_ARG, "internal error in vqc_evaluate_host");
     }
+}
+
+extern "C" int32_t vqc_host_direct(int32_t device) {
+    return env_flag("VQC_HOST_DIRECT", true) && host_direct(device) ? 1 : 0;
 }

@@ -39,8 +39,20 @@ def host(a, dtype):
     return np.ascontiguousarray(a, dtype=np.float32 if dtype == "c64" else np.float64)
 
 
+@pytest.fixture(params=["direct", "staged"])
+def access(request, monkeypatch):
+    """Both transfer modes: kernels on the host arrays in place (where the
+    device supports it) and the pinned staging copies."""
+    if request.param == "staged":
+        monkeypatch.setenv("VQC_HOST_DIRECT", "0")
+        assert B.vqc_host_direct(0) == 0
+    elif not B.vqc_host_direct(0):
+        pytest.skip("this device does not access pageable host memory")
+    return request.param
+
+
 @pytest.mark.parametrize("batch", [1024, 37])
-def test_matches_device_calls_and_oracle(batch):
+def test_matches_device_calls_and_oracle(access, batch):
     w_ = wl.config(2)[0]
     if batch != w_.batch:
         w_ = rows(w_, np.arange(batch) * 7 % w_.batch)
@@ -59,7 +71,7 @@ def test_matches_device_calls_and_oracle(batch):
         assert maxerr(dw, dw_ref) <= TOL["c64"]["grad"]
 
 
-def test_forward_only_c128_and_batch_changes():
+def test_forward_only_c128_and_batch_changes(access):
     w_ = wl.config(1, dtype="c128")[0]
     c = C(w_.spec, "c128")
     for b in (5, 64, 3, 64):
@@ -79,7 +91,7 @@ def test_forward_only_c128_and_batch_changes():
     assert not dw0.any()
 
 
-def test_hbm_path_circuit():
+def test_hbm_path_circuit(access):
     n = 16
     spec = wl.layered(n, 2, ("RX", "RY", "RZ"), "CX", ring_range=lambda l: 2 * l + 1)
     rng = np.random.default_rng(1616)
@@ -117,18 +129,24 @@ def test_argument_errors():
         c.evaluate_host(w_.x, w)
 
 
-def test_graph_replay_sees_new_inputs(monkeypatch):
+def test_graph_replay_sees_new_inputs(access, monkeypatch):
     """From the second call of one shape on, the device work is a replayed CUDA
-    graph: it must read each call's inputs, and agree bit for bit with direct
-    launches (VQC_HOST_GRAPH=0)."""
+    graph: it must read each call's inputs (new arrays, or new contents of the
+    same arrays), and agree bit for bit with plain launches (VQC_HOST_GRAPH=0)."""
     w_ = wl.config(2, batch=64)[0]
     c = C(w_.spec, "c64")
     x1, w1, g1 = host(w_.x, "c64"), host(w_.w, "c64"), host(w_.gE, "c64")
     x2 = np.ascontiguousarray(x1[::-1])
     w2 = np.ascontiguousarray(w1 * 0.5)
-    first = c.evaluate_host(x1, w1, g1)
-    again = c.evaluate_host(x1, w1, g1)        # captured here
-    other = c.evaluate_host(x2, w2, g1)        # replayed with new inputs
+    outs = tuple(np.empty_like(a) for a in (np.empty((64, w_.spec.n), np.float32), x1, w1))
+    first = [a.copy() for a in c.evaluate_host(x1, w1, g1, out=outs)]
+    again = [a.copy() for a in c.evaluate_host(x1, w1, g1, out=outs)]   # captured here
+    xs, ws_ = x1.copy(), w1.copy()
+    x1[:] = x2
+    w1[:] = w2
+    other = [a.copy() for a in c.evaluate_host(x1, w1, g1, out=outs)]   # replayed, new contents
+    x1[:] = xs
+    w1[:] = ws_
     for a, b in zip(first, again):
         assert np.array_equal(a, b)
     monkeypatch.setenv("VQC_HOST_GRAPH", "0")
