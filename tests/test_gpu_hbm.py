@@ -7,6 +7,8 @@
   tile-outer controls and phases), against the oracle, with and without psi0
   and the saved final state, ragged batches;
 * cross-path agreement: the 12-qubit workload on the resident and HBM paths;
+* the largest plan (24 qubits): forward against the oracle, backward against
+  central differences of the complex128 forward;
 * the thread-block-cluster forward (VQC_FORCE_PATH=cluster) at 14-16 qubits
   against the oracle and against the HBM passes, and on the 16-qubit workload.
 """
@@ -135,6 +137,44 @@ def test_hbm_18_qubits_sampled():
     dx, dw = run_bwd(c, w_)
     dx_ref, dw_ref = orc.backward(spec, x, w, gE)
     assert maxerr(dx, dx_ref) <= 5e-4 and maxerr(dw, dw_ref) <= 5e-4
+
+
+def test_max_qubits_24():
+    """The largest plan the ABI accepts (24 qubits: 128 MiB complex64 / 256 MiB
+    complex128 per state).  Forward: E of one row against the oracle (complex64,
+    batch of 2).  Backward, where the oracle would take minutes: the adjoint
+    directional derivatives dL/dw . v and dL/dx . u match central differences
+    of L = sum gE * E computed with the complex128 forward (a property that
+    holds at any size; the forward itself is pinned above)."""
+    n = 24
+    spec = wl.layered(n, 1, ("RX", "RY", "RZ"), "CX")
+    rng = np.random.default_rng(2400)
+    x = wl._round(rng.uniform(-np.pi, np.pi, (2, n)), "c64")
+    w = wl._round(rng.uniform(-np.pi, np.pi, spec.num_w), "c64")
+    gE = wl._round(rng.standard_normal((2, n)), "c64")
+    c = C(spec, "c64")
+    assert c.info(2)["fwd_path"] == 1
+    E = run_fwd(c, wl.Workload("n24", spec, 2, x, w, gE, "c64", 2400), want_state=False)
+    assert maxerr(E[:1], orc.forward(spec, x[:1], w)) <= 1e-4
+    assert np.all(np.abs(E) <= 1 + 1e-5)
+    del c
+    torch.cuda.empty_cache()
+
+    c = C(spec, "c128")
+    x1, g1 = x[:1], gE[:1]
+    dx, dw = run_bwd(c, wl.Workload("n24", spec, 1, x1, w, g1, "c128", 2400))
+
+    def loss(xv, wv):
+        Ev = run_fwd(c, wl.Workload("n24", spec, 1, xv, wv, g1, "c128", 2400), want_state=False)
+        return float(np.sum(g1 * Ev))
+
+    v = rng.standard_normal(spec.num_w)
+    u = rng.standard_normal((1, n))
+    h = 1e-4
+    fd_w = (loss(x1, w + h * v) - loss(x1, w - h * v)) / (2 * h)
+    fd_x = (loss(x1 + h * u, w) - loss(x1 - h * u, w)) / (2 * h)
+    assert abs(fd_w - float(dw @ v)) <= 1e-6 * max(1.0, abs(fd_w))
+    assert abs(fd_x - float(np.sum(dx * u))) <= 1e-6 * max(1.0, abs(fd_x))
 
 
 @pytest.mark.parametrize("dtype,n", [("c64", 15), ("c64", 16), ("c128", 14), ("c128", 15), ("c128", 16)])
