@@ -176,7 +176,7 @@ vqc_status vqc_compile_qasm(const char* source, int32_t num_x, int32_t num_w, vq
 void vqc_free(vqc_plan* plan);
 
 /* Bytes of device workspace a call needs: mode 0 = vqc_forward, 1 = vqc_backward,
- * 2 = vqc_probabilities.  Returns 0 when no workspace is needed; (size_t)-1 for
+ * 2 = vqc_probabilities, 3 = vqc_forward_backward.  Returns 0 when no workspace is needed; (size_t)-1 for
  * a NULL plan. */
 size_t vqc_workspace_bytes(const vqc_plan* plan, int32_t batch, int32_t mode);
 
@@ -215,6 +215,23 @@ vqc_status vqc_backward(const vqc_plan* plan, int32_t batch, const void* x, cons
                         const void* psi0, const void* psi_final, const void* grad_expz,
                         void* grad_x, void* grad_w, void* workspace, size_t workspace_bytes,
                         void* stream);
+
+/* Forward and adjoint backward together, for a loss whose gradient gE is known
+ * before the call (L = sum gE * E with fixed weights; the paper's own objective,
+ * the mean of <Z_j>, has gE = 1/n): E, dL/dx and dL/dw of one batch.  Where the
+ * state fits one SM (the resident path) it is ONE launch: the backward kernel
+ * runs the forward sweep itself, keeps the final states in shared memory,
+ * writes E and sweeps back, so no state goes through HBM; otherwise it is
+ * vqc_forward followed by vqc_backward recomputing the states.
+ *   expz_out  device [B, n] real (required); grad_expz device [B, n] (required);
+ *   grad_x, grad_w as vqc_backward; psi0 as vqc_forward.
+ *   workspace vqc_workspace_bytes(plan, B, 3) bytes, 256-byte aligned,
+ *             initialised once with vqc_workspace_init.
+ * E agrees with vqc_forward and the gradients with vqc_backward to rounding (the
+ * sweeps may group the gates into different stages).  Errors as vqc_backward. */
+vqc_status vqc_forward_backward(const vqc_plan* plan, int32_t batch, const void* x, const void* w,
+                                const void* psi0, const void* grad_expz, void* expz_out, void* grad_x,
+                                void* grad_w, void* workspace, size_t workspace_bytes, void* stream);
 
 /* Measurement probabilities |psi_b[k]|^2 of the final states (paper, Sec. 3:
  * the engine's outputs are the statevector or its probabilities, and <Z>):
@@ -268,8 +285,9 @@ vqc_status vqc_backward_noalloc(const vqc_plan* plan, int32_t batch, const void*
  *   grad_x    host [B, num_x] real dL/dx, or NULL (ignored without grad_expz).
  *   grad_w    host [num_w] real dL/dw summed over the batch, or NULL.
  *   stream    cudaStream_t the work is enqueued on.
+ * The work is vqc_forward_backward (vqc_forward without grad_expz).
  * Initial states are |0...0>.  The plan owns a device arena (packed inputs and
- * outputs, final states, both workspaces) and a pinned host mirror, sized for
+ * outputs, the workspace) and a pinned host mirror, sized for
  * the largest batch seen on the current device and released by vqc_free; calls
  * on one plan are serialised by the plan.  Blocking: returns after `stream`
  * has finished the call's work.  Errors as vqc_forward / vqc_backward, plus

@@ -80,6 +80,7 @@ SIGNATURES = [
     ("vqc_compile_qasm", _I, [ctypes.c_char_p, _I, _I, _I, ctypes.POINTER(_P)]),
     ("vqc_evaluate_host", _I, [_P, _I, _P, _P, _P, _P, _P, _P, _P]),
     ("vqc_host_direct", _I, [_I]),
+    ("vqc_forward_backward", _I, [_P, _I, _P, _P, _P, _P, _P, _P, _P, _P, _S, _P]),
 ]
 
 
@@ -172,6 +173,12 @@ def vqc_backward(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x, grad_w, 
                  workspace_bytes, stream):
     _check(lib().vqc_backward(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x, grad_w,
                               workspace, workspace_bytes, stream))
+
+
+def vqc_forward_backward(plan, batch, x, w, psi0, grad_expz, expz_out, grad_x, grad_w, workspace,
+                         workspace_bytes, stream):
+    _check(lib().vqc_forward_backward(plan, batch, x, w, psi0, grad_expz, expz_out, grad_x, grad_w,
+                                      workspace, workspace_bytes, stream))
 
 
 def vqc_backward_noalloc(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x, grad_w, stream):

@@ -24,7 +24,8 @@ NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2",
 UNITS = ["compiler.cpp", "qasm.cpp", "capi.cu", "noalloc.cu", "host_eval.cu",
          "kernels_f32_fwd.cu", "kernels_f32_bwd.cu", "kernels_f64_fwd.cu", "kernels_f64_bwd.cu",
          "kernels_f32_fwd_small.cu", "kernels_f32_bwd_small.cu", "kernels_f64_fwd_small.cu",
-         "kernels_f64_bwd_small.cu", "kernels_hbm.cu", "kernels_cluster.cu"]
+         "kernels_f64_bwd_small.cu", "kernels_hbm.cu", "kernels_cluster.cu",
+         "kernels_f32_fused.cu", "kernels_f64_fused.cu"]
 
 
 def nvcc() -> str:

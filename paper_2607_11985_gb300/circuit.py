@@ -141,6 +141,27 @@ class Circuit:
                        _ptr(gE), _ptr(dx), _ptr(dw), _ptr(ws), wsb, stream.cuda_stream)
         return dx, dw
 
+    def forward_backward(self, x, w, grad_expz, psi0=None, out=None):
+        """(E [B, n], dL/dx [B, num_x], dL/dw [num_w]) for L = sum(grad_expz * E)
+        with grad_expz known up front (vqc_forward_backward: one launch on the
+        resident path).  ``out`` = (E, dx, dw) preallocated CUDA tensors."""
+        batch = grad_expz.shape[0]
+        x = self._check(x, self.real, (batch, self.num_x), "x") if self.num_x else None
+        w = self._check(w, self.real, (self.num_w,), "w") if self.num_w else None
+        gE = self._check(grad_expz, self.real, (batch, self.n), "grad_expz")
+        psi0 = self._check(psi0, self.cplx, (batch, 1 << self.n), "psi0")
+        if out is None:
+            E = torch.empty(batch, self.n, dtype=self.real, device="cuda")
+            dx = torch.empty(batch, self.num_x, dtype=self.real, device="cuda") if self.num_x else None
+            dw = torch.empty(self.num_w, dtype=self.real, device="cuda") if self.num_w else None
+        else:
+            E, dx, dw = out
+        stream = torch.cuda.current_stream()
+        ws, wsb = self.workspace(batch, 3, stream)
+        B.vqc_forward_backward(self.plan, batch, _ptr(x), _ptr(w), _ptr(psi0), _ptr(gE), _ptr(E),
+                               _ptr(dx), _ptr(dw), _ptr(ws), wsb, stream.cuda_stream)
+        return E, dx, dw
+
     def evaluate_host(self, x, w, grad_expz=None, out=None, stream=None):
         """One evaluation from and to host memory (numpy arrays): E [B, n] and,
         given grad_expz [B, n], (dL/dx [B, num_x], dL/dw [num_w]) for

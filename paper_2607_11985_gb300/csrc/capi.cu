@@ -78,7 +78,9 @@ vqc_status device_info(int dev, DevInfo& out) {
     return VQC_OK;
 }
 
+// mode 2: the backward with the forward sweep and E inside (vqc_forward_backward)
 const void* kernel_ptr(int dtype, int mode, int K, bool full) {
+    if (mode == 2) return dtype == VQC_C64 ? sweep_ptr_f32_fused(K, full) : sweep_ptr_f64_fused(K, full);
     if (full) {
         if (dtype == VQC_C64) return mode == 0 ? sweep_ptr_f32_fwd(K) : sweep_ptr_f32_bwd(K);
         return mode == 0 ? sweep_ptr_f64_fwd(K) : sweep_ptr_f64_bwd(K);
@@ -152,7 +154,9 @@ int choose_k(const HostPlan& p, int mode, int B) {
     return K;
 }
 
-vqc_status plan_launch_uncached(const HostPlan& p, int mode, int B, Launch& L) {
+vqc_status plan_launch_uncached(const HostPlan& p, int launch_mode, int B, Launch& L) {
+    // mode 2 (fused) has the backward's schedule and layout, its own kernel
+    const int mode = launch_mode == 2 ? 1 : launch_mode;
     int dev = 0;
     VQC_CUDA(cudaGetDevice(&dev));
     DevInfo di;
@@ -177,8 +181,8 @@ vqc_status plan_launch_uncached(const HostPlan& p, int mode, int B, Launch& L) {
                          align16((size_t)p.num_w * rs) + 10 * 16;
     const size_t per_sample = (size_t)p.n_ps * ew * rs + dim * cs * (mode == 1 ? 2 : 1) +
                               (size_t)(p.num_x + p.n) * rs +
-                              (mode == 1 ? p.accs.size() * L.wg * 8 * rs + p.term_src.size() * rs
-                                         : (size_t)L.wg * p.n * rs);
+                              (mode == 1 ? p.accs.size() * L.wg * 8 * rs + p.term_src.size() * rs : 0) +
+                              (size_t)L.wg * p.n * rs;
     // samples per CTA: groups up to VQC_CTA_THREADS (default 128) threads
     int S = std::max(1, cta_threads() / L.T);
     if ((size_t)di.smem_optin > fixed) {
@@ -211,7 +215,7 @@ vqc_status plan_launch_uncached(const HostPlan& p, int mode, int B, Launch& L) {
     L.sm_acc = take(mode == 1 ? (size_t)L.S * p.accs.size() * L.wg * 8 * rs : 0);
     L.sm_terms = take(mode == 1 ? (size_t)L.S * p.term_src.size() * rs : 0);
     L.sm_dw = take(mode == 1 ? (size_t)p.num_w * rs : 0);
-    L.sm_red = take(mode == 0 ? (size_t)L.S * L.wg * p.n * rs : 0);
+    L.sm_red = take((size_t)L.S * L.wg * p.n * rs);   // <Z> partials (forward, or recompute with E)
     L.sm_w = take((size_t)p.num_w * rs);
     L.sm_xg = take((size_t)L.S * (p.num_x + p.n) * rs);
     // the plan's table data and this schedule go to shared memory when they fit
@@ -222,7 +226,7 @@ vqc_status plan_launch_uncached(const HostPlan& p, int mode, int B, Launch& L) {
     L.smem = off;
     if (L.smem > (size_t)di.smem_optin)
         return fail(VQC_ERR_UNSUPPORTED, "shared-memory layout exceeds the per-CTA limit");
-    L.fn = kernel_ptr(p.dtype, mode, L.K, L.T >= 32);
+    L.fn = kernel_ptr(p.dtype, launch_mode, L.K, L.T >= 32);
     if (!L.fn) return fail(VQC_ERR_UNSUPPORTED, "kernel not instantiated for this K");
     VQC_CUDA(cudaFuncSetAttribute(L.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem));
     int per_sm = 0;
@@ -399,7 +403,7 @@ vqc_status run(const HostPlan& p, int mode, int B, const void* x, const void* w,
     a.state_out = static_cast<C*>(state_out);
     a.dx = static_cast<R*>(dx);
     a.dw = static_cast<R*>(dw);
-    if (mode == 1) {
+    if (mode >= 1) {
         size_t need = bwd_workspace(p, L);
         if (!ws || ws_bytes < need || misaligned(ws, 256))
             return fail(VQC_ERR_WORKSPACE, "backward workspace must be >= " + std::to_string(need) +
@@ -409,7 +413,7 @@ vqc_status run(const HostPlan& p, int mode, int B, const void* x, const void* w,
     }
     void* args[] = {&a};
     VQC_CUDA(launch(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
-    if (mode == 1 && dw && p.num_w > 0) {
+    if (mode >= 1 && dw && p.num_w > 0) {
         const R* part = a.dw_part;
         int rows = L.grid, cols = p.num_w;
         R* out = static_cast<R*>(dw);
@@ -981,6 +985,17 @@ void vqc_free(vqc_plan* plan) {
 
 size_t vqc_workspace_bytes(const vqc_plan* plan, int32_t batch, int32_t mode) {
     if (!plan) return (size_t)-1;
+    if (mode == 3) {   // vqc_forward_backward: its one-launch form, or either call's workspace
+        size_t need = std::max(vqc_workspace_bytes(plan, batch, 0), vqc_workspace_bytes(plan, batch, 1));
+        const HostPlan& p = plan->hp;
+        Launch L;
+        const std::string saved = g_err;
+        if (batch > 0 && !use_cluster(p, 0) && !use_hbm(p, 0, batch) && !use_hbm(p, 1, batch) &&
+            plan_launch(p, 2, batch, L) == VQC_OK)
+            need = std::max(need, bwd_workspace(p, L));
+        g_err = saved;
+        return need;
+    }
     if (mode == 2 && batch > 0) {   // vqc_probabilities: forward workspace + state + E
         const HostPlan& p = plan->hp;
         const size_t rs = p.dtype == VQC_C128 ? 8 : 4;
@@ -1106,6 +1121,42 @@ vqc_status vqc_backward(const vqc_plan* plan, int32_t batch, const void* x, cons
                            grad_w, workspace, workspace_bytes, s);
     } catch (...) {
         return fail(VQC_ERR_INVALID_ARG, "internal error in vqc_backward");
+    }
+}
+
+vqc_status vqc_forward_backward(const vqc_plan* plan, int32_t batch, const void* x, const void* w,
+                                const void* psi0, const void* grad_expz, void* expz_out, void* grad_x,
+                                void* grad_w, void* workspace, size_t workspace_bytes, void* stream) {
+    try {
+        vqc_status st = check_common(plan, batch);
+        if (st != VQC_OK) return st;
+        const HostPlan& p = plan->hp;
+        cudaStream_t s = static_cast<cudaStream_t>(stream);
+        if (batch == 0) {
+            if (grad_w && p.num_w > 0)
+                VQC_CUDA(cudaMemsetAsync(grad_w, 0, (size_t)p.num_w * (p.dtype == VQC_C128 ? 8 : 4), s));
+            return VQC_OK;
+        }
+        st = check_ptrs(p, x, w, psi0, nullptr);
+        if (st != VQC_OK) return st;
+        if (!grad_expz) return fail(VQC_ERR_INVALID_ARG, "grad_expz is NULL");
+        if (!expz_out) return fail(VQC_ERR_INVALID_ARG, "expz_out is NULL");
+        if (!use_cluster(p, 0) && !use_hbm(p, 0, batch) && !use_hbm(p, 1, batch)) {
+            // one launch: the backward kernel sweeps forward itself (the state stays in
+            // shared memory), writes E, then sweeps back
+            if (p.dtype == VQC_C64)
+                return run<float>(p, 2, batch, x, w, psi0, nullptr, grad_expz, expz_out, nullptr, grad_x,
+                                  grad_w, workspace, workspace_bytes, s);
+            return run<double>(p, 2, batch, x, w, psi0, nullptr, grad_expz, expz_out, nullptr, grad_x,
+                               grad_w, workspace, workspace_bytes, s);
+        }
+        // states beyond one SM: the forward passes, then the backward recomputing them
+        st = vqc_forward(plan, batch, x, w, psi0, expz_out, nullptr, workspace, workspace_bytes, stream);
+        if (st != VQC_OK) return st;
+        return vqc_backward(plan, batch, x, w, psi0, nullptr, grad_expz, grad_x, grad_w, workspace,
+                            workspace_bytes, stream);
+    } catch (...) {
+        return fail(VQC_ERR_INVALID_ARG, "internal error in vqc_forward_backward");
     }
 }
 

@@ -5,10 +5,10 @@
 // side, a service answering requests) would otherwise pay three host-to-device
 // copies, the forward, the backward, three device-to-host copies and their
 // per-call overheads.  Here the plan keeps a device arena (packed inputs,
-// packed outputs, final states, both workspaces) and a pinned host mirror of
-// the packed inputs and outputs, sized for the largest batch seen:
+// packed outputs, the workspace) and a pinned host mirror of the packed inputs
+// and outputs, sized for the largest batch seen:
 //   host x, w, gE  --memcpy-->  pinned [x | w | gE]  --1 copy-->  device
-//   vqc_forward (E, final states) ; vqc_backward (dx, dw) from those states
+//   vqc_forward_backward (E, dx, dw; one launch on the resident path)
 //   device [E | dx | dw]  --1 copy-->  pinned  --memcpy-->  host E, dx, dw
 // and the call returns after the stream has finished.  Where the device can
 // access pageable host memory coherently (cudaDevAttrPageableMemoryAccess, e.g.
@@ -17,8 +17,7 @@
 // (VQC_HOST_DIRECT=0 forces the staged copies).  From the second call with the
 // same batch and outputs (and, direct, the same arrays) on, the device part is
 // one CUDA graph launch (captured once on a private stream; VQC_HOST_GRAPH=0
-// turns this off).  The arena is released
-// by vqc_free.
+// turns this off).  The arena is released by vqc_free.
 #include <cuda_runtime.h>
 
 #include <cstdlib>
@@ -43,7 +42,7 @@ size_t up256(size_t v) { return (v + 255) & ~(size_t)255; }
 struct Layout {
     size_t x = 0, w = 0, g = 0, in_bytes = 0;
     size_t out = 0, E = 0, dx = 0, dw = 0, out_bytes = 0;
-    size_t state = 0, ws0 = 0, ws0_bytes = 0, ws1 = 0, ws1_bytes = 0, dev_bytes = 0;
+    size_t ws0 = 0, ws0_bytes = 0, ws1 = 0, ws1_bytes = 0, dev_bytes = 0;
     bool operator==(const Layout& o) const { return std::memcmp(this, &o, sizeof(Layout)) == 0; }
 };
 
@@ -99,10 +98,10 @@ Layout layout_for(const vqc_plan* plan, int B, bool bwd) {
     L.dx = o - L.out; o = up256(o + (bwd ? (size_t)B * p.num_x * rs : 0));
     L.dw = o - L.out; o = up256(o + (bwd ? (size_t)p.num_w * rs : 0));
     L.out_bytes = o - L.out;
-    L.state = o; o = up256(o + (bwd ? ((size_t)B << p.n) * 2 * rs : 0));
-    L.ws0_bytes = vqc_workspace_bytes(plan, B, 0);
+    // forward only: vqc_forward's workspace; with gE: vqc_forward_backward's
+    L.ws0_bytes = bwd ? 0 : vqc_workspace_bytes(plan, B, 0);
     L.ws0 = o; o = up256(o + L.ws0_bytes);
-    L.ws1_bytes = bwd ? vqc_workspace_bytes(plan, B, 1) : 0;
+    L.ws1_bytes = bwd ? vqc_workspace_bytes(plan, B, 3) : 0;
     L.ws1 = o; o = up256(o + L.ws1_bytes);
     L.dev_bytes = o;
     return L;
@@ -283,18 +282,17 @@ extern "C" vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, con
         }
 
         // Direct access: the kernels read x, w, gE and write E, dx, dw in the
-        // caller's host arrays themselves; only states and workspaces are in
-        // the arena.
+        // caller's host arrays themselves; only the workspace is in the arena.
         auto enqueue_direct = [&](cudaStream_t q) -> vqc_status {
             const void* xh = p.num_x > 0 ? x : nullptr;
             const void* wh = p.num_w > 0 ? w : nullptr;
-            vqc_status r = vqc_forward(plan, batch, xh, wh, nullptr, expz_out, bwd ? D + L.state : nullptr,
-                                       L.ws0_bytes ? D + L.ws0 : nullptr, L.ws0_bytes, q);
-            if (r != VQC_OK || !bwd) return r;
-            return vqc_backward(plan, batch, xh, wh, nullptr, D + L.state, grad_expz,
-                                (flags & 2) && p.num_x > 0 ? grad_x : nullptr,
-                                (flags & 4) && p.num_w > 0 ? grad_w : nullptr,
-                                L.ws1_bytes ? D + L.ws1 : nullptr, L.ws1_bytes, q);
+            if (!bwd)
+                return vqc_forward(plan, batch, xh, wh, nullptr, expz_out, nullptr,
+                                   L.ws0_bytes ? D + L.ws0 : nullptr, L.ws0_bytes, q);
+            return vqc_forward_backward(plan, batch, xh, wh, nullptr, grad_expz, expz_out,
+                                        (flags & 2) && p.num_x > 0 ? grad_x : nullptr,
+                                        (flags & 4) && p.num_w > 0 ? grad_w : nullptr,
+                                        L.ws1_bytes ? D + L.ws1 : nullptr, L.ws1_bytes, q);
         };
 
         // inputs: caller memory -> pinned mirror (one copy to the device below)
@@ -311,16 +309,14 @@ extern "C" vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, con
             const void* xd = p.num_x > 0 ? D + L.x : nullptr;
             const void* wd = p.num_w > 0 ? D + L.w : nullptr;
             unsigned char* O = D + L.out;
-            vqc_status r = vqc_forward(plan, batch, xd, wd, nullptr, O + L.E, bwd ? D + L.state : nullptr,
-                                       L.ws0_bytes ? D + L.ws0 : nullptr, L.ws0_bytes, q);
+            const vqc_status r =
+                bwd ? vqc_forward_backward(plan, batch, xd, wd, nullptr, D + L.g, O + L.E,
+                                           (flags & 2) && p.num_x > 0 ? O + L.dx : nullptr,
+                                           (flags & 4) && p.num_w > 0 ? O + L.dw : nullptr,
+                                           L.ws1_bytes ? D + L.ws1 : nullptr, L.ws1_bytes, q)
+                    : vqc_forward(plan, batch, xd, wd, nullptr, O + L.E, nullptr,
+                                  L.ws0_bytes ? D + L.ws0 : nullptr, L.ws0_bytes, q);
             if (r != VQC_OK) return r;
-            if (bwd) {
-                r = vqc_backward(plan, batch, xd, wd, nullptr, D + L.state, D + L.g,
-                                 (flags & 2) && p.num_x > 0 ? O + L.dx : nullptr,
-                                 (flags & 4) && p.num_w > 0 ? O + L.dw : nullptr,
-                                 L.ws1_bytes ? D + L.ws1 : nullptr, L.ws1_bytes, q);
-                if (r != VQC_OK) return r;
-            }
             ce = cudaMemcpyAsync(H + L.in_bytes, O, L.out_bytes, cudaMemcpyDeviceToHost, q);
             if (ce != cudaSuccess) return cuda_err(ce, "cudaMemcpyAsync(outputs)");
             return VQC_OK;

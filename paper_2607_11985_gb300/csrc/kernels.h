@@ -13,6 +13,8 @@ const void* sweep_ptr_f32_fwd_small(int K);    // sample groups of < 32 threads
 const void* sweep_ptr_f32_bwd_small(int K);
 const void* sweep_ptr_f64_fwd_small(int K);
 const void* sweep_ptr_f64_bwd_small(int K);
+const void* sweep_ptr_f32_fused(int K, bool full);   // backward that also writes E
+const void* sweep_ptr_f64_fused(int K, bool full);
 
 // HBM-tiled pass kernels (K fixed per type and mode) and partial reductions.
 const void* pass_ptr(bool dbl, int mode, int K, bool full);   // full: tile groups >= 32 threads

@@ -7,10 +7,10 @@ namespace vqc {
 
 const void* sweep_ptr_f32_bwd(int K) {
     switch (K) {
-    case 1: return reinterpret_cast<const void*>(&sweep_kernel<float, 1, 1, true>);
-    case 2: return reinterpret_cast<const void*>(&sweep_kernel<float, 2, 1, true>);
-    case 3: return reinterpret_cast<const void*>(&sweep_kernel<float, 3, 1, true>);
-    case 4: return reinterpret_cast<const void*>(&sweep_kernel<float, 4, 1, true>);
+    case 1: return reinterpret_cast<const void*>(&sweep_kernel<float, 1, 1, true, false>);
+    case 2: return reinterpret_cast<const void*>(&sweep_kernel<float, 2, 1, true, false>);
+    case 3: return reinterpret_cast<const void*>(&sweep_kernel<float, 3, 1, true, false>);
+    case 4: return reinterpret_cast<const void*>(&sweep_kernel<float, 4, 1, true, false>);
     default: return nullptr;
     }
 }

@@ -7,11 +7,11 @@ namespace vqc {
 
 const void* sweep_ptr_f32_fwd_small(int K) {
     switch (K) {
-    case 1: return reinterpret_cast<const void*>(&sweep_kernel<float, 1, 0, false>);
-    case 2: return reinterpret_cast<const void*>(&sweep_kernel<float, 2, 0, false>);
-    case 3: return reinterpret_cast<const void*>(&sweep_kernel<float, 3, 0, false>);
-    case 4: return reinterpret_cast<const void*>(&sweep_kernel<float, 4, 0, false>);
-    case 5: return reinterpret_cast<const void*>(&sweep_kernel<float, 5, 0, false>);
+    case 1: return reinterpret_cast<const void*>(&sweep_kernel<float, 1, 0, false, false>);
+    case 2: return reinterpret_cast<const void*>(&sweep_kernel<float, 2, 0, false, false>);
+    case 3: return reinterpret_cast<const void*>(&sweep_kernel<float, 3, 0, false, false>);
+    case 4: return reinterpret_cast<const void*>(&sweep_kernel<float, 4, 0, false, false>);
+    case 5: return reinterpret_cast<const void*>(&sweep_kernel<float, 5, 0, false, false>);
     default: return nullptr;
     }
 }

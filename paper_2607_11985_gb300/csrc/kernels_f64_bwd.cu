@@ -7,9 +7,9 @@ namespace vqc {
 
 const void* sweep_ptr_f64_bwd(int K) {
     switch (K) {
-    case 1: return reinterpret_cast<const void*>(&sweep_kernel<double, 1, 1, true>);
-    case 2: return reinterpret_cast<const void*>(&sweep_kernel<double, 2, 1, true>);
-    case 3: return reinterpret_cast<const void*>(&sweep_kernel<double, 3, 1, true>);
+    case 1: return reinterpret_cast<const void*>(&sweep_kernel<double, 1, 1, true, false>);
+    case 2: return reinterpret_cast<const void*>(&sweep_kernel<double, 2, 1, true, false>);
+    case 3: return reinterpret_cast<const void*>(&sweep_kernel<double, 3, 1, true, false>);
     default: return nullptr;
     }
 }

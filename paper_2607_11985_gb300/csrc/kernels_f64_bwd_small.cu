@@ -7,9 +7,9 @@ namespace vqc {
 
 const void* sweep_ptr_f64_bwd_small(int K) {
     switch (K) {
-    case 1: return reinterpret_cast<const void*>(&sweep_kernel<double, 1, 1, false>);
-    case 2: return reinterpret_cast<const void*>(&sweep_kernel<double, 2, 1, false>);
-    case 3: return reinterpret_cast<const void*>(&sweep_kernel<double, 3, 1, false>);
+    case 1: return reinterpret_cast<const void*>(&sweep_kernel<double, 1, 1, false, false>);
+    case 2: return reinterpret_cast<const void*>(&sweep_kernel<double, 2, 1, false, false>);
+    case 3: return reinterpret_cast<const void*>(&sweep_kernel<double, 3, 1, false, false>);
     default: return nullptr;
     }
 }

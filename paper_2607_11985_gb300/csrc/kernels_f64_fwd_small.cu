@@ -7,10 +7,10 @@ namespace vqc {
 
 const void* sweep_ptr_f64_fwd_small(int K) {
     switch (K) {
-    case 1: return reinterpret_cast<const void*>(&sweep_kernel<double, 1, 0, false>);
-    case 2: return reinterpret_cast<const void*>(&sweep_kernel<double, 2, 0, false>);
-    case 3: return reinterpret_cast<const void*>(&sweep_kernel<double, 3, 0, false>);
-    case 4: return reinterpret_cast<const void*>(&sweep_kernel<double, 4, 0, false>);
+    case 1: return reinterpret_cast<const void*>(&sweep_kernel<double, 1, 0, false, false>);
+    case 2: return reinterpret_cast<const void*>(&sweep_kernel<double, 2, 0, false, false>);
+    case 3: return reinterpret_cast<const void*>(&sweep_kernel<double, 3, 0, false, false>);
+    case 4: return reinterpret_cast<const void*>(&sweep_kernel<double, 4, 0, false, false>);
     default: return nullptr;
     }
 }

@@ -1166,7 +1166,10 @@ __device__ void acc_terms(const DAcc& ac, const DEntry& e, const R* ap, int wg,
 // MODE 0: forward, MODE 1: backward.
 // FULL: every sample group spans whole warps (2^(n-K) >= 32 threads), so warp
 // reductions are fixed full-warp butterflies; the launch picks the variant.
-template <typename R, int K, int MODE, bool FULL>
+// FUSED (MODE 1 only): the backward that recomputes the states also writes E
+// (vqc_forward_backward); a separate instantiation keeps that code out of the
+// plain backward kernel.
+template <typename R, int K, int MODE, bool FULL, bool FUSED>
 __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArgs<R> A) {
     extern __shared__ __align__(16) unsigned char smem[];
     R* sh_tab = reinterpret_cast<R*>(smem + A.sm_sh);
@@ -1297,8 +1300,10 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
         const bool recompute = MODE == 1 && A.psi_final == nullptr;
         const int ns = A.nstages;
 
-        // -------- forward sweep (forward mode, or backward recompute)
+        // -------- forward sweep (forward mode, or backward recompute; the
+        // recompute also writes E when the caller asks for it)
         R* red = red_all + (size_t)q.g * q.wg * n;
+        const bool want_E = MODE == 0 || (FUSED && recompute && A.E != nullptr);
         if (MODE == 0 || recompute) {
             for (int s = 0; s < ns; ++s) {
                 const DStage* sp = P.stages + s;
@@ -1317,7 +1322,7 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                     }
                     run_ops<R, K, 0, false, FULL>(P.ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
                                      sh_tab, ps_tab, nullptr, q, lane, warp_in_group);
-                    if (MODE == 0 && last) {   // <Z_j> partials from the final blocks
+                    if (want_E && last) {   // <Z_j> partials from the final blocks
                         if constexpr (FULL) {   // butterfly over the warp (n <= 16 here)
                             if (n <= 8) {
                                 R ez[8];
@@ -1347,7 +1352,7 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                         block_store<R, K>(a, psi, b2, s2);
                     }
                 }
-                if (MODE == 0 && last && FULL) {
+                if (want_E && last && FULL) {
                     // a single-warp group writes E itself
                     const int low = n <= 8 ? 3 : 1;   // lane bits below the scatter bits
                     if ((lane & low) == 0 && eidx < n) {
@@ -1382,6 +1387,16 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
             }
             if (unit + (int)gridDim.x < A.nunits) __syncthreads();
             continue;
+        }
+
+        if (MODE == 1 && want_E && !(FULL && q.wg == 1)) {   // E of the recomputed states
+            __syncthreads();
+            if (valid)
+                for (int j = q.t; j < n; j += q.T) {
+                    R e = 0;
+                    for (int k = 0; k < q.wg; ++k) e += red[k * n + j];
+                    A.E[(size_t)b * n + j] = e;
+                }
         }
 
         // -------- backward: reverse sweep with psi and lam

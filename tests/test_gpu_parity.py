@@ -316,3 +316,59 @@ def test_largest_resident_forward_n14():
     for psi_final in (None, devc(st, "c64")):
         dx, dw = run_bwd(c, w_, psi_final=psi_final)
         assert maxerr(dx, dx_ref) <= 5e-4 and maxerr(dw, dw_ref) <= 5e-4
+
+
+# ------------------------------------------------------------------ fused forward + backward
+@pytest.mark.parametrize("case", ["cfg1", "cfg2", "cfg3_rows", "rand_c128_psi0", "hbm16"])
+def test_forward_backward_fused(case, monkeypatch):
+    """vqc_forward_backward (one launch on the resident path: the backward kernel
+    sweeps forward itself and writes E) against the oracle and against the
+    separate vqc_forward + vqc_backward.  Covers sub-warp groups (4 qubits),
+    one-warp groups (8), multi-warp groups (12), complex128 with psi0, and a
+    16-qubit plan that runs as forward passes + recomputing backward passes."""
+    psi0 = None
+    if case == "cfg1":
+        w_ = wl.config(1)[0]
+    elif case == "cfg2":
+        w_ = wl.config(2)[0]
+    elif case == "cfg3_rows":
+        full = wl.config(3)[0]
+        idx = np.arange(40) * 97 % full.batch
+        w_ = wl.Workload(full.name, full.spec, 40, full.x[idx], full.w, full.gE[idx], "c64", full.seed)
+    elif case == "rand_c128_psi0":
+        w_, psi0 = wl.small_random(777, 9, 180, batch=6, dtype="c128", with_psi0=True)
+    else:
+        spec = wl.layered(16, 1, ("RX", "RY", "RZ"), "CX")
+        rng = np.random.default_rng(1616)
+        w_ = wl.Workload("hbm16", spec, 2, wl._round(rng.uniform(-3, 3, (2, 16)), "c64"),
+                         wl._round(rng.uniform(-3, 3, spec.num_w), "c64"),
+                         wl._round(rng.standard_normal((2, 16)), "c64"), "c64", 1616)
+    dt = w_.dtype
+    c = C(w_.spec, dt)
+    x = dev(w_.x, dt) if w_.spec.num_x else None
+    w = dev(w_.w, dt) if w_.spec.num_w else None
+    gE = dev(w_.gE, dt)
+    p0 = devc(psi0, dt) if psi0 is not None else None
+    E, dx, dw = c.forward_backward(x, w, gE, psi0=p0)
+    torch.cuda.synchronize()
+    E, dx, dw = E.cpu().numpy(), (dx.cpu().numpy() if dx is not None else None), \
+        (dw.cpu().numpy() if dw is not None else None)
+    E2 = run_fwd(c, w_, psi0, want_state=False)
+    dx2, dw2 = run_bwd(c, w_, psi0)
+    tol = TOL[dt]
+    close = 1e-5 if dt == "c64" else 1e-12
+    assert maxerr(E, E2) <= close
+    if dx is not None:
+        assert maxerr(dx, dx2) <= 10 * close
+    if dw is not None:
+        assert maxerr(dw, dw2) <= 10 * close * max(1.0, float(np.abs(dw2).max()))
+    rows = [0, w_.batch - 1]
+    E_ref = orc.forward(w_.spec, w_.x[rows], w_.w, psi0=None if psi0 is None else psi0[rows])
+    dx_ref, _ = orc.backward(w_.spec, w_.x[rows], w_.w, w_.gE[rows],
+                             psi0=None if psi0 is None else psi0[rows])
+    assert maxerr(E[rows], E_ref) <= tol["E"]
+    if dx is not None:
+        assert maxerr(dx[rows], dx_ref) <= tol["grad"]
+    if w_.batch <= 64 and dw is not None:
+        _, dw_ref = orc.backward(w_.spec, w_.x, w_.w, w_.gE, psi0=psi0)
+        assert maxerr(dw, dw_ref) <= tol["grad"]
