@@ -269,8 +269,10 @@ def run_ours(args, rank, world, local_rank):
     h2d = xh.nbytes + wh.nbytes + gh.nbytes
     d2h = Eh.nbytes + dxh.nbytes + dwh.nbytes
 
+    host_step = c.prepare_host(xh, wh, gh, out=(Eh, dxh, dwh), stream=sp)
+
     def e2e_step():
-        c.evaluate_host(xh, wh, gh, out=(Eh, dxh, dwh), stream=sp)
+        host_step()
         if world > 1:   # the data-parallel dw sum of the step
             t = torch.from_numpy(dwh).to("cuda")
             dist.all_reduce(t)
@@ -367,7 +369,7 @@ def run_ours(args, rank, world, local_rank):
                      "launch_ms": bwd_avg_s * 1e3,
                      "fwd_frac": ach_fwd / peak},
         "e2e": {"value": e2e_value, "unit": "circuit evals/s (fwd+adjoint bwd, host buffers)",
-                "call": "vqc_evaluate_host (pageable numpy in/out; %s)" % (
+                "call": "Circuit.prepare_host -> vqc_evaluate_host (pageable numpy in/out; %s)" % (
                     "kernels access the host arrays in place over NVLink-C2C"
                     if B.vqc_host_direct(local_rank) else "one packed copy each way"),
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": Ke},

@@ -199,8 +199,61 @@ class Circuit:
         B.vqc_evaluate_host(self.plan, batch, hp(x), hp(w), hp(gE), hp(E), hp(dx), hp(dw), stream)
         return E if gE is None else (E, dx, dw)
 
+    def prepare_host(self, x, w, grad_expz=None, out=None, stream=None):
+        """A prepared ``evaluate_host`` on fixed host arrays: the arrays are
+        checked and their addresses taken once; each call of the returned
+        ``HostStep`` evaluates whatever the arrays hold then (refill them in
+        place between calls) and returns the output arrays."""
+        return HostStep(self, x, w, grad_expz, out, stream)
+
     def __call__(self, x, w, psi0=None):
         return VQCFunction.apply(x, w, self, psi0)
+
+
+class HostStep:
+    """``Circuit.prepare_host``: one vqc_evaluate_host call on fixed host arrays."""
+
+    def __init__(self, circuit, x, w, grad_expz=None, out=None, stream=None):
+        import numpy as np
+        c = circuit
+        rdt = np.float32 if c.dtype == "c64" else np.float64
+        batch = x.shape[0] if x is not None and c.num_x else \
+            (grad_expz.shape[0] if grad_expz is not None else 1)
+
+        def arr(a, shape, name):
+            if a is None:
+                return None
+            if not isinstance(a, np.ndarray) or a.dtype != rdt or a.shape != tuple(shape) \
+                    or not a.flags.c_contiguous:
+                raise ValueError("%s must be a C-contiguous %s array of shape %s"
+                                 % (name, np.dtype(rdt).name, tuple(shape)))
+            return a
+
+        x = arr(x, (batch, c.num_x), "x") if c.num_x else None
+        w = arr(w, (c.num_w,), "w") if c.num_w else None
+        gE = arr(grad_expz, (batch, c.n), "grad_expz")
+        if out is None:
+            out = (np.empty((batch, c.n), rdt),
+                   np.empty((batch, c.num_x), rdt) if gE is not None and c.num_x else None,
+                   np.empty((c.num_w,), rdt) if gE is not None and c.num_w else None)
+        E, dx, dw = out
+        E = arr(E, (batch, c.n), "E")
+        dx = arr(dx, (batch, c.num_x), "dx")
+        dw = arr(dw, (c.num_w,), "dw")
+        self.circuit = c                              # keeps the plan alive
+        self.arrays = (x, w, gE, E, dx, dw)           # keeps the addresses valid
+        hp = lambda a: None if a is None else a.ctypes.data   # noqa: E731
+        if stream is None:
+            stream = torch.cuda.current_stream().cuda_stream
+        self._args = (c.plan, batch) + tuple(hp(a) for a in self.arrays) + (stream,)
+        self._fn = B.lib().vqc_evaluate_host
+        self.result = E if gE is None else (E, dx, dw)
+
+    def __call__(self):
+        st = self._fn(*self._args)
+        if st != 0:
+            B._check(st)
+        return self.result
 
 
 class VQCFunction(torch.autograd.Function):

@@ -157,3 +157,23 @@ def test_graph_replay_sees_new_inputs(access, monkeypatch):
     sub = wl.Workload(w_.name, w_.spec, 64, x2.astype(np.float64), w2.astype(np.float64),
                       g1.astype(np.float64), "c64", w_.seed)
     assert maxerr(other[0], orc.forward(w_.spec, sub.x, sub.w)) <= TOL["c64"]["E"]
+
+
+def test_prepared_host_step_refills(access):
+    """Circuit.prepare_host: the arrays are bound once; refilling them in place
+    between calls gives the results evaluate_host gives on the new contents."""
+    w_ = wl.config(2, batch=64)[0]
+    c = C(w_.spec, "c64")
+    x, w, g = host(w_.x, "c64"), host(w_.w, "c64"), host(w_.gE, "c64")
+    step = c.prepare_host(x, w, g)
+    E1, dx1, dw1 = [a.copy() for a in step()]
+    ref1 = c.evaluate_host(host(w_.x, "c64"), host(w_.w, "c64"), host(w_.gE, "c64"))
+    x[:] = x[::-1].copy()
+    g *= -0.5
+    E2, dx2, dw2 = [a.copy() for a in step()]
+    ref2 = c.evaluate_host(x.copy(), w.copy(), g.copy())
+    for a, b in zip((E1, dx1, dw1, E2, dx2, dw2), tuple(ref1) + tuple(ref2)):
+        assert np.array_equal(a, b)
+    assert not np.array_equal(E1, E2)
+    with pytest.raises(ValueError):
+        c.prepare_host(w_.x, w, g)          # float64 x for a complex64 plan
