@@ -372,3 +372,59 @@ def test_forward_backward_fused(case, monkeypatch):
     if w_.batch <= 64 and dw is not None:
         _, dw_ref = orc.backward(w_.spec, w_.x, w_.w, w_.gE, psi0=psi0)
         assert maxerr(dw, dw_ref) <= tol["grad"]
+
+
+# ------------------------------------------------------------------ degenerate circuits
+@pytest.mark.parametrize("dtype", ["c64", "c128"])
+@pytest.mark.parametrize("which", ["empty", "no_params", "one_long_run"])
+def test_degenerate_circuits(dtype, which):
+    """An empty gate list (E = <Z> of psi0; the state passes through), a circuit
+    without any angle parameter (gradients have no entries), and one qubit
+    carrying a single fused run of 40 rotations (far more than a table entry's
+    four constituents) with a gradient for every angle: forward, backward and
+    the fused call against the oracle, with and without psi0."""
+    rng = np.random.default_rng({"empty": 11, "no_params": 12, "one_long_run": 13}[which])
+    if which == "empty":
+        spec = wl.CircuitSpec(3, 0, 0)
+    elif which == "no_params":
+        spec = wl.CircuitSpec(5, 0, 0).add("H", (0,)).add("CX", (0, 4)).add("T", (4,)) \
+            .add("SWAP", (1, 3)).add("U3", (2,), [("c", 0.3), ("c", -1.1), ("c", 2.0)]).add("CZ", (2, 4))
+    else:
+        spec = wl.CircuitSpec(4, 2, 20).add("H", (1,)).add("CX", (1, 2))
+        for k in range(40):
+            g = ("RX", "RY", "RZ")[k % 3]
+            spec.add(g, (2,), [("x", k % 2)] if k % 4 == 0 else [("w", k % 20)])
+        spec.add("CRZ", (2, 3), [("w", 3)])
+    Bt = 5
+    x = wl._round(rng.uniform(-np.pi, np.pi, (Bt, spec.num_x)), dtype)
+    w = wl._round(rng.uniform(-np.pi, np.pi, spec.num_w), dtype)
+    gE = wl._round(rng.standard_normal((Bt, spec.n)), dtype)
+    z = rng.standard_normal((Bt, 1 << spec.n)) + 1j * rng.standard_normal((Bt, 1 << spec.n))
+    z /= np.linalg.norm(z, axis=1, keepdims=True)
+    if dtype == "c64":
+        z = z.astype(np.complex64).astype(np.complex128)
+    c = C(spec, dtype)
+    tol = TOL[dtype]
+    real = torch.float32 if dtype == "c64" else torch.float64
+    xd = torch.tensor(x, dtype=real, device="cuda")   # [B, 0] when there is no x: carries B
+    wd = dev(w, dtype) if spec.num_w else None
+    gd = dev(gE, dtype)
+    for psi0 in (None, z):
+        p0 = devc(psi0, dtype) if psi0 is not None else None
+        E, st = c.forward(xd, wd, psi0=p0, want_state=True)
+        dx, dw = c.backward(xd if spec.num_x else None, wd, gd, psi0=p0)
+        Ef, dxf, dwf = c.forward_backward(xd if spec.num_x else None, wd, gd, psi0=p0)
+        torch.cuda.synchronize()
+        E_ref, st_ref = orc.forward(spec, x, w, psi0=psi0, want_state=True)
+        dx_ref, dw_ref = orc.backward(spec, x, w, gE, psi0=psi0)
+        assert maxerr(E.cpu().numpy(), E_ref) <= tol["E"]
+        assert maxerr(Ef.cpu().numpy(), E_ref) <= tol["E"]
+        assert maxerr(st.cpu().numpy(), st_ref) <= tol["state"]
+        if which == "empty":
+            assert maxerr(st.cpu().numpy(), psi0 if psi0 is not None else
+                          np.eye(1, 1 << spec.n).repeat(Bt, 0)) <= tol["state"]
+        for got, ref in ((dx, dx_ref), (dw, dw_ref), (dxf, dx_ref), (dwf, dw_ref)):
+            if got is None:
+                assert np.asarray(ref).size == 0
+            else:
+                assert maxerr(got.cpu().numpy(), ref) <= tol["grad"]
