@@ -448,9 +448,9 @@ vqc_status plan_cluster(const HostPlan& p, int B, Launch& L) {
     const bool dbl = p.dtype == VQC_C128;
     const size_t rs = dbl ? 8 : 4, cs = 2 * rs, ew = dbl ? 8 : 32;
     L.K = L.s->K;
-    L.cl = p.n - L.K - 9;
+    L.cl = p.n - L.K - L.s->cta_bits;
     L.T = 1 << (p.n - L.K);           // threads of a sample group, over the whole cluster
-    L.block = L.T >> L.cl;            // 512
+    L.block = L.T >> L.cl;            // 2^cta_bits: 256 or 512
     L.S = 1;
     L.bpt = 1;
     L.wg = L.block / 32;

@@ -656,18 +656,21 @@ vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx,
         }
     }
     // Cluster schedules (forward): states up to 16 qubits over 2..8 CTAs of a
-    // thread-block cluster, one register block per thread (2^(n-K) threads, at
-    // most 512 per CTA) and at most 128 KiB of state per CTA.
+    // thread-block cluster, one register block per thread (2^(n-K) threads) and
+    // at most 128 KiB of state per CTA.  CTAs of 512 threads (2^cta_bits):
+    // 256-thread CTAs, two clusters' CTAs per SM, measured 12% slower on the
+    // 16-qubit workload (more cross-CTA stages, wider cluster barriers).
     {
         const int K = max_k(0, dtype);
-        const int cl = n - K - 9;
         const size_t cs = dtype == VQC_C128 ? 16 : 8;
+        const int ctb = 9, cl = n - K - ctb;
         if (n > resident_max_qubits(0, dtype) && n <= 16 && cl >= 1 && cl <= 3 &&
             (((size_t)1 << (n - cl)) * cs) <= 128 * 1024) {
             Schedule s;
             s.mode = 0;
             s.K = K;
             s.path = VQC_PATH_CLUSTER;
+            s.cta_bits = ctb;
             build_schedule(p, s);
             // A map keeps every block in its thread's own CTA when no local offset
             // reaches the top cl slot bits (those index the CTA) and the top cl
@@ -733,7 +736,7 @@ const Schedule* find_hbm_schedule(const HostPlan& p, int mode) {
 
 std::vector<uint8_t> export_plan(const HostPlan& p) {
     std::vector<uint8_t> out = {'V', 'Q', 'C', 'P'};
-    put_i32(out, 2);   // export format version
+    put_i32(out, 3);   // export format version
     for (int v : {p.n, p.num_x, p.num_w, p.dtype, p.num_gates_in, p.G_swz, p.n_ps, p.n_sh,
                   p.n_runs})
         put_i32(out, v);
@@ -759,7 +762,8 @@ std::vector<uint8_t> export_plan(const HostPlan& p) {
     put_vec(out, p.wocc);
     put_i32(out, (int32_t)p.scheds.size());
     for (const auto& s : p.scheds) {
-        for (int v : {s.mode, s.K, s.m, s.path, s.thread_bits, s.group_lanes_log2}) put_i32(out, v);
+        for (int v : {s.mode, s.K, s.m, s.path, s.thread_bits, s.group_lanes_log2, s.cta_bits})
+            put_i32(out, v);
         put_vec(out, s.ops);
         put_vec(out, s.stages);
         put_vec(out, s.passes);

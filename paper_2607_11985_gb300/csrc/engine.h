@@ -30,6 +30,7 @@ struct Schedule {
     int path = VQC_PATH_RESIDENT;
     int thread_bits = 0;   // m - K
     int group_lanes_log2 = 0;   // log2(threads per sample group) when < 2^G
+    int cta_bits = 0;           // cluster path: log2(threads per CTA); 2^(m-K-cta_bits) CTAs
     std::vector<DOp> ops;
     std::vector<DStage> stages;
     std::vector<DPass> passes;            // HBM path: one record per pass

@@ -96,7 +96,7 @@ class Plan:
         assert blob[:4] == b"VQCP"
         r = Reader(blob)
         r.off = 4
-        assert r.i32() == 2
+        assert r.i32() == 3
         (self.n, self.num_x, self.num_w, self.dtype, self.num_gates_in, self.G, self.n_ps,
          self.n_sh, self.n_runs) = [r.i32() for _ in range(9)]
         self.hops = r.vec("<i4").reshape(-1, 5)
@@ -113,14 +113,14 @@ class Plan:
         self.wocc = r.vec("<i4")
         self.scheds = []
         for _ in range(r.i32()):
-            mode, K, m, path, tb, gl = [r.i32() for _ in range(6)]
+            mode, K, m, path, tb, gl, ctb = [r.i32() for _ in range(7)]
             ops = r.vec(DOP)
             stages = r.vec(DSTAGE)
             passes = r.vec(DPASS)
             pass_entries = r.vec("<i4")
             pass_accs = r.vec("<i4")
             store_masks = r.vec("<u4").reshape(len(stages), 5 + 16)
-            self.scheds.append(dict(mode=mode, K=K, m=m, path=path, thread_bits=tb, ops=ops,
+            self.scheds.append(dict(mode=mode, K=K, m=m, path=path, thread_bits=tb, cta_bits=ctb, ops=ops,
                                     stages=stages, passes=passes, pass_entries=pass_entries,
                                     pass_accs=pass_accs, store_masks=store_masks))
         assert r.off == len(blob)

@@ -248,17 +248,18 @@ def slots_all(st, K, sig, tau):
 
 
 def test_cluster_locality_flags():
-    """Cluster schedules (512 threads per CTA, 2^(n-K-9) CTAs): a stage's
-    cl_local bit 0 / bit 1 is set exactly when every slot its load / store map
-    gives a thread lies in the slice of that thread's own CTA."""
+    """Cluster schedules (2^cta_bits threads per CTA, 2^(n-K-cta_bits) CTAs): a
+    stage's cl_local bit 0 / bit 1 is set exactly when every slot its load /
+    store map gives a thread lies in the slice of that thread's own CTA."""
     w_ = wl.config(5, batch=1)[0]
     seen = 0
     for dtype in (0, 1):
         pl = Plan(B.vqc_plan_export(compile_spec(w_.spec, dtype)))
         for s in (s for s in pl.scheds if s["path"] == 2):
-            n, K = pl.n, s["K"]
-            slice_ = K + 9
-            rank = (np.arange(1 << (n - K)) >> 9)[:, None]
+            n, K, ctb = pl.n, s["K"], s["cta_bits"]
+            assert ctb == 9 and 1 <= n - K - ctb <= 3
+            slice_ = K + ctb
+            rank = (np.arange(1 << (n - K)) >> ctb)[:, None]
             flags = []
             for st in s["stages"]:
                 ld = bool(((slots_all(st, K, "sigma", "tau") >> slice_) == rank).all())
