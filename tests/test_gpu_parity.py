@@ -428,3 +428,33 @@ def test_degenerate_circuits(dtype, which):
                 assert np.asarray(ref).size == 0
             else:
                 assert maxerr(got.cpu().numpy(), ref) <= tol["grad"]
+
+
+def test_two_streams_share_a_plan():
+    """One plan used on two CUDA streams at once (each with its own workspace,
+    different batches): results equal those of the same calls made one after
+    the other on the default stream."""
+    w_ = wl.config(2)[0]
+    c = C(w_.spec, "c64")
+    x = dev(w_.x, "c64")
+    w = dev(w_.w, "c64")
+    gE = dev(w_.gE, "c64")
+    halves = [slice(0, 400), slice(400, 1024)]
+    ref = []
+    for h in halves:
+        E, st = c.forward(x[h], w, want_state=True)
+        dx, dw = c.backward(x[h], w, gE[h], psi_final=st)
+        ref.append((E.clone(), dx.clone(), dw.clone()))
+    torch.cuda.synchronize()
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    got = []
+    for _ in range(3):
+        got.clear()
+        for h, s in zip(halves, streams):
+            with torch.cuda.stream(s):
+                E, st = c.forward(x[h], w, want_state=True)
+                dx, dw = c.backward(x[h], w, gE[h], psi_final=st)
+                got.append((E, dx, dw))
+        torch.cuda.synchronize()
+        for (E, dx, dw), (E0, dx0, dw0) in zip(got, ref):
+            assert torch.equal(E, E0) and torch.equal(dx, dx0) and torch.equal(dw, dw0)
