@@ -311,8 +311,12 @@ vqc_status vqc_plan_info(const vqc_plan* plan, int32_t batch, vqc_plan_stats* ou
  * are a deterministic function of the vqc_compile arguments. */
 vqc_status vqc_plan_export(const vqc_plan* plan, void* buf, size_t* inout_bytes);
 
-/* Synchronise `stream` and report any CUDA error or tripped device check
- * raised by enqueued work on plans of this process. */
+/* Synchronise `stream` and report any CUDA error, then read (and clear) the
+ * error word of every plan of this process on the current device: each kernel
+ * checks its launch geometry against the plan before touching memory and, on
+ * a mismatch (an engine bug, never the caller's data), records it there and
+ * skips its work; such a record returns VQC_ERR_DEVICE_CHECK naming the
+ * kernel kind. */
 vqc_status vqc_sync_check(void* stream);
 
 /* Thread-local message of the last failing call ("" if none). */

@@ -11,6 +11,7 @@
 #include <memory>
 #include <mutex>
 #include <new>
+#include <set>
 #include <string>
 #include <vector>
 
@@ -314,6 +315,10 @@ void fill_plan_args(const HostPlan& p, const Launch& L, KArgs<R>& a) {
 }
 
 // Device buffer layout of a plan (all sections 16-byte aligned).
+// Uploaded plans (their device error words are read by vqc_sync_check).
+std::mutex g_plans_mu;
+std::set<const HostPlan*> g_plans;
+
 vqc_status upload(HostPlan& p) {
     const bool dbl = p.dtype == VQC_C128;
     std::vector<uint8_t> blob;
@@ -368,6 +373,8 @@ vqc_status upload(HostPlan& p) {
     p.dbuf = d;
     p.dbytes = blob.size();
     p.dev_error = reinterpret_cast<unsigned*>(static_cast<char*>(d) + err_off);
+    std::lock_guard<std::mutex> lk(g_plans_mu);
+    g_plans.insert(&p);
     return VQC_OK;
 }
 
@@ -678,6 +685,7 @@ void fill_pass_args(const HostPlan& p, const PassGeo& L, const DPass& ps, PArgs<
     const char* base = static_cast<const char*>(p.dbuf);
     a.ops = reinterpret_cast<const DOp*>(base + L.s->dev_ops);
     a.stages = reinterpret_cast<const DStage*>(base + L.s->dev_stages);
+    a.err = p.dev_error;
     a.pass_entries = reinterpret_cast<const int32_t*>(base + L.s->dev_pass_entries);
     a.pass_accs = reinterpret_cast<const int32_t*>(base + L.s->dev_pass_accs);
     a.entries = reinterpret_cast<const DEntry*>(base + p.dev_entries);
@@ -971,6 +979,10 @@ vqc_status vqc_compile(const vqc_gate* gates, int32_t num_gates, int32_t num_qub
 
 void vqc_free(vqc_plan* plan) {
     if (!plan) return;
+    {
+        std::lock_guard<std::mutex> lk(g_plans_mu);
+        g_plans.erase(&plan->hp);
+    }
     forget_plan(&plan->hp);
     release_host_arena(plan);
     if (plan->hp.dbuf) {
@@ -1242,6 +1254,30 @@ vqc_status vqc_sync_check(void* stream) {
     if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
     e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "cudaGetLastError");
+    // the kernels' launch self-checks: each plan's error word on this device
+    int dev = -1;
+    VQC_CUDA(cudaGetDevice(&dev));
+    std::vector<const HostPlan*> plans;
+    {
+        std::lock_guard<std::mutex> lk(g_plans_mu);
+        plans.assign(g_plans.begin(), g_plans.end());
+    }
+    unsigned tripped = 0;
+    for (const HostPlan* p : plans) {
+        if (p->device != dev || !p->dev_error) continue;
+        unsigned w = 0;
+        VQC_CUDA(cudaMemcpy(&w, p->dev_error, sizeof(w), cudaMemcpyDeviceToHost));
+        if (w) {
+            tripped |= w;
+            VQC_CUDA(cudaMemset(p->dev_error, 0, sizeof(w)));
+        }
+    }
+    if (tripped)
+        return fail(VQC_ERR_DEVICE_CHECK,
+                    std::string("a kernel's launch self-check tripped:") +
+                        ((tripped & 1u) ? " resident sweep geometry" : "") +
+                        ((tripped & 2u) ? " HBM pass geometry" : "") +
+                        ((tripped & 4u) ? " cluster geometry" : "") + " (the work was skipped)");
     return VQC_OK;
 }
 

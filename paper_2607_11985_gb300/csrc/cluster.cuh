@@ -88,6 +88,13 @@ __device__ __forceinline__ void cl_block_store(const C2<R> (&a)[1 << K], uint32_
 // per-warp <Z> sums, sm_ecl rank 0's [2^cl][n] gather of per-CTA sums), cl.
 template <typename R, int K>
 __global__ void __launch_bounds__(512) cluster_fwd_kernel(const __grid_constant__ KArgs<R> A) {
+    // every CTA of every cluster takes the same branch, before any cluster barrier
+    uint32_t nrank;
+    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(nrank));
+    if (geometry_bad(((unsigned)blockDim.x << A.cl) != (unsigned)A.tpg || nrank != (1u << A.cl) ||
+                         A.tpg != (1 << (A.n - K)) || A.nstages < 1,
+                     A.err, kErrClusterGeometry))
+        return;
     extern __shared__ __align__(16) unsigned char smem[];
     R* sh_tab = reinterpret_cast<R*>(smem + A.sm_sh);
     R* ps_tab = reinterpret_cast<R*>(smem + A.sm_ps);

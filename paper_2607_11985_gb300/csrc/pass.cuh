@@ -46,6 +46,7 @@ struct PArgs {
     const unsigned char* plan;   // plan regions copied to shared memory (see KArgs)
     int tab_off, tab_bytes, sched_off, sched_bytes, sm_plan, plan_smem;
     int sm_koff;                 // per-pass tile-copy offsets: [ceil(2^m / (APV * T))] uint2
+    unsigned* err;               // the plan's error word (launch self-check)
 };
 
 // Global amplitude index of tile-local index u (the low G tile bits are the
@@ -126,6 +127,10 @@ __device__ __forceinline__ void tile_scatter(const C2<R>* sm, C2<R>* gs, uint32_
 // tile), see sweep_kernel.
 template <typename R, int K, int MODE, bool FULL>
 __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PArgs<R> A) {
+    if (geometry_bad(blockDim.x != (unsigned)(A.S << A.tbits) || A.tbits != A.m - K ||
+                         A.stage_end <= A.stage_begin,
+                     A.err, kErrPassGeometry))
+        return;
     extern __shared__ __align__(16) unsigned char smem[];
     R* sh_tab = reinterpret_cast<R*>(smem + A.sm_sh);
     R* ps_all = reinterpret_cast<R*>(smem + A.sm_ps);

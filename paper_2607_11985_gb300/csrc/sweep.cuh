@@ -1169,8 +1169,23 @@ __device__ void acc_terms(const DAcc& ac, const DEntry& e, const R* ap, int wg,
 // FUSED (MODE 1 only): the backward that recomputes the states also writes E
 // (vqc_forward_backward); a separate instantiation keeps that code out of the
 // plain backward kernel.
+// Launch-geometry self-check (kernel side): the host derives the block size,
+// the sample groups and the register blocks from one plan; a launch whose
+// numbers disagree records `code` in the plan's error word (read back by
+// vqc_sync_check) and does no work.  Uniform over the grid: every thread takes
+// the same branch.
+__device__ __forceinline__ bool geometry_bad(bool bad, unsigned* err, unsigned code) {
+    if (bad && threadIdx.x == 0 && err) atomicOr(err, code);
+    return bad;
+}
+enum : unsigned { kErrSweepGeometry = 1u, kErrPassGeometry = 2u, kErrClusterGeometry = 4u };
+
 template <typename R, int K, int MODE, bool FULL, bool FUSED>
 __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArgs<R> A) {
+    if (geometry_bad(blockDim.x != (unsigned)(A.S * A.tpg) || A.bpt * A.tpg != (1 << A.tbits) ||
+                         A.tbits != A.n - K || A.nstages < 1,
+                     A.err, kErrSweepGeometry))
+        return;
     extern __shared__ __align__(16) unsigned char smem[];
     R* sh_tab = reinterpret_cast<R*>(smem + A.sm_sh);
     R* ps_all = reinterpret_cast<R*>(smem + A.sm_ps);

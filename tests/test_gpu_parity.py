@@ -15,6 +15,7 @@ torch = pytest.importorskip("torch")
 
 from oracle import oracle as orc  # noqa: E402
 from paper_2607_11985_gb300 import workloads as wl  # noqa: E402
+from paper_2607_11985_gb300 import binding as B  # noqa: E402
 
 pytestmark = pytest.mark.gpu
 
@@ -458,3 +459,28 @@ def test_two_streams_share_a_plan():
         torch.cuda.synchronize()
         for (E, dx, dw), (E0, dx0, dw0) in zip(got, ref):
             assert torch.equal(E, E0) and torch.equal(dx, dx0) and torch.equal(dw, dw0)
+
+
+def test_sync_check_after_every_kernel_kind(monkeypatch):
+    """vqc_sync_check reads every plan's error word: after resident forward,
+    backward and fused launches, HBM passes, the cluster forward and the
+    probabilities kernel, no launch self-check has tripped."""
+    w_ = wl.config(2, batch=64)[0]
+    c = C(w_.spec, "c64")
+    x, w, gE = dev(w_.x, "c64"), dev(w_.w, "c64"), dev(w_.gE, "c64")
+    E, st = c.forward(x, w, want_state=True)
+    c.backward(x, w, gE, psi_final=st)
+    c.forward_backward(x, w, gE)
+    c.probabilities(x, w)
+    spec = wl.layered(15, 1, ("RX", "RY", "RZ"), "CX")
+    rng = np.random.default_rng(15)
+    c2 = C(spec, "c64")
+    x2 = dev(rng.uniform(-3, 3, (2, 15)), "c64")
+    w2 = dev(rng.uniform(-3, 3, spec.num_w), "c64")
+    g2 = dev(rng.standard_normal((2, 15)), "c64")
+    E2, st2 = c2.forward(x2, w2, want_state=True)          # HBM passes
+    c2.backward(x2, w2, g2, psi_final=st2)
+    monkeypatch.setenv("VQC_FORCE_PATH", "cluster")
+    assert c2.info(2)["fwd_path"] == 2
+    c2.forward(x2, w2)                                      # cluster forward
+    B.vqc_sync_check(torch.cuda.current_stream().cuda_stream)
