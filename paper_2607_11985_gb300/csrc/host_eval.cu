@@ -225,7 +225,6 @@ extern "C" vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, con
             return vqc::set_error(VQC_ERR_INVALID_ARG, "vqc_evaluate_host: the plan's arena is on device " +
                                                            std::to_string(A->device) + ", current device is " +
                                                            std::to_string(dev));
-        const Layout L = layout_for(plan, batch, bwd);
         const bool direct = env_flag("VQC_HOST_DIRECT", true) && host_direct(dev);
         const int flags = (bwd ? 1 : 0) | (bwd && grad_x ? 2 : 0) | (bwd && grad_w ? 4 : 0) |
                           (direct ? 8 : 0);
@@ -234,6 +233,9 @@ extern "C" vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, con
         if (direct)
             for (int i = 0; i < 6; ++i) same_shape = same_shape && A->shape_ptrs[i] == ptrs[i];
         if (!same_shape) A->drop_graph();
+        // A captured graph holds this shape's layout (the arena and workspaces it
+        // was recorded on): reuse it instead of planning the launches again.
+        const Layout L = (A->exec && A->have_last) ? A->last : layout_for(plan, batch, bwd);
         if (L.dev_bytes > A->dev_cap) {
             A->drop_graph();
             if (A->dev) {
