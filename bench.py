@@ -352,6 +352,11 @@ def run_ours(args, rank, world, local_rank):
                    "fwd_stages": info["fwd_stages"], "bwd_stages": info["bwd_stages"]},
         "fwd": {"value": world * Bt / fwd_avg_s, "unit": "circuit evals/s (fwd)",
                 "ms": fwd_avg_s * 1e3, "achieved": ach_fwd},
+        # per-call device times (ms) of this rank: median, mean, std (the paper reports mean +- std)
+        "time_stats_ms": {name: {"median": statistics.median(v), "mean": statistics.mean(v),
+                                 "std": statistics.pstdev(v), "n": len(v)}
+                          for name, v in (("step", step_ms), ("fwd", fwd_ms), ("bwd", bwd_ms),
+                                          ("fused", fused_ms))},
         "fused": {"value": world * Bt / (statistics.mean(fused_ms) / 1e3),
                   "unit": "circuit evals/s (fwd+adjoint bwd)",
                   "ms_per_step": statistics.mean(fused_ms),
