@@ -340,9 +340,9 @@ def run_ours(args, rank, world, local_rank):
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "c64 (fp32 arithmetic)",
+        "dtype": "f32",   # arithmetic type; states are complex64 (config.state)
         "data": "synthetic (seeded; RY(x) encoding + RX/RY/RZ layers + CZ ring)",
-        "config": {"workload": w_.name.split("_rank")[0], "qubits": w_.spec.n,
+        "config": {"workload": w_.name.split("_rank")[0], "qubits": w_.spec.n, "state": "complex64",
                    "batch_per_gpu": Bt,
                    "gates": len(w_.spec.gates), "num_x": w_.spec.num_x, "num_w": w_.spec.num_w,
                    "parallelism": "dp%d (batch-sharded replicas, dw all-reduce)" % world,
@@ -624,7 +624,7 @@ def run_reference(args, rank, world):
     return {"metric": METRIC, "value": value, "unit": "circuit evals/s (fwd+adjoint bwd)",
             "impl": "reference", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": total / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "c128 (fp64 arithmetic)",
+            "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded)", "config": {"workload": w_.name, "qubits": w_.spec.n,
                                                     "batch_per_step": chunk},
             "cpu_baseline": {"value": value, "unit": "circuit evals/s (fwd+adjoint bwd)",
