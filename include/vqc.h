@@ -106,9 +106,11 @@ typedef enum {
     VQC_PATH_RESIDENT = 0,  /* each sample's state stays in one CTA's shared memory */
     VQC_PATH_HBM = 1,       /* state in HBM, swept in shared-memory tiles, one launch per pass */
     VQC_PATH_CLUSTER = 2    /* forward: each sample's state spread over the shared memory of a
-                               thread-block cluster (2..8 CTAs), one launch; taken only when the
-                               environment sets VQC_FORCE_PATH=cluster (otherwise such states
-                               go through VQC_PATH_HBM, measured faster) */
+                               thread-block cluster (2..8 CTAs), one launch; taken by default for
+                               2-CTA clusters (complex64 15 qubits, complex128 14 qubits), for
+                               larger ones only when the environment sets VQC_FORCE_PATH=cluster
+                               (they measured slower than VQC_PATH_HBM); VQC_FORCE_PATH=hbm
+                               turns it off */
 } vqc_path;
 
 typedef struct {

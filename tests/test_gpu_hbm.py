@@ -195,7 +195,9 @@ def test_cluster_forward(monkeypatch, dtype, n):
         z = z.astype(np.complex64).astype(np.complex128)
     w_ = wl.Workload("cluster_n%d" % n, spec, B, x, w, gE, dtype, 1500 + n)
     c = C(spec, dtype)
-    assert c.info(B)["fwd_path"] == 1   # the HBM passes unless asked for the cluster
+    # default: the cluster for 2-CTA clusters (complex64 15 qubits, complex128 14), else the passes
+    two_cta = (dtype, n) in (("c64", 15), ("c128", 14))
+    assert c.info(B)["fwd_path"] == (2 if two_cta else 1)
     monkeypatch.setenv("VQC_FORCE_PATH", "cluster")
     assert c.info(B)["fwd_path"] == 2
     tol = TOL[dtype]

@@ -478,6 +478,8 @@ def test_sync_check_after_every_kernel_kind(monkeypatch):
     x2 = dev(rng.uniform(-3, 3, (2, 15)), "c64")
     w2 = dev(rng.uniform(-3, 3, spec.num_w), "c64")
     g2 = dev(rng.standard_normal((2, 15)), "c64")
+    monkeypatch.setenv("VQC_FORCE_PATH", "hbm")
+    assert c2.info(2)["fwd_path"] == 1
     E2, st2 = c2.forward(x2, w2, want_state=True)          # HBM passes
     c2.backward(x2, w2, g2, psi_final=st2)
     monkeypatch.setenv("VQC_FORCE_PATH", "cluster")
