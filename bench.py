@@ -479,7 +479,7 @@ def ablation(torch, Circuit, w_):
     return out
 
 
-def regime_map(torch, Circuit, qubits=(4, 8, 12, 16, 18, 20), batches=(1, 8, 32, 128), layers=4):
+def regime_map(torch, Circuit, qubits=(4, 8, 12, 15, 16, 18, 20), batches=(1, 8, 32, 128), layers=4):
     """Qubits x batch sweep (the paper's regime map, Sec. 4.4): RY(x) encoding,
     `layers` x (RX RY RZ per qubit + CX ring), complex64.  Per point: path, passes,
     device workspace bytes of the backward (the memory the caller must provide
@@ -514,8 +514,10 @@ def regime_map(torch, Circuit, qubits=(4, 8, 12, 16, 18, 20), batches=(1, 8, 32,
                 torch.cuda.synchronize()
                 tf += a.elapsed_time(b2) / reps
                 tb += b2.elapsed_time(d) / reps
+            paths = {0: "resident", 1: "hbm-tiled", 2: "cluster"}
             pts.append({"qubits": n, "batch": Bt,
-                        "path": "hbm-tiled" if inf["bwd_path"] == 1 else "resident",
+                        "path": paths[inf["fwd_path"]] if inf["fwd_path"] == inf["bwd_path"] else
+                        "%s fwd / %s bwd" % (paths[inf["fwd_path"]], paths[inf["bwd_path"]]),
                         "passes_fwd_bwd": [inf["fwd_passes"], inf["bwd_passes"]],
                         "state_bytes": Bt * (8 << n),
                         "bwd_workspace_bytes": int(Bd.vqc_workspace_bytes(c.plan, Bt, 1)),
