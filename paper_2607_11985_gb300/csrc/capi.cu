@@ -7,6 +7,7 @@
 #include <algorithm>
 #include <cstdlib>
 #include <cstring>
+#include <initializer_list>
 #include <map>
 #include <memory>
 #include <mutex>
@@ -887,6 +888,19 @@ vqc_status check_common(const vqc_plan* plan, int32_t batch) {
     return VQC_OK;
 }
 
+// Real arrays (E, gE, dx, dw, probabilities) must be aligned to the real type,
+// state arrays to the complex type; NULL passes (each call checks presence).
+vqc_status check_out_ptrs(const HostPlan& p, std::initializer_list<const void*> reals,
+                          std::initializer_list<const void*> states) {
+    const size_t rs = p.dtype == VQC_C128 ? 8 : 4;
+    for (const void* q : reals)
+        if (q && misaligned(q, rs)) return fail(VQC_ERR_INVALID_ARG, "real arrays must be aligned to the real type");
+    for (const void* q : states)
+        if (q && misaligned(q, 2 * rs))
+            return fail(VQC_ERR_INVALID_ARG, "state arrays must be aligned to the complex type");
+    return VQC_OK;
+}
+
 vqc_status check_ptrs(const HostPlan& p, const void* x, const void* w, const void* psi0,
                       const void* psi_final) {
     const size_t rs = p.dtype == VQC_C128 ? 8 : 4;
@@ -925,6 +939,8 @@ vqc_status backward_with_scratch(const vqc_plan* plan, int32_t batch, const void
     st = check_ptrs(p, x, w, psi0, psi_final);
     if (st != VQC_OK) return st;
     if (!grad_expz) return fail(VQC_ERR_INVALID_ARG, "grad_expz is NULL");
+    st = check_out_ptrs(p, {grad_expz, grad_x, grad_w}, {});
+    if (st != VQC_OK) return st;
     Launch L;
     st = plan_launch(p, 1, batch, L);
     if (st != VQC_OK) return st;
@@ -1043,6 +1059,8 @@ vqc_status vqc_probabilities(const vqc_plan* plan, int32_t batch, const void* x,
         if (batch == 0) return VQC_OK;
         const HostPlan& p = plan->hp;
         if (!probs_out) return fail(VQC_ERR_INVALID_ARG, "probs_out is NULL");
+        st = check_out_ptrs(p, {probs_out}, {});
+        if (st != VQC_OK) return st;
         const bool dbl = p.dtype == VQC_C128;
         const size_t rs = dbl ? 8 : 4;
         const size_t fws = vqc_workspace_bytes(plan, batch, 0);
@@ -1085,6 +1103,8 @@ vqc_status vqc_forward(const vqc_plan* plan, int32_t batch, const void* x, const
         st = check_ptrs(p, x, w, psi0, nullptr);
         if (st != VQC_OK) return st;
         if (!expz_out) return fail(VQC_ERR_INVALID_ARG, "expz_out is NULL");
+        st = check_out_ptrs(p, {expz_out}, {state_out});
+        if (st != VQC_OK) return st;
         cudaStream_t s = static_cast<cudaStream_t>(stream);
         if (use_cluster(p, 0)) {
             if (p.dtype == VQC_C64)
@@ -1125,6 +1145,8 @@ vqc_status vqc_backward(const vqc_plan* plan, int32_t batch, const void* x, cons
         st = check_ptrs(p, x, w, psi0, psi_final);
         if (st != VQC_OK) return st;
         if (!grad_expz) return fail(VQC_ERR_INVALID_ARG, "grad_expz is NULL");
+        st = check_out_ptrs(p, {grad_expz, grad_x, grad_w}, {});
+        if (st != VQC_OK) return st;
         if (use_hbm(p, 1, batch)) {
             if (p.dtype == VQC_C64)
                 return run_hbm_backward<float>(p, batch, x, w, psi0, psi_final, grad_expz, grad_x,
@@ -1159,6 +1181,8 @@ vqc_status vqc_forward_backward(const vqc_plan* plan, int32_t batch, const void*
         if (st != VQC_OK) return st;
         if (!grad_expz) return fail(VQC_ERR_INVALID_ARG, "grad_expz is NULL");
         if (!expz_out) return fail(VQC_ERR_INVALID_ARG, "expz_out is NULL");
+        st = check_out_ptrs(p, {expz_out, grad_expz, grad_x, grad_w}, {});
+        if (st != VQC_OK) return st;
         if (!use_cluster(p, 0) && !use_hbm(p, 0, batch) && !use_hbm(p, 1, batch)) {
             // one launch: the backward kernel sweeps forward itself (the state stays in
             // shared memory), writes E, then sweeps back

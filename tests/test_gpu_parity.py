@@ -486,3 +486,42 @@ def test_sync_check_after_every_kernel_kind(monkeypatch):
     assert c2.info(2)["fwd_path"] == 2
     c2.forward(x2, w2)                                      # cluster forward
     B.vqc_sync_check(torch.cuda.current_stream().cuda_stream)
+
+
+def test_argument_errors_before_any_launch():
+    """Every argument check of the device calls fails before anything is
+    launched: NULL / misaligned pointers, negative batch, short or misaligned
+    workspace, NULL plan.  The stream stays clean (vqc_sync_check)."""
+    w_ = wl.config(2, batch=8)[0]
+    c = C(w_.spec, "c64")
+    s = torch.cuda.current_stream().cuda_stream
+    x, w, gE = dev(w_.x, "c64"), dev(w_.w, "c64"), dev(w_.gE, "c64")
+    E = torch.empty(8, w_.spec.n, device="cuda")
+    st = torch.empty(8, 1 << w_.spec.n, dtype=torch.complex64, device="cuda")
+    dx, dw = torch.empty_like(x), torch.empty_like(w)
+    ws, wsb = c.workspace(8, 1, torch.cuda.current_stream())
+    ws3, ws3b = c.workspace(8, 3, torch.cuda.current_stream())
+
+    def P(t, off=0):
+        return t.data_ptr() + off
+
+    fwd = lambda **k: B.vqc_forward(k.get("plan", c.plan), k.get("b", 8), k.get("x", P(x)), P(w), None,   # noqa: E731
+                                    k.get("E", P(E)), k.get("st"), None, 0, s)
+    bwd = lambda **k: B.vqc_backward(c.plan, 8, P(x), P(w), None, k.get("psi", P(st)), k.get("g", P(gE)),   # noqa: E731
+                                     k.get("dx", P(dx)), P(dw), k.get("ws", P(ws)), k.get("wsb", wsb), s)
+    fb = lambda **k: B.vqc_forward_backward(c.plan, 8, P(x), P(w), None, k.get("g", P(gE)),   # noqa: E731
+                                            k.get("E", P(E)), P(dx), k.get("dw", P(dw)),
+                                            P(ws3) if ws3 is not None else None, ws3b, s)
+    cases = [
+        (lambda: fwd(plan=None), 1), (lambda: fwd(b=-1), 1), (lambda: fwd(x=None), 1),
+        (lambda: fwd(E=None), 1), (lambda: fwd(x=P(x, 2)), 1), (lambda: fwd(E=P(E, 2)), 1),
+        (lambda: fwd(st=P(st, 4)), 1),
+        (lambda: bwd(g=None), 1), (lambda: bwd(dx=P(dx, 2)), 1), (lambda: bwd(psi=P(st, 4)), 1),
+        (lambda: bwd(wsb=16), 8), (lambda: bwd(ws=P(ws, 16), wsb=wsb - 16), 8), (lambda: bwd(ws=None), 8),
+        (lambda: fb(E=None), 1), (lambda: fb(g=None), 1), (lambda: fb(dw=P(dw, 2)), 1),
+    ]
+    for i, (call, code) in enumerate(cases):
+        with pytest.raises(B.VQCError) as e:
+            call()
+        assert e.value.status == code, (i, str(e.value))
+    B.vqc_sync_check(s)
