@@ -705,6 +705,9 @@ vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx,
             K = std::min(hbm_k(mode, dtype), m - 1);
         }
         if (K != hbm_k(mode, dtype)) continue;   // pass kernels exist for this K only
+        // the backward passes recompute the final state with the forward passes
+        // when the caller gives none: no backward schedule without a forward one
+        if (mode == 1 && !find_hbm_schedule(p, 0)) continue;
         Schedule s;
         s.mode = mode;
         s.K = K;

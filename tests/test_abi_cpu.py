@@ -217,6 +217,17 @@ def test_hbm_schedules_small_tiles(monkeypatch, seed, n, G):
                 assert np.allclose(dw, dw_ref, atol=1e-10)
 
 
+@pytest.mark.parametrize("n", range(2, 14))
+def test_hbm_backward_schedule_implies_forward(n):
+    # the HBM backward recomputes the final state with the forward passes when
+    # none is given, so a plan never holds the backward passes alone
+    w_, _ = wl.small_random(520 + n, n, 4 * n, batch=1, dtype="c128")
+    for dtype in (0, 1):
+        pl = Plan(B.vqc_plan_export(compile_spec(w_.spec, dtype)))
+        modes = {s["mode"] for s in pl.scheds if s["path"] == 1}
+        assert 1 not in modes or 0 in modes, (n, dtype, modes)
+
+
 def test_config5_hbm_schedule_structure():
     w_ = wl.config(5, batch=1)[0]
     for dtype in (0, 1):

@@ -5,7 +5,8 @@
   small slice against the oracle and, at full size, as the sum over two halves;
 * small circuits forced onto the HBM path with 6-qubit tiles (many passes,
   tile-outer controls and phases), against the oracle, with and without psi0
-  and the saved final state, ragged batches;
+  and the saved final state, ragged batches; the smallest circuits with the
+  path forced (recomputing backward and the one-call forward+backward);
 * cross-path agreement: the 12-qubit workload on the resident and HBM paths;
 * the largest plan (24 qubits): forward against the oracle, backward against
   central differences of the complex128 forward;
@@ -87,6 +88,32 @@ def test_forced_hbm_small_tiles(monkeypatch, seed, n, G, dtype):
     assert maxerr(dx, dx_ref) <= tol["grad"] and maxerr(dw, dw_ref) <= tol["grad"]
     dx, dw = run_bwd(c, w_, psi0, psi_final=devc(st, dtype))
     assert maxerr(dx, dx_ref) <= tol["grad"] and maxerr(dw, dw_ref) <= tol["grad"]
+
+
+@pytest.mark.parametrize("dtype,n", [("c64", 6), ("c128", 5), ("c64", 7)])
+def test_forced_hbm_smallest_circuits(monkeypatch, dtype, n):
+    # at these sizes the backward's tile fits a pass kernel but the forward's
+    # does not: the compiler then keeps both on the resident path, and the
+    # recomputing backward and the one-call forward+backward still run
+    monkeypatch.setenv("VQC_FORCE_PATH", "hbm")
+    w_, psi0 = wl.small_random(640 + n, n, 60, batch=5, dtype=dtype, with_psi0=True)
+    c = C(w_.spec, dtype)
+    info = c.info(w_.batch)
+    assert (info["bwd_path"] == 1) <= (info["fwd_path"] == 1)
+    tol = TOL[dtype]
+    E_ref = orc.forward(w_.spec, w_.x, w_.w, psi0=psi0)
+    dx_ref, dw_ref = orc.backward(w_.spec, w_.x, w_.w, w_.gE, psi0=psi0)
+    dx, dw = run_bwd(c, w_, psi0)
+    assert maxerr(dx, dx_ref) <= tol["grad"] and maxerr(dw, dw_ref) <= tol["grad"]
+    x = dev(w_.x, dtype) if w_.spec.num_x else None
+    w = dev(w_.w, dtype) if w_.spec.num_w else None
+    E, dx, dw = c.forward_backward(x, w, dev(w_.gE, dtype), psi0=devc(psi0, dtype))
+    torch.cuda.synchronize()
+    assert maxerr(E.cpu().numpy(), E_ref) <= tol["E"]
+    if dx is not None:
+        assert maxerr(dx.cpu().numpy(), dx_ref) <= tol["grad"]
+    if dw is not None:
+        assert maxerr(dw.cpu().numpy(), dw_ref) <= tol["grad"]
 
 
 def test_forced_hbm_ragged_batches(monkeypatch):
