@@ -329,6 +329,10 @@ def run_ours(args, rank, world, local_rank):
                 if len(parts) >= 4 and not line.startswith("#") and parts[0] == w_.name.split("_rank")[0] \
                         and parts[1] == "bwd" and parts[2] == info_digest():
                     traffic = float(parts[3])
+    # measured FMA rates (outside the timed region): packed FP32 for complex64
+    # sweeps, FP64 for complex128 ones
+    fma = {"fp32_tflops": B.vqc_fma_peak(0), "fp64_tflops": B.vqc_fma_peak(1),
+           "kernel": "independent FMA chains over every SM (vqc_fma_peak), best of 5 launches"}
     out = {
         "metric": METRIC,
         "value": value,
@@ -372,7 +376,9 @@ def run_ours(args, rank, world, local_rank):
                       % (pk.get("sm_max_mhz", SM_MAX_MHZ), pk_kind)),
                      ("bytes_per_call" if hbm_path else "flops_per_launch"): bwd_flops,
                      "launch_ms": bwd_avg_s * 1e3,
-                     "fwd_frac": ach_fwd / peak},
+                     "fwd_frac": ach_fwd / peak,
+                     "frac_of_measured_fma": None if hbm_path else ach_bwd / fma["fp32_tflops"]},
+        "fma_measured": fma,
         "e2e": {"value": e2e_value, "unit": "circuit evals/s (fwd+adjoint bwd, host buffers)",
                 "call": "Circuit.prepare_host -> vqc_evaluate_host (pageable numpy in/out; %s)" % (
                     "kernels access the host arrays in place over NVLink-C2C"
@@ -394,7 +400,7 @@ def run_ours(args, rank, world, local_rank):
             "kind": "oracle, batch-parallel threads",
             "sample": "%d rows of the workload (cycled), fwd+bwd, %.1f s" % (pdone, pdt)}
     if args.extra:
-        out["configs"] = extra_configs(torch, Circuit, B)
+        out["configs"] = extra_configs(torch, Circuit, B, fma)
     if args.ablation:
         out["ablation"] = ablation(torch, Circuit, w_)
     if args.regime:
@@ -529,25 +535,27 @@ def regime_map(torch, Circuit, qubits=(4, 8, 12, 15, 16, 18, 20), batches=(1, 8,
     return pts
 
 
-def extra_configs(torch, Circuit, B):
+def extra_configs(torch, Circuit, B, fma=None):
     """Forward and fwd+bwd evaluations/s and roofline fractions of the other
     workloads (device time, L2 flushed before each timed call)."""
     from paper_2607_11985_gb300 import workloads as wl
     pk, _ = peaks()
     fp32 = fp32_peak_tflops(pk.get("sm_max_mhz", SM_MAX_MHZ))
     hbm = pk.get("hbm_gbs", 6800.0)
+    fp64 = fma["fp64_tflops"] if fma else None
     res = {}
     flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
     # (name, config, dtype, batch): the 8-qubit circuit also at a large batch, where
     # the sweep is throughput-bound rather than latency-bound
     cases = [("cfg1", 1, None, None), ("cfg2_B65536", 2, None, 65536), ("cfg3", 3, None, None),
-             ("cfg4", 4, None, None), ("cfg5_c64", 5, "c64", None), ("cfg5_c128", 5, "c128", None)]
+             ("cfg3_c128", 3, "c128", None), ("cfg4", 4, None, None), ("cfg5_c64", 5, "c64", None),
+             ("cfg5_c128", 5, "c128", None)]
     for key, k, dt, bsz in cases:
         try:
             ws_ = wl.config(k, dtype=dt, batch=bsz)
             tot_f = tot_b = 0.0
             evals = 0
-            work_f = work_b = 0.0
+            work_f = work_b = flop_f = flop_b = 0.0
             path = None
             for w_ in ws_:
                 real = torch.float32 if w_.dtype == "c64" else torch.float64
@@ -578,24 +586,27 @@ def extra_configs(torch, Circuit, B):
                 if path == "hbm-tiled":
                     work_f += n_rep * w_.batch * inf["fwd_hbm_bytes_per_eval"]
                     work_b += n_rep * w_.batch * inf["bwd_hbm_bytes_per_eval"] if w_.backward else 0
-                else:
-                    work_f += n_rep * w_.batch * inf["fwd_flops_per_eval"]
-                    work_b += n_rep * w_.batch * inf["bwd_flops_per_eval"] if w_.backward else 0
+                flop_f += n_rep * w_.batch * inf["fwd_flops_per_eval"]
+                flop_b += n_rep * w_.batch * inf["bwd_flops_per_eval"] if w_.backward else 0
                 del c
             r = {"path": path, "circuits": len(ws_), "batch": ws_[0].batch,
                  "qubits": sorted({w_.spec.n for w_ in ws_}), "dtype": ws_[0].dtype,
                  "fwd_evals_per_s": evals / tot_f,
-                 "fwd_bwd_evals_per_s": (evals / (tot_f + tot_b)) if work_b else None}
+                 "fwd_bwd_evals_per_s": (evals / (tot_f + tot_b)) if flop_b else None}
             if path == "hbm-tiled":
                 r["fwd_gbs"] = work_f / tot_f / 1e9
                 r["bwd_gbs"] = work_b / tot_b / 1e9 if work_b else None
                 r["fwd_frac_hbm"] = r["fwd_gbs"] / hbm
                 r["bwd_frac_hbm"] = r["bwd_gbs"] / hbm if work_b else None
-            else:
-                r["fwd_tflops"] = work_f / tot_f / 1e12
-                r["bwd_tflops"] = work_b / tot_b / 1e12 if work_b else None
+            # algorithmic flop rates against the arithmetic ceiling of the state type
+            r["fwd_tflops"] = flop_f / tot_f / 1e12
+            r["bwd_tflops"] = flop_b / tot_b / 1e12 if flop_b else None
+            if r["dtype"] == "c64":
                 r["fwd_frac_fp32"] = r["fwd_tflops"] / fp32
-                r["bwd_frac_fp32"] = r["bwd_tflops"] / fp32 if work_b else None
+                r["bwd_frac_fp32"] = r["bwd_tflops"] / fp32 if flop_b else None
+            elif fp64:
+                r["fwd_frac_fp64_measured"] = r["fwd_tflops"] / fp64
+                r["bwd_frac_fp64_measured"] = r["bwd_tflops"] / fp64 if flop_b else None
             res[key] = r
         except Exception as e:   # report, do not hide
             res[key] = {"error": str(e)[:200]}

@@ -303,6 +303,17 @@ vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, const void* x,
  * set VQC_HOST_DIRECT=0), else 0 (staged copies). */
 int32_t vqc_host_direct(int32_t device);
 
+/* The fused multiply-add rate of the current device for the arithmetic of
+ * `dtype`'s sweeps (VQC_C64: packed FP32 pairs; VQC_C128: FP64), in TFLOP/s
+ * (an FMA counts as two flops), measured: a kernel of independent FMA chains
+ * over every SM, calibrated to launches of about 5 ms, best of five timed
+ * launches.  This is the arithmetic ceiling against which the sweep kernels'
+ * algorithmic flop rates are reported (roofline of the resident path, Sec. 3
+ * complexity O(B * G * 2^n)).  Blocking; runs on a private stream; takes
+ * about 50 ms.  Errors: VQC_ERR_INVALID_ARG (NULL out, bad dtype),
+ * VQC_ERR_CUDA. */
+vqc_status vqc_fma_peak(vqc_dtype dtype, double* tflops_out);
+
 /* Plan statistics (paths, stage counts, algorithmic flop and byte counts per
  * evaluation) for a batch of `batch` samples. */
 vqc_status vqc_plan_info(const vqc_plan* plan, int32_t batch, vqc_plan_stats* out);

@@ -80,6 +80,7 @@ SIGNATURES = [
     ("vqc_compile_qasm", _I, [ctypes.c_char_p, _I, _I, _I, ctypes.POINTER(_P)]),
     ("vqc_evaluate_host", _I, [_P, _I, _P, _P, _P, _P, _P, _P, _P]),
     ("vqc_host_direct", _I, [_I]),
+    ("vqc_fma_peak", _I, [_I, ctypes.POINTER(ctypes.c_double)]),
     ("vqc_forward_backward", _I, [_P, _I, _P, _P, _P, _P, _P, _P, _P, _P, _S, _P]),
 ]
 
@@ -194,6 +195,13 @@ def vqc_evaluate_host(plan, batch, x, w, grad_expz, expz_out, grad_x, grad_w, st
 
 def vqc_host_direct(device):
     return int(lib().vqc_host_direct(device))
+
+
+def vqc_fma_peak(dtype):
+    """Measured FMA rate (TFLOP/s) of the current device for dtype's arithmetic."""
+    out = ctypes.c_double(0.0)
+    _check(lib().vqc_fma_peak(dtype, ctypes.byref(out)))
+    return out.value
 
 
 def vqc_plan_info(plan, batch):
