@@ -548,8 +548,8 @@ def extra_configs(torch, Circuit, B, fma=None):
     # (name, config, dtype, batch): the 8-qubit circuit also at a large batch, where
     # the sweep is throughput-bound rather than latency-bound
     cases = [("cfg1", 1, None, None), ("cfg2_B65536", 2, None, 65536), ("cfg3", 3, None, None),
-             ("cfg3_c128", 3, "c128", None), ("cfg4", 4, None, None), ("cfg5_c64", 5, "c64", None),
-             ("cfg5_c128", 5, "c128", None)]
+             ("cfg3_c128", 3, "c128", None), ("cfg3_c128df", 3, "c128df", None), ("cfg4", 4, None, None),
+             ("cfg5_c64", 5, "c64", None), ("cfg5_c128", 5, "c128", None), ("cfg5_c128df", 5, "c128df", None)]
     for key, k, dt, bsz in cases:
         try:
             ws_ = wl.config(k, dtype=dt, batch=bsz)
@@ -605,8 +605,15 @@ def extra_configs(torch, Circuit, B, fma=None):
                 r["fwd_frac_fp32"] = r["fwd_tflops"] / fp32
                 r["bwd_frac_fp32"] = r["bwd_tflops"] / fp32 if flop_b else None
             elif fp64:
+                # complex128 flops against the native FP64 ceiling (double-float
+                # runs on the FP32 units, so it can exceed 1)
                 r["fwd_frac_fp64_measured"] = r["fwd_tflops"] / fp64
                 r["bwd_frac_fp64_measured"] = r["bwd_tflops"] / fp64 if flop_b else None
+            if r["dtype"] == "c128df" and key.replace("df", "") in res and "fwd_evals_per_s" in res[key.replace("df", "")]:
+                ref = res[key.replace("df", "")]
+                r["fwd_speedup_vs_fp64"] = r["fwd_evals_per_s"] / ref["fwd_evals_per_s"]
+                if flop_b and ref.get("fwd_bwd_evals_per_s"):
+                    r["fwd_bwd_speedup_vs_fp64"] = r["fwd_bwd_evals_per_s"] / ref["fwd_bwd_evals_per_s"]
             res[key] = r
         except Exception as e:   # report, do not hide
             res[key] = {"error": str(e)[:200]}

@@ -23,9 +23,9 @@
  *
  * Conventions.  Qubit q is bit q of the amplitude index (little endian).  A
  * gate list is in time order.  States are interleaved (re, im) pairs: float2
- * for VQC_C64, double2 for VQC_C128; arrays are row-major and sample-major.
- * Real arrays (x, w, E, gradients) are float for VQC_C64 and double for
- * VQC_C128.  Gate matrices: RX/RY/RZ(t) = exp(-i t P / 2); U3 is
+ * for VQC_C64, double2 for VQC_C128 and VQC_C128_DF; arrays are row-major
+ * and sample-major.  Real arrays (x, w, E, gradients) are float for VQC_C64
+ * and double for VQC_C128 and VQC_C128_DF.  Gate matrices: RX/RY/RZ(t) = exp(-i t P / 2); U3 is
  * [[c, -e^{i l} s], [e^{i p} s, e^{i(p+l)} c]] with c, s = cos, sin(t/2);
  * CRZ(t) = |0><0|_q0 (x) I + |1><1|_q0 (x) RZ_q1(t); RZZ(t) = exp(-i t Z Z / 2);
  * CX/CRZ control is q0, target q1.
@@ -69,7 +69,16 @@ typedef enum {
     VQC_ERR_UNSUPPORTED = 10       /* valid request this build cannot run (e.g. too large) */
 } vqc_status;
 
-typedef enum { VQC_C64 = 0, VQC_C128 = 1 } vqc_dtype;
+/* VQC_C128_DF: complex128 in memory (every array, layout, workspace size and
+ * plan schedule exactly as VQC_C128) with the kernels computing in double-float
+ * arithmetic on the FP32 units: each real is an unevaluated sum of two floats
+ * (about 48 significant bits; error-free sums and FMA products, Dekker 1971),
+ * split when read and rejoined when written.  Results agree with VQC_C128 to
+ * about 1e-13 (the complex128 parity bound, 1e-10, holds); on parts whose FP64
+ * rate is a small fraction of the FP32 rate (GB300: about 1/75) it is the
+ * faster way to complex128 accuracy.  vqc_plan_export gives the same bytes as
+ * for VQC_C128 (the arithmetic is chosen at launch, not in the plan). */
+typedef enum { VQC_C64 = 0, VQC_C128 = 1, VQC_C128_DF = 2 } vqc_dtype;
 
 /* The 16-gate set.  Angles per gate: RX/RY/RZ/CRZ/RZZ one (theta),
  * U3 three (theta, phi, lambda), the rest none. */
@@ -304,7 +313,8 @@ vqc_status vqc_evaluate_host(const vqc_plan* plan, int32_t batch, const void* x,
 int32_t vqc_host_direct(int32_t device);
 
 /* The fused multiply-add rate of the current device for the arithmetic of
- * `dtype`'s sweeps (VQC_C64: packed FP32 pairs; VQC_C128: FP64), in TFLOP/s
+ * `dtype`'s sweeps (VQC_C64 and VQC_C128_DF: packed FP32 pairs, the FP32
+ * lanes double-float also runs on; VQC_C128: FP64), in TFLOP/s
  * (an FMA counts as two flops), measured: a kernel of independent FMA chains
  * over every SM, calibrated to launches of about 5 ms, best of five timed
  * launches.  This is the arithmetic ceiling against which the sweep kernels'

@@ -20,7 +20,7 @@ GATE_CODE = {g: i for i, g in enumerate(GATE_OPS)}
 NUM_ANGLES = {"RX": 1, "RY": 1, "RZ": 1, "CRZ": 1, "RZZ": 1, "U3": 3}
 PKIND = {"c": 1, "x": 2, "w": 3}
 
-VQC_C64, VQC_C128 = 0, 1
+VQC_C64, VQC_C128, VQC_C128_DF = 0, 1, 2
 STATUS = {0: "VQC_OK", 1: "VQC_ERR_INVALID_ARG", 2: "VQC_ERR_UNSUPPORTED_GATE",
           3: "VQC_ERR_QUBIT_RANGE", 4: "VQC_ERR_TOO_MANY_QUBITS", 5: "VQC_ERR_PARAM_RANGE",
           6: "VQC_ERR_OUT_OF_MEMORY", 7: "VQC_ERR_CUDA", 8: "VQC_ERR_WORKSPACE",

@@ -13,7 +13,9 @@ import torch
 from . import binding as B
 
 _DT = {"c64": (B.VQC_C64, torch.float32, torch.complex64),
-       "c128": (B.VQC_C128, torch.float64, torch.complex128)}
+       "c128": (B.VQC_C128, torch.float64, torch.complex128),
+       # complex128 storage, double-float arithmetic on the FP32 units
+       "c128df": (B.VQC_C128_DF, torch.float64, torch.complex128)}
 
 
 def _ptr(t):
@@ -25,7 +27,7 @@ class Circuit:
 
     def __init__(self, spec, dtype: str = "c64"):
         if dtype not in _DT:
-            raise ValueError("dtype must be 'c64' or 'c128'")
+            raise ValueError("dtype must be 'c64', 'c128' or 'c128df'")
         self.spec = spec
         self.n, self.num_x, self.num_w = int(spec.n), int(spec.num_x), int(spec.num_w)
         self.dtype = dtype
@@ -40,7 +42,7 @@ class Circuit:
         """Compile an OpenQASM 2 program (gate set, parameter references x[i] /
         w[j]: see vqc_compile_qasm in include/vqc.h)."""
         if dtype not in _DT:
-            raise ValueError("dtype must be 'c64' or 'c128'")
+            raise ValueError("dtype must be 'c64', 'c128' or 'c128df'")
         self = cls.__new__(cls)
         self.spec = None
         self.dtype = dtype

@@ -81,7 +81,9 @@ vqc_status device_info(int dev, DevInfo& out) {
 }
 
 // mode 2: the backward with the forward sweep and E inside (vqc_forward_backward)
-const void* kernel_ptr(int dtype, int mode, int K, bool full) {
+const void* kernel_ptr(int dtype, bool dfloat, int mode, int K, bool full) {
+    if (dfloat)
+        return mode == 2 ? sweep_ptr_dd_fused(K, full) : mode == 0 ? sweep_ptr_dd_fwd(K, full) : sweep_ptr_dd_bwd(K, full);
     if (mode == 2) return dtype == VQC_C64 ? sweep_ptr_f32_fused(K, full) : sweep_ptr_f64_fused(K, full);
     if (full) {
         if (dtype == VQC_C64) return mode == 0 ? sweep_ptr_f32_fwd(K) : sweep_ptr_f32_bwd(K);
@@ -228,7 +230,7 @@ vqc_status plan_launch_uncached(const HostPlan& p, int launch_mode, int B, Launc
     L.smem = off;
     if (L.smem > (size_t)di.smem_optin)
         return fail(VQC_ERR_UNSUPPORTED, "shared-memory layout exceeds the per-CTA limit");
-    L.fn = kernel_ptr(p.dtype, launch_mode, L.K, L.T >= 32);
+    L.fn = kernel_ptr(p.dtype, p.dfloat, launch_mode, L.K, L.T >= 32);
     if (!L.fn) return fail(VQC_ERR_UNSUPPORTED, "kernel not instantiated for this K");
     VQC_CUDA(cudaFuncSetAttribute(L.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem));
     int per_sm = 0;
@@ -335,6 +337,19 @@ vqc_status upload(HostPlan& p) {
     // the kernels index lists by slot order, which is entry order within each list
     std::vector<double> cm_d = p.cmat, ca_d = p.cang;
     std::vector<float> cm_f(cm_d.begin(), cm_d.end()), ca_f(ca_d.begin(), ca_d.end());
+    if (p.dfloat) {
+        // double-float kernels read constants as (hi, lo) float pairs in the 8
+        // bytes a double takes: hi = the double rounded to float, lo = the rest
+        auto split = [](std::vector<double>& v) {
+            for (double& d : v) {
+                const float hi = (float)d, lo = (float)(d - (double)hi);
+                std::memcpy(reinterpret_cast<char*>(&d), &hi, 4);
+                std::memcpy(reinterpret_cast<char*>(&d) + 4, &lo, 4);
+            }
+        };
+        split(cm_d);
+        split(ca_d);
+    }
     p.dev_entries = put(p.entries.data(), p.entries.size() * sizeof(DEntry));
     p.dev_ps_list = put(ps_list.data(), ps_list.size() * 4);
     p.dev_sh_list = put(sh_list.data(), sh_list.size() * 4);
@@ -482,7 +497,7 @@ vqc_status plan_cluster(const HostPlan& p, int B, Launch& L) {
     L.smem = off;
     if (L.smem > (size_t)di.smem_optin)
         return fail(VQC_ERR_UNSUPPORTED, "cluster slice does not fit in shared memory");
-    L.fn = cluster_ptr(dbl);
+    L.fn = p.dfloat ? cluster_ptr_dd() : cluster_ptr(dbl);
     VQC_CUDA(cudaFuncSetAttribute(L.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem));
     cudaLaunchConfig_t cfg{};
     cudaLaunchAttribute attr[1];
@@ -624,7 +639,7 @@ vqc_status plan_hbm_uncached(const HostPlan& p, int mode, int B, PassGeo& L) {
     L.plan_smem = off + plan_bytes <= (size_t)di.smem_optin && plan_bytes <= 48 * 1024;
     L.sm_plan = L.plan_smem ? take(plan_bytes) : 0;
     L.smem = off;
-    L.fn = pass_ptr(dbl, mode, L.K, L.T >= 32);
+    L.fn = p.dfloat ? pass_ptr_dd(mode, L.K, L.T >= 32) : pass_ptr(dbl, mode, L.K, L.T >= 32);
     if (!L.fn) return fail(VQC_ERR_UNSUPPORTED, "pass kernel not instantiated for this K");
     VQC_CUDA(cudaFuncSetAttribute(L.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem));
     int per_sm = 0;
@@ -970,14 +985,19 @@ vqc_status vqc_compile(const vqc_gate* gates, int32_t num_gates, int32_t num_qub
         *out_plan = nullptr;
         if (num_gates < 0 || num_x < 0 || num_w < 0 || (num_gates > 0 && !gates))
             return fail(VQC_ERR_INVALID_ARG, "negative count or NULL gate list");
-        if (dtype != VQC_C64 && dtype != VQC_C128) return fail(VQC_ERR_INVALID_ARG, "bad dtype");
+        if (dtype != VQC_C64 && dtype != VQC_C128 && dtype != VQC_C128_DF)
+            return fail(VQC_ERR_INVALID_ARG, "bad dtype");
         if (num_qubits < 1 || num_qubits > VQC_MAX_QUBITS)
             return fail(VQC_ERR_TOO_MANY_QUBITS, "num_qubits must be in 1.." +
                                                      std::to_string(VQC_MAX_QUBITS));
         std::unique_ptr<vqc_plan> p(new vqc_plan());
         std::string err;
-        vqc_status st = compile_host(gates, num_gates, num_qubits, num_x, num_w, dtype, p->hp, err);
+        // VQC_C128_DF plans are complex128 plans (same layouts and schedules)
+        // whose kernels compute in double-float
+        const vqc_dtype store = dtype == VQC_C128_DF ? VQC_C128 : dtype;
+        vqc_status st = compile_host(gates, num_gates, num_qubits, num_x, num_w, store, p->hp, err);
         if (st != VQC_OK) return fail(st, err);
+        p->hp.dfloat = dtype == VQC_C128_DF;
         // Upload now when a CUDA device is present; a host-only plan (no device
         // in this process) still serves vqc_plan_export and vqc_plan_info, and
         // is uploaded by the first launching call.
@@ -1209,7 +1229,7 @@ vqc_status vqc_plan_info(const vqc_plan* plan, int32_t batch, vqc_plan_stats* ou
     out->num_qubits = p.n;
     out->num_x = p.num_x;
     out->num_w = p.num_w;
-    out->dtype = p.dtype;
+    out->dtype = p.dfloat ? VQC_C128_DF : p.dtype;
     out->num_gates_in = p.num_gates_in;
     out->num_ops = (int32_t)p.ops.size();
     out->num_runs = p.n_runs;

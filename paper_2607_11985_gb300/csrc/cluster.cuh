@@ -59,6 +59,20 @@ __device__ __forceinline__ void dsm_store(uint32_t a, float v) {
 __device__ __forceinline__ void dsm_store(uint32_t a, double v) {
     asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(a), "d"(v) : "memory");
 }
+// double-float: (hi, lo) pairs, complex values as (re.hi, re.lo, im.hi, im.lo)
+__device__ __forceinline__ dd2 dsm_load(uint32_t a, dd2*) {
+    dd2 v;
+    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x.hi), "=f"(v.x.lo), "=f"(v.y.hi), "=f"(v.y.lo) : "r"(a) : "memory");
+    return v;
+}
+__device__ __forceinline__ void dsm_store(uint32_t a, dd2 v) {
+    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(a), "f"(v.x.hi), "f"(v.x.lo),
+                 "f"(v.y.hi), "f"(v.y.lo) : "memory");
+}
+__device__ __forceinline__ void dsm_store(uint32_t a, dd v) {
+    asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(a), "f"(v.hi), "f"(v.lo) : "memory");
+}
 
 // Cluster address of slot s of the distributed state (psi_sa: this CTA's local
 // shared address of its slice; slices are 2^slice amplitudes).
@@ -87,7 +101,7 @@ __device__ __forceinline__ void cl_block_store(const C2<R> (&a)[1 << K], uint32_
 // carve-up (sm_psi holds this CTA's slice of 2^(n - cl) amplitudes, sm_red the
 // per-warp <Z> sums, sm_ecl rank 0's [2^cl][n] gather of per-CTA sums), cl.
 template <typename R, int K>
-__global__ void __launch_bounds__(512) cluster_fwd_kernel(const __grid_constant__ KArgs<R> A) {
+__global__ void __launch_bounds__(512) cluster_fwd_kernel(const __grid_constant__ KArgs<St<R>> A) {
     // every CTA of every cluster takes the same branch, before any cluster barrier
     uint32_t nrank;
     asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(nrank));
@@ -136,8 +150,11 @@ __global__ void __launch_bounds__(512) cluster_fwd_kernel(const __grid_constant_
     }
     grid_dep_wait();
     grid_dep_launch();
-    for (int i = threadIdx.x; i < A.Pw; i += nthr) async_elem<R>(w_sm + i, A.w + i);
+    for (int i = threadIdx.x; i < A.Pw; i += nthr)
+        async_elem<St<R>>(reinterpret_cast<St<R>*>(w_sm) + i, A.w + i);
     async_wait();
+    if constexpr (!std::is_same<St<R>, R>::value)   // each thread splits the values it copied
+        for (int i = threadIdx.x; i < A.Pw; i += nthr) w_sm[i] = R(reinterpret_cast<const St<R>*>(w_sm)[i]);
     PlanPtrs P;
     P.ops = rebase(A.ops, A.plan, A.sched_off, sms);
     P.stages = rebase(A.stages, A.plan, A.sched_off, sms);
@@ -152,18 +169,19 @@ __global__ void __launch_bounds__(512) cluster_fwd_kernel(const __grid_constant_
     __syncthreads();
     for (int i = threadIdx.x; i < A.n_sh; i += nthr) {
         const DEntry e = P.entries[vqc_ld(&P.sh_list[i])];
-        eval_entry<R>(e, P.consts, nullptr, w_sm, Pcang, Pcmat, sh_tab + EntryWords<R>::value * e.slot);
+        eval_entry<R>(e, P.consts, static_cast<const R*>(nullptr), w_sm, Pcang, Pcmat,
+                      sh_tab + EntryWords<R>::value * e.slot);
     }
 
     const int ns = A.nstages;
     for (int b = cid; b < A.nunits; b += ncl) {
         // this sample's x row, per-sample table and (given psi0) this CTA's slice
-        for (int i = threadIdx.x; i < A.Px; i += nthr) xrow[i] = A.x[(size_t)b * A.Px + i];
+        for (int i = threadIdx.x; i < A.Px; i += nthr) xrow[i] = as_r<R>(A.x[(size_t)b * A.Px + i]);
         if (A.psi0) {
-            const C2<R>* gs = A.psi0 + ((size_t)b << n) + ((size_t)rank << slice);
+            const SC2<R>* gs = A.psi0 + ((size_t)b << n) + ((size_t)rank << slice);
             const uint32_t u0 = rank << slice;
             for (uint32_t v = threadIdx.x; v < (1u << slice); v += nthr)
-                psi[swz(u0 + v, G) & ((1u << slice) - 1u)] = gs[v];
+                psi[swz(u0 + v, G) & ((1u << slice) - 1u)] = c2_in<R>(gs[v]);
         }
         __syncthreads();
         for (int i = threadIdx.x; i < A.n_ps; i += nthr) {
@@ -231,13 +249,13 @@ __global__ void __launch_bounds__(512) cluster_fwd_kernel(const __grid_constant_
             for (int j = threadIdx.x; j < n; j += nthr) {
                 R e = 0;
                 for (int r = 0; r < (1 << CL); ++r) e += ecl[r * n + j];
-                A.E[(size_t)b * n + j] = e;
+                A.E[(size_t)b * n + j] = as_out<St<R>>(e);
             }
         if (A.state_out) {   // this CTA's slice, logical order
-            C2<R>* go = A.state_out + ((size_t)b << n) + ((size_t)rank << slice);
+            SC2<R>* go = A.state_out + ((size_t)b << n) + ((size_t)rank << slice);
             const uint32_t u0 = rank << slice;
             for (uint32_t v = threadIdx.x; v < (1u << slice); v += nthr)
-                go[v] = psi[swz(u0 + v, G) & ((1u << slice) - 1u)];
+                go[v] = c2_out<R>(psi[swz(u0 + v, G) & ((1u << slice) - 1u)]);
         }
         cluster_sync();   // slices and rank 0's gather area are reused by the next sample
     }

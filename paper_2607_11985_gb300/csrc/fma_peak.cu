@@ -63,7 +63,9 @@ __global__ void __launch_bounds__(kThreads) fma_f64_kernel(int iters, double b, 
 extern "C" vqc_status vqc_fma_peak(vqc_dtype dtype, double* tflops_out) {
     using vqc::set_error;
     if (!tflops_out) return set_error(VQC_ERR_INVALID_ARG, "tflops_out is NULL");
-    if (dtype != VQC_C64 && dtype != VQC_C128) return set_error(VQC_ERR_INVALID_ARG, "bad dtype");
+    if (dtype != VQC_C64 && dtype != VQC_C128 && dtype != VQC_C128_DF)
+        return set_error(VQC_ERR_INVALID_ARG, "bad dtype");
+    if (dtype == VQC_C128_DF) dtype = VQC_C64;   // double-float runs on the FP32 units
     *tflops_out = 0.0;
     int dev = 0, sms = 0, per_sm = 0;
     cudaError_t e = cudaGetDevice(&dev);

@@ -15,6 +15,12 @@ const void* sweep_ptr_f64_fwd_small(int K);
 const void* sweep_ptr_f64_bwd_small(int K);
 const void* sweep_ptr_f32_fused(int K, bool full);   // backward that also writes E
 const void* sweep_ptr_f64_fused(int K, bool full);
+// double-float arithmetic on complex128 storage (VQC_C128_DF plans)
+const void* sweep_ptr_dd_fwd(int K, bool full);
+const void* sweep_ptr_dd_bwd(int K, bool full);
+const void* sweep_ptr_dd_fused(int K, bool full);
+const void* pass_ptr_dd(int mode, int K, bool full);
+const void* cluster_ptr_dd();
 
 // HBM-tiled pass kernels (K fixed per type and mode) and partial reductions.
 const void* pass_ptr(bool dbl, int mode, int K, bool full);   // full: tile groups >= 32 threads

@@ -16,6 +16,7 @@
 
 namespace vqc {
 
+// R here is the storage real type (pass kernels take PArgs<St<R>>).
 template <typename R>
 struct PArgs {
     const DOp* ops;
@@ -78,6 +79,12 @@ template <> struct Vec16<double> {
     __device__ __forceinline__ void ld(const double2* p) { a[0] = __ldcs(p); }
     __device__ __forceinline__ void st(double2* p) const { __stcs(p, a[0]); }
 };
+// double-float kernels: complex128 in HBM, split on the way in, rejoined on the way out
+template <> struct Vec16<dd> {
+    dd2 a[1];
+    __device__ __forceinline__ void ld(const double2* p) { a[0] = c2_in<dd>(__ldcs(p)); }
+    __device__ __forceinline__ void st(double2* p) const { __stcs(p, c2_out<dd>(a[0])); }
+};
 
 // Tile copies between HBM and shared memory.  A CTA-thread t moves vectors
 // v = t + k*T; the tile-local index of v splits into disjoint bit fields of t
@@ -85,7 +92,7 @@ template <> struct Vec16<double> {
 // linear in those fields, so each is a per-thread part XOR a per-k part
 // (tabulated once per pass in shared memory: koff[k] = (global, slot)).
 template <typename R>
-__device__ __forceinline__ void tile_gather(C2<R>* sm, const C2<R>* gs, uint32_t gt, uint32_t st,
+__device__ __forceinline__ void tile_gather(C2<R>* sm, const SC2<R>* gs, uint32_t gt, uint32_t st,
                                             const uint2* koff, int nk, int T, int t) {
     constexpr int APV = 16 / sizeof(C2<R>);
     constexpr int U = 8;
@@ -111,7 +118,7 @@ __device__ __forceinline__ void tile_gather(C2<R>* sm, const C2<R>* gs, uint32_t
 }
 
 template <typename R>
-__device__ __forceinline__ void tile_scatter(const C2<R>* sm, C2<R>* gs, uint32_t gt, uint32_t st,
+__device__ __forceinline__ void tile_scatter(const C2<R>* sm, SC2<R>* gs, uint32_t gt, uint32_t st,
                                              const uint2* koff, int nk, int T, int t) {
     constexpr int APV = 16 / sizeof(C2<R>);
     for (int k = 0; k < nk; ++k) {
@@ -126,7 +133,7 @@ __device__ __forceinline__ void tile_scatter(const C2<R>* sm, C2<R>* gs, uint32_
 // FULL: tile groups span whole warps (2^(m-K) >= 32 threads; every production
 // tile), see sweep_kernel.
 template <typename R, int K, int MODE, bool FULL>
-__global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PArgs<R> A) {
+__global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PArgs<St<R>> A) {
     if (geometry_bad(blockDim.x != (unsigned)(A.S << A.tbits) || A.tbits != A.m - K ||
                          A.stage_end <= A.stage_begin,
                      A.err, kErrPassGeometry))
@@ -193,7 +200,8 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
 
     for (int i = threadIdx.x; i < A.sh_count; i += nthr) {
         const DEntry e = P_entries[vqc_ld(&P_pass_entries[A.sh_begin + i])];
-        eval_entry<R>(e, P_consts, nullptr, A.w, P_cang, P_cmat, sh_tab + EntryWords<R>::value * i);
+        eval_entry<R>(e, P_consts, static_cast<const St<R>*>(nullptr), A.w, P_cang, P_cmat,
+                      sh_tab + EntryWords<R>::value * i);
     }
     __syncthreads();
 
@@ -259,7 +267,7 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
                     for (int j = q.t; j < n; j += q.T) {
                         R e = 0;
                         for (int k = 0; k < q.wg; ++k) e += red[k * n + j];
-                        A.E_part[tile_id * n + j] = e;
+                        A.E_part[tile_id * n + j] = as_out<St<R>>(e);
                     }
             }
             __syncthreads();
@@ -307,7 +315,7 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
             const int bb = (int)(tt / A.ntiles);
             const DAcc ac = P_accs[vqc_ld(&P_pass_accs[A.acc_begin + k])];
             acc_terms<R>(ac, P_entries[ac.entry], acc_all + ((size_t)gg * A.acc_count + k) * q.wg * 8,
-                         q.wg, P_consts, A.x ? A.x + (size_t)bb * A.Px : nullptr, A.w, P_cang,
+                         q.wg, P_consts, A.x ? A.x + (size_t)bb * A.Px : static_cast<const St<R>*>(nullptr), A.w, P_cang,
                          P_cmat, A.terms + tt * A.n_terms);
         }
         __syncthreads();

@@ -24,6 +24,9 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <type_traits>
+
+#include "dd.cuh"
 #include "plan.h"
 
 namespace vqc {
@@ -31,7 +34,38 @@ namespace vqc {
 template <typename R> struct V2;
 template <> struct V2<float> { using t = float2; };
 template <> struct V2<double> { using t = double2; };
+template <> struct V2<dd> { using t = dd2; };
 template <typename R> using C2 = typename V2<R>::t;
+
+// The real type arrays have outside a kernel (caller memory, workspaces,
+// partials) for the kernel's arithmetic type R: R itself, except double for
+// double-float kernels, which split values on reading and rejoin them on
+// writing.  For float and double every conversion below is the identity.
+template <typename R> struct StoreOf { using t = R; };
+template <> struct StoreOf<dd> { using t = double; };
+template <typename R> using St = typename StoreOf<R>::t;
+template <typename R> using SC2 = C2<St<R>>;
+
+template <typename R, typename T>
+__device__ __forceinline__ R as_r(T v) {
+    if constexpr (std::is_same<T, R>::value) return v;
+    else return R(v);
+}
+template <typename O, typename R>
+__device__ __forceinline__ O as_out(R v) {
+    if constexpr (std::is_same<O, R>::value) return v;
+    else return v.to_double();
+}
+template <typename R>
+__device__ __forceinline__ C2<R> c2_in(SC2<R> v) {
+    if constexpr (std::is_same<St<R>, R>::value) return v;
+    else { C2<R> r; r.x = R(v.x); r.y = R(v.y); return r; }
+}
+template <typename R>
+__device__ __forceinline__ SC2<R> c2_out(C2<R> v) {
+    if constexpr (std::is_same<St<R>, R>::value) return v;
+    else { SC2<R> r; r.x = v.x.to_double(); r.y = v.y.to_double(); return r; }
+}
 
 template <typename R>
 __device__ __forceinline__ C2<R> cm(R x, R y) { C2<R> r; r.x = x; r.y = y; return r; }
@@ -157,8 +191,16 @@ __device__ __forceinline__ void sc(float t, float* s, float* c) {
     *c = ((q + 1) & 2) ? -cv : cv;
 }
 __device__ __forceinline__ void sc(double t, double* s, double* c) { sincos(t, s, c); }
+// double-float: the library routine in double (once per angle), then split
+__device__ __forceinline__ void sc(dd t, dd* s, dd* c) {
+    double sd, cd;
+    sincos(t.to_double(), &sd, &cd);
+    *s = dd(sd);
+    *c = dd(cd);
+}
 
 // ---------------------------------------------------------------- kernel args
+// R here is the storage real type (kernels take KArgs<St<R>>).
 template <typename R>
 struct KArgs {
     // plan
@@ -244,17 +286,17 @@ __device__ __forceinline__ void store_matrix(const M2<R>& m, R* out) {
         out[4] = m.c.x; out[5] = m.c.y; out[6] = m.d.x; out[7] = m.d.y;
     }
 }
-template <typename R>
-__device__ __forceinline__ R angle_of(uint8_t src, int32_t idx, const R* xb, const R* w,
+template <typename R, typename XI, typename WI>
+__device__ __forceinline__ R angle_of(uint8_t src, int32_t idx, const XI* xb, const WI* w,
                                       const R* cang) {
-    if (src == SRC_X) return xb[idx];
-    if (src == SRC_W) return w[idx];
+    if (src == SRC_X) return as_r<R>(xb[idx]);
+    if (src == SRC_W) return as_r<R>(w[idx]);
     return cang[idx];
 }
 
 // Matrix of one constituent of a run.
-template <typename R>
-__device__ __forceinline__ M2<R> constituent(const DConst& c, const R* xb, const R* w, const R* cang,
+template <typename R, typename XI, typename WI>
+__device__ __forceinline__ M2<R> constituent(const DConst& c, const XI* xb, const WI* w, const R* cang,
                              const R* cmat) {
     M2<R> u;
     if (c.kind == CK_CONST) {
@@ -278,8 +320,8 @@ __device__ __forceinline__ M2<R> constituent(const DConst& c, const R* xb, const
 }
 
 // Evaluate one table entry (8 reals) for sample row xb.
-template <typename R>
-__device__ __forceinline__ void eval_entry(const DEntry& e, const DConst* consts, const R* xb, const R* w,
+template <typename R, typename XI, typename WI>
+__device__ __forceinline__ void eval_entry(const DEntry& e, const DConst* consts, const XI* xb, const WI* w,
                            const R* cang, const R* cmat, R* out) {
     if (e.phase) {
         const DConst c = consts[e.cfirst];
@@ -828,6 +870,12 @@ template <> __device__ __forceinline__ M2<double> load_m2v<double>(const double*
     m.a = q[0]; m.b = q[1]; m.c = q[2]; m.d = q[3];
     return m;
 }
+template <> __device__ __forceinline__ M2<dd> load_m2v<dd>(const dd* p) {
+    const dd2* q = reinterpret_cast<const dd2*>(p);
+    M2<dd> m;
+    m.a = q[0]; m.b = q[1]; m.c = q[2]; m.d = q[3];
+    return m;
+}
 
 __device__ __forceinline__ bool physbit(uint32_t pb, int ref) {
     return ((pb >> (ref - kRefPhys)) & 1u) != 0;
@@ -981,8 +1029,8 @@ __device__ __forceinline__ void run_ops(const DOp* ops, int ob, int oe, uint32_t
 
 // lam = O psi on the block, O = sum_j gE_j Z_j (diagonal): the sign of Z_j comes
 // from local bit j of r for active qubits and from the block base pb otherwise.
-template <typename R, int K>
-__device__ __forceinline__ void lambda_init(const DStage* sp, uint32_t pb, const R* gb, int n,
+template <typename R, int K, typename GI>
+__device__ __forceinline__ void lambda_init(const DStage* sp, uint32_t pb, const GI* gb, int n,
                                             const C2<R> (&a)[1 << K], C2<R> (&l)[1 << K]) {
     R ge_loc[K];
     R cst = 0;
@@ -991,10 +1039,10 @@ __device__ __forceinline__ void lambda_init(const DStage* sp, uint32_t pb, const
     for (int j = 0; j < K; ++j) {
         const int aq = vqc_ld(&sp->active[j]);
         actmask |= 1u << aq;
-        ge_loc[j] = gb[aq];
+        ge_loc[j] = as_r<R>(gb[aq]);
     }
     for (int j = 0; j < n; ++j)
-        if (!((actmask >> j) & 1)) cst += ((pb >> j) & 1u) ? -gb[j] : gb[j];
+        if (!((actmask >> j) & 1)) cst += ((pb >> j) & 1u) ? -as_r<R>(gb[j]) : as_r<R>(gb[j]);
 #pragma unroll
     for (int r = 0; r < (1 << K); ++r) {
         R o = cst;
@@ -1106,14 +1154,14 @@ __device__ __forceinline__ void expz_partials(const DStage* sp, uint32_t pb,
 // Gradient terms of one accumulator slot (summed over the wg per-warp
 // partials at ap): a phase op's scalar, or Im Tr(W_j P_j W_j^dag rho) for each
 // parametrised constituent j of a run.  Writes out[term].
-template <typename R>
+template <typename R, typename XI, typename WI, typename O>
 __device__ void acc_terms(const DAcc& ac, const DEntry& e, const R* ap, int wg,
-                          const DConst* consts, const R* xg, const R* w, const R* cang,
-                          const R* cmat, R* out) {
+                          const DConst* consts, const XI* xg, const WI* w, const R* cang,
+                          const R* cmat, O* out) {
     if (ac.kind == 1) {
         R sum = 0;
         for (int k2 = 0; k2 < wg; ++k2) sum += ap[k2 * 8];
-        out[consts[e.cfirst].term] = sum;
+        out[consts[e.cfirst].term] = as_out<O>(sum);
         return;
     }
     R vx = 0, vy = 0, vz = 0;
@@ -1130,7 +1178,7 @@ __device__ void acc_terms(const DAcc& ac, const DEntry& e, const R* ap, int wg,
     // P's axis; a scalar phase leaves it; a constant 2x2 goes through its matrix.
     for (int c = e.ccount - 1; c >= 0; --c) {
         const DConst cn = consts[e.cfirst + c];
-        if (cn.term >= 0) out[cn.term] = cn.kind == CK_RX ? vx : cn.kind == CK_RY ? vy : vz;
+        if (cn.term >= 0) out[cn.term] = as_out<O>(cn.kind == CK_RX ? vx : cn.kind == CK_RY ? vy : vz);
         if (c == 0) break;
         if (cn.kind == CK_RX || cn.kind == CK_RY || cn.kind == CK_RZ) {
             R sn, co;
@@ -1181,7 +1229,7 @@ __device__ __forceinline__ bool geometry_bad(bool bad, unsigned* err, unsigned c
 enum : unsigned { kErrSweepGeometry = 1u, kErrPassGeometry = 2u, kErrClusterGeometry = 4u };
 
 template <typename R, int K, int MODE, bool FULL, bool FUSED>
-__global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArgs<R> A) {
+__global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArgs<St<R>> A) {
     if (geometry_bad(blockDim.x != (unsigned)(A.S * A.tpg) || A.bpt * A.tpg != (1 << A.tbits) ||
                          A.tbits != A.n - K || A.nstages < 1,
                      A.err, kErrSweepGeometry))
@@ -1218,24 +1266,43 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
     C2<R>* lam = lam_all + (size_t)q.g * dim;
 
     // initial (forward) or final (backward) state source; null: |0...0>
-    const C2<R>* src = MODE == 1 ? A.psi_final : A.psi0;
+    const SC2<R>* src = MODE == 1 ? A.psi_final : A.psi0;
     if (MODE == 1 && !src) src = A.psi0;
     const bool from_global = src != nullptr;
 
     // One unit's inputs to shared memory, asynchronously: x (and, backward,
     // gE) rows of its samples and each sample's initial / final state
     // (coalesced reads, swizzled slots).
+    // (Double-float kernels copy the stored doubles as they are and split them
+    // in place afterwards, unit_to_dd: both types are 8 bytes.)
+    St<R>* xg_st = reinterpret_cast<St<R>*>(xg_all);
+    SC2<R>* psi_st = reinterpret_cast<SC2<R>*>(psi);
     auto stage_unit = [&](int unit) {
         for (int i = threadIdx.x; i < A.S * xgw; i += nthr) {
             const int gg = i / xgw, c = i % xgw;
             const int bb = min(unit * A.S + gg, A.B - 1);
-            if (c < A.Px) async_elem<R>(xg_all + i, A.x + (size_t)bb * A.Px + c);
-            else if (MODE == 1) async_elem<R>(xg_all + i, A.gE + (size_t)bb * n + (c - A.Px));
+            if (c < A.Px) async_elem<St<R>>(xg_st + i, A.x + (size_t)bb * A.Px + c);
+            else if (MODE == 1) async_elem<St<R>>(xg_st + i, A.gE + (size_t)bb * n + (c - A.Px));
         }
         if (from_global) {
             const int b = min(unit * A.S + q.g, A.B - 1);
-            const C2<R>* gs = src + (size_t)b * dim;
-            for (int u = q.t; u < dim; u += q.T) async_elem<C2<R>>(psi + (swz(u, G) ^ q.h), gs + u);
+            const SC2<R>* gs = src + (size_t)b * dim;
+            for (int u = q.t; u < dim; u += q.T) async_elem<SC2<R>>(psi_st + (swz(u, G) ^ q.h), gs + u);
+        }
+    };
+    // after async_wait(): stored doubles -> dd in place, each by the thread that
+    // issued its copy (its own copies are visible to it); a barrier follows
+    auto unit_to_dd = [&]() {
+        if constexpr (!std::is_same<St<R>, R>::value) {
+            for (int i = threadIdx.x; i < A.S * xgw; i += nthr) {
+                const int c = i % xgw;
+                if (c < A.Px || MODE == 1) xg_all[i] = R(xg_st[i]);
+            }
+            if (from_global)
+                for (int u = q.t; u < dim; u += q.T) {
+                    const int sl = swz(u, G) ^ q.h;
+                    psi[sl] = c2_in<R>(psi_st[sl]);
+                }
         }
     };
 
@@ -1253,7 +1320,8 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
     }
     grid_dep_wait();
     grid_dep_launch();
-    for (int i = threadIdx.x; i < A.Pw; i += nthr) async_elem<R>(w_sm + i, A.w + i);
+    for (int i = threadIdx.x; i < A.Pw; i += nthr)
+        async_elem<St<R>>(reinterpret_cast<St<R>*>(w_sm) + i, A.w + i);
     if ((int)blockIdx.x < A.nunits) stage_unit(blockIdx.x);
     if (MODE == 1)
         for (int i = threadIdx.x; i < A.Pw; i += nthr) dw_cta[i] = 0;
@@ -1274,6 +1342,10 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
     const R* Pcmat = reinterpret_cast<const R*>(P.cmat);
     const R* Pcang = reinterpret_cast<const R*>(P.cang);
     async_wait();
+    if constexpr (!std::is_same<St<R>, R>::value) {
+        for (int i = threadIdx.x; i < A.Pw; i += nthr) w_sm[i] = R(reinterpret_cast<const St<R>*>(w_sm)[i]);
+        if ((int)blockIdx.x < A.nunits) unit_to_dd();
+    }
     __syncthreads();
 
     // shared table (w and constants) once per CTA, on the CTA's last threads
@@ -1281,7 +1353,8 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
     for (int i = nthr - 1 - threadIdx.x; i < A.n_sh; i += nthr) {
         const int id = vqc_ld(&P.sh_list[i]);
         const DEntry e = P.entries[id];
-        eval_entry<R>(e, P.consts, nullptr, w_sm, Pcang, Pcmat, sh_tab + EntryWords<R>::value * e.slot);
+        eval_entry<R>(e, P.consts, static_cast<const R*>(nullptr), w_sm, Pcang, Pcmat,
+                      sh_tab + EntryWords<R>::value * e.slot);
     }
 
     R* ps_tab = ps_all + (size_t)q.g * A.n_ps * EntryWords<R>::value;
@@ -1295,6 +1368,7 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
         if (unit != (int)blockIdx.x) {
             stage_unit(unit);
             async_wait();
+            if constexpr (!std::is_same<St<R>, R>::value) unit_to_dd();
             __syncthreads();
         }
         const R* xrow = xg_all + (size_t)q.g * xgw;
@@ -1372,7 +1446,7 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                     const int low = n <= 8 ? 3 : 1;   // lane bits below the scatter bits
                     if ((lane & low) == 0 && eidx < n) {
                         if (q.wg == 1) {
-                            if (valid) A.E[(size_t)b * n + eidx] = eacc;
+                            if (valid) A.E[(size_t)b * n + eidx] = as_out<St<R>>(eacc);
                         } else {
                             red[warp_in_group * n + eidx] = eacc;
                         }
@@ -1391,12 +1465,12 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                         for (int j = q.t; j < n; j += q.T) {
                             R e = 0;
                             for (int k = 0; k < q.wg; ++k) e += red[k * n + j];
-                            A.E[(size_t)b * n + j] = e;
+                            A.E[(size_t)b * n + j] = as_out<St<R>>(e);
                         }
                     }
                     if (A.state_out) {
-                        C2<R>* go = A.state_out + (size_t)b * dim;
-                        for (int u = q.t; u < dim; u += q.T) go[u] = psi[swz(u, G) ^ q.h];
+                        SC2<R>* go = A.state_out + (size_t)b * dim;
+                        for (int u = q.t; u < dim; u += q.T) go[u] = c2_out<R>(psi[swz(u, G) ^ q.h]);
                     }
                 }
             }
@@ -1410,7 +1484,7 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                 for (int j = q.t; j < n; j += q.T) {
                     R e = 0;
                     for (int k = 0; k < q.wg; ++k) e += red[k * n + j];
-                    A.E[(size_t)b * n + j] = e;
+                    A.E[(size_t)b * n + j] = as_out<St<R>>(e);
                 }
         }
 
@@ -1462,7 +1536,7 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
                 const int k0 = vqc_ld(&P.xocc_ptr[p]), k1 = vqc_ld(&P.xocc_ptr[p + 1]);
                 R sum = 0;
                 for (int k = k0; k < k1; ++k) sum += tm[vqc_ld(&P.xocc[k])];
-                A.dx[(size_t)bb * A.Px + p] = sum;
+                A.dx[(size_t)bb * A.Px + p] = as_out<St<R>>(sum);
             }
         }
         const int nvalid = min(A.S, A.B - unit * A.S);
@@ -1487,7 +1561,7 @@ __global__ void __launch_bounds__(512) sweep_kernel(const __grid_constant__ KArg
     if (MODE == 1 && A.Pw > 0 && A.dw) {
         // per-CTA partial of dw; reduce_cols sums the partials in CTA order
         for (int p = threadIdx.x; p < A.Pw; p += nthr)
-            A.dw_part[(size_t)blockIdx.x * A.Pw + p] = dw_cta[p];
+            A.dw_part[(size_t)blockIdx.x * A.Pw + p] = as_out<St<R>>(dw_cta[p]);
     }
 }
 

@@ -54,7 +54,7 @@ class Workload:
     x: np.ndarray          # [B, num_x] float64 holding dtype-rounded values
     w: np.ndarray          # [num_w]
     gE: np.ndarray         # [B, n]
-    dtype: str             # "c64" or "c128"
+    dtype: str             # "c64", "c128" or "c128df" (complex128 storage)
     seed: int
     backward: bool = True
 

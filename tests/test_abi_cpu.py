@@ -98,6 +98,21 @@ def test_export_deterministic_and_info():
         B.vqc_free(p2)
 
 
+def test_double_float_plan_is_a_complex128_plan():
+    # VQC_C128_DF changes only the kernels' arithmetic: the plan bytes (layouts,
+    # schedules, tables) equal the complex128 plan's; plan_info reports the dtype
+    for k in (2, 3, 5):
+        spec = wl.config(k)[0].spec
+        p1, p2 = compile_spec(spec, B.VQC_C128), compile_spec(spec, B.VQC_C128_DF)
+        assert B.vqc_plan_export(p1) == B.vqc_plan_export(p2)
+        i1, i2 = B.vqc_plan_info(p1, 512), B.vqc_plan_info(p2, 512)
+        assert i1["dtype"] == B.VQC_C128 and i2["dtype"] == B.VQC_C128_DF
+        assert {k: v for k, v in i1.items() if k != "dtype"} == {k: v for k, v in i2.items() if k != "dtype"}
+        B.vqc_free(p1)
+        B.vqc_free(p2)
+    assert status_of(wl.config(1)[0].spec, dtype=3) == 1   # VQC_ERR_INVALID_ARG
+
+
 def slot_of(st, K, t, r, sig, tau):
     sl = 0
     for i in range(int(st["nthreadbits"])):

@@ -34,7 +34,7 @@ def cuda_ready():
     torch.cuda.set_device(0)
 
 
-@pytest.mark.parametrize("dtype", ["c64", "c128"])
+@pytest.mark.parametrize("dtype", ["c64", "c128", "c128df"])
 def test_config5_full_batch(dtype):
     w_ = wl.config(5, dtype=dtype)[0]
     c = C(w_.spec, dtype)
@@ -67,7 +67,7 @@ def test_config5_full_batch(dtype):
 SMALL = [(601, 8, 160), (602, 9, 200), (603, 10, 240), (604, 11, 200)]
 
 
-@pytest.mark.parametrize("dtype", ["c64", "c128"])
+@pytest.mark.parametrize("dtype", ["c64", "c128", "c128df"])
 @pytest.mark.parametrize("seed,n,G", SMALL)
 def test_forced_hbm_small_tiles(monkeypatch, seed, n, G, dtype):
     monkeypatch.setenv("VQC_HBM_TILE_QUBITS", "6")
@@ -90,7 +90,7 @@ def test_forced_hbm_small_tiles(monkeypatch, seed, n, G, dtype):
     assert maxerr(dx, dx_ref) <= tol["grad"] and maxerr(dw, dw_ref) <= tol["grad"]
 
 
-@pytest.mark.parametrize("dtype,n", [("c64", 6), ("c128", 5), ("c64", 7)])
+@pytest.mark.parametrize("dtype,n", [("c64", 6), ("c128", 5), ("c64", 7), ("c128df", 5)])
 def test_forced_hbm_smallest_circuits(monkeypatch, dtype, n):
     # at these sizes the backward's tile fits a pass kernel but the forward's
     # does not: the compiler then keeps both on the resident path, and the
@@ -204,7 +204,8 @@ def test_max_qubits_24():
     assert abs(fd_x - float(np.sum(dx * u))) <= 1e-6 * max(1.0, abs(fd_x))
 
 
-@pytest.mark.parametrize("dtype,n", [("c64", 15), ("c64", 16), ("c128", 14), ("c128", 15), ("c128", 16)])
+@pytest.mark.parametrize("dtype,n", [("c64", 15), ("c64", 16), ("c128", 14), ("c128", 15), ("c128", 16),
+                                     ("c128df", 14), ("c128df", 16)])
 def test_cluster_forward(monkeypatch, dtype, n):
     """Forward with the state spread over a thread-block cluster (2, 4 or 8 CTAs):
     E and the final states against the oracle, from |0...0> and from a given
@@ -223,7 +224,7 @@ def test_cluster_forward(monkeypatch, dtype, n):
     w_ = wl.Workload("cluster_n%d" % n, spec, B, x, w, gE, dtype, 1500 + n)
     c = C(spec, dtype)
     # default: the cluster for 2-CTA clusters (complex64 15 qubits, complex128 14), else the passes
-    two_cta = (dtype, n) in (("c64", 15), ("c128", 14))
+    two_cta = (dtype, n) in (("c64", 15), ("c128", 14), ("c128df", 14))
     assert c.info(B)["fwd_path"] == (2 if two_cta else 1)
     monkeypatch.setenv("VQC_FORCE_PATH", "cluster")
     assert c.info(B)["fwd_path"] == 2
@@ -240,7 +241,7 @@ def test_cluster_forward(monkeypatch, dtype, n):
         assert maxerr(E3, E) <= tol["E"] and maxerr(st3, st) <= tol["state"]
 
 
-@pytest.mark.parametrize("dtype", ["c64", "c128"])
+@pytest.mark.parametrize("dtype", ["c64", "c128", "c128df"])
 def test_config5_cluster_forward(monkeypatch, dtype):
     """The 16-qubit, 8-layer batch through the cluster forward: sampled rows
     against the oracle."""

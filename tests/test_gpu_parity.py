@@ -19,7 +19,8 @@ from paper_2607_11985_gb300 import binding as B  # noqa: E402
 
 pytestmark = pytest.mark.gpu
 
-TOL = {"c64": dict(E=1e-4, state=1e-4, grad=5e-4), "c128": dict(E=1e-10, state=1e-10, grad=1e-10)}
+TOL = {"c64": dict(E=1e-4, state=1e-4, grad=5e-4), "c128": dict(E=1e-10, state=1e-10, grad=1e-10),
+       "c128df": dict(E=1e-10, state=1e-10, grad=1e-10)}   # complex128 storage, double-float arithmetic
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -81,7 +82,7 @@ SMALL = [(201, 1, 10), (202, 2, 40), (203, 3, 80), (204, 4, 120), (205, 5, 160),
          (207, 7, 200), (208, 8, 240), (209, 9, 200), (210, 10, 160)]
 
 
-@pytest.mark.parametrize("dtype", ["c64", "c128"])
+@pytest.mark.parametrize("dtype", ["c64", "c128", "c128df"])
 @pytest.mark.parametrize("seed,n,G", SMALL)
 def test_random_forward_and_gradients(seed, n, G, dtype):
     w_, psi0 = wl.small_random(seed, n, G, batch=37, dtype=dtype, with_psi0=(seed % 2 == 0))
@@ -320,7 +321,7 @@ def test_largest_resident_forward_n14():
 
 
 # ------------------------------------------------------------------ fused forward + backward
-@pytest.mark.parametrize("case", ["cfg1", "cfg2", "cfg3_rows", "rand_c128_psi0", "hbm16"])
+@pytest.mark.parametrize("case", ["cfg1", "cfg2", "cfg3_rows", "rand_c128_psi0", "rand_c128df_psi0", "hbm16"])
 def test_forward_backward_fused(case, monkeypatch):
     """vqc_forward_backward (one launch on the resident path: the backward kernel
     sweeps forward itself and writes E) against the oracle and against the
@@ -336,8 +337,8 @@ def test_forward_backward_fused(case, monkeypatch):
         full = wl.config(3)[0]
         idx = np.arange(40) * 97 % full.batch
         w_ = wl.Workload(full.name, full.spec, 40, full.x[idx], full.w, full.gE[idx], "c64", full.seed)
-    elif case == "rand_c128_psi0":
-        w_, psi0 = wl.small_random(777, 9, 180, batch=6, dtype="c128", with_psi0=True)
+    elif case in ("rand_c128_psi0", "rand_c128df_psi0"):
+        w_, psi0 = wl.small_random(777, 9, 180, batch=6, dtype=case[5:-5], with_psi0=True)
     else:
         spec = wl.layered(16, 1, ("RX", "RY", "RZ"), "CX")
         rng = np.random.default_rng(1616)
@@ -375,8 +376,31 @@ def test_forward_backward_fused(case, monkeypatch):
         assert maxerr(dw, dw_ref) <= tol["grad"]
 
 
+@pytest.mark.parametrize("case", ["cfg3_rows", "rand_psi0"])
+def test_double_float_agrees_with_fp64(case):
+    """complex128 with double-float arithmetic against native FP64 on the same
+    inputs: E, final states and gradients agree far inside the complex128
+    parity bound (48-bit double-float against 53-bit double)."""
+    if case == "cfg3_rows":
+        full = wl.config(3, dtype="c128")[0]
+        idx = np.arange(64) * 61 % full.batch
+        w_ = wl.Workload(full.name, full.spec, 64, full.x[idx], full.w, full.gE[idx], "c128", full.seed)
+        psi0 = None
+    else:
+        w_, psi0 = wl.small_random(778, 10, 220, batch=8, dtype="c128", with_psi0=True)
+    out = {}
+    for dt in ("c128", "c128df"):
+        c = C(w_.spec, dt)
+        E, st = run_fwd(c, w_, psi0)
+        dx, dw = run_bwd(c, w_, psi0)
+        out[dt] = (E, st, dx, dw)
+    for a, b in zip(out["c128"], out["c128df"]):
+        scale = max(1.0, float(np.abs(a).max())) if a.size else 1.0
+        assert maxerr(a, b) <= 1e-12 * scale
+
+
 # ------------------------------------------------------------------ degenerate circuits
-@pytest.mark.parametrize("dtype", ["c64", "c128"])
+@pytest.mark.parametrize("dtype", ["c64", "c128", "c128df"])
 @pytest.mark.parametrize("which", ["empty", "no_params", "one_long_run"])
 def test_degenerate_circuits(dtype, which):
     """An empty gate list (E = <Z> of psi0; the state passes through), a circuit

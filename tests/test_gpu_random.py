@@ -9,7 +9,9 @@ forward+backward on:
 * the default path choice;
 * the HBM-tiled passes with 6-qubit tiles (VQC_FORCE_PATH=hbm), from 7 qubits;
 * the resident sweep with the smallest register blocks (K = 1 below 3 qubits,
-  else 2), so the stage cuts differ from the default ones.
+  else 2), so the stage cuts differ from the default ones;
+* the same circuit in complex128 with double-float arithmetic (c128df) on the
+  default path.
 
 Every output is compared with the oracle element by element at the parity
 tolerances.
@@ -56,12 +58,15 @@ def cases():
         if n >= 7:
             out.append((i, "hbm"))
         out.append((i, "small_k"))
+        out.append((i, "df"))
     return out
 
 
 @pytest.mark.parametrize("i,mode", cases())
 def test_random_circuit(monkeypatch, i, mode):
     n, G, dtype, seed, batch, with_psi0 = draw(i)
+    if mode == "df":
+        dtype = "c128df"
     for k in ENV:
         monkeypatch.delenv(k, raising=False)
     if mode == "hbm":
