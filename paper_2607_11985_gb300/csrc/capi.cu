@@ -775,6 +775,11 @@ vqc_status run_hbm_forward(const HostPlan& p, int B, const void* x, const void* 
         const bool last = i == np - 1;
         a.dst_psi = (last && want_E && !state_out) ? nullptr : W;
         a.E_part = (last && want_E) ? E_part : nullptr;
+        // double-float: raw pairs between passes, complex128 in and out (a
+        // pass reads its whole tile before writing it, so W may change format
+        // in place)
+        a.src_raw = i > 0;
+        a.dst_raw = !last;
         void* args[] = {&a};
         VQC_CUDA(launch(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
     }
@@ -822,6 +827,8 @@ vqc_status run_hbm_backward(const HostPlan& p, int B, const void* x, const void*
             a.w = static_cast<const R*>(w);
             a.src_psi = i == 0 ? static_cast<const C*>(psi0) : Psi;
             a.dst_psi = Psi;
+            a.src_raw = i > 0;
+            a.dst_raw = 1;   // read only by the backward passes below
             void* args[] = {&a};
             VQC_CUDA(launch(Lf.fn, dim3(Lf.grid), dim3(Lf.block), args, Lf.smem, stream));
         }
@@ -840,6 +847,9 @@ vqc_status run_hbm_backward(const HostPlan& p, int B, const void* x, const void*
         a.src_lam = first ? nullptr : Lam;
         a.dst_psi = last ? nullptr : Psi;
         a.dst_lam = last ? nullptr : Lam;
+        a.src_raw = first ? psi_final == nullptr : 1;   // recomputed states are raw
+        a.lam_raw = 1;
+        a.dst_raw = 1;
         a.terms = terms;
         void* args[] = {&a};
         VQC_CUDA(launch(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));

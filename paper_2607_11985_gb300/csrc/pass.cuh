@@ -48,6 +48,10 @@ struct PArgs {
     int tab_off, tab_bytes, sched_off, sched_bytes, sm_plan, plan_smem;
     int sm_koff;                 // per-pass tile-copy offsets: [ceil(2^m / (APV * T))] uint2
     unsigned* err;               // the plan's error word (launch self-check)
+    // double-float kernels only: src_psi / src_lam / dst_psi and dst_lam hold
+    // raw (hi, lo) float pairs (workspace state passed between passes) rather
+    // than complex128 values (caller buffers); ignored by other kernels
+    int src_raw, lam_raw, dst_raw;
 };
 
 // Global amplitude index of tile-local index u (the low G tile bits are the
@@ -85,20 +89,36 @@ template <> struct Vec16<dd> {
     __device__ __forceinline__ void ld(const double2* p) { a[0] = c2_in<dd>(__ldcs(p)); }
     __device__ __forceinline__ void st(double2* p) const { __stcs(p, c2_out<dd>(a[0])); }
 };
+// raw (hi, lo) pairs in a workspace buffer between double-float passes: no
+// conversion (the conversions run on the FP64 units, a pass's slowest work)
+struct Vec16Raw {
+    dd2 a[1];
+    __device__ __forceinline__ void ld(const double2* p) {
+        const float4 v = __ldcs(reinterpret_cast<const float4*>(p));
+        a[0].x = dd(v.x, v.y);
+        a[0].y = dd(v.z, v.w);
+    }
+    __device__ __forceinline__ void st(double2* p) const {
+        __stcs(reinterpret_cast<float4*>(p), make_float4(a[0].x.hi, a[0].x.lo, a[0].y.hi, a[0].y.lo));
+    }
+};
+template <typename R, bool RAW> struct VecSel { using t = Vec16<R>; };
+template <> struct VecSel<dd, true> { using t = Vec16Raw; };
 
 // Tile copies between HBM and shared memory.  A CTA-thread t moves vectors
 // v = t + k*T; the tile-local index of v splits into disjoint bit fields of t
 // and of k, and both the index deposit into global qubits and the swizzle are
 // linear in those fields, so each is a per-thread part XOR a per-k part
 // (tabulated once per pass in shared memory: koff[k] = (global, slot)).
-template <typename R>
+template <typename R, bool RAW = false>
 __device__ __forceinline__ void tile_gather(C2<R>* sm, const SC2<R>* gs, uint32_t gt, uint32_t st,
                                             const uint2* koff, int nk, int T, int t) {
+    using V = typename VecSel<R, RAW>::t;
     constexpr int APV = 16 / sizeof(C2<R>);
     constexpr int U = 8;
     int k = 0;
     for (; k + U <= nk; k += U) {
-        Vec16<R> v[U];
+        V v[U];
 #pragma unroll
         for (int j = 0; j < U; ++j) v[j].ld(gs + (gt | koff[k + j].x));
 #pragma unroll
@@ -109,7 +129,7 @@ __device__ __forceinline__ void tile_gather(C2<R>* sm, const SC2<R>* gs, uint32_
         }
     }
     for (; k < nk; ++k) {
-        Vec16<R> v;
+        V v;
         v.ld(gs + (gt | koff[k].x));
         const uint32_t sl = st ^ koff[k].y;
 #pragma unroll
@@ -117,12 +137,13 @@ __device__ __forceinline__ void tile_gather(C2<R>* sm, const SC2<R>* gs, uint32_
     }
 }
 
-template <typename R>
+template <typename R, bool RAW = false>
 __device__ __forceinline__ void tile_scatter(const C2<R>* sm, SC2<R>* gs, uint32_t gt, uint32_t st,
                                              const uint2* koff, int nk, int T, int t) {
+    using V = typename VecSel<R, RAW>::t;
     constexpr int APV = 16 / sizeof(C2<R>);
     for (int k = 0; k < nk; ++k) {
-        Vec16<R> v;
+        V v;
         const uint32_t sl = st ^ koff[k].y;
 #pragma unroll
         for (int e = 0; e < APV; ++e) v.a[e] = sm[sl ^ e];
@@ -173,6 +194,7 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
 
     const int n = A.n, G = A.G, tdim = 1 << A.m;
     const long long total_tiles = (long long)A.B * A.ntiles;
+    constexpr bool DDK = !std::is_same<St<R>, R>::value;   // double-float kernel
     Geo q;
     q.T = 1 << A.tbits;
     q.lanes = q.T < 32 ? q.T : 32;
@@ -230,8 +252,14 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
         }
         const size_t sbase = (size_t)b << n;
         const uint32_t gt = tile_global(u_t, tile_base, A.tile_q, G);
-        if (A.src_psi) tile_gather<R>(psi, A.src_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
-        if (MODE == 1 && A.src_lam) tile_gather<R>(lam, A.src_lam + sbase, gt, st_t, koff, nk, q.T, q.t);
+        if (A.src_psi) {
+            if (DDK && A.src_raw) tile_gather<R, DDK>(psi, A.src_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
+            else tile_gather<R>(psi, A.src_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
+        }
+        if (MODE == 1 && A.src_lam) {
+            if (DDK && A.lam_raw) tile_gather<R, DDK>(lam, A.src_lam + sbase, gt, st_t, koff, nk, q.T, q.t);
+            else tile_gather<R>(lam, A.src_lam + sbase, gt, st_t, koff, nk, q.T, q.t);
+        }
         __syncthreads();
 
         C2<R> a[1 << K];
@@ -271,8 +299,10 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
                     }
             }
             __syncthreads();
-            if (A.dst_psi && valid)
-                tile_scatter<R>(psi, A.dst_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
+            if (A.dst_psi && valid) {
+                if (DDK && A.dst_raw) tile_scatter<R, DDK>(psi, A.dst_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
+                else tile_scatter<R>(psi, A.dst_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
+            }
             __syncthreads();
             continue;
         }
@@ -305,8 +335,13 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
         }
         __syncthreads();
         if (valid && A.dst_psi) {
-            tile_scatter<R>(psi, A.dst_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
-            tile_scatter<R>(lam, A.dst_lam + sbase, gt, st_t, koff, nk, q.T, q.t);
+            if (DDK && A.dst_raw) {
+                tile_scatter<R, DDK>(psi, A.dst_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
+                tile_scatter<R, DDK>(lam, A.dst_lam + sbase, gt, st_t, koff, nk, q.T, q.t);
+            } else {
+                tile_scatter<R>(psi, A.dst_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
+                tile_scatter<R>(lam, A.dst_lam + sbase, gt, st_t, koff, nk, q.T, q.t);
+            }
         }
         for (int i = threadIdx.x; i < A.S * A.acc_count; i += nthr) {
             const int gg = i / A.acc_count, k = i % A.acc_count;
