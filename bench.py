@@ -104,10 +104,16 @@ class ClockSampler:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
-def workload(cfg=2, rank=0, world=1):
+def workload(cfg=2, rank=0, world=1, dtype="c64"):
     """This rank's shard of the global batch (world x per-rank batch rows)."""
     from paper_2607_11985_gb300 import workloads as wl
-    return wl.config(cfg, rank=rank, world=world)[0]
+    return wl.config(cfg, dtype=dtype, rank=rank, world=world)[0]
+
+
+# state type -> (torch real, torch complex, numpy real, arithmetic label, state label)
+DTYPES = {"c64": ("float32", "complex64", np.float32, "f32", "complex64"),
+          "c128": ("float64", "complex128", np.float64, "f64", "complex128"),
+          "c128df": ("float64", "complex128", np.float64, "f32x2 (double-float)", "complex128")}
 
 
 # ------------------------------------------------------------------ CPU oracle baseline
@@ -165,17 +171,19 @@ def run_ours(args, rank, world, local_rank):
 
     __graft_entry__.build()
     torch.cuda.set_device(local_rank)
-    w_ = workload(args.config, rank, world)
+    w_ = workload(args.config, rank, world, args.dtype)
     Bt = w_.batch
-    c = Circuit(w_.spec, "c64")
+    c = Circuit(w_.spec, args.dtype)
     info = c.info(Bt)
     stream = torch.cuda.current_stream()
     sp = stream.cuda_stream
-    x = torch.tensor(w_.x, dtype=torch.float32, device="cuda")
-    w = torch.tensor(w_.w, dtype=torch.float32, device="cuda")
-    gE = torch.tensor(w_.gE, dtype=torch.float32, device="cuda")
-    E = torch.empty(Bt, w_.spec.n, dtype=torch.float32, device="cuda")
-    st = torch.empty(Bt, 1 << w_.spec.n, dtype=torch.complex64, device="cuda")
+    t_real, t_cplx, np_real, arith, state_kind = DTYPES[args.dtype]
+    t_real, t_cplx = getattr(torch, t_real), getattr(torch, t_cplx)
+    x = torch.tensor(w_.x, dtype=t_real, device="cuda")
+    w = torch.tensor(w_.w, dtype=t_real, device="cuda")
+    gE = torch.tensor(w_.gE, dtype=t_real, device="cuda")
+    E = torch.empty(Bt, w_.spec.n, dtype=t_real, device="cuda")
+    st = torch.empty(Bt, 1 << w_.spec.n, dtype=t_cplx, device="cuda")
     dx = torch.empty_like(x)
     dw = torch.empty_like(w)
     ws, wsb = c.workspace(Bt, 1, stream)
@@ -260,10 +268,10 @@ def run_ours(args, rank, world, local_rank):
 
     # ---- end to end through the C ABI with HOST buffers (vqc_evaluate_host):
     # every step copies x, w, gE in and E, dx, dw out (one packed copy each way)
-    xh = np.ascontiguousarray(w_.x, dtype=np.float32)
-    wh = np.ascontiguousarray(w_.w, dtype=np.float32)
-    gh = np.ascontiguousarray(w_.gE, dtype=np.float32)
-    Eh = np.empty((Bt, w_.spec.n), np.float32)
+    xh = np.ascontiguousarray(w_.x, dtype=np_real)
+    wh = np.ascontiguousarray(w_.w, dtype=np_real)
+    gh = np.ascontiguousarray(w_.gE, dtype=np_real)
+    Eh = np.empty((Bt, w_.spec.n), np_real)
     dxh = np.empty_like(xh)
     dwh = np.empty_like(wh)
     h2d = xh.nbytes + wh.nbytes + gh.nbytes
@@ -307,7 +315,12 @@ def run_ours(args, rank, world, local_rank):
     launches_per_step = launches_fwd + launches_bwd
     bwd_avg_s = statistics.mean(bwd_ms) / 1e3
     fwd_avg_s = statistics.mean(fwd_ms) / 1e3
-    if hbm_path:
+    # measured FMA rates (outside the timed region): packed FP32 for complex64
+    # sweeps, FP64 for complex128 ones
+    fma = {"fp32_tflops": B.vqc_fma_peak(0), "fp64_tflops": B.vqc_fma_peak(1),
+           "kernel": "independent FMA chains over every SM (vqc_fma_peak), best of 5 launches"}
+    rname = {"c64": "float", "c128": "double", "c128df": "dd"}[args.dtype]
+    if hbm_path and args.dtype == "c64":
         # state bytes the passes move through HBM (vqc_plan_info), against copy bandwidth
         peak = pk.get("hbm_gbs", 6800.0)
         bwd_flops = info["bwd_hbm_bytes_per_eval"] * Bt
@@ -315,7 +328,17 @@ def run_ours(args, rank, world, local_rank):
         ach_bwd = bwd_flops / bwd_avg_s / 1e9
         ach_fwd = fwd_flops / fwd_avg_s / 1e9
     else:
-        peak = fp32_peak_tflops(pk.get("sm_max_mhz", SM_MAX_MHZ))
+        if args.dtype == "c64":
+            peak = fp32_peak_tflops(pk.get("sm_max_mhz", SM_MAX_MHZ))
+            basis = ("FP32 FFMA: 152 SMs x 128 lanes x 2 x %.0f MHz (%s sm_max_mhz)"
+                     % (pk.get("sm_max_mhz", SM_MAX_MHZ), pk_kind))
+        elif args.dtype == "c128":
+            peak = fma["fp64_tflops"]
+            basis = "measured FP64 FMA rate (vqc_fma_peak); complex128 sweeps are FP64-bound on GB300"
+        else:
+            peak = fma["fp32_tflops"] / 15.0
+            basis = ("measured FP32 FMA rate / 15: a double-float FMA (2 flops) is 15 FP32 "
+                     "instructions on the FMA pipe")
         bwd_flops = info["bwd_flops_per_eval"] * Bt
         fwd_flops = info["fwd_flops_per_eval"] * Bt
         ach_bwd = bwd_flops / bwd_avg_s / 1e12
@@ -329,10 +352,7 @@ def run_ours(args, rank, world, local_rank):
                 if len(parts) >= 4 and not line.startswith("#") and parts[0] == w_.name.split("_rank")[0] \
                         and parts[1] == "bwd" and parts[2] == info_digest():
                     traffic = float(parts[3])
-    # measured FMA rates (outside the timed region): packed FP32 for complex64
-    # sweeps, FP64 for complex128 ones
-    fma = {"fp32_tflops": B.vqc_fma_peak(0), "fp64_tflops": B.vqc_fma_peak(1),
-           "kernel": "independent FMA chains over every SM (vqc_fma_peak), best of 5 launches"}
+    bytes_bound = hbm_path and args.dtype == "c64"
     out = {
         "metric": METRIC,
         "value": value,
@@ -344,9 +364,9 @@ def run_ours(args, rank, world, local_rank):
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "f32",   # arithmetic type; states are complex64 (config.state)
+        "dtype": arith,   # arithmetic type; the state type is config.state
         "data": "synthetic (seeded; RY(x) encoding + RX/RY/RZ layers + CZ ring)",
-        "config": {"workload": w_.name.split("_rank")[0], "qubits": w_.spec.n, "state": "complex64",
+        "config": {"workload": w_.name.split("_rank")[0], "qubits": w_.spec.n, "state": state_kind,
                    "batch_per_gpu": Bt,
                    "gates": len(w_.spec.gates), "num_x": w_.spec.num_x, "num_w": w_.spec.num_w,
                    "parallelism": "dp%d (batch-sharded replicas, dw all-reduce)" % world,
@@ -366,18 +386,17 @@ def run_ours(args, rank, world, local_rank):
                   "ms_per_step": statistics.mean(fused_ms),
                   "call": "vqc_forward_backward (gE known before the call, e.g. the mean-<Z> "
                           "objective; one launch)"},
-        "roofline": {"kernel": ("pass_kernel<float,K=%d,bwd> x %d passes" % (info["bwd_k"], info["bwd_passes"]))
-                     if hbm_path else "sweep_kernel<float,K=%d,bwd>" % info["bwd_k"],
-                     "bound": "hbm" if hbm_path else "alu",
-                     "achieved": ach_bwd, "peak": peak, "unit": "GB/s" if hbm_path else "TFLOP/s",
+        "roofline": {"kernel": ("pass_kernel<%s,K=%d,bwd> x %d passes" % (rname, info["bwd_k"], info["bwd_passes"]))
+                     if hbm_path else "sweep_kernel<%s,K=%d,bwd>" % (rname, info["bwd_k"]),
+                     "bound": "hbm" if bytes_bound else "alu",
+                     "achieved": ach_bwd, "peak": peak, "unit": "GB/s" if bytes_bound else "TFLOP/s",
                      "frac": ach_bwd / peak, "traffic": traffic,
-                     "peak_basis": ("copy bandwidth, %s hbm_gbs" % pk_kind) if hbm_path else
-                     ("FP32 FFMA: 152 SMs x 128 lanes x 2 x %.0f MHz (%s sm_max_mhz)"
-                      % (pk.get("sm_max_mhz", SM_MAX_MHZ), pk_kind)),
-                     ("bytes_per_call" if hbm_path else "flops_per_launch"): bwd_flops,
+                     "peak_basis": ("copy bandwidth, %s hbm_gbs" % pk_kind) if bytes_bound else basis,
+                     ("bytes_per_call" if bytes_bound else "flops_per_launch"): bwd_flops,
                      "launch_ms": bwd_avg_s * 1e3,
                      "fwd_frac": ach_fwd / peak,
-                     "frac_of_measured_fma": None if hbm_path else ach_bwd / fma["fp32_tflops"]},
+                     "frac_of_measured_fma": ach_bwd / fma["fp32_tflops"]
+                     if not bytes_bound and args.dtype == "c64" else None},
         "fma_measured": fma,
         "e2e": {"value": e2e_value, "unit": "circuit evals/s (fwd+adjoint bwd, host buffers)",
                 "call": "Circuit.prepare_host -> vqc_evaluate_host (pageable numpy in/out; %s)" % (
@@ -609,6 +628,11 @@ def extra_configs(torch, Circuit, B, fma=None):
                 # runs on the FP32 units, so it can exceed 1)
                 r["fwd_frac_fp64_measured"] = r["fwd_tflops"] / fp64
                 r["bwd_frac_fp64_measured"] = r["bwd_tflops"] / fp64 if flop_b else None
+            if r["dtype"] == "c128df" and fma:
+                # and against the double-float ceiling: measured FP32 rate / 15
+                # (a double-float FMA, 2 flops, is 15 FP32 instructions)
+                r["fwd_frac_df_ceiling"] = r["fwd_tflops"] / (fma["fp32_tflops"] / 15.0)
+                r["bwd_frac_df_ceiling"] = r["bwd_tflops"] / (fma["fp32_tflops"] / 15.0) if flop_b else None
             if r["dtype"] == "c128df" and key.replace("df", "") in res and "fwd_evals_per_s" in res[key.replace("df", "")]:
                 ref = res[key.replace("df", "")]
                 r["fwd_speedup_vs_fp64"] = r["fwd_evals_per_s"] / ref["fwd_evals_per_s"]
@@ -625,7 +649,7 @@ def run_reference(args, rank, world):
     """The oracle on the host cores, same metric and workload (bounded sample)."""
     if rank != 0:
         return None
-    w_ = workload(args.config)
+    w_ = workload(args.config, dtype=args.dtype)
     chunk = 8
     from oracle import oracle as orc
     orc.build()
@@ -662,6 +686,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=50)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", type=int, default=2)
+    ap.add_argument("--dtype", default="c64", choices=sorted(DTYPES),
+                    help="state type of the timed workload (c128df: complex128 in double-float)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--extra", action="store_true", help="also time configs 1, 3, 4 and 5")
