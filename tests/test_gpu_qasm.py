@@ -38,7 +38,7 @@ def qasm_ring(n, layers):
     return "\n".join(lines) + "\n"
 
 
-@pytest.mark.parametrize("dtype", ["c64", "c128"])
+@pytest.mark.parametrize("dtype", ["c64", "c128", "c128df"])
 @pytest.mark.parametrize("source", ["program", "ring6", "ring11"])
 def test_qasm_forward_backward(dtype, source):
     from paper_2607_11985_gb300.circuit import Circuit
@@ -64,7 +64,7 @@ def test_qasm_forward_backward(dtype, source):
     assert maxerr(dw.cpu().numpy(), dw_ref) <= tol["grad"]
 
 
-@pytest.mark.parametrize("dtype", ["c64", "c128"])
+@pytest.mark.parametrize("dtype", ["c64", "c128", "c128df"])
 @pytest.mark.parametrize("force_hbm", [False, True])
 def test_probabilities(monkeypatch, dtype, force_hbm):
     from paper_2607_11985_gb300.circuit import Circuit
