@@ -34,8 +34,8 @@ def ready():
     torch.cuda.set_device(0)
 
 
-def _inputs(w_):
-    f = lambda a: torch.tensor(np.asarray(a), dtype=torch.float32, device="cuda")
+def _inputs(w_, real=torch.float32):
+    f = lambda a: torch.tensor(np.asarray(a), dtype=real, device="cuda")
     return f(w_.x), f(w_.w), f(w_.gE)
 
 
@@ -74,6 +74,23 @@ def test_noalloc_backward_matches_workspace_backward_twice(k):
         assert torch.isfinite(dx).all() and torch.isfinite(dw).all()
         assert float((dx - dx_ref).abs().max()) <= GRAD_TOL
         assert float((dw - dw_ref).abs().max()) <= GRAD_TOL
+
+
+@pytest.mark.parametrize("dt", ["c128", "c128df"])
+def test_noalloc_backward_complex128(dt):
+    # complex128 storage (native FP64 and double-float kernels): the workspace
+    # backward's gradients
+    from paper_2607_11985_gb300 import binding as B
+    from paper_2607_11985_gb300.circuit import Circuit
+    w_ = wl.config(1, dtype=dt)[0]
+    c = Circuit(w_.spec, dt)
+    x, w, gE = _inputs(w_, torch.float64)
+    E, st = c.forward(x, w, want_state=True)
+    dx_ref, dw_ref = _workspace_backward(B, c, x, w, gE, st)
+    dx, dw = _noalloc_backward(B, c, x, w, gE, st)
+    torch.cuda.synchronize()
+    assert torch.isfinite(dx).all() and torch.isfinite(dw).all()
+    assert float((dx - dx_ref).abs().max()) <= 1e-12 and float((dw - dw_ref).abs().max()) <= 1e-12
 
 
 def test_noalloc_rejects_batches_beyond_the_builtin_scratch():
