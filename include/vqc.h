@@ -66,7 +66,7 @@ typedef enum {
     VQC_ERR_CUDA = 7,              /* a CUDA runtime call failed (message has the name) */
     VQC_ERR_WORKSPACE = 8,         /* workspace NULL, too small or not 256-byte aligned */
     VQC_ERR_DEVICE_CHECK = 9,      /* a kernel's own bounds/consistency check tripped */
-    VQC_ERR_UNSUPPORTED = 10       /* valid request this build cannot run (e.g. too large) */
+    VQC_ERR_UNSUPPORTED = 10       /* valid request the library cannot run (e.g. too large) */
 } vqc_status;
 
 /* VQC_C128_DF: complex128 in memory (every array, layout, workspace size and
@@ -123,7 +123,7 @@ typedef enum {
 } vqc_path;
 
 typedef struct {
-    int32_t num_qubits, num_x, num_w, dtype;
+    int32_t num_qubits, num_x, num_w, dtype;   /* dtype as given to vqc_compile */
     int32_t num_gates_in;        /* gates given to vqc_compile */
     int32_t num_ops;             /* fused ops after lowering (1q runs, CX, CZ, phase ops) */
     int32_t num_runs;            /* fused single-qubit runs */
@@ -147,7 +147,9 @@ typedef struct {
  * device, uploads the plan to the current device (one synchronous copy);
  * otherwise the plan is host-only (vqc_plan_info / vqc_plan_export work) and
  * the first vqc_forward / vqc_backward uploads it, so that first call must
- * not be made inside CUDA stream capture.  On success *out_plan owns the result.
+ * not be made inside CUDA stream capture.  dtype is VQC_C64, VQC_C128 or
+ * VQC_C128_DF (a VQC_C128 plan whose kernels compute in double-float; see
+ * vqc_dtype).  On success *out_plan owns the result.
  * Errors: VQC_ERR_INVALID_ARG (NULL gates with num_gates > 0, NULL out_plan,
  * negative counts, bad dtype, nonzero reserved bytes), VQC_ERR_UNSUPPORTED_GATE,
  * VQC_ERR_QUBIT_RANGE, VQC_ERR_TOO_MANY_QUBITS, VQC_ERR_PARAM_RANGE,
