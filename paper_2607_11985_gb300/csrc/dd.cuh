@@ -75,14 +75,6 @@ struct __align__(8) dd {
     friend __device__ __forceinline__ dd& operator+=(dd& a, dd b) { return a = a + b; }
     friend __device__ __forceinline__ dd& operator-=(dd& a, dd b) { return a = a - b; }
     friend __device__ __forceinline__ dd& operator*=(dd& a, dd b) { return a = a * b; }
-
-    // warp exchange of both parts (found by argument-dependent lookup from the
-    // generic reductions)
-    friend __device__ __forceinline__ dd __shfl_xor_sync(unsigned mask, dd v, int lane_mask,
-                                                         int width = 32) {
-        return dd(::__shfl_xor_sync(mask, v.hi, lane_mask, width),
-                  ::__shfl_xor_sync(mask, v.lo, lane_mask, width));
-    }
 };
 
 struct __align__(16) dd2 {

@@ -585,8 +585,14 @@ __device__ __forceinline__ int refbit(int ref, int r, uint32_t pb) {
 }
 
 // ---------------------------------------------------------------- reductions
+// Butterfly exchange with lane ^ m (double-float: both parts).
 template <typename R>
-__device__ __forceinline__ R shx(R v, int m, unsigned mask) { return __shfl_xor_sync(mask, v, m); }
+__device__ __forceinline__ R shx(R v, int m, unsigned mask) {
+    if constexpr (std::is_same<R, dd>::value)
+        return dd(__shfl_xor_sync(mask, v.hi, m), __shfl_xor_sync(mask, v.lo, m));
+    else
+        return __shfl_xor_sync(mask, v, m);
+}
 
 // Reduce 4 values over a group of `lanes` lanes (power of two <= 32) and write
 // the 4 sums to dst[0..3] (reduce-scatter: 2 + 1 exchanges, then plain steps).
@@ -632,16 +638,16 @@ __device__ __forceinline__ void reduce4_full(R (&v)[4], int lane, R* dst, bool a
     for (int i = 0; i < 2; ++i) {
         const R send = u0 ? v[i] : v[i + 2];
         const R keep = u0 ? v[i + 2] : v[i];
-        v[i] = keep + __shfl_xor_sync(full, send, 16);
+        v[i] = keep + shx<R>(send, 16, full);
     }
     {
         const R send = u1 ? v[0] : v[1];
         const R keep = u1 ? v[1] : v[0];
-        v[0] = keep + __shfl_xor_sync(full, send, 8);
+        v[0] = keep + shx<R>(send, 8, full);
     }
-    v[0] += __shfl_xor_sync(full, v[0], 4);
-    v[0] += __shfl_xor_sync(full, v[0], 2);
-    v[0] += __shfl_xor_sync(full, v[0], 1);
+    v[0] += shx<R>(v[0], 4, full);
+    v[0] += shx<R>(v[0], 2, full);
+    v[0] += shx<R>(v[0], 1, full);
     if ((lane & 7) == 0) {
         R* d = dst + 2 * u0 + u1;
         *d = add ? *d + v[0] : v[0];
@@ -772,7 +778,7 @@ template <typename R, bool FULL>
 __device__ __forceinline__ void ph2_term_store(R tv, const Geo& q, R* accp, bool acc_add) {
     if (FULL) {
 #pragma unroll
-        for (int m = 16; m >= 1; m >>= 1) tv += __shfl_xor_sync(0xffffffffu, tv, m);
+        for (int m = 16; m >= 1; m >>= 1) tv += shx<R>(tv, m, 0xffffffffu);
     } else {
         tv = reduce1<R>(tv, q.lanes, q.mask);
     }
@@ -1101,12 +1107,12 @@ __device__ __forceinline__ int warp_reduce_scatter(R (&v)[NV], int lane) {
         for (int i = 0; i < h; ++i) {
             const R send = u ? v[i] : v[i + h];
             const R keep = u ? v[i + h] : v[i];
-            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, m);
+            v[i] = keep + shx<R>(send, m, 0xffffffffu);
         }
         idx = 2 * idx + u;
     }
 #pragma unroll
-    for (; m >= 1; m >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], m);
+    for (; m >= 1; m >>= 1) v[0] += shx<R>(v[0], m, 0xffffffffu);
     return idx;
 }
 
