@@ -81,4 +81,32 @@ struct __align__(16) dd2 {
     dd x, y;
 };
 
+// a0 b0 + a1 b1 + a2 b2 + a3 b3 with a single normalisation (the compensated
+// dot product of Ogita, Rump and Oishi, 2005): the high products are summed by
+// TwoSum, every rounding error (of the sums, of the products, the cross terms
+// hi*lo) is gathered in one float, and one FastTwoSum ends it.  43 FP32
+// operations instead of 52 for a product and three fused multiply-adds.
+__device__ __forceinline__ dd dot4(dd a0, dd b0, dd a1, dd b1, dd a2, dd b2, dd a3, dd b3) {
+    float s = __fmul_rn(a0.hi, b0.hi);
+    float err = __fmaf_rn(a0.hi, b0.hi, -s);
+    err = __fmaf_rn(a0.hi, b0.lo, err);
+    err = __fmaf_rn(a0.lo, b0.hi, err);
+    const dd A[3] = {a1, a2, a3}, Bv[3] = {b1, b2, b3};
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+        const float p = __fmul_rn(A[k].hi, Bv[k].hi);
+        const float e = __fmaf_rn(A[k].hi, Bv[k].hi, -p);
+        const float t = __fadd_rn(s, p);
+        const float v = __fsub_rn(t, s);
+        const float r = __fadd_rn(__fsub_rn(s, __fsub_rn(t, v)), __fsub_rn(p, v));
+        s = t;
+        err = __fadd_rn(err, r);
+        err = __fmaf_rn(A[k].hi, Bv[k].lo, err);
+        err = __fmaf_rn(A[k].lo, Bv[k].hi, err);
+        err = __fadd_rn(err, e);
+    }
+    const float h = __fadd_rn(s, err);
+    return dd(h, __fsub_rn(err, __fsub_rn(h, s)));
+}
+
 }  // namespace vqc

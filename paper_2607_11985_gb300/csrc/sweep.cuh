@@ -77,6 +77,12 @@ __device__ __forceinline__ C2<R> cmul(C2<R> a, C2<R> b) {
 // m0 * u + m1 * v
 template <typename R>
 __device__ __forceinline__ C2<R> cmv2(C2<R> m0, C2<R> u, C2<R> m1, C2<R> v) {
+    if constexpr (std::is_same<R, dd>::value) {   // each component one compensated dot product
+        C2<R> r;
+        r.x = dot4(m0.x, u.x, -m0.y, u.y, m1.x, v.x, -m1.y, v.y);
+        r.y = dot4(m0.x, u.y, m0.y, u.x, m1.x, v.y, m1.y, v.x);
+        return r;
+    }
     R x = fma(m0.x, u.x, fma(-m0.y, u.y, fma(m1.x, v.x, -m1.y * v.y)));
     R y = fma(m0.x, u.y, fma(m0.y, u.x, fma(m1.x, v.y, m1.y * v.x)));
     return cm<R>(x, y);
