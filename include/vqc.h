@@ -163,7 +163,10 @@ vqc_status vqc_compile(const vqc_gate* gates, int32_t num_gates, int32_t num_qub
  * registers are numbered in declaration order, qubit 0 first), the gate set
  * under its qelib1 names -- h x y z s t sx rx ry rz u3 (also u, U) cx (CX) cz
  * swap crz rzz -- and the exact U3 special cases u1 / p, u2, sdg, tdg, id;
- * `barrier` and `measure` are accepted and ignored (the engine returns <Z>).
+ * `barrier` and terminal `measure` are accepted and ignored (the engine
+ * returns <Z>); a gate or barrier on a qubit after its measurement is rejected
+ * with VQC_ERR_UNSUPPORTED_GATE (a mid-circuit measurement is outside the
+ * static-circuit scope).
  * Whole-register operands broadcast over equal-sized registers.  An angle is a
  * constant expression (numbers, pi, + - * / ^, unary minus, parentheses, sin
  * cos tan exp ln sqrt) or, as the variational extension, exactly one parameter
@@ -276,7 +279,9 @@ vqc_status vqc_probabilities(const vqc_plan* plan, int32_t batch, const void* x,
  *   on a device share the array, so calls that overlap on the GPU race and must
  *   be ordered by the caller.  The first call on a device (with that device
  *   current) looks up the array's device address; make it before any CUDA
- *   stream capture begins. */
+ *   stream capture begins.  That address is cached for the process: the entry
+ *   point assumes the CUDA runtime's primary context and no cudaDeviceReset
+ *   while the library is loaded. */
 vqc_status vqc_backward_noalloc(const vqc_plan* plan, int32_t batch, const void* x,
                                 const void* w, const void* psi0, const void* psi_final,
                                 const void* grad_expz, void* grad_x, void* grad_w, void* stream);

@@ -171,3 +171,59 @@ def gate_matrix_deriv(name, theta, p):
         raise ValueError("gate %s has no parameter %d" % (name, p))
     m = out[:2 * d * d:2] + 1j * out[1:2 * d * d:2]
     return m.reshape(d, d)
+
+
+# ------------------------------------------------------------------ batch-parallel calls
+def _row_chunks(B, workers):
+    """Contiguous row ranges, about four per worker thread."""
+    parts = max(1, min(B, 4 * workers))
+    edges = np.linspace(0, B, parts + 1).astype(int)
+    return [(int(a), int(b)) for a, b in zip(edges[:-1], edges[1:]) if b > a]
+
+
+def _pool_map(fn, items, workers):
+    import concurrent.futures as cf
+    _load()   # build and load the library before the threads start
+    with cf.ThreadPoolExecutor(max_workers=workers) as ex:
+        return list(ex.map(fn, items))
+
+
+def forward_parallel(spec, x, w, psi0=None, want_state=False, workers=None):
+    """forward() over row chunks on a thread pool: samples are independent and the
+    C oracle releases the GIL during each call, so every host core works on its
+    own rows.  Same results as forward() on the whole batch."""
+    workers = workers or os.cpu_count() or 1
+    Px = int(spec.num_x)
+    x = None if not Px else np.asarray(x)
+    B = x.shape[0] if x is not None else np.asarray(psi0).shape[0]
+
+    def one(rg):
+        a, b = rg
+        return forward(spec, None if x is None else x[a:b], w,
+                       psi0=None if psi0 is None else np.asarray(psi0)[a:b], want_state=want_state)
+
+    outs = _pool_map(one, _row_chunks(B, workers), workers)
+    if want_state:
+        return (np.concatenate([o[0] for o in outs]), np.concatenate([o[1] for o in outs]))
+    return np.concatenate(outs)
+
+
+def backward_parallel(spec, x, w, gE, psi0=None, workers=None):
+    """backward() over row chunks on a thread pool: dx rows are independent and
+    dw is the sum of the chunks' dw (in chunk order, float64)."""
+    workers = workers or os.cpu_count() or 1
+    gE = np.asarray(gE)
+    B = gE.shape[0]
+    Px = int(spec.num_x)
+
+    def one(rg):
+        a, b = rg
+        return backward(spec, None if not Px else np.asarray(x)[a:b], w, gE[a:b],
+                        psi0=None if psi0 is None else np.asarray(psi0)[a:b])
+
+    outs = _pool_map(one, _row_chunks(B, workers), workers)
+    dx = np.concatenate([o[0] for o in outs])
+    dw = np.zeros(int(spec.num_w), np.float64)
+    for o in outs:
+        dw += o[1]
+    return dx, dw

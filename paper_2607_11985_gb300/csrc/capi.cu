@@ -80,6 +80,22 @@ vqc_status device_info(int dev, DevInfo& out) {
     return VQC_OK;
 }
 
+// Let `fn` take up to the device's opt-in shared memory per CTA, once per
+// (kernel, device).  The attribute is per kernel, not per launch geometry:
+// setting it to each geometry's own need would let a later, smaller geometry of
+// the same kernel (another plan, batch or environment setting) lower it below a
+// cached larger geometry's need, whose launch would then fail.
+std::mutex g_smem_attr_mu;
+std::set<std::pair<const void*, int>> g_smem_attr_done;
+
+vqc_status allow_max_smem(const void* fn, int dev, int smem_optin) {
+    std::lock_guard<std::mutex> lk(g_smem_attr_mu);
+    if (g_smem_attr_done.count({fn, dev})) return VQC_OK;
+    VQC_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_optin));
+    g_smem_attr_done.insert({fn, dev});
+    return VQC_OK;
+}
+
 // mode 2: the backward with the forward sweep and E inside (vqc_forward_backward)
 const void* kernel_ptr(int dtype, bool dfloat, int mode, int K, bool full) {
     if (dfloat)
@@ -232,7 +248,8 @@ vqc_status plan_launch_uncached(const HostPlan& p, int launch_mode, int B, Launc
         return fail(VQC_ERR_UNSUPPORTED, "shared-memory layout exceeds the per-CTA limit");
     L.fn = kernel_ptr(p.dtype, p.dfloat, launch_mode, L.K, L.T >= 32);
     if (!L.fn) return fail(VQC_ERR_UNSUPPORTED, "kernel not instantiated for this K");
-    VQC_CUDA(cudaFuncSetAttribute(L.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem));
+    st = allow_max_smem(L.fn, dev, di.smem_optin);
+    if (st != VQC_OK) return st;
     int per_sm = 0;
     VQC_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, L.fn, L.block, L.smem));
     if (per_sm < 1) return fail(VQC_ERR_UNSUPPORTED, "kernel cannot be resident with this geometry");
@@ -498,7 +515,8 @@ vqc_status plan_cluster(const HostPlan& p, int B, Launch& L) {
     if (L.smem > (size_t)di.smem_optin)
         return fail(VQC_ERR_UNSUPPORTED, "cluster slice does not fit in shared memory");
     L.fn = p.dfloat ? cluster_ptr_dd() : cluster_ptr(dbl);
-    VQC_CUDA(cudaFuncSetAttribute(L.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem));
+    st = allow_max_smem(L.fn, dev, di.smem_optin);
+    if (st != VQC_OK) return st;
     cudaLaunchConfig_t cfg{};
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -641,7 +659,8 @@ vqc_status plan_hbm_uncached(const HostPlan& p, int mode, int B, PassGeo& L) {
     L.smem = off;
     L.fn = p.dfloat ? pass_ptr_dd(mode, L.K, L.T >= 32) : pass_ptr(dbl, mode, L.K, L.T >= 32);
     if (!L.fn) return fail(VQC_ERR_UNSUPPORTED, "pass kernel not instantiated for this K");
-    VQC_CUDA(cudaFuncSetAttribute(L.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem));
+    st = allow_max_smem(L.fn, dev, di.smem_optin);
+    if (st != VQC_OK) return st;
     int per_sm = 0;
     VQC_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, L.fn, L.block, L.smem));
     if (per_sm < 1) return fail(VQC_ERR_UNSUPPORTED, "pass kernel cannot be resident");
@@ -966,15 +985,33 @@ vqc_status backward_with_scratch(const vqc_plan* plan, int32_t batch, const void
     if (!grad_expz) return fail(VQC_ERR_INVALID_ARG, "grad_expz is NULL");
     st = check_out_ptrs(p, {grad_expz, grad_x, grad_w}, {});
     if (st != VQC_OK) return st;
-    Launch L;
-    st = plan_launch(p, 1, batch, L);
-    if (st != VQC_OK) return st;
-    const size_t need = bwd_workspace(p, L);
+    // the same path choice as vqc_backward: resident when the batch fits a
+    // resident launch, else the HBM-tiled passes (their workspace layout)
+    const bool hbm = use_hbm(p, 1, batch);
+    size_t need = 0;
+    if (hbm) {
+        PassGeo L;
+        st = plan_hbm(p, 1, batch, L);
+        if (st != VQC_OK) return st;
+        need = hbm_layout(p, 1, batch, L.ntiles).total;
+    } else {
+        Launch L;
+        st = plan_launch(p, 1, batch, L);
+        if (st != VQC_OK) return st;
+        need = bwd_workspace(p, L);
+    }
     if (need > scratch_bytes)
         return fail(VQC_ERR_WORKSPACE, "this batch needs " + std::to_string(need) +
                                            " bytes of scratch; the built-in scratch holds " +
                                            std::to_string(scratch_bytes));
     if (clear_control) VQC_CUDA(cudaMemsetAsync(scratch, 0, 256, s));
+    if (hbm) {
+        if (p.dtype == VQC_C64)
+            return run_hbm_backward<float>(p, batch, x, w, psi0, psi_final, grad_expz, grad_x,
+                                           grad_w, scratch, scratch_bytes, s);
+        return run_hbm_backward<double>(p, batch, x, w, psi0, psi_final, grad_expz, grad_x,
+                                        grad_w, scratch, scratch_bytes, s);
+    }
     if (p.dtype == VQC_C64)
         return run<float>(p, 1, batch, x, w, psi0, psi_final, grad_expz, nullptr, nullptr, grad_x,
                           grad_w, scratch, scratch_bytes, s);
@@ -1222,7 +1259,27 @@ vqc_status vqc_forward_backward(const vqc_plan* plan, int32_t batch, const void*
             return run<double>(p, 2, batch, x, w, psi0, nullptr, grad_expz, expz_out, nullptr, grad_x,
                                grad_w, workspace, workspace_bytes, s);
         }
-        // states beyond one SM: the forward passes, then the backward recomputing them
+        // states beyond one SM: the forward (passes or cluster) leaves the final
+        // states in the psi region of the backward's HBM layout, in this
+        // workspace, and the backward passes start from them (the forward's own
+        // working state is that region too, and its <Z> partials sit where the
+        // backward's lam goes: both are consumed before the backward starts)
+        if (use_hbm(p, 1, batch)) {
+            PassGeo Lb;
+            st = plan_hbm(p, 1, batch, Lb);
+            if (st != VQC_OK) return st;
+            const HbmWs lay = hbm_layout(p, 1, batch, Lb.ntiles);
+            const size_t need = vqc_workspace_bytes(plan, batch, 3);
+            if (!workspace || workspace_bytes < need || misaligned(workspace, 256))
+                return fail(VQC_ERR_WORKSPACE, "workspace must be >= " + std::to_string(need) +
+                                                   " bytes and 256-byte aligned");
+            void* psi_final = static_cast<char*>(workspace) + lay.state;
+            st = vqc_forward(plan, batch, x, w, psi0, expz_out, psi_final, workspace, workspace_bytes,
+                             stream);
+            if (st != VQC_OK) return st;
+            return vqc_backward(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x, grad_w,
+                                workspace, workspace_bytes, stream);
+        }
         st = vqc_forward(plan, batch, x, w, psi0, expz_out, nullptr, workspace, workspace_bytes, stream);
         if (st != VQC_OK) return st;
         return vqc_backward(plan, batch, x, w, psi0, nullptr, grad_expz, grad_x, grad_w, workspace,

@@ -18,7 +18,10 @@
 //
 // The device address of the array is looked up once per device, on the first
 // call made while that device is current (cudaGetSymbolAddress); make that first
-// call before any CUDA stream capture begins.
+// call before any CUDA stream capture begins.  The cached address belongs to the
+// device's primary context (the one the CUDA runtime uses): the entry point
+// assumes callers stay in it and do not reset the device (cudaDeviceReset)
+// while the library is loaded; after a reset the cached address is stale.
 #include <cuda_runtime.h>
 
 #include <mutex>

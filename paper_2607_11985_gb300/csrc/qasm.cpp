@@ -7,7 +7,9 @@
 // This front end accepts OPENQASM 2.0 with qreg/creg declarations, the gates of
 // the engine's set under their qelib1 names, the single-qubit phase forms that
 // are exact special cases of U3 (u1, p, u2, sdg, tdg, id), `barrier` and
-// `measure` (both ignored: the engine returns expectations), and one extension
+// terminal `measure` (both ignored: the engine returns expectations; a gate or
+// barrier on a qubit after its measurement is rejected, since a mid-circuit
+// measurement is outside the static-circuit scope), and one extension
 // for variational circuits: an angle may be a per-sample parameter `x[i]` or a
 // shared weight `w[j]` instead of a constant expression.  Constant expressions
 // use numbers, pi, + - * / ^, unary minus, parentheses and sin cos tan exp ln
@@ -108,6 +110,7 @@ struct Parser {
     std::map<std::string, int> qbase, qsize;
     std::map<std::string, int> cregs;
     int nq = 0;
+    std::vector<char> measured;   // per qubit: a measure statement has named it
     std::vector<vqc_gate> gates;
     int32_t max_x = -1, max_w = -1;
 
@@ -229,6 +232,14 @@ struct Parser {
         for (int k = 0; k < qsize[r]; ++k) all.push_back(b->second + k);
         return all;
     }
+    // Only terminal measurements: nothing may act on a qubit after its measure.
+    void not_measured(const std::vector<int>& qs, const std::string& what) {
+        for (int q : qs)
+            if (measured[q])
+                err(what + " on qubit " + std::to_string(q) +
+                    " after its measurement (only terminal measurements are in the static-circuit scope)",
+                    VQC_ERR_UNSUPPORTED_GATE);
+    }
     void skip_classical_operand() {
         const std::string r = expect_id();
         if (!cregs.count(r)) err("unknown classical register '" + r + "'");
@@ -297,6 +308,7 @@ struct Parser {
             const int q0 = ops[0].size() > 1 ? ops[0][k] : ops[0][0];
             const int q1 = g.nq == 2 ? (ops[1].size() > 1 ? ops[1][k] : ops[1][0]) : -1;
             if (g.nq == 2 && q0 == q1) err("a two-qubit gate needs two different qubits", VQC_ERR_QUBIT_RANGE);
+            not_measured(g.nq == 2 ? std::vector<int>{q0, q1} : std::vector<int>{q0}, "gate '" + name + "'");
             const double pi = 3.14159265358979323846;
             switch (g.na) {
             case -1: emit(VQC_U3, q0, -1, {cst(0), cst(0), args[0]}); break;          // u1 / p
@@ -336,17 +348,18 @@ struct Parser {
                     qbase[r] = nq;
                     qsize[r] = n;
                     nq += n;
+                    measured.resize(nq > 0 ? nq : 0, 0);
                     if (nq > VQC_MAX_QUBITS) err("more than " + std::to_string(VQC_MAX_QUBITS) + " qubits",
                                                  VQC_ERR_TOO_MANY_QUBITS);
                 } else {
                     cregs[r] = n;
                 }
             } else if (kw == "barrier") {
-                operand();
-                while (is_sym(",")) { ++i; operand(); }
+                not_measured(operand(), "barrier");
+                while (is_sym(",")) { ++i; not_measured(operand(), "barrier"); }
                 expect_sym(";");
             } else if (kw == "measure") {   // expectations are returned instead
-                operand();
+                for (int q : operand()) measured[q] = 1;
                 expect_sym("->");
                 skip_classical_operand();
                 expect_sym(";");

@@ -174,9 +174,14 @@ __device__ __forceinline__ const T* rebase(const T* g, const unsigned char* plan
 // with pi/2 split in three parts (the head has 8 significant bits, so k *
 // head is exact for |k| < 2^16), |r| <= pi/4, then the Taylor polynomials of
 // sin (through r^9) and cos (through r^10), whose truncation errors on
-// [-pi/4, pi/4] are below 2e-9, and the quadrant of k.  complex128 uses the
-// library routine.
+// [-pi/4, pi/4] are below 2e-9, and the quadrant of k.  The reduction is exact
+// only while |k| < 2^16; arguments beyond |t| = 65536 (|k| <= 41722), and NaN,
+// go to the library sincosf instead.  complex128 uses the library routine.
 __device__ __forceinline__ void sc(float t, float* s, float* c) {
+    if (!(fabsf(t) <= 65536.0f)) {
+        sincosf(t, s, c);
+        return;
+    }
     const float k = rintf(t * 0.636619772367581343f);   // t / (pi/2)
     float r = fmaf(-k, 1.5703125f, t);
     r = fmaf(-k, 4.838267923332751e-4f, r);

@@ -434,3 +434,22 @@ def test_gradient_finite_difference_mean_objective():
             xp[b, j] += h
             xm[b, j] -= h
             assert abs(dx[b, j] - (L(xp, w_.w) - L(xm, w_.w)) / (2 * h)) < 1e-8
+
+
+@pytest.mark.parametrize("t", [1e3, -1e5, 131072.0, 1e6, -3e7])
+def test_large_angle_rotations_closed_form(t):
+    """Angles far outside [-pi, pi] (the range the GPU trig test covers): the
+    oracle's RY, RX and RZ states equal the closed forms from the float64
+    half-angle, and the adjoint gradient of <Z> after RY(t) RX(s) equals its
+    closed form (d/dt cos t cos s = -sin t cos s)."""
+    c, s = np.cos(t / 2), np.sin(t / 2)
+    for name, want in (("RY", [c, s]), ("RX", [c, -1j * s]), ("RZ", [c - 1j * s, 0])):
+        spec = wl.CircuitSpec(1, 1, 0).add(name, (0,), [("x", 0)])
+        _, st = orc.forward(spec, np.array([[t]]), None, want_state=True)
+        assert np.allclose(st[0], want, atol=1e-12, rtol=0), name
+    u = 0.37 * t
+    spec = wl.CircuitSpec(1, 2, 0).add("RY", (0,), [("x", 0)]).add("RX", (0,), [("x", 1)])
+    x = np.array([[t, u]])
+    assert abs(orc.forward(spec, x, None)[0, 0] - np.cos(t) * np.cos(u)) <= 1e-12
+    dx, _ = orc.backward(spec, x, None, np.ones((1, 1)))
+    assert np.allclose(dx[0], [-np.sin(t) * np.cos(u), -np.cos(t) * np.sin(u)], atol=1e-11, rtol=0)

@@ -139,12 +139,28 @@ def test_broadcast_and_expressions():
     ("reset q[0];", 2, 3),
     ("h q[0];\nrx(0.1, 0.2) q[1];", 1, 4),
     ("h z[0];", 3, 3),
+    # only terminal measurements (Sec. 3 "Static Circuit Scope"): nothing acts
+    # on a qubit after its measure
+    ("creg c[3];\nmeasure q[0] -> c[0];\nh q[0];", 2, 5),
+    ("creg c[3];\nmeasure q -> c;\ncx q[1], q[2];", 2, 5),
+    ("creg c[3];\nmeasure q[2] -> c[2];\nbarrier q;", 2, 5),
+    ("creg c[3];\nmeasure q[1] -> c[1];\nrzz(0.3) q[0], q[1];", 2, 5),
 ])
 def test_errors_name_the_line(body, code, line):
     with pytest.raises(B.VQCError) as e:
         B.vqc_parse_qasm("OPENQASM 2.0;\nqreg q[3];\n" + body + "\n")
     assert e.value.status == code
     assert "line %d" % line in str(e.value)
+
+
+def test_terminal_measurements_accepted():
+    # measuring one qubit leaves the others free; measurements at the end pass
+    arr, n, nq, nx, nw = B.vqc_parse_qasm(
+        "OPENQASM 2.0;\nqreg q[3];\ncreg c[3];\nh q[0];\nmeasure q[0] -> c[0];\n"
+        "cx q[1], q[2];\nbarrier q[1], q[2];\nmeasure q[1] -> c[1];\nmeasure q[2] -> c[2];\n")
+    assert n == 2 and nq == 3
+    assert [(g.op, g.q0, g.q1) for g in arr[:n]] == [(B.GATE_CODE["H"], 0, 0),
+                                                     (B.GATE_CODE["CX"], 1, 2)]
 
 
 def test_header_required():

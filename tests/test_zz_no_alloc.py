@@ -4,11 +4,13 @@ vqc_backward_noalloc serves callers that cannot allocate device memory (a
 plugin whose host application owns every device allocation, a real-time loop
 that cannot afford cudaMalloc's latency and implicit synchronisation, code under
 a fixed device-memory budget): it takes no workspace and uses scratch built
-into the library instead.  Its gradients must equal those of the workspace
-entry point within the engine's complex64 gradient tolerance (5e-4), on two
-calls in a row (the second call finds the first call's leftovers in the shared
-scratch).  A batch whose scratch need exceeds the built-in size must be
-rejected with VQC_ERR_WORKSPACE.
+into the library instead.  It runs the same kernels with the same fixed-order
+reductions as the workspace entry point, so its gradients must be bit-identical
+to those of vqc_backward, on two calls in a row (the second call finds the first
+call's leftovers in the shared scratch): on the resident path and on the
+HBM-tiled passes (15 qubits), from a saved final state and recomputing it.  A
+batch whose scratch need exceeds the built-in size must be rejected with
+VQC_ERR_WORKSPACE.
 
 This file is collected last so that a run stopping at its first failure has
 already run every other test; it also passes on its own in a fresh process.
@@ -21,8 +23,6 @@ torch = pytest.importorskip("torch")
 from paper_2607_11985_gb300 import workloads as wl  # noqa: E402
 
 pytestmark = pytest.mark.gpu
-
-GRAD_TOL = 5e-4
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -39,12 +39,16 @@ def _inputs(w_, real=torch.float32):
     return f(w_.x), f(w_.w), f(w_.gE)
 
 
+def _ptr(t):
+    return None if t is None else t.data_ptr()
+
+
 def _workspace_backward(B, c, x, w, gE, st):
     dx = torch.empty_like(x)
     dw = torch.empty_like(w)
     stream = torch.cuda.current_stream()
     ws, wsb = c.workspace(x.shape[0], 1, stream)
-    B.vqc_backward(c.plan, x.shape[0], x.data_ptr(), w.data_ptr(), None, st.data_ptr(),
+    B.vqc_backward(c.plan, x.shape[0], x.data_ptr(), w.data_ptr(), None, _ptr(st),
                    gE.data_ptr(), dx.data_ptr(), dw.data_ptr(), ws.data_ptr(), wsb,
                    stream.cuda_stream)
     return dx, dw
@@ -53,7 +57,7 @@ def _workspace_backward(B, c, x, w, gE, st):
 def _noalloc_backward(B, c, x, w, gE, st):
     dx = torch.full_like(x, float("nan"))
     dw = torch.full_like(w, float("nan"))
-    B.vqc_backward_noalloc(c.plan, x.shape[0], x.data_ptr(), w.data_ptr(), None, st.data_ptr(),
+    B.vqc_backward_noalloc(c.plan, x.shape[0], x.data_ptr(), w.data_ptr(), None, _ptr(st),
                            gE.data_ptr(), dx.data_ptr(), dw.data_ptr(),
                            torch.cuda.current_stream().cuda_stream)
     return dx, dw
@@ -72,8 +76,30 @@ def test_noalloc_backward_matches_workspace_backward_twice(k):
         dx, dw = _noalloc_backward(B, c, x, w, gE, st)
         torch.cuda.synchronize()
         assert torch.isfinite(dx).all() and torch.isfinite(dw).all()
-        assert float((dx - dx_ref).abs().max()) <= GRAD_TOL
-        assert float((dw - dw_ref).abs().max()) <= GRAD_TOL
+        assert torch.equal(dx, dx_ref) and torch.equal(dw, dw_ref)
+
+
+@pytest.mark.parametrize("saved_state", [True, False])
+def test_noalloc_backward_hbm_passes(saved_state):
+    # 15 qubits complex64: the backward runs HBM-tiled passes whose psi / lam
+    # working states (about 0.5 MiB at batch 1) live in the built-in scratch
+    from paper_2607_11985_gb300 import binding as B
+    from paper_2607_11985_gb300.circuit import Circuit
+    spec = wl.layered(15, 1, ("RX", "RY", "RZ"), "CX")
+    rng = np.random.default_rng(1515)
+    c = Circuit(spec, "c64")
+    assert c.info(1)["bwd_path"] == 1
+    assert B.vqc_workspace_bytes(c.plan, 1, 1) <= (1 << 20)
+    x = torch.tensor(rng.uniform(-3, 3, (1, 15)), dtype=torch.float32, device="cuda")
+    w = torch.tensor(rng.uniform(-3, 3, spec.num_w), dtype=torch.float32, device="cuda")
+    gE = torch.tensor(rng.standard_normal((1, 15)), dtype=torch.float32, device="cuda")
+    st = c.forward(x, w, want_state=True)[1] if saved_state else None
+    dx_ref, dw_ref = _workspace_backward(B, c, x, w, gE, st)
+    for _ in range(2):
+        dx, dw = _noalloc_backward(B, c, x, w, gE, st)
+        torch.cuda.synchronize()
+        assert torch.isfinite(dx).all() and torch.isfinite(dw).all()
+        assert torch.equal(dx, dx_ref) and torch.equal(dw, dw_ref)
 
 
 @pytest.mark.parametrize("dt", ["c128", "c128df"])
@@ -87,10 +113,11 @@ def test_noalloc_backward_complex128(dt):
     x, w, gE = _inputs(w_, torch.float64)
     E, st = c.forward(x, w, want_state=True)
     dx_ref, dw_ref = _workspace_backward(B, c, x, w, gE, st)
-    dx, dw = _noalloc_backward(B, c, x, w, gE, st)
-    torch.cuda.synchronize()
-    assert torch.isfinite(dx).all() and torch.isfinite(dw).all()
-    assert float((dx - dx_ref).abs().max()) <= 1e-12 and float((dw - dw_ref).abs().max()) <= 1e-12
+    for _ in range(2):
+        dx, dw = _noalloc_backward(B, c, x, w, gE, st)
+        torch.cuda.synchronize()
+        assert torch.isfinite(dx).all() and torch.isfinite(dw).all()
+        assert torch.equal(dx, dx_ref) and torch.equal(dw, dw_ref)
 
 
 def test_noalloc_rejects_batches_beyond_the_builtin_scratch():
