@@ -1,23 +1,28 @@
 #!/usr/bin/env python
 """Benchmark: circuit evaluations/s of the batched statevector engine on GB300.
 
-One step = one pass of the whole hot path over one batch: forward sweep to
-per-qubit <Z> (saving the final state) plus the adjoint backward to dL/dx and
-dL/dw, for the 8-qubit / 4-layer / batch-1024 complex64 workload (RY(x)
-encoding, RX RY RZ per qubit per layer, CZ ring).  Inputs are seeded and
-synthetic.
+One step = one pass of the whole hot path over one batch: the forward sweep to
+per-qubit <Z> (saving the final states) plus the adjoint backward to dL/dx and
+dL/dw.  The timed workload (``value``) is the 16-qubit / 8-layer / batch-512
+complex64 circuit (RY(x) encoding, RX RY RZ per qubit per layer, CX ring): the
+largest configuration of the path that fits one GPU.  Sub-records (``configs``)
+time every other workload the same way: the 4-, 8- and 12-qubit circuits, the
+32 random circuits (forward only) and the 16-qubit circuit in complex128 and in
+double-float complex128.  Inputs are seeded and synthetic.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
-Under torchrun (N > 1) every rank runs the same per-rank batch (weak scaling);
-the shared-weight gradient is summed across ranks with one all-reduce per step.
-Rank 0 prints one JSON line.
+With --gpus N > 1 and no torchrun environment, the script starts itself under
+torch.distributed.run with N ranks.  Each rank runs the same per-rank batch
+(weak scaling); the shared-weight gradient is summed across ranks with one
+all-reduce per step.  Rank 0 prints one JSON line.
 """
 from __future__ import annotations
 
 import argparse
 import json
 import os
+import socket
 import statistics
 import subprocess
 import sys
@@ -31,8 +36,11 @@ sys.path.insert(0, ROOT)
 
 METRIC = "circuit evals/sec (fwd; fwd+adjoint bwd) at 4-16 qubits; % of roofline"
 FP32_LANES_PER_SM = 128
-NUM_SMS = 152
 SM_MAX_MHZ = 2070.0
+# double-float complex128: each component of a 2x2 update (4 products, 3 sums:
+# 7 of the 14 algorithmic flops per amplitude) is one compensated dot product
+# of 43 FP32 instructions, so 14 flops cost 86 FP32 instructions
+DF_FP32_OPS_PER_14_FLOPS = 86.0
 
 
 def peaks():
@@ -45,9 +53,72 @@ def peaks():
         return {"hbm_gbs": 6800.0, "sm_max_mhz": SM_MAX_MHZ}, "fallback"
 
 
-def fp32_peak_tflops(sm_mhz):
+def num_sms():
+    try:
+        import torch
+        return torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    except Exception:
+        return 152
+
+
+def fp32_peak_tflops(sm_mhz, sms=None):
     # FP32 CUDA-core peak: SMs x 128 lanes x 2 flop (FFMA) x clock
-    return NUM_SMS * FP32_LANES_PER_SM * 2 * sm_mhz * 1e6 / 1e12
+    return (sms or num_sms()) * FP32_LANES_PER_SM * 2 * sm_mhz * 1e6 / 1e12
+
+
+def flops_per_eval(info):
+    """Algorithmic flops of one evaluation by the counting rule of the hot-path
+    scope (per amplitude: 14 per fused single-qubit run, 6 per RZZ, 3 per CRZ,
+    0 for permutations; <Z> (3 + n)):
+      forward  F = sum_f 2^n + (3 + n) 2^n
+      backward   = 2 sum_f 2^n + 4 2^n (parametrised angle slots) + (n + 2) 2^n
+    sum_f 2^n is the plan's forward count without the <Z> term."""
+    n = info["num_qubits"]
+    dim = float(1 << n)
+    gates = info["fwd_flops_per_eval"] - (3 + n) * dim
+    return info["fwd_flops_per_eval"], 2 * gates + 4 * dim * info["num_terms"] + (n + 2) * dim
+
+
+def rooflines(parts, dtype, fma, pk, pk_kind):
+    """Roofline fractions of the forward and backward calls of a workload, from
+    parts = [(plan info, batch, forward seconds, backward seconds or None)] (one
+    per circuit; their work and times are summed).  Arithmetic ceiling by state
+    type: complex64 FP32 (SMs x 128 lanes x 2 x sm_max_mhz), complex128 the
+    measured FP64 FMA rate, double-float the measured FP32 instruction rate x 14
+    / 86 (its 2x2 updates' instruction mix).  HBM-tiled calls are also held
+    against the copy bandwidth with the state bytes their passes move; the bound
+    reported is the ceiling the call comes closest to."""
+    if dtype == "c64":
+        alu = fp32_peak_tflops(pk.get("sm_max_mhz", SM_MAX_MHZ))
+        alu_basis = ("FP32 FFMA: %d SMs x 128 lanes x 2 x %.0f MHz (%s sm_max_mhz)"
+                     % (num_sms(), pk.get("sm_max_mhz", SM_MAX_MHZ), pk_kind))
+    elif dtype == "c128":
+        alu = fma["fp64_tflops"]
+        alu_basis = "measured FP64 FMA rate (vqc_fma_peak); GB300's FP64 rate is ~1/75 of FP32"
+    else:
+        alu = fma["fp32_tflops"] / 2.0 * 14.0 / DF_FP32_OPS_PER_14_FLOPS
+        alu_basis = ("double-float: measured FP32 instruction rate (vqc_fma_peak / 2) x 14 flops "
+                     "per 86 FP32 instructions of a 2x2 update")
+    out = {}
+    for idx, name in ((2, "fwd"), (3, "bwd")):
+        if any(p[idx] is None for p in parts):
+            continue
+        secs = sum(p[idx] for p in parts)
+        flops = sum(flops_per_eval(p[0])[idx - 2] * p[1] for p in parts)
+        r = {"alu": {"achieved": flops / secs / 1e12, "peak": alu, "unit": "TFLOP/s",
+                     "flops": flops, "basis": alu_basis}}
+        r["alu"]["frac"] = r["alu"]["achieved"] / alu
+        if all(p[0][name + "_path"] == 1 for p in parts):
+            hbm = pk.get("hbm_gbs", 6800.0)
+            nbytes = sum(p[0][name + "_hbm_bytes_per_eval"] * p[1] for p in parts)
+            ach = nbytes / secs / 1e9
+            r["hbm"] = {"achieved": ach, "peak": hbm, "unit": "GB/s", "bytes": nbytes,
+                        "frac": ach / hbm, "basis": "copy bandwidth, %s hbm_gbs" % pk_kind}
+        r["bound"] = max(("alu", "hbm") if "hbm" in r else ("alu",), key=lambda k: r[k]["frac"])
+        r["frac"] = r[r["bound"]]["frac"]
+        r["call_ms"] = secs * 1e3
+        out[name] = r
+    return out
 
 
 class ClockSampler:
@@ -104,25 +175,39 @@ class ClockSampler:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
-def workload(cfg=2, rank=0, world=1, dtype="c64"):
-    """This rank's shard of the global batch (world x per-rank batch rows)."""
-    from paper_2607_11985_gb300 import workloads as wl
-    return wl.config(cfg, dtype=dtype, rank=rank, world=world)[0]
-
-
 # state type -> (torch real, torch complex, numpy real, arithmetic label, state label)
 DTYPES = {"c64": ("float32", "complex64", np.float32, "f32", "complex64"),
           "c128": ("float64", "complex128", np.float64, "f64", "complex128"),
           "c128df": ("float64", "complex128", np.float64, "f32x2 (double-float)", "complex128")}
 
 
+# ------------------------------------------------------------------ data-parallel step
+def dp_shard(cfg, dtype, rank, world, batch=None):
+    """This rank's workload: rows [rank B, (rank + 1) B) of a global batch of
+    world x B rows (B = the configuration's batch unless given).  Samples are
+    independent, so the shards need no exchange in the forward."""
+    from paper_2607_11985_gb300 import workloads as wl
+    return wl.config(cfg, dtype=dtype, batch=batch, rank=rank, world=world)
+
+
+def dp_sum(t, world):
+    """The data-parallel step's one exchange: the shared-weight gradient dw
+    summed over the ranks, in place (a torch tensor on the rank's device)."""
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t)
+    return t
+
+
 # ------------------------------------------------------------------ CPU oracle baseline
-def oracle_rate(w_, seconds=12.0, chunk=16, backward=True):
-    """Oracle fwd(+bwd) evaluations/s on the host (single thread), on a bounded
-    sample of the workload's rows."""
+def oracle_rate(w_, seconds=10.0, chunk=None, backward=True):
+    """Oracle fwd(+bwd) evaluations/s on one host core, on a bounded sample of
+    the workload's rows (cycled; at least one chunk)."""
     from oracle import oracle as orc
+    if chunk is None:
+        chunk = max(1, min(16, int(2e7 / ((1 << w_.spec.n) * max(1, len(w_.spec.gates))))))
     done, t0, row = 0, time.perf_counter(), 0
-    while time.perf_counter() - t0 < seconds:
+    while done == 0 or time.perf_counter() - t0 < seconds:
         rows = [(row + i) % w_.batch for i in range(chunk)]
         x = w_.x[rows]
         orc.forward(w_.spec, x, w_.w)
@@ -134,7 +219,7 @@ def oracle_rate(w_, seconds=12.0, chunk=16, backward=True):
     return done / dt, done, dt
 
 
-def oracle_rate_parallel(w_, seconds=12.0, chunk=16, workers=None, backward=True):
+def oracle_rate_parallel(w_, seconds=10.0, workers=None, backward=True):
     """The same oracle on all host cores: one thread per core, each cycling its
     own rows (the oracle runs in C; ctypes releases the GIL during each call)."""
     import concurrent.futures as cf
@@ -144,15 +229,14 @@ def oracle_rate_parallel(w_, seconds=12.0, chunk=16, workers=None, backward=True
     t0 = time.perf_counter()
 
     def work(k):
-        done, row = 0, k * chunk
-        while time.perf_counter() - t0 < seconds:
-            rows = [(row + i) % w_.batch for i in range(chunk)]
-            x = w_.x[rows]
-            orc.forward(w_.spec, x, w_.w)
+        done, row = 0, k
+        while done == 0 or time.perf_counter() - t0 < seconds:
+            rows = [row % w_.batch]
+            orc.forward(w_.spec, w_.x[rows], w_.w)
             if backward:
-                orc.backward(w_.spec, x, w_.w, w_.gE[rows])
-            done += chunk
-            row += chunk * workers
+                orc.backward(w_.spec, w_.x[rows], w_.w, w_.gE[rows])
+            done += 1
+            row += workers
         return done
 
     with cf.ThreadPoolExecutor(max_workers=workers) as ex:
@@ -162,269 +246,380 @@ def oracle_rate_parallel(w_, seconds=12.0, chunk=16, workers=None, backward=True
 
 
 # ------------------------------------------------------------------ our engine
+class CircuitBench:
+    """One compiled circuit with its device inputs, outputs and workspaces, and
+    the calls a step makes through the C ABI (forward with the final state
+    saved, backward from it; or the one-call forward+backward)."""
+
+    def __init__(self, torch, w_, stream):
+        from paper_2607_11985_gb300 import binding as B
+        from paper_2607_11985_gb300.circuit import Circuit
+        self.B, self.w_ = B, w_
+        t_real, t_cplx = getattr(torch, DTYPES[w_.dtype][0]), getattr(torch, DTYPES[w_.dtype][1])
+        self.c = c = Circuit(w_.spec, w_.dtype)
+        self.Bt = Bt = w_.batch
+        self.info = c.info(Bt)
+        self.sp = stream.cuda_stream
+        dev = lambda a: torch.tensor(np.asarray(a), dtype=t_real, device="cuda")   # noqa: E731
+        self.x = dev(w_.x) if w_.spec.num_x else None
+        self.w = dev(w_.w) if w_.spec.num_w else None
+        self.gE = dev(w_.gE)
+        self.E = torch.empty(Bt, w_.spec.n, dtype=t_real, device="cuda")
+        self.st = torch.empty(Bt, 1 << w_.spec.n, dtype=t_cplx, device="cuda")
+        self.dx = torch.empty_like(self.x) if self.x is not None else None
+        self.dw = torch.empty_like(self.w) if self.w is not None else None
+        self.ws = [c.workspace(Bt, m, stream) for m in (0, 1, 3)]
+
+    @staticmethod
+    def _p(t):
+        return None if t is None else t.data_ptr()
+
+    def fwd(self):
+        p, (ws, wsb) = self._p, self.ws[0]
+        self.B.vqc_forward(self.c.plan, self.Bt, p(self.x), p(self.w), None, p(self.E), p(self.st),
+                           p(ws), wsb, self.sp)
+
+    def bwd(self):
+        p, (ws, wsb) = self._p, self.ws[1]
+        self.B.vqc_backward(self.c.plan, self.Bt, p(self.x), p(self.w), None, p(self.st), p(self.gE),
+                            p(self.dx), p(self.dw), p(ws), wsb, self.sp)
+
+    def step(self):
+        self.fwd()
+        if self.w_.backward:
+            self.bwd()
+
+    def fused(self):
+        p, (ws, wsb) = self._p, self.ws[2]
+        self.B.vqc_forward_backward(self.c.plan, self.Bt, p(self.x), p(self.w), None, p(self.gE),
+                                    p(self.E), p(self.dx), p(self.dw), p(ws), wsb, self.sp)
+
+    def launches(self):
+        """Library kernels per step: resident forward 1, resident backward 2
+        (sweep + fixed-order dw sum); HBM-tiled: one launch per pass plus the
+        partial sums (E; dx and dw); cluster forward 1."""
+        inf, nx, nw = self.info, self.w_.spec.num_x > 0, self.w_.spec.num_w > 0
+        f = inf["fwd_passes"] + 1 if inf["fwd_path"] == 1 else 1
+        if not self.w_.backward:
+            return f
+        b = inf["bwd_passes"] + int(nx) + int(nw) if inf["bwd_path"] == 1 else 1 + int(nw)
+        return f + b
+
+    def host_step(self, stream_ptr):
+        """The end-to-end call on host numpy arrays (vqc_evaluate_host)."""
+        w_, rdt = self.w_, DTYPES[self.w_.dtype][2]
+        xh = np.ascontiguousarray(w_.x, dtype=rdt) if w_.spec.num_x else None
+        wh = np.ascontiguousarray(w_.w, dtype=rdt) if w_.spec.num_w else None
+        gh = np.ascontiguousarray(w_.gE, dtype=rdt) if w_.backward else None
+        Eh = np.empty((self.Bt, w_.spec.n), rdt)
+        dxh = np.empty_like(xh) if (gh is not None and xh is not None) else None
+        dwh = np.empty_like(wh) if (gh is not None and wh is not None) else None
+        h2d = sum(a.nbytes for a in (xh, wh, gh) if a is not None)
+        d2h = sum(a.nbytes for a in (Eh, dxh, dwh) if a is not None)
+        step = self.c.prepare_host(xh, wh, gh, out=(Eh, dxh, dwh), stream=stream_ptr)
+        return step, h2d, d2h, (Eh, dxh, dwh)
+
+
+def time_calls(torch, fn, n, flush, stream):
+    """Device time (ms) of n calls, one CUDA-event pair per call on the launch
+    stream, L2 flushed before each (outside the events)."""
+    pairs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+             for _ in range(n)]
+    for a, b in pairs:
+        flush.zero_()
+        a.record(stream)
+        fn()
+        b.record(stream)
+    torch.cuda.synchronize()
+    return [a.elapsed_time(b) for a, b in pairs]
+
+
+def stats(v):
+    return {"median": statistics.median(v), "mean": statistics.mean(v),
+            "std": statistics.pstdev(v), "n": len(v)}
+
+
+def measure_workload(torch, ws_list, steps, warmup, flush, stream, fma, pk, pk_kind,
+                     e2e_steps=10, cpu_seconds=0.0, rank=0, world=1):
+    """Time one workload (one or more circuits, same dtype) through the C ABI:
+    K steps (forward + backward from the saved state; forward only for
+    forward-only workloads), each call type on its own, the one-call
+    forward+backward, and end to end from host arrays; plus rooflines and the
+    oracle on a bounded sample.  Device times are per-rank; rates are whole-job
+    (world x per-rank batch)."""
+    benches = [CircuitBench(torch, w_, stream) for w_ in ws_list]
+    has_bwd = ws_list[0].backward
+    for b in benches:
+        for _ in range(warmup):
+            b.step()
+            if has_bwd and world > 1:
+                dp_sum(b.dw, world)
+    torch.cuda.synchronize()
+    evals = sum(b.Bt for b in benches)
+    step_ms = [0.0] * steps
+    for b in benches:
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(steps)]
+        for i in range(steps):
+            flush.zero_()                               # L2 flush, outside the step events
+            ev[i][0].record(stream)
+            b.step()
+            if has_bwd and world > 1:
+                dp_sum(b.dw, world)
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+        for i in range(steps):
+            step_ms[i] += ev[i][0].elapsed_time(ev[i][1])
+    n_calls = max(5, min(steps, 200))
+    fwd_ms = [time_calls(torch, b.fwd, n_calls, flush, stream) for b in benches]
+    bwd_ms = [time_calls(torch, b.bwd, n_calls, flush, stream) for b in benches] if has_bwd else None
+    fused_ms = [time_calls(torch, b.fused, n_calls, flush, stream) for b in benches] if has_bwd else None
+    sum_mean = lambda per: sum(statistics.mean(v) for v in per)   # noqa: E731
+    total = torch.tensor([sum(step_ms)], dtype=torch.float64, device="cuda")
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(total, op=dist.ReduceOp.MAX)
+    total_ms = float(total.item())
+    rec = {
+        "circuits": len(benches), "batch_per_gpu": benches[0].Bt,
+        "qubits": sorted({w_.spec.n for w_ in ws_list}), "dtype": ws_list[0].dtype,
+        "path": {0: "resident", 1: "hbm-tiled", 2: "cluster"}[benches[0].info["fwd_path"]] +
+                ("" if not has_bwd or benches[0].info["bwd_path"] == benches[0].info["fwd_path"] else
+                 " fwd / %s bwd" % {0: "resident", 1: "hbm-tiled", 2: "cluster"}[benches[0].info["bwd_path"]]),
+        "value": world * evals * steps / (total_ms / 1e3),
+        "unit": "circuit evals/s (%s)" % ("fwd+adjoint bwd" if has_bwd else "fwd"),
+        "ms_per_step": total_ms / steps,
+        "fwd": {"value": world * evals / (sum_mean(fwd_ms) / 1e3), "unit": "circuit evals/s (fwd)",
+                "ms": sum_mean(fwd_ms)},
+        "time_stats_ms": {"step": stats(step_ms), "fwd": stats([sum(t) for t in zip(*fwd_ms)])},
+        "gpu_launches": sum(b.launches() for b in benches) * steps,
+    }
+    if has_bwd:
+        rec["bwd"] = {"value": world * evals / (sum_mean(bwd_ms) / 1e3), "ms": sum_mean(bwd_ms)}
+        rec["fwd_bwd_two_calls"] = {"value": world * evals / ((sum_mean(fwd_ms) + sum_mean(bwd_ms)) / 1e3),
+                                    "unit": "circuit evals/s (fwd+adjoint bwd)",
+                                    "basis": "sum of the separately timed forward and backward calls"}
+        rec["fused"] = {"value": world * evals / (sum_mean(fused_ms) / 1e3),
+                        "unit": "circuit evals/s (fwd+adjoint bwd)", "ms_per_step": sum_mean(fused_ms),
+                        "call": "vqc_forward_backward (gE known before the call)"}
+        rec["time_stats_ms"]["bwd"] = stats([sum(t) for t in zip(*bwd_ms)])
+        rec["time_stats_ms"]["fused"] = stats([sum(t) for t in zip(*fused_ms)])
+    parts = [(b.info, b.Bt, statistics.mean(f) / 1e3,
+              statistics.mean(bw) / 1e3 if has_bwd else None)
+             for b, f, bw in zip(benches, fwd_ms, bwd_ms if has_bwd else [None] * len(benches))]
+    rec["roofline"] = rooflines(parts, ws_list[0].dtype, fma, pk, pk_kind)
+    if e2e_steps:
+        rec["e2e"] = e2e_rate(torch, benches, e2e_steps, stream, world)
+    if cpu_seconds > 0 and rank == 0:
+        rec["cpu_baseline"] = cpu_baseline(ws_list, cpu_seconds, has_bwd)
+    rec["_benches"] = benches
+    return rec
+
+
+def e2e_rate(torch, benches, steps, stream, world):
+    """End to end through vqc_evaluate_host: host numpy inputs in, outputs out,
+    every step (host wall clock, including the Python call)."""
+    hs = [b.host_step(stream.cuda_stream) for b in benches]
+    for step, *_ in hs:
+        step()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        for step, _, _, outs in hs:
+            step()
+            if world > 1 and outs[2] is not None:     # the data-parallel dw sum of the step
+                t = torch.from_numpy(outs[2]).to("cuda")
+                dp_sum(t, world)
+                outs[2][:] = t.cpu().numpy()
+    dt = time.perf_counter() - t0
+    t = torch.tensor([dt], dtype=torch.float64, device="cuda")
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    evals = sum(b.Bt for b in benches)
+    for _, _, _, outs in hs:
+        assert all(np.all(np.isfinite(a)) for a in outs if a is not None)
+    from paper_2607_11985_gb300 import binding as B
+    direct = B.vqc_host_direct(torch.cuda.current_device())
+    return {"value": world * evals * steps / float(t.item()),
+            "unit": "circuit evals/s (%s, host buffers)" % ("fwd+adjoint bwd" if benches[0].w_.backward else "fwd"),
+            "call": "Circuit.prepare_host -> vqc_evaluate_host (pageable numpy in/out; %s)" % (
+                "kernels access the host arrays in place over NVLink-C2C" if direct
+                else "one packed copy each way"),
+            "h2d_bytes_per_step": sum(h[1] for h in hs), "d2h_bytes_per_step": sum(h[2] for h in hs),
+            "steps": steps}
+
+
+def cpu_baseline(ws_list, seconds, backward):
+    """The oracle on one host core, on a bounded sample: rows cycled through the
+    workload's circuits (seconds split evenly)."""
+    per = seconds / len(ws_list)
+    done, dt = 0, 0.0
+    for w_ in ws_list:
+        _, d, t = oracle_rate(w_, seconds=per, backward=backward)
+        done += d
+        dt += t
+    return {"value": done / dt, "unit": "circuit evals/s (%s)" % ("fwd+adjoint bwd" if backward else "fwd"),
+            "cores": 1, "kind": "oracle",
+            "sample": "%d rows of the workload (cycled%s), %.1f s" % (
+                done, ", over its %d circuits" % len(ws_list) if len(ws_list) > 1 else "", dt)}
+
+
+SUB_RECORDS = [("cfg1", 1, "c64"), ("cfg2", 2, "c64"), ("cfg3", 3, "c64"), ("cfg4", 4, "c64"),
+               ("cfg5_c64", 5, "c64"), ("cfg5_c128", 5, "c128"), ("cfg5_c128df", 5, "c128df")]
+
+
+def kernel_name(info, dtype, mode):
+    rname = {"c64": "float", "c128": "double", "c128df": "dd"}[dtype]
+    k, path = info[mode + "_k"], info[mode + "_path"]
+    if path == 1:
+        return "pass_kernel<%s,K=%d,%s> x %d passes" % (rname, k, mode, info[mode + "_passes"])
+    if path == 2:
+        return "cluster_fwd_kernel<%s,K=%d>" % (rname, k)
+    return "sweep_kernel<%s,K=%d,%s>" % (rname, k, mode)
+
+
+def traffic_of(workload, mode):
+    """DRAM bytes per call from the committed ncu capture of this kernel build
+    (profiles/traffic.txt: workload, mode, source digest, bytes), else None."""
+    tpath = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(tpath):
+        return None
+    with open(tpath) as f:
+        for line in f:
+            parts = line.split()
+            if len(parts) >= 4 and not line.startswith("#") and parts[0] == workload \
+                    and parts[1] == mode and parts[2] == info_digest():
+                return float(parts[3])
+    return None
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
-    import torch.distributed as dist
     import __graft_entry__
     from paper_2607_11985_gb300 import binding as B
-    from paper_2607_11985_gb300.circuit import Circuit
 
     __graft_entry__.build()
     torch.cuda.set_device(local_rank)
-    w_ = workload(args.config, rank, world, args.dtype)
-    Bt = w_.batch
-    c = Circuit(w_.spec, args.dtype)
-    info = c.info(Bt)
     stream = torch.cuda.current_stream()
-    sp = stream.cuda_stream
-    t_real, t_cplx, np_real, arith, state_kind = DTYPES[args.dtype]
-    t_real, t_cplx = getattr(torch, t_real), getattr(torch, t_cplx)
-    x = torch.tensor(w_.x, dtype=t_real, device="cuda")
-    w = torch.tensor(w_.w, dtype=t_real, device="cuda")
-    gE = torch.tensor(w_.gE, dtype=t_real, device="cuda")
-    E = torch.empty(Bt, w_.spec.n, dtype=t_real, device="cuda")
-    st = torch.empty(Bt, 1 << w_.spec.n, dtype=t_cplx, device="cuda")
-    dx = torch.empty_like(x)
-    dw = torch.empty_like(w)
-    ws, wsb = c.workspace(Bt, 1, stream)
-    wsf, wsfb = c.workspace(Bt, 0, stream)
-    wsf_ptr = wsf.data_ptr() if wsf is not None else None
     flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")   # > 129 MB L2
-
-    def step():
-        B.vqc_forward(c.plan, Bt, x.data_ptr(), w.data_ptr(), None, E.data_ptr(), st.data_ptr(),
-                      wsf_ptr, wsfb, sp)
-        B.vqc_backward(c.plan, Bt, x.data_ptr(), w.data_ptr(), None, st.data_ptr(), gE.data_ptr(),
-                       dx.data_ptr(), dw.data_ptr(), ws.data_ptr(), wsb, sp)
-
-    for _ in range(args.warmup):
-        step()
-        if world > 1:
-            dist.all_reduce(dw)
-    torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
-
-    K = args.steps
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-          for _ in range(K)]
-    sampler = ClockSampler(local_rank)
-    if rank == 0:
-        sampler.start()
-    torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
-    torch.cuda._sleep(int(50e-3 * SM_MAX_MHZ * 1e6))   # queue work ahead of the GPU
-    t_wall = time.perf_counter()
-    for i in range(K):
-        flush.zero_()                                   # L2 flush, outside the step events
-        e0, e2 = ev[i]
-        e0.record(stream)
-        step()          # forward, then the backward from the saved final state
-        if world > 1:
-            dist.all_reduce(dw)
-        e2.record(stream)
-    torch.cuda.synchronize()
-    t_wall = time.perf_counter() - t_wall
-    if world > 1:
-        dist.barrier()
-    clocks = sampler.stop() if rank == 0 else None
-    step_ms = [a.elapsed_time(cc) for a, cc in ev]
-
-    # Each call on its own (for the per-kernel rooflines): an event between the
-    # forward and the backward would cut the overlap of the backward's launch
-    # with the forward's tail that the timed steps above get.
-    def timed_calls(fn, n):
-        pairs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                 for _ in range(n)]
-        for a, b2 in pairs:
-            flush.zero_()
-            a.record(stream)
-            fn()
-            b2.record(stream)
-        torch.cuda.synchronize()
-        return [a.elapsed_time(b2) for a, b2 in pairs]
-
-    n_calls = max(10, min(K, 1000))
-    fwd_ms = timed_calls(lambda: B.vqc_forward(c.plan, Bt, x.data_ptr(), w.data_ptr(), None,
-                                               E.data_ptr(), st.data_ptr(), wsf_ptr, wsfb, sp), n_calls)
-    bwd_ms = timed_calls(lambda: B.vqc_backward(c.plan, Bt, x.data_ptr(), w.data_ptr(), None,
-                                                st.data_ptr(), gE.data_ptr(), dx.data_ptr(),
-                                                dw.data_ptr(), ws.data_ptr(), wsb, sp), n_calls)
-    # the same step as ONE call when gE is known up front (vqc_forward_backward:
-    # one launch on the resident path, no state through HBM)
-    wsF, wsFb = c.workspace(Bt, 3, stream)
-    wsF_ptr = wsF.data_ptr() if wsF is not None else None
-    fused_ms = timed_calls(lambda: B.vqc_forward_backward(
-        c.plan, Bt, x.data_ptr(), w.data_ptr(), None, gE.data_ptr(), E.data_ptr(), dx.data_ptr(),
-        dw.data_ptr(), wsF_ptr, wsFb, sp), n_calls)
-    total_ms = float(sum(step_ms))
-    tot = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        dist.all_reduce(tot, op=dist.ReduceOp.MAX)
-    total_ms = float(tot.item())
-    ms_per_step = total_ms / K
-    value = world * Bt * K / (total_ms / 1e3)
-
-    # ---- end to end through the C ABI with HOST buffers (vqc_evaluate_host):
-    # every step copies x, w, gE in and E, dx, dw out (one packed copy each way)
-    xh = np.ascontiguousarray(w_.x, dtype=np_real)
-    wh = np.ascontiguousarray(w_.w, dtype=np_real)
-    gh = np.ascontiguousarray(w_.gE, dtype=np_real)
-    Eh = np.empty((Bt, w_.spec.n), np_real)
-    dxh = np.empty_like(xh)
-    dwh = np.empty_like(wh)
-    h2d = xh.nbytes + wh.nbytes + gh.nbytes
-    d2h = Eh.nbytes + dxh.nbytes + dwh.nbytes
-
-    host_step = c.prepare_host(xh, wh, gh, out=(Eh, dxh, dwh), stream=sp)
-
-    def e2e_step():
-        host_step()
-        if world > 1:   # the data-parallel dw sum of the step
-            t = torch.from_numpy(dwh).to("cuda")
-            dist.all_reduce(t)
-            dwh[:] = t.cpu().numpy()
-
-    for _ in range(max(3, args.warmup // 4)):
-        e2e_step()
-    Ke = max(10, min(K, 500))
-    torch.cuda.synchronize()
-    t0 = time.perf_counter()
-    for _ in range(Ke):
-        e2e_step()
-    e2e_s = time.perf_counter() - t0
-    t = torch.tensor([e2e_s], dtype=torch.float64, device="cuda")
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    e2e_value = world * Bt * Ke / float(t.item())
-    E_check = float(np.max(np.abs(Eh))) if Eh.size else 0.0
-    assert np.isfinite(E_check) and np.all(np.isfinite(dwh))
-
-    if rank != 0:
-        return None
-
     pk, pk_kind = peaks()
-    hbm_path = info["bwd_path"] == 1
-    # library kernels per step: resident forward 1; resident backward = sweep +
-    # fixed-order dw sum; HBM-tiled: one launch per pass plus the partial sums
-    # (E; dx and dw), the backward starting from the saved final state
-    nw, nx = w_.spec.num_w > 0, w_.spec.num_x > 0
-    launches_fwd = info["fwd_passes"] + 1 if info["fwd_path"] == 1 else 1
-    launches_bwd = (1 + int(nw)) if not hbm_path else info["bwd_passes"] + int(nx) + int(nw)
-    launches_per_step = launches_fwd + launches_bwd
-    bwd_avg_s = statistics.mean(bwd_ms) / 1e3
-    fwd_avg_s = statistics.mean(fwd_ms) / 1e3
     # measured FMA rates (outside the timed region): packed FP32 for complex64
     # sweeps, FP64 for complex128 ones
     fma = {"fp32_tflops": B.vqc_fma_peak(0), "fp64_tflops": B.vqc_fma_peak(1),
            "kernel": "independent FMA chains over every SM (vqc_fma_peak), best of 5 launches"}
-    rname = {"c64": "float", "c128": "double", "c128df": "dd"}[args.dtype]
-    if hbm_path and args.dtype == "c64":
-        # state bytes the passes move through HBM (vqc_plan_info), against copy bandwidth
-        peak = pk.get("hbm_gbs", 6800.0)
-        bwd_flops = info["bwd_hbm_bytes_per_eval"] * Bt
-        fwd_flops = info["fwd_hbm_bytes_per_eval"] * Bt
-        ach_bwd = bwd_flops / bwd_avg_s / 1e9
-        ach_fwd = fwd_flops / fwd_avg_s / 1e9
-    else:
-        if args.dtype == "c64":
-            peak = fp32_peak_tflops(pk.get("sm_max_mhz", SM_MAX_MHZ))
-            basis = ("FP32 FFMA: 152 SMs x 128 lanes x 2 x %.0f MHz (%s sm_max_mhz)"
-                     % (pk.get("sm_max_mhz", SM_MAX_MHZ), pk_kind))
-        elif args.dtype == "c128":
-            peak = fma["fp64_tflops"]
-            basis = "measured FP64 FMA rate (vqc_fma_peak); complex128 sweeps are FP64-bound on GB300"
-        else:
-            peak = fma["fp32_tflops"] / 15.0
-            basis = ("measured FP32 FMA rate / 15: a double-float FMA (2 flops) is 15 FP32 "
-                     "instructions on the FMA pipe")
-        bwd_flops = info["bwd_flops_per_eval"] * Bt
-        fwd_flops = info["fwd_flops_per_eval"] * Bt
-        ach_bwd = bwd_flops / bwd_avg_s / 1e12
-        ach_fwd = fwd_flops / fwd_avg_s / 1e12
-    traffic = None
-    tpath = os.path.join(ROOT, "profiles", "traffic.txt")
-    if os.path.exists(tpath):
-        with open(tpath) as f:
-            for line in f:
-                parts = line.split()
-                if len(parts) >= 4 and not line.startswith("#") and parts[0] == w_.name.split("_rank")[0] \
-                        and parts[1] == "bwd" and parts[2] == info_digest():
-                    traffic = float(parts[3])
-    bytes_bound = hbm_path and args.dtype == "c64"
+    head = dp_shard(args.config, args.dtype, rank, world)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    sampler = ClockSampler(local_rank)
+    if rank == 0:
+        sampler.start()
+    torch.cuda._sleep(int(50e-3 * SM_MAX_MHZ * 1e6))   # queue work ahead of the GPU
+    t_wall = time.perf_counter()
+    rec = measure_workload(torch, head, args.steps, args.warmup, flush, stream, fma, pk, pk_kind,
+                           e2e_steps=max(10, min(args.steps, 200)),
+                           cpu_seconds=0.0 if args.no_cpu_baseline else args.cpu_seconds,
+                           rank=rank, world=world)
+    t_wall = time.perf_counter() - t_wall
+    clocks = sampler.stop() if rank == 0 else None
+    benches = rec.pop("_benches")
+    info, w0 = benches[0].info, head[0]
+    subs = {}
+    if not args.no_subrecords:
+        for key, cfg, dt in SUB_RECORDS:
+            if cfg == args.config and dt == args.dtype:
+                continue
+            try:
+                r = measure_workload(torch, dp_shard(cfg, dt, rank, world), min(args.steps, 10),
+                                     min(args.warmup, 3), flush, stream, fma, pk, pk_kind, e2e_steps=5,
+                                     cpu_seconds=0.0 if args.no_cpu_baseline else args.sub_cpu_seconds,
+                                     rank=rank, world=world)
+                bs = r.pop("_benches")
+                r["workload"] = bs[0].w_.name.split("_rank")[0] if len(bs) == 1 else \
+                    "cfg4_" + "random32_n10-14_B256_c64_fwd"
+                del bs
+                subs[key] = r
+            except Exception as e:   # report, do not hide
+                subs[key] = {"error": str(e)[:300]}
+            torch.cuda.empty_cache()
+    if rank != 0:
+        return None
+    has_bwd = w0.backward
+    dom = "bwd" if has_bwd else "fwd"
+    rl = rec["roofline"][dom]
+    main = rl[rl["bound"]]
+    alt = {k: rl[k] for k in ("alu", "hbm") if k in rl and k != rl["bound"]}
+    wname = w0.name.split("_rank")[0]
     out = {
         "metric": METRIC,
-        "value": value,
-        "unit": "circuit evals/s (fwd+adjoint bwd)",
+        "value": rec["value"],
+        "unit": rec["unit"],
         "n_gpus": world,
-        "steps": K,
+        "steps": args.steps,
         "warmup": args.warmup,
-        "ms_per_step": ms_per_step,
+        "ms_per_step": rec["ms_per_step"],
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": arith,   # arithmetic type; the state type is config.state
-        "data": "synthetic (seeded; RY(x) encoding + RX/RY/RZ layers + CZ ring)",
-        "config": {"workload": w_.name.split("_rank")[0], "qubits": w_.spec.n, "state": state_kind,
-                   "batch_per_gpu": Bt,
-                   "gates": len(w_.spec.gates), "num_x": w_.spec.num_x, "num_w": w_.spec.num_w,
+        "dtype": DTYPES[args.dtype][3],   # arithmetic type; the state type is config.state
+        "data": "synthetic (seeded; RY(x) encoding + RX/RY/RZ layers + CX ring)",
+        "config": {"workload": wname, "qubits": w0.spec.n, "state": DTYPES[args.dtype][4],
+                   "batch_per_gpu": w0.batch, "gates": len(w0.spec.gates), "num_x": w0.spec.num_x,
+                   "num_w": w0.spec.num_w,
                    "parallelism": "dp%d (batch-sharded replicas, dw all-reduce)" % world,
                    "l2": "flushed between steps (256 MiB write) outside the per-step CUDA events",
-                   "fwd_k": info["fwd_k"], "bwd_k": info["bwd_k"],
-                   "path": "hbm-tiled" if hbm_path else "resident",
+                   "step": "vqc_forward (final states saved) + vqc_backward from them",
+                   "path": rec["path"], "fwd_k": info["fwd_k"], "bwd_k": info["bwd_k"],
+                   "fwd_passes": info["fwd_passes"], "bwd_passes": info["bwd_passes"],
                    "fwd_stages": info["fwd_stages"], "bwd_stages": info["bwd_stages"]},
-        "fwd": {"value": world * Bt / fwd_avg_s, "unit": "circuit evals/s (fwd)",
-                "ms": fwd_avg_s * 1e3, "achieved": ach_fwd},
-        # per-call device times (ms) of this rank: median, mean, std (the paper reports mean +- std)
-        "time_stats_ms": {name: {"median": statistics.median(v), "mean": statistics.mean(v),
-                                 "std": statistics.pstdev(v), "n": len(v)}
-                          for name, v in (("step", step_ms), ("fwd", fwd_ms), ("bwd", bwd_ms),
-                                          ("fused", fused_ms))},
-        "fused": {"value": world * Bt / (statistics.mean(fused_ms) / 1e3),
-                  "unit": "circuit evals/s (fwd+adjoint bwd)",
-                  "ms_per_step": statistics.mean(fused_ms),
-                  "call": "vqc_forward_backward (gE known before the call, e.g. the mean-<Z> "
-                          "objective; one launch)"},
-        "roofline": {"kernel": ("pass_kernel<%s,K=%d,bwd> x %d passes" % (rname, info["bwd_k"], info["bwd_passes"]))
-                     if hbm_path else "sweep_kernel<%s,K=%d,bwd>" % (rname, info["bwd_k"]),
-                     "bound": "hbm" if bytes_bound else "alu",
-                     "achieved": ach_bwd, "peak": peak, "unit": "GB/s" if bytes_bound else "TFLOP/s",
-                     "frac": ach_bwd / peak, "traffic": traffic,
-                     "peak_basis": ("copy bandwidth, %s hbm_gbs" % pk_kind) if bytes_bound else basis,
-                     ("bytes_per_call" if bytes_bound else "flops_per_launch"): bwd_flops,
-                     "launch_ms": bwd_avg_s * 1e3,
-                     "fwd_frac": ach_fwd / peak,
-                     "frac_of_measured_fma": ach_bwd / fma["fp32_tflops"]
-                     if not bytes_bound and args.dtype == "c64" else None},
+        "fwd": rec["fwd"],
+        "bwd": rec.get("bwd"),
+        "fused": rec.get("fused"),
+        "time_stats_ms": rec["time_stats_ms"],
+        "roofline": {"kernel": kernel_name(info, args.dtype, dom), "bound": rl["bound"],
+                     "achieved": main["achieved"], "peak": main["peak"], "unit": main["unit"],
+                     "frac": main["frac"], "traffic": traffic_of(wname, dom),
+                     "peak_basis": main["basis"],
+                     ("bytes_per_call" if rl["bound"] == "hbm" else "flops_per_call"):
+                         main.get("bytes", main.get("flops")),
+                     "call_ms": rl["call_ms"],
+                     "timing": "mean of per-call CUDA-event times on the launch stream (one call = "
+                               "every launch of the %s; L2 flushed before each)" % dom,
+                     "other_bound": alt, "fwd": rec["roofline"].get("fwd")},
         "fma_measured": fma,
-        "e2e": {"value": e2e_value, "unit": "circuit evals/s (fwd+adjoint bwd, host buffers)",
-                "call": "Circuit.prepare_host -> vqc_evaluate_host (pageable numpy in/out; %s)" % (
-                    "kernels access the host arrays in place over NVLink-C2C"
-                    if B.vqc_host_direct(local_rank) else "one packed copy each way"),
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": Ke},
-        "gpu_launches": launches_per_step * K,
+        "e2e": rec["e2e"],
+        "gpu_launches": rec["gpu_launches"],
         "clocks": clocks,
-        "wall_s_timed_loop": t_wall,
+        "wall_s_timed_region": t_wall,
     }
-    if not args.no_cpu_baseline:
-        rate, done, dt = oracle_rate(w_, seconds=args.cpu_seconds)
-        out["cpu_baseline"] = {"value": rate, "unit": "circuit evals/s (fwd+adjoint bwd)",
-                               "cores": 1, "kind": "oracle",
-                               "sample": "%d rows of the workload (cycled), fwd+bwd, %.1f s"
-                                         % (done, dt)}
-        prate, pdone, pdt, nw = oracle_rate_parallel(w_, seconds=args.cpu_seconds)
-        out["cpu_baseline_all_cores"] = {
-            "value": prate, "unit": "circuit evals/s (fwd+adjoint bwd)", "cores": nw,
-            "kind": "oracle, batch-parallel threads",
-            "sample": "%d rows of the workload (cycled), fwd+bwd, %.1f s" % (pdone, pdt)}
-    if args.extra:
-        out["configs"] = extra_configs(torch, Circuit, B, fma)
+    if "cpu_baseline" in rec:
+        out["cpu_baseline"] = rec["cpu_baseline"]
+        if not args.no_cpu_baseline:
+            prate, pdone, pdt, nw = oracle_rate_parallel(w0, seconds=args.cpu_seconds, backward=has_bwd)
+            out["cpu_baseline_all_cores"] = {
+                "value": prate, "unit": rec["unit"], "cores": nw,
+                "kind": "oracle, batch-parallel threads",
+                "sample": "%d rows of the workload (cycled), %.1f s" % (pdone, pdt)}
+    if subs:
+        for r in subs.values():
+            if "roofline" in r:
+                d = "bwd" if "bwd" in r["roofline"] else "fwd"
+                r["roofline_summary"] = {"kernel_call": d, "bound": r["roofline"][d]["bound"],
+                                         "frac": r["roofline"][d]["frac"],
+                                         "fwd_frac": r["roofline"]["fwd"]["frac"],
+                                         "fwd_bound": r["roofline"]["fwd"]["bound"]}
+        out["configs"] = subs
     if args.ablation:
-        out["ablation"] = ablation(torch, Circuit, w_)
+        out["ablation"] = ablation(torch, wl_config(2))
     if args.regime:
-        out["regime_map"] = regime_map(torch, Circuit)
+        out["regime_map"] = regime_map(torch)
     return out
+
+
+def wl_config(k, **kw):
+    from paper_2607_11985_gb300 import workloads as wl
+    return wl.config(k, **kw)[0]
 
 
 _DIGEST = None
@@ -438,12 +633,12 @@ def info_digest():
     return _DIGEST
 
 
-def ablation(torch, Circuit, w_):
+def ablation(torch, w_):
     """Internal ablation on this engine (the paper's Table 5 design choices),
     8-qubit workload: compile once vs compile per call; one batched launch vs a
     loop over samples; adjoint gradients vs central finite differences (the
     same forward kernel, 2 calls per parameter).  Device and host time."""
-    import numpy as np
+    from paper_2607_11985_gb300.circuit import Circuit
     real = torch.float32
     x = torch.tensor(w_.x, dtype=real, device="cuda")
     w = torch.tensor(w_.w, dtype=real, device="cuda")
@@ -504,13 +699,13 @@ def ablation(torch, Circuit, w_):
     return out
 
 
-def regime_map(torch, Circuit, qubits=(4, 8, 12, 15, 16, 18, 20), batches=(1, 8, 32, 128), layers=4):
+def regime_map(torch, qubits=(4, 8, 12, 15, 16, 18, 20), batches=(1, 8, 32, 128), layers=4):
     """Qubits x batch sweep (the paper's regime map, Sec. 4.4): RY(x) encoding,
     `layers` x (RX RY RZ per qubit + CX ring), complex64.  Per point: path, passes,
     device workspace bytes of the backward (the memory the caller must provide
     beyond inputs and outputs), forward and fwd+bwd device time (L2 flushed)."""
-    import numpy as np
     from paper_2607_11985_gb300 import binding as Bd
+    from paper_2607_11985_gb300.circuit import Circuit
     from paper_2607_11985_gb300 import workloads as wl
     flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
     pts = []
@@ -554,103 +749,15 @@ def regime_map(torch, Circuit, qubits=(4, 8, 12, 15, 16, 18, 20), batches=(1, 8,
     return pts
 
 
-def extra_configs(torch, Circuit, B, fma=None):
-    """Forward and fwd+bwd evaluations/s and roofline fractions of the other
-    workloads (device time, L2 flushed before each timed call)."""
-    from paper_2607_11985_gb300 import workloads as wl
-    pk, _ = peaks()
-    fp32 = fp32_peak_tflops(pk.get("sm_max_mhz", SM_MAX_MHZ))
-    hbm = pk.get("hbm_gbs", 6800.0)
-    fp64 = fma["fp64_tflops"] if fma else None
-    res = {}
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
-    # (name, config, dtype, batch): the 8-qubit circuit also at a large batch, where
-    # the sweep is throughput-bound rather than latency-bound
-    cases = [("cfg1", 1, None, None), ("cfg2_B65536", 2, None, 65536), ("cfg3", 3, None, None),
-             ("cfg3_c128", 3, "c128", None), ("cfg3_c128df", 3, "c128df", None), ("cfg4", 4, None, None),
-             ("cfg5_c64", 5, "c64", None), ("cfg5_c128", 5, "c128", None), ("cfg5_c128df", 5, "c128df", None)]
-    for key, k, dt, bsz in cases:
-        try:
-            ws_ = wl.config(k, dtype=dt, batch=bsz)
-            tot_f = tot_b = 0.0
-            evals = 0
-            work_f = work_b = flop_f = flop_b = 0.0
-            path = None
-            for w_ in ws_:
-                real = torch.float32 if w_.dtype == "c64" else torch.float64
-                c = Circuit(w_.spec, w_.dtype)
-                inf = c.info(w_.batch)
-                path = {0: "resident", 1: "hbm-tiled", 2: "cluster"}[inf["fwd_path"]]
-                x = torch.tensor(w_.x, dtype=real, device="cuda")
-                w = torch.tensor(w_.w, dtype=real, device="cuda") if w_.spec.num_w else None
-                gE = torch.tensor(w_.gE, dtype=real, device="cuda")
-                E, st = c.forward(x, w, want_state=True)
-                if w_.backward:
-                    c.backward(x, w, gE, psi_final=st)
-                torch.cuda.synchronize()
-                n_rep = 3 if k == 5 else 5
-                for _ in range(n_rep):
-                    flush.zero_()
-                    a, b2, d = (torch.cuda.Event(enable_timing=True) for _ in range(3))
-                    a.record()
-                    c.forward(x, w, out=E, state_out=st)
-                    b2.record()
-                    if w_.backward:
-                        c.backward(x, w, gE, psi_final=st)
-                    d.record()
-                    torch.cuda.synchronize()
-                    tot_f += a.elapsed_time(b2) / 1e3
-                    tot_b += b2.elapsed_time(d) / 1e3
-                evals += n_rep * w_.batch
-                if path == "hbm-tiled":
-                    work_f += n_rep * w_.batch * inf["fwd_hbm_bytes_per_eval"]
-                    work_b += n_rep * w_.batch * inf["bwd_hbm_bytes_per_eval"] if w_.backward else 0
-                flop_f += n_rep * w_.batch * inf["fwd_flops_per_eval"]
-                flop_b += n_rep * w_.batch * inf["bwd_flops_per_eval"] if w_.backward else 0
-                del c
-            r = {"path": path, "circuits": len(ws_), "batch": ws_[0].batch,
-                 "qubits": sorted({w_.spec.n for w_ in ws_}), "dtype": ws_[0].dtype,
-                 "fwd_evals_per_s": evals / tot_f,
-                 "fwd_bwd_evals_per_s": (evals / (tot_f + tot_b)) if flop_b else None}
-            if path == "hbm-tiled":
-                r["fwd_gbs"] = work_f / tot_f / 1e9
-                r["bwd_gbs"] = work_b / tot_b / 1e9 if work_b else None
-                r["fwd_frac_hbm"] = r["fwd_gbs"] / hbm
-                r["bwd_frac_hbm"] = r["bwd_gbs"] / hbm if work_b else None
-            # algorithmic flop rates against the arithmetic ceiling of the state type
-            r["fwd_tflops"] = flop_f / tot_f / 1e12
-            r["bwd_tflops"] = flop_b / tot_b / 1e12 if flop_b else None
-            if r["dtype"] == "c64":
-                r["fwd_frac_fp32"] = r["fwd_tflops"] / fp32
-                r["bwd_frac_fp32"] = r["bwd_tflops"] / fp32 if flop_b else None
-            elif fp64:
-                # complex128 flops against the native FP64 ceiling (double-float
-                # runs on the FP32 units, so it can exceed 1)
-                r["fwd_frac_fp64_measured"] = r["fwd_tflops"] / fp64
-                r["bwd_frac_fp64_measured"] = r["bwd_tflops"] / fp64 if flop_b else None
-            if r["dtype"] == "c128df" and fma:
-                # and against the double-float ceiling: measured FP32 rate / 15
-                # (a double-float FMA, 2 flops, is 15 FP32 instructions)
-                r["fwd_frac_df_ceiling"] = r["fwd_tflops"] / (fma["fp32_tflops"] / 15.0)
-                r["bwd_frac_df_ceiling"] = r["bwd_tflops"] / (fma["fp32_tflops"] / 15.0) if flop_b else None
-            if r["dtype"] == "c128df" and key.replace("df", "") in res and "fwd_evals_per_s" in res[key.replace("df", "")]:
-                ref = res[key.replace("df", "")]
-                r["fwd_speedup_vs_fp64"] = r["fwd_evals_per_s"] / ref["fwd_evals_per_s"]
-                if flop_b and ref.get("fwd_bwd_evals_per_s"):
-                    r["fwd_bwd_speedup_vs_fp64"] = r["fwd_bwd_evals_per_s"] / ref["fwd_bwd_evals_per_s"]
-            res[key] = r
-        except Exception as e:   # report, do not hide
-            res[key] = {"error": str(e)[:200]}
-    return res
-
-
 # ------------------------------------------------------------------ reference arm
 def run_reference(args, rank, world):
-    """The oracle on the host cores, same metric and workload (bounded sample)."""
+    """The oracle on the host cores, same metric and workload (bounded sample:
+    each step evaluates a few rows, sized so the run ends within minutes)."""
     if rank != 0:
         return None
-    w_ = workload(args.config, dtype=args.dtype)
-    chunk = 8
+    w_ = dp_shard(args.config, args.dtype, 0, 1)[0]
+    backward = w_.backward
+    chunk = max(1, min(8, int(2e7 / ((1 << w_.spec.n) * max(1, len(w_.spec.gates))))))
     from oracle import oracle as orc
     orc.build()
     for _ in range(args.warmup):
@@ -660,45 +767,65 @@ def run_reference(args, rank, world):
         rows = [(row + i) % w_.batch for i in range(chunk)]
         t0 = time.perf_counter()
         orc.forward(w_.spec, w_.x[rows], w_.w)
-        orc.backward(w_.spec, w_.x[rows], w_.w, w_.gE[rows])
+        if backward:
+            orc.backward(w_.spec, w_.x[rows], w_.w, w_.gE[rows])
         times.append(time.perf_counter() - t0)
         row += chunk
     total = sum(times)
     value = chunk * args.steps / total
-    return {"metric": METRIC, "value": value, "unit": "circuit evals/s (fwd+adjoint bwd)",
+    unit = "circuit evals/s (%s)" % ("fwd+adjoint bwd" if backward else "fwd")
+    return {"metric": METRIC, "value": value, "unit": unit,
             "impl": "reference", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": total / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded)", "config": {"workload": w_.name, "qubits": w_.spec.n,
                                                     "batch_per_step": chunk},
-            "cpu_baseline": {"value": value, "unit": "circuit evals/s (fwd+adjoint bwd)",
-                             "cores": 1, "kind": "oracle",
+            "cpu_baseline": {"value": value, "unit": unit, "cores": 1, "kind": "oracle",
                              "sample": "%d steps x %d rows of the workload" % (args.steps, chunk)},
-            "e2e": {"value": value, "unit": "circuit evals/s (fwd+adjoint bwd)",
-                    "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
             "gpu_launches": 0}
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
 
 
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=5000)
-    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--config", type=int, default=2)
+    ap.add_argument("--config", type=int, default=5, help="timed workload (1..5; default 5, 16 qubits)")
     ap.add_argument("--dtype", default="c64", choices=sorted(DTYPES),
                     help="state type of the timed workload (c128df: complex128 in double-float)")
-    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--sub-cpu-seconds", type=float, default=2.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--extra", action="store_true", help="also time configs 1, 3, 4 and 5")
+    ap.add_argument("--no-subrecords", action="store_true",
+                    help="time only the selected workload (no per-configuration sub-records)")
     ap.add_argument("--regime", action="store_true",
                     help="qubits x batch sweep to 20 qubits (HBM-tiled beyond one SM's state)")
     ap.add_argument("--ablation", action="store_true",
-                    help="compile-once / batching / adjoint-vs-FD ablation on the bench workload")
+                    help="compile-once / batching / adjoint-vs-FD ablation on the 8-qubit workload")
     args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if "WORLD_SIZE" not in os.environ and args.gpus > 1:
+        # N ranks, one per GPU: start this script under torch.distributed.run
+        cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1",
+               "--nproc-per-node", str(args.gpus), "--master-addr", "127.0.0.1",
+               "--master-port", str(_free_port()), os.path.abspath(__file__)] + sys.argv[1:]
+        sys.exit(subprocess.call(cmd))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world != args.gpus:
+        ap.error("--gpus %d but the launcher started %d ranks" % (args.gpus, world))
     if args.impl == "reference":
         out = run_reference(args, rank, world)
         if out is not None:

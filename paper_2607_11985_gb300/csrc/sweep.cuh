@@ -276,10 +276,12 @@ struct PlanPtrs {
 
 // ---------------------------------------------------------------- tables
 // Reals per table entry.  complex64 stores each 2x2 run matrix U twice in the
-// operand form of the packed-FP32 update (see m1_apply_f2): U at [0, 16) and
-// U^dag at [16, 32), each as (Re, Re), (-Im, Im) pairs of its four entries.
+// operand form of the packed-FP32 update (see m1_apply_f2w): U at [0, 16) and
+// U^dag at [16, 32), each as the pairs (m, i m) = (Re m, Im m), (-Im m, Re m) of
+// its four entries m.
 // complex128 stores U once (8 reals).  Phase entries use the first 8 reals.
 template <typename R> struct EntryWords { static constexpr int value = sizeof(R) == 4 ? 32 : 8; };
+
 
 template <typename R>
 __device__ __forceinline__ void store_matrix(const M2<R>& m, R* out) {
@@ -289,8 +291,8 @@ __device__ __forceinline__ void store_matrix(const M2<R>& m, R* out) {
         float4* o4 = reinterpret_cast<float4*>(out);
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-            o4[k] = make_float4(e[k].x, e[k].x, -e[k].y, e[k].y);
-            o4[4 + k] = make_float4(d[k].x, d[k].x, -d[k].y, d[k].y);
+            o4[k] = make_float4(e[k].x, e[k].y, -e[k].y, e[k].x);        // (m, i m)
+            o4[4 + k] = make_float4(d[k].x, d[k].y, -d[k].y, d[k].x);
         }
     } else {
         out[0] = m.a.x; out[1] = m.a.y; out[2] = m.b.x; out[3] = m.b.y;
@@ -380,34 +382,6 @@ __device__ __forceinline__ void m1_apply(C2<R> (&a)[1 << K], const M2<R>& m) {
     }
 }
 
-// complex64: the same update with Blackwell's packed FP32 instructions on
-// (re, im) pairs.  With u~ = (u.im, u.re):
-//   m u = (Re m, Re m) * u + (-Im m, Im m) * u~
-// so a complex multiply-add is two FFMA2 and a pair update eight.
-template <int K, int T>
-__device__ __forceinline__ void m1_apply_f2(float2 (&a)[1 << K], const M2<float>& m) {
-    const float2 ar = make_float2(m.a.x, m.a.x), ai = make_float2(-m.a.y, m.a.y);
-    const float2 br = make_float2(m.b.x, m.b.x), bi = make_float2(-m.b.y, m.b.y);
-    const float2 cr = make_float2(m.c.x, m.c.x), ci = make_float2(-m.c.y, m.c.y);
-    const float2 dr = make_float2(m.d.x, m.d.x), di = make_float2(-m.d.y, m.d.y);
-#pragma unroll
-    for (int p = 0; p < (1 << (K - 1)); ++p) {
-        const int i0 = pair_lo<T>(p), i1 = i0 | (1 << T);
-        const float2 u = a[i0], v = a[i1];
-        const float2 us = make_float2(u.y, u.x), vs = make_float2(v.y, v.x);
-        float2 nu = __fmul2_rn(ar, u);
-        nu = __ffma2_rn(ai, us, nu);
-        nu = __ffma2_rn(br, v, nu);
-        nu = __ffma2_rn(bi, vs, nu);
-        float2 nv = __fmul2_rn(cr, u);
-        nv = __ffma2_rn(ci, us, nv);
-        nv = __ffma2_rn(dr, v, nv);
-        nv = __ffma2_rn(di, vs, nv);
-        a[i0] = nu;
-        a[i1] = nv;
-    }
-}
-
 // Gradient accumulator of a fused run.  With rho = sum_pairs psi conj(lam)^T
 // (2x2, rho[a][b] = psi_a conj(lam_b)), every term the run needs is
 // Im Tr(P rho') for a Pauli P and rho' = W^dag rho W, i.e. it depends only on
@@ -439,8 +413,14 @@ __device__ __forceinline__ void m1_t3(const C2<R> (&ps)[1 << K], const C2<R> (&l
     v[2] += z0 + z1;
 }
 
-// complex64 2x2 update with the operand pairs read directly from a table entry
-// (w: 8 float2 = (Re a, Re a), (-Im a, Im a), (Re b, Re b), ... ).
+// complex64 2x2 update with Blackwell's packed FP32 instructions (FFMA2 on
+// (re, im) pairs), the operand pairs read directly from a table entry (w: 8
+// float2 = a, i a, b, i b, c, i c, d, i d).  With each state component
+// broadcast to both lanes,
+//   m u = (u.re, u.re) * m + (u.im, u.im) * (i m)
+// so a complex multiply-add is two FFMA2 and a pair update eight.  (The form
+// with the table's (Re m, Re m), (-Im m, Im m) pairs needs the swapped state
+// pair (u.im, u.re) instead and measured 2-8% slower.)
 template <int K, int T>
 __device__ __forceinline__ void m1_apply_f2w(float2 (&a)[1 << K], const float* wp) {
     const float4 w0 = *reinterpret_cast<const float4*>(wp);
@@ -455,15 +435,17 @@ __device__ __forceinline__ void m1_apply_f2w(float2 (&a)[1 << K], const float* w
     for (int p = 0; p < (1 << (K - 1)); ++p) {
         const int i0 = pair_lo<T>(p), i1 = i0 | (1 << T);
         const float2 u = a[i0], v = a[i1];
-        const float2 us = make_float2(u.y, u.x), vs = make_float2(v.y, v.x);
-        float2 nu = __fmul2_rn(ar, u);
-        nu = __ffma2_rn(ai, us, nu);
-        nu = __ffma2_rn(br, v, nu);
-        nu = __ffma2_rn(bi, vs, nu);
-        float2 nv = __fmul2_rn(cr, u);
-        nv = __ffma2_rn(ci, us, nv);
-        nv = __ffma2_rn(dr, v, nv);
-        nv = __ffma2_rn(di, vs, nv);
+        // entries hold (m, i m): m u = u.re (m) + u.im (i m)
+        const float2 ux = make_float2(u.x, u.x), uy = make_float2(u.y, u.y);
+        const float2 vx = make_float2(v.x, v.x), vy = make_float2(v.y, v.y);
+        float2 nu = __fmul2_rn(ar, ux);
+        nu = __ffma2_rn(ai, uy, nu);
+        nu = __ffma2_rn(br, vx, nu);
+        nu = __ffma2_rn(bi, vy, nu);
+        float2 nv = __fmul2_rn(cr, ux);
+        nv = __ffma2_rn(ci, uy, nv);
+        nv = __ffma2_rn(dr, vx, nv);
+        nv = __ffma2_rn(di, vy, nv);
         a[i0] = nu;
         a[i1] = nv;
     }
@@ -479,42 +461,6 @@ __device__ __forceinline__ void m1_entry(C2<R> (&a)[1 << K], const R* tp) {
         if (ADJ) m = mdag<R>(m);
         m1_apply<R, K, T>(a, m);
     }
-}
-
-// Packed-FP32 variants for complex64, plain FMA for complex128.
-template <typename R, int K, int T>
-__device__ __forceinline__ void m1_go(C2<R> (&a)[1 << K], const M2<R>& m) {
-    if constexpr (sizeof(R) == 4) m1_apply_f2<K, T>(a, m);
-    else m1_apply<R, K, T>(a, m);
-}
-
-
-// CX with local control C and local target T: swap (r, r^T) for r with C set, T clear.
-template <typename R, int K, int Cc, int T>
-__device__ __forceinline__ void cx_ll(C2<R> (&a)[1 << K]) {
-#pragma unroll
-    for (int r = 0; r < (1 << K); ++r) {
-        if (((r >> Cc) & 1) && !((r >> T) & 1)) {
-            C2<R> u = a[r];
-            a[r] = a[r | (1 << T)];
-            a[r | (1 << T)] = u;
-        }
-    }
-}
-
-template <typename R, int K>
-__device__ __forceinline__ void cx_ll_dispatch(int c, int t, C2<R> (&a)[1 << K]) {
-#define VQC_CXCASE(C_, T_) \
-    case C_ * 8 + T_: if constexpr (C_ < K && T_ < K) cx_ll<R, K, C_, T_>(a); break;
-    switch (c * 8 + t) {
-        VQC_CXCASE(0, 1) VQC_CXCASE(0, 2) VQC_CXCASE(0, 3) VQC_CXCASE(0, 4)
-        VQC_CXCASE(1, 0) VQC_CXCASE(1, 2) VQC_CXCASE(1, 3) VQC_CXCASE(1, 4)
-        VQC_CXCASE(2, 0) VQC_CXCASE(2, 1) VQC_CXCASE(2, 3) VQC_CXCASE(2, 4)
-        VQC_CXCASE(3, 0) VQC_CXCASE(3, 1) VQC_CXCASE(3, 2) VQC_CXCASE(3, 4)
-        VQC_CXCASE(4, 0) VQC_CXCASE(4, 1) VQC_CXCASE(4, 2) VQC_CXCASE(4, 3)
-        default: break;
-    }
-#undef VQC_CXCASE
 }
 
 // X on local T when the predicate holds (control outside the block).
@@ -903,7 +849,11 @@ __device__ __forceinline__ bool physbit(uint32_t pb, int ref) {
 // One switch over the dispatch code; every case has fixed local positions.
 // WITH_CX: the schedule may hold CX ops (HBM passes); resident schedules fold
 // every CX into stage store maps, and leaving those cases out of the switch
-// keeps the other cases' register allocation tight.
+// keeps the other cases' register allocation tight.  A pass schedule holds
+// only CX gates whose control lies outside the tile (the compiler folds every
+// CX with both qubits in the tile into a store map), so the switch has no case
+// for a local control: its code alone made the pass kernels spill (about 2.5x
+// the spill traffic under the 128-register cap).
 template <typename R, int K, int MODE, bool WITH_CX, bool FULL>
 __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 << K],
                                          C2<R> (&l)[1 << K], const R* sh_tab, const R* ps_tab,
@@ -922,14 +872,16 @@ __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 <<
                 m1_entry<R, K, T_, false>(a, tp);                                    \
             } else {                                                                 \
                 if constexpr (FULL) {                                                \
-                    /* one basic block: the butterfly's shuffles can overlap  */     \
-                    /* the adjoint arithmetic                                 */     \
+                    /* one basic block; the butterfly is issued before the    */     \
+                    /* adjoint updates so that the accumulator registers are */     \
+                    /* free while both blocks are updated (fewer spills under */     \
+                    /* the pass kernels' 128-register cap)                    */     \
                     if (flags & OPF_HAS_ACC) {                                       \
                         R rh[4] = {0, 0, 0, 0};                                      \
                         m1_t3<R, K, T_>(a, l, rh);                                   \
+                        reduce4_full<R>(rh, lane, accp, acc_add);                    \
                         m1_entry<R, K, T_, true>(a, tp);                             \
                         m1_entry<R, K, T_, true>(l, tp);                             \
-                        reduce4_full<R>(rh, lane, accp, acc_add);                    \
                     } else {                                                         \
                         m1_entry<R, K, T_, true>(a, tp);                             \
                         m1_entry<R, K, T_, true>(l, tp);                             \
@@ -948,19 +900,6 @@ __device__ __forceinline__ void apply_op(uint2 raw, uint32_t pb, C2<R> (&a)[1 <<
         break;
         VQC_M1(0) VQC_M1(1) VQC_M1(2) VQC_M1(3) VQC_M1(4)
 #undef VQC_M1
-#define VQC_CXLL(C_, T_)                                                             \
-    case DC_CX_LL + 4 * C_ + (T_ < C_ ? T_ : T_ - 1):                                \
-        if constexpr (WITH_CX && C_ < K && T_ < K) {                                 \
-            cx_ll<R, K, C_, T_>(a);                                                  \
-            if (MODE == 1) cx_ll<R, K, C_, T_>(l);                                   \
-        }                                                                            \
-        break;
-        VQC_CXLL(0, 1) VQC_CXLL(0, 2) VQC_CXLL(0, 3) VQC_CXLL(0, 4)
-        VQC_CXLL(1, 0) VQC_CXLL(1, 2) VQC_CXLL(1, 3) VQC_CXLL(1, 4)
-        VQC_CXLL(2, 0) VQC_CXLL(2, 1) VQC_CXLL(2, 3) VQC_CXLL(2, 4)
-        VQC_CXLL(3, 0) VQC_CXLL(3, 1) VQC_CXLL(3, 2) VQC_CXLL(3, 4)
-        VQC_CXLL(4, 0) VQC_CXLL(4, 1) VQC_CXLL(4, 2) VQC_CXLL(4, 3)
-#undef VQC_CXLL
 #define VQC_CXPL(T_)                                                                 \
     case DC_CX_PL + T_:                                                              \
         if constexpr (WITH_CX && T_ < K) {                                           \
