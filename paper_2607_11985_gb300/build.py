@@ -19,7 +19,7 @@ OUT = os.path.join(HERE, "libvqc.so")
 BUILD = os.path.join(HERE, "_build")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2",
+NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2,-ffp-contract=off",
               "--expt-relaxed-constexpr", "-I" + os.path.join(ROOT, "include")]
 UNITS = ["compiler.cpp", "qasm.cpp", "capi.cu", "noalloc.cu", "host_eval.cu",
          "kernels_f32_fwd.cu", "kernels_f32_bwd.cu", "kernels_f64_fwd.cu", "kernels_f64_bwd.cu",
