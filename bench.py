@@ -610,11 +610,49 @@ def run_ours(args, rank, world, local_rank):
                                          "fwd_frac": r["roofline"]["fwd"]["frac"],
                                          "fwd_bound": r["roofline"]["fwd"]["bound"]}
         out["configs"] = subs
+    if not args.no_subrecords:
+        out["f4_tensor_core_stage"] = tc_stage_measurement(torch, torch.empty(256 << 20, dtype=torch.uint8,
+                                                                              device="cuda"), torch.cuda.current_stream())
     if args.ablation:
         out["ablation"] = ablation(torch, wl_config(2))
     if args.regime:
         out["regime_map"] = regime_map(torch)
     return out
+
+
+def tc_stage_measurement(torch, flush, stream, repeats=32, n=16, batch=512):
+    """One batch-shared 5-qubit stage (the dense 32 x 32 product of five 2x2
+    runs) on the tensor cores (tcgen05, tf32 split three products) and on the
+    FP32 units (packed FP32 register blocks), applied `repeats` times to states
+    kept on chip: device time per application, algorithmic flops (5 runs x 14
+    per amplitude, the FP32 form's count) per second, agreement of the two."""
+    from paper_2607_11985_gb300 import binding as B
+    rng = np.random.default_rng(1616)
+    th = rng.uniform(-np.pi, np.pi, (5, 3))
+
+    def u3(t, p, l):
+        c, s = np.cos(t / 2), np.sin(t / 2)
+        return np.array([[c, -np.exp(1j * l) * s], [np.exp(1j * p) * s, np.exp(1j * (p + l)) * c]])
+
+    factors = np.stack([u3(*t) for t in th])
+    z = torch.randn(batch, 1 << n, dtype=torch.complex64, device="cuda")
+    z /= torch.linalg.vector_norm(z, dim=1, keepdim=True)
+    outs, res = {}, {}
+    sp = stream.cuda_stream
+    for method, name in ((0, "fp32_cores"), (1, "tcgen05_tf32x3")):
+        out = torch.empty_like(z)
+        B.vqc_stage_apply(method, batch, n, factors, z.data_ptr(), out.data_ptr(), repeats, sp)
+        ms = time_calls(torch, lambda: B.vqc_stage_apply(method, batch, n, factors, z.data_ptr(),
+                                                          out.data_ptr(), repeats, sp), 5, flush, stream)
+        B.vqc_sync_check(sp)
+        per_app = statistics.median(ms) / repeats
+        flops = 5 * 14 * float(batch << n)
+        res[name] = {"ms_per_application": per_app, "tflops_algorithmic": flops / (per_app / 1e3) / 1e12}
+        outs[name] = out
+    res["tc_over_fp32_speedup"] = res["fp32_cores"]["ms_per_application"] / res["tcgen05_tf32x3"]["ms_per_application"]
+    res["max_abs_diff_after_%d" % repeats] = float((outs["fp32_cores"] - outs["tcgen05_tf32x3"]).abs().max())
+    res["workload"] = "%d-qubit states x %d, %d applications on chip per call" % (n, batch, repeats)
+    return res
 
 
 def wl_config(k, **kw):

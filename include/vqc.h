@@ -331,6 +331,30 @@ int32_t vqc_host_direct(int32_t device);
  * VQC_ERR_CUDA. */
 vqc_status vqc_fma_peak(vqc_dtype dtype, double* tflops_out);
 
+/* One batch-shared 5-qubit stage applied to a batch of complex64 states, on
+ * the tensor cores or on the FP32 CUDA cores: the measurement behind the
+ * engine's choice of FP32 register blocks over tensor-core stages (paper,
+ * Sec. 3 "Gate Application and Differentiation": the prior art applies gates
+ * as batched matrix products).  Not used by the evaluation calls above.
+ *   method    1: the dense 32 x 32 complex Kronecker product of the factors
+ *             as a real 64 x 64 matrix product on tcgen05 tensor cores (tf32
+ *             operands split into high and low parts, three products
+ *             accumulated in FP32 in tensor memory); 0: the five 2x2 factors in
+ *             packed FP32 register blocks.
+ *   batch, num_qubits  B >= 0 states of n (5..VQC_MAX_QUBITS) qubits.
+ *   factors   host [5][8] doubles: factor q (row-major 2x2, (re, im) pairs)
+ *             acts on qubit q; the stage is U_4 (x) ... (x) U_0 on qubits 0..4.
+ *   psi_in, psi_out  device [B, 2^n] complex64, 16-byte aligned (may be equal).
+ *   repeats   the stage is applied this many times to data kept on chip
+ *             (psi_out = U^repeats psi_in), so that timing the call measures
+ *             arithmetic rather than HBM traffic.
+ *   stream    cudaStream_t.
+ * Asynchronous.  A tensor-core completion wait that runs out (about a second)
+ * is reported by the next vqc_sync_check as VQC_ERR_DEVICE_CHECK.  Errors:
+ * VQC_ERR_INVALID_ARG, VQC_ERR_CUDA. */
+vqc_status vqc_stage_apply(int32_t method, int32_t batch, int32_t num_qubits, const double* factors,
+                           const void* psi_in, void* psi_out, int32_t repeats, void* stream);
+
 /* Plan statistics (paths, stage counts, algorithmic flop and byte counts per
  * evaluation) for a batch of `batch` samples. */
 vqc_status vqc_plan_info(const vqc_plan* plan, int32_t batch, vqc_plan_stats* out);

@@ -69,6 +69,7 @@ SIGNATURES = [
     ("vqc_forward", _I, [_P, _I, _P, _P, _P, _P, _P, _P, _S, _P]),
     ("vqc_backward", _I, [_P, _I, _P, _P, _P, _P, _P, _P, _P, _P, _S, _P]),
     ("vqc_backward_noalloc", _I, [_P, _I, _P, _P, _P, _P, _P, _P, _P, _P]),
+    ("vqc_stage_apply", _I, [_I, _I, _I, ctypes.POINTER(ctypes.c_double), _P, _P, _I, _P]),
     ("vqc_plan_info", _I, [_P, _I, ctypes.POINTER(vqc_plan_stats)]),
     ("vqc_plan_export", _I, [_P, _P, ctypes.POINTER(_S)]),
     ("vqc_sync_check", _I, [_P]),
@@ -185,6 +186,17 @@ def vqc_forward_backward(plan, batch, x, w, psi0, grad_expz, expz_out, grad_x, g
 def vqc_backward_noalloc(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x, grad_w, stream):
     _check(lib().vqc_backward_noalloc(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x,
                                       grad_w, stream))
+
+
+def vqc_stage_apply(method, batch, num_qubits, factors, psi_in, psi_out, repeats, stream):
+    """factors: 5 complex 2x2 matrices (any array of shape [5, 2, 2]), factor q
+    on qubit q; psi_in / psi_out device addresses of complex64 states."""
+    import numpy as np
+    f = np.ascontiguousarray(np.stack([np.asarray(factors, np.complex128).real,
+                                       np.asarray(factors, np.complex128).imag], -1).reshape(5, 8))
+    _check(lib().vqc_stage_apply(method, batch, num_qubits,
+                                 f.ctypes.data_as(ctypes.POINTER(ctypes.c_double)), psi_in, psi_out,
+                                 repeats, stream))
 
 
 def vqc_evaluate_host(plan, batch, x, w, grad_expz, expz_out, grad_x, grad_w, stream):

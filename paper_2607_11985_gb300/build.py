@@ -26,7 +26,8 @@ UNITS = ["compiler.cpp", "qasm.cpp", "capi.cu", "noalloc.cu", "host_eval.cu",
          "kernels_f32_fwd_small.cu", "kernels_f32_bwd_small.cu", "kernels_f64_fwd_small.cu",
          "kernels_f64_bwd_small.cu", "kernels_hbm.cu", "kernels_cluster.cu",
          "kernels_f32_fused.cu", "kernels_f64_fused.cu", "fma_peak.cu",
-         "kernels_dd_fwd.cu", "kernels_dd_bwd.cu", "kernels_dd_fused.cu", "kernels_dd_hbm.cu"]
+         "kernels_dd_fwd.cu", "kernels_dd_bwd.cu", "kernels_dd_fused.cu", "kernels_dd_hbm.cu",
+         "tc_stage.cu"]
 
 
 def nvcc() -> str:

@@ -961,6 +961,9 @@ vqc_status check_ptrs(const HostPlan& p, const void* x, const void* w, const voi
 
 vqc_status set_error(vqc_status s, const std::string& msg) { return fail(s, msg); }
 
+// tc_stage.cu: the error word of vqc_stage_apply's kernels (read and cleared).
+vqc_status stage_error_check();
+
 // host_eval.cu: the per-plan arena of vqc_evaluate_host.
 void release_host_arena(const vqc_plan* plan);
 
@@ -1395,7 +1398,7 @@ vqc_status vqc_sync_check(void* stream) {
                         ((tripped & 1u) ? " resident sweep geometry" : "") +
                         ((tripped & 2u) ? " HBM pass geometry" : "") +
                         ((tripped & 4u) ? " cluster geometry" : "") + " (the work was skipped)");
-    return VQC_OK;
+    return stage_error_check();   // vqc_stage_apply's tensor-core waits
 }
 
 const char* vqc_last_error(void) { return g_err.c_str(); }
