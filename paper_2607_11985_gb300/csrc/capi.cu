@@ -157,9 +157,13 @@ int cta_threads() {
 }
 
 // Pick the register-block size: the largest K that still gives the batch
-// enough threads to cover every SM's schedulers (>= 152 * 4 warps), but not
-// below 3 (a block of 8 amplitudes) where the circuit allows it.
-int choose_k(const HostPlan& p, int mode, int B) {
+// enough threads to cover every SM's schedulers (SMs x 4 warps), but not below
+// 3 (a block of 8 amplitudes) where the circuit allows it.  A forced-K sweep on
+// GB300 (8-qubit batch 1024 and 8192, 12-qubit batch 4096; forward, backward
+// and the fused call) found no smaller K faster than this choice: smaller
+// blocks add stages (shared-memory round trips and barriers) faster than the
+// extra warps hide latency.
+int choose_k(const HostPlan& p, int mode, int B, int sms) {
     int forced = env_int(mode == 0 ? "VQC_FORCE_K_FWD" : "VQC_FORCE_K_BWD", 0);
     if (forced > 0 && find_schedule(p, mode, forced)) return forced;
     int kmax = 0;
@@ -167,7 +171,7 @@ int choose_k(const HostPlan& p, int mode, int B) {
         if (s.mode == mode && s.path == VQC_PATH_RESIDENT) kmax = std::max(kmax, s.K);
     if (kmax == 0) return 0;
     const int kmin = std::min(kmax, 3);
-    const double want = 152.0 * 4 * 32;
+    const double want = (double)sms * 4 * 32;
     int K = kmax;
     while (K > kmin && (double)B * std::ldexp(1.0, p.n - K) < want && find_schedule(p, mode, K - 1))
         --K;
@@ -182,7 +186,7 @@ vqc_status plan_launch_uncached(const HostPlan& p, int launch_mode, int B, Launc
     DevInfo di;
     vqc_status st = device_info(dev, di);
     if (st != VQC_OK) return st;
-    L.K = choose_k(p, mode, B);
+    L.K = choose_k(p, mode, B, di.sms);
     L.s = L.K ? find_schedule(p, mode, L.K) : nullptr;
     if (!L.s)
         return fail(VQC_ERR_UNSUPPORTED, "no resident schedule for this circuit (n = " +
@@ -1314,6 +1318,13 @@ vqc_status vqc_plan_info(const vqc_plan* plan, int32_t batch, vqc_plan_stats* ou
         ndev = 0;
     }
     const std::string saved = g_err;
+    int sms = 152;   // without a device: GB300's SM count
+    if (ndev > 0) {
+        int dev = 0;
+        DevInfo di;
+        if (cudaGetDevice(&dev) == cudaSuccess && device_info(dev, di) == VQC_OK) sms = di.sms;
+        else (void)cudaGetLastError();
+    }
     const double sbytes = std::ldexp(1.0, p.n) * (p.dtype == VQC_C128 ? 16.0 : 8.0);
     for (int mode = 0; mode < 2; ++mode) {
         int* path = mode == 0 ? &out->fwd_path : &out->bwd_path;
@@ -1323,7 +1334,7 @@ vqc_status vqc_plan_info(const vqc_plan* plan, int32_t batch, vqc_plan_stats* ou
         int* tps = mode == 0 ? &out->fwd_threads_per_sample : &out->bwd_threads_per_sample;
         int* tq = mode == 0 ? &out->fwd_tile_qubits : &out->bwd_tile_qubits;
         double* hb = mode == 0 ? &out->fwd_hbm_bytes_per_eval : &out->bwd_hbm_bytes_per_eval;
-        const int K = choose_k(p, mode, B);
+        const int K = choose_k(p, mode, B, sms);
         const bool clu = use_cluster(p, mode);
         const bool hbm = !clu && (ndev > 0 ? use_hbm(p, mode, B)
                                            : (K == 0 && find_hbm_schedule(p, mode) != nullptr));
