@@ -824,6 +824,20 @@ def run_reference(args, rank, world):
             "gpu_launches": 0}
 
 
+def one_call(args):
+    """One forward with the final states saved and one backward of the selected
+    workload (launch order: the forward's passes, then the backward's)."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    torch.cuda.set_device(0)
+    for w_ in dp_shard(args.config, args.dtype, 0, 1):
+        b = CircuitBench(torch, w_, torch.cuda.current_stream())
+        b.step()
+        torch.cuda.synchronize()
+        print("one call: %s, E sum %.6g" % (w_.name, float(b.E.double().abs().sum())))
+
+
 def _free_port():
     s = socket.socket()
     s.bind(("127.0.0.1", 0))
@@ -850,6 +864,12 @@ def main():
                     help="qubits x batch sweep to 20 qubits (HBM-tiled beyond one SM's state)")
     ap.add_argument("--ablation", action="store_true",
                     help="compile-once / batching / adjoint-vs-FD ablation on the 8-qubit workload")
+    ap.add_argument("--stage-once", action="store_true",
+                    help="no timing: the batch-shared 5-qubit stage once on the FP32 units and once on "
+                         "the tensor cores (16-qubit states x 512, 8 applications), for a profiler")
+    ap.add_argument("--one-call", action="store_true",
+                    help="no timing: one forward (final states saved) and one backward of the selected "
+                         "workload, for a profiler to capture")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -864,6 +884,18 @@ def main():
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if world != args.gpus:
         ap.error("--gpus %d but the launcher started %d ranks" % (args.gpus, world))
+    if args.one_call:
+        one_call(args)
+        return
+    if args.stage_once:
+        import torch
+        torch.cuda.set_device(0)
+        import __graft_entry__
+        __graft_entry__.build()
+        r = tc_stage_measurement(torch, torch.empty(256 << 20, dtype=torch.uint8, device="cuda"),
+                                 torch.cuda.current_stream(), repeats=8)
+        print(json.dumps(r))
+        return
     if args.impl == "reference":
         out = run_reference(args, rank, world)
         if out is not None:

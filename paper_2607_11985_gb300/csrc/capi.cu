@@ -97,7 +97,11 @@ vqc_status allow_max_smem(const void* fn, int dev, int smem_optin) {
 }
 
 // mode 2: the backward with the forward sweep and E inside (vqc_forward_backward)
-const void* kernel_ptr(int dtype, bool dfloat, int mode, int K, bool full) {
+const void* kernel_ptr(int dtype, bool dfloat, int mode, int K, bool full, bool ph2) {
+    // complex64 forward / backward sweeps of plans without CRZ / RZZ: the
+    // instantiations without the phase cases (fewer spills)
+    if (!dfloat && dtype == VQC_C64 && !ph2 && mode != 2)
+        return mode == 0 ? sweep_ptr_f32_fwd_nph(K, full) : sweep_ptr_f32_bwd_nph(K, full);
     if (dfloat)
         return mode == 2 ? sweep_ptr_dd_fused(K, full) : mode == 0 ? sweep_ptr_dd_fwd(K, full) : sweep_ptr_dd_bwd(K, full);
     if (mode == 2) return dtype == VQC_C64 ? sweep_ptr_f32_fused(K, full) : sweep_ptr_f64_fused(K, full);
@@ -250,7 +254,7 @@ vqc_status plan_launch_uncached(const HostPlan& p, int launch_mode, int B, Launc
     L.smem = off;
     if (L.smem > (size_t)di.smem_optin)
         return fail(VQC_ERR_UNSUPPORTED, "shared-memory layout exceeds the per-CTA limit");
-    L.fn = kernel_ptr(p.dtype, p.dfloat, launch_mode, L.K, L.T >= 32);
+    L.fn = kernel_ptr(p.dtype, p.dfloat, launch_mode, L.K, L.T >= 32, p.has_ph2);
     if (!L.fn) return fail(VQC_ERR_UNSUPPORTED, "kernel not instantiated for this K");
     st = allow_max_smem(L.fn, dev, di.smem_optin);
     if (st != VQC_OK) return st;
@@ -661,7 +665,9 @@ vqc_status plan_hbm_uncached(const HostPlan& p, int mode, int B, PassGeo& L) {
     L.plan_smem = off + plan_bytes <= (size_t)di.smem_optin && plan_bytes <= 48 * 1024;
     L.sm_plan = L.plan_smem ? take(plan_bytes) : 0;
     L.smem = off;
-    L.fn = p.dfloat ? pass_ptr_dd(mode, L.K, L.T >= 32) : pass_ptr(dbl, mode, L.K, L.T >= 32);
+    L.fn = p.dfloat ? pass_ptr_dd(mode, L.K, L.T >= 32)
+           : (!dbl && mode == 0 && !p.has_ph2) ? pass_ptr_f32_fwd_nph(L.K, L.T >= 32)   // no phase cases
+                                               : pass_ptr(dbl, mode, L.K, L.T >= 32);
     if (!L.fn) return fail(VQC_ERR_UNSUPPORTED, "pass kernel not instantiated for this K");
     st = allow_max_smem(L.fn, dev, di.smem_optin);
     if (st != VQC_OK) return st;

@@ -624,6 +624,7 @@ vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx,
             else p.wocc[fw[p.term_idx[t]]++] = (int32_t)t;
         }
     }
+    for (const HOp& o : p.ops) p.has_ph2 = p.has_ph2 || o.type == OP_PH2;
     // Algorithmic flops per evaluation (counted on the fused op list).
     const double dim = std::ldexp(1.0, n);
     double f = 0, fb = 0;

@@ -49,6 +49,7 @@ struct HostPlan {
     int n = 0, num_x = 0, num_w = 0, dtype = 0, num_gates_in = 0;
     int G_swz = 4;                         // swizzle chunk bits (4: c64, 3: c128)
     bool dfloat = false;                   // VQC_C128_DF: complex128 storage, double-float kernels
+    bool has_ph2 = false;                  // the op list holds diagonal two-qubit phases (CRZ / RZZ)
     std::vector<HOp> ops;
     std::vector<DEntry> entries;
     std::vector<DConst> consts;

@@ -14,6 +14,10 @@ const void* sweep_ptr_f32_bwd_small(int K);
 const void* sweep_ptr_f64_fwd_small(int K);
 const void* sweep_ptr_f64_bwd_small(int K);
 const void* sweep_ptr_f32_fused(int K, bool full);   // backward that also writes E
+// plans without CRZ / RZZ phase ops: instantiations without the phase cases
+const void* sweep_ptr_f32_fwd_nph(int K, bool full);
+const void* sweep_ptr_f32_bwd_nph(int K, bool full);
+const void* pass_ptr_f32_fwd_nph(int K, bool full);
 const void* sweep_ptr_f64_fused(int K, bool full);
 // double-float arithmetic on complex128 storage (VQC_C128_DF plans)
 const void* sweep_ptr_dd_fwd(int K, bool full);

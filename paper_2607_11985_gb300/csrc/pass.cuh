@@ -153,7 +153,7 @@ __device__ __forceinline__ void tile_scatter(const C2<R>* sm, SC2<R>* gs, uint32
 
 // FULL: tile groups span whole warps (2^(m-K) >= 32 threads; every production
 // tile), see sweep_kernel.
-template <typename R, int K, int MODE, bool FULL>
+template <typename R, int K, int MODE, bool FULL, bool PH2 = true>
 __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PArgs<St<R>> A) {
     if (geometry_bad(blockDim.x != (unsigned)(A.S << A.tbits) || A.tbits != A.m - K ||
                          A.stage_end <= A.stage_begin,
@@ -277,7 +277,7 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
                 } else {
                     block_load<R, K>(a, psi, v.swb, sg);
                 }
-                run_ops<R, K, 0, true, FULL>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
+                run_ops<R, K, 0, true, FULL, PH2>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, a,
                                  sh_tab, ps_tab, nullptr, q, lane, warp_in_group);
                 if (s + 1 < A.stage_end || A.dst_psi) {   // store map: absorbed CX gates
                     if (vqc_ld(&sp->nperm)) group_sync<R>(q);   // all loads of the stage first
@@ -322,7 +322,7 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
                 else
                     block_load<R, K>(l, lam, b2, s2);
             }
-            run_ops<R, K, 1, true, FULL>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l, sh_tab,
+            run_ops<R, K, 1, true, FULL, PH2>(P_ops, vqc_ld(&sp->op_begin), vqc_ld(&sp->op_end), v.pb, a, l, sh_tab,
                              ps_tab, acc, q, lane, warp_in_group);
             if (s > A.stage_begin || A.dst_psi) {   // back to the stage's load map
                 if (vqc_ld(&sp->nperm)) group_sync<R>(q);   // all loads of the stage first
