@@ -237,8 +237,11 @@ vqc_status vqc_backward(const vqc_plan* plan, int32_t batch, const void* x, cons
  * the mean of <Z_j>, has gE = 1/n): E, dL/dx and dL/dw of one batch.  Where the
  * state fits one SM (the resident path) it is ONE launch: the backward kernel
  * runs the forward sweep itself, keeps the final states in shared memory,
- * writes E and sweeps back, so no state goes through HBM; otherwise it is
- * vqc_forward followed by vqc_backward recomputing the states.
+ * writes E and sweeps back, so no state goes through HBM -- unless the forward
+ * alone would take larger register blocks than the backward, when it is
+ * vqc_forward saving the final states in the workspace followed by
+ * vqc_backward from them (faster there).  Beyond one SM it is vqc_forward
+ * (final states into the workspace) followed by the backward passes.
  *   expz_out  device [B, n] real (required); grad_expz device [B, n] (required);
  *   grad_x, grad_w as vqc_backward; psi0 as vqc_forward.
  *   workspace vqc_workspace_bytes(plan, B, 3) bytes, 256-byte aligned,

@@ -17,6 +17,7 @@ const void* sweep_ptr_f32_fused(int K, bool full);   // backward that also write
 // plans without CRZ / RZZ phase ops: instantiations without the phase cases
 const void* sweep_ptr_f32_fwd_nph(int K, bool full);
 const void* sweep_ptr_f32_bwd_nph(int K, bool full);
+const void* sweep_ptr_f32_fused_nph(int K, bool full);
 const void* pass_ptr_f32_fwd_nph(int K, bool full);
 const void* sweep_ptr_f64_fused(int K, bool full);
 // double-float arithmetic on complex128 storage (VQC_C128_DF plans)
