@@ -114,12 +114,15 @@ typedef struct {
 typedef enum {
     VQC_PATH_RESIDENT = 0,  /* each sample's state stays in one CTA's shared memory */
     VQC_PATH_HBM = 1,       /* state in HBM, swept in shared-memory tiles, one launch per pass */
-    VQC_PATH_CLUSTER = 2    /* forward: each sample's state spread over the shared memory of a
-                               thread-block cluster (2..8 CTAs), one launch; taken by default for
-                               2-CTA clusters (complex64 15 qubits, complex128 14 qubits), for
-                               larger ones only when the environment sets VQC_FORCE_PATH=cluster
-                               (they measured slower than VQC_PATH_HBM); VQC_FORCE_PATH=hbm
-                               turns it off */
+    VQC_PATH_CLUSTER = 2    /* each sample's state (forward) or its psi and lambda (backward)
+                               spread over the shared memory of a thread-block cluster (2..8
+                               CTAs of 512 threads), one launch (plus the fixed-order dw sum);
+                               taken by default for 2-CTA clusters (forward: complex64 15
+                               qubits, complex128 14; backward: complex64 14, complex128 13),
+                               for larger ones only when the environment sets
+                               VQC_FORCE_PATH=cluster (they measured slower than VQC_PATH_HBM);
+                               VQC_FORCE_PATH=hbm turns it off.  The backward's workspace is a
+                               256-byte control block and one dw partial per cluster. */
 } vqc_path;
 
 typedef struct {
@@ -241,7 +244,8 @@ vqc_status vqc_backward(const vqc_plan* plan, int32_t batch, const void* x, cons
  * alone would take larger register blocks than the backward, when it is
  * vqc_forward saving the final states in the workspace followed by
  * vqc_backward from them (faster there).  Beyond one SM it is vqc_forward
- * (final states into the workspace) followed by the backward passes.
+ * (final states into the workspace) followed by the backward passes or the
+ * cluster backward from them.
  *   expz_out  device [B, n] real (required); grad_expz device [B, n] (required);
  *   grad_x, grad_w as vqc_backward; psi0 as vqc_forward.
  *   workspace vqc_workspace_bytes(plan, B, 3) bytes, 256-byte aligned,

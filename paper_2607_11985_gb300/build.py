@@ -28,7 +28,7 @@ UNITS = ["compiler.cpp", "qasm.cpp", "capi.cu", "noalloc.cu", "host_eval.cu",
          "kernels_f32_fused.cu", "kernels_f64_fused.cu", "fma_peak.cu",
          "kernels_dd_fwd.cu", "kernels_dd_bwd.cu", "kernels_dd_fused.cu", "kernels_dd_hbm.cu",
          "tc_stage.cu", "kernels_f32_fwd_nph.cu", "kernels_f32_bwd_nph.cu", "kernels_hbm_nph.cu",
-         "kernels_f32_fused_nph.cu"]
+         "kernels_f32_fused_nph.cu", "kernels_cluster_bwd.cu"]
 
 
 def nvcc() -> str:

@@ -476,8 +476,8 @@ vqc_status run(const HostPlan& p, int mode, int B, const void* x, const void* w,
 
 // ---------------------------------------------------------------- cluster path
 
-vqc_status plan_cluster(const HostPlan& p, int B, Launch& L) {
-    const GeoKey k = geo_key(p, 0, B, 2);
+vqc_status plan_cluster(const HostPlan& p, int mode, int B, Launch& L) {
+    const GeoKey k = geo_key(p, mode, B, 2);
     {
         std::lock_guard<std::mutex> lk(g_geo_mu);
         auto it = g_cluster_cache.find(k);
@@ -487,7 +487,7 @@ vqc_status plan_cluster(const HostPlan& p, int B, Launch& L) {
         }
     }
     L = Launch();
-    L.s = find_cluster_schedule(p, 0);
+    L.s = find_cluster_schedule(p, mode);
     if (!L.s) return fail(VQC_ERR_UNSUPPORTED, "no cluster schedule for this circuit");
     int dev = 0;
     VQC_CUDA(cudaGetDevice(&dev));
@@ -509,13 +509,23 @@ vqc_status plan_cluster(const HostPlan& p, int B, Launch& L) {
         off = align16(off + bytes);
         return (int)o;
     };
+    const size_t slice = ((size_t)1 << (p.n - L.cl)) * cs;
     L.sm_sh = take((size_t)p.n_sh * ew * rs);
     L.sm_ps = take((size_t)p.n_ps * ew * rs);
-    L.sm_psi = take(((size_t)1 << (p.n - L.cl)) * cs);
-    L.sm_red = take((size_t)L.wg * p.n * rs);
-    L.sm_ecl = take(((size_t)1 << L.cl) * p.n * rs);
-    L.sm_w = take((size_t)p.num_w * rs);
-    L.sm_xg = take((size_t)p.num_x * rs);
+    L.sm_psi = take(slice);
+    if (mode == 0) {
+        L.sm_red = take((size_t)L.wg * p.n * rs);
+        L.sm_ecl = take(((size_t)1 << L.cl) * p.n * rs);
+        L.sm_w = take((size_t)p.num_w * rs);
+        L.sm_xg = take((size_t)p.num_x * rs);
+    } else {   // lam, rho partials [accs][warps][4], terms, dw partial, x and gE rows
+        L.sm_lam = take(slice);
+        L.sm_acc = take(std::max<size_t>(p.accs.size(), 1) * L.wg * 4 * rs);
+        L.sm_terms = take(std::max<size_t>(p.term_src.size(), 1) * rs);
+        L.sm_dw = take((size_t)std::max(p.num_w, 1) * rs);
+        L.sm_w = take((size_t)std::max(p.num_w, 1) * rs);
+        L.sm_xg = take((size_t)(p.num_x + p.n) * rs);
+    }
     const size_t plan_bytes = align16(p.dev_tab_end - p.dev_tab_begin) +
                               (L.s->dev_region_end - L.s->dev_region_begin);
     L.plan_smem = off + plan_bytes <= (size_t)di.smem_optin && env_int("VQC_PLAN_IN_SMEM", 1) != 0;
@@ -523,7 +533,7 @@ vqc_status plan_cluster(const HostPlan& p, int B, Launch& L) {
     L.smem = off;
     if (L.smem > (size_t)di.smem_optin)
         return fail(VQC_ERR_UNSUPPORTED, "cluster slice does not fit in shared memory");
-    L.fn = p.dfloat ? cluster_ptr_dd() : cluster_ptr(dbl);
+    L.fn = mode == 0 ? (p.dfloat ? cluster_ptr_dd() : cluster_ptr(dbl)) : cluster_bwd_ptr(dbl, p.dfloat);
     st = allow_max_smem(L.fn, dev, di.smem_optin);
     if (st != VQC_OK) return st;
     cudaLaunchConfig_t cfg{};
@@ -552,14 +562,25 @@ vqc_status plan_cluster(const HostPlan& p, int B, Launch& L) {
 // Larger clusters measured slower (0.7x at 16 qubits: one sample per cluster
 // leaves too few warps per SM to hide the per-stage cluster barriers), so they
 // run only when VQC_FORCE_PATH=cluster asks; VQC_FORCE_PATH=hbm turns it off.
+// The cluster backward (psi and lam over the cluster) follows the same rule:
+// by default for 2-CTA clusters (complex64 14 qubits, complex128 13), where it
+// measured 1-7% faster than the backward passes, and 0.78-0.90x with 4-8 CTAs
+// (0.80x on the 16-qubit / batch-512 workload); it also needs its shared-memory
+// layout (two slices, the per-warp rho partials, the tables) to fit one CTA.
 bool use_cluster(const HostPlan& p, int mode) {
-    if (mode != 0) return false;
-    const Schedule* s = find_cluster_schedule(p, 0);
+    const Schedule* s = find_cluster_schedule(p, mode);
     if (!s) return false;
     const char* f = std::getenv("VQC_FORCE_PATH");
-    if (f && std::string(f) == "cluster") return true;
+    const bool forced = f && std::string(f) == "cluster";
     if (f && std::string(f) == "hbm") return false;
-    return p.n - s->K - s->cta_bits == 1;
+    const bool two_cta = p.n - s->K - s->cta_bits == 1;
+    if (mode == 0) return forced || two_cta;
+    if (!forced && !two_cta) return false;
+    Launch L;
+    const std::string saved = g_err;
+    const bool ok = plan_cluster(p, 1, 1, L) == VQC_OK;
+    g_err = saved;
+    return ok;
 }
 
 template <typename R>
@@ -567,7 +588,7 @@ vqc_status run_cluster_forward(const HostPlan& p, int B, const void* x, const vo
                                const void* psi0, void* E, void* state_out, cudaStream_t stream) {
     using C = C2<R>;
     Launch L;
-    vqc_status st = plan_cluster(p, B, L);
+    vqc_status st = plan_cluster(p, 0, B, L);
     if (st != VQC_OK) return st;
     KArgs<R> a{};
     fill_plan_args<R>(p, L, a);
@@ -594,6 +615,64 @@ vqc_status run_cluster_forward(const HostPlan& p, int B, const void* x, const vo
     cfg.attrs = attr;
     cfg.numAttrs = env_int("VQC_PDL", 1) != 0 ? 2 : 1;
     VQC_CUDA(cudaLaunchKernelExC(&cfg, L.fn, args));
+    return VQC_OK;
+}
+
+// Workspace of a cluster backward: [0, 256) control block, then the per-cluster
+// dw partials [clusters, num_w].
+size_t cluster_bwd_workspace(const HostPlan& p, const Launch& L) {
+    const size_t rs = p.dtype == VQC_C128 ? 8 : 4;
+    return 256 + align256((size_t)(L.grid >> L.cl) * std::max(p.num_w, 1) * rs);
+}
+
+template <typename R>
+vqc_status run_cluster_backward(const HostPlan& p, int B, const void* x, const void* w,
+                                const void* psi0, const void* psi_final, const void* gE, void* dx,
+                                void* dw, void* ws, size_t ws_bytes, cudaStream_t stream) {
+    using C = C2<R>;
+    Launch L;
+    vqc_status st = plan_cluster(p, 1, B, L);
+    if (st != VQC_OK) return st;
+    const size_t need = cluster_bwd_workspace(p, L);
+    if (!ws || ws_bytes < need || misaligned(ws, 256))
+        return fail(VQC_ERR_WORKSPACE, "backward workspace must be >= " + std::to_string(need) +
+                                           " bytes and 256-byte aligned");
+    KArgs<R> a{};
+    fill_plan_args<R>(p, L, a);
+    a.B = B;
+    a.nunits = B;
+    a.x = static_cast<const R*>(x);
+    a.w = static_cast<const R*>(w);
+    a.psi0 = static_cast<const C*>(psi0);
+    a.psi_final = static_cast<const C*>(psi_final);
+    a.gE = static_cast<const R*>(gE);
+    a.dx = static_cast<R*>(dx);
+    a.dw = static_cast<R*>(dw);
+    a.counter = static_cast<unsigned*>(ws);
+    a.dw_part = reinterpret_cast<R*>(static_cast<char*>(ws) + 256);
+    void* args[] = {&a};
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1u << L.cl;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(L.grid);
+    cfg.blockDim = dim3(L.block);
+    cfg.dynamicSmemBytes = L.smem;
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = env_int("VQC_PDL", 1) != 0 ? 2 : 1;
+    VQC_CUDA(cudaLaunchKernelExC(&cfg, L.fn, args));
+    if (dw && p.num_w > 0) {
+        const R* part = a.dw_part;
+        int rows = L.grid >> L.cl, cols = p.num_w;
+        R* out = static_cast<R*>(dw);
+        void* rargs[] = {&part, &rows, &cols, &out};
+        VQC_CUDA(launch(reduce_cols_ptr(p.dtype == VQC_C128), dim3(cols), dim3(256), rargs, 0, stream));
+    }
     return VQC_OK;
 }
 
@@ -1021,11 +1100,18 @@ vqc_status backward_with_scratch(const vqc_plan* plan, int32_t batch, const void
     if (!grad_expz) return fail(VQC_ERR_INVALID_ARG, "grad_expz is NULL");
     st = check_out_ptrs(p, {grad_expz, grad_x, grad_w}, {});
     if (st != VQC_OK) return st;
-    // the same path choice as vqc_backward: resident when the batch fits a
-    // resident launch, else the HBM-tiled passes (their workspace layout)
-    const bool hbm = use_hbm(p, 1, batch);
+    // the same path choice as vqc_backward: the cluster backward when the
+    // environment asks for it, resident when the batch fits a resident launch,
+    // else the HBM-tiled passes (each with its own workspace layout)
+    const bool clu = use_cluster(p, 1);
+    const bool hbm = !clu && use_hbm(p, 1, batch);
     size_t need = 0;
-    if (hbm) {
+    if (clu) {
+        Launch L;
+        st = plan_cluster(p, 1, batch, L);
+        if (st != VQC_OK) return st;
+        need = cluster_bwd_workspace(p, L);
+    } else if (hbm) {
         PassGeo L;
         st = plan_hbm(p, 1, batch, L);
         if (st != VQC_OK) return st;
@@ -1041,6 +1127,13 @@ vqc_status backward_with_scratch(const vqc_plan* plan, int32_t batch, const void
                                            " bytes of scratch; the built-in scratch holds " +
                                            std::to_string(scratch_bytes));
     if (clear_control) VQC_CUDA(cudaMemsetAsync(scratch, 0, 256, s));
+    if (clu) {
+        if (p.dtype == VQC_C64)
+            return run_cluster_backward<float>(p, batch, x, w, psi0, psi_final, grad_expz, grad_x,
+                                               grad_w, scratch, scratch_bytes, s);
+        return run_cluster_backward<double>(p, batch, x, w, psi0, psi_final, grad_expz, grad_x,
+                                            grad_w, scratch, scratch_bytes, s);
+    }
     if (hbm) {
         if (p.dtype == VQC_C64)
             return run_hbm_backward<float>(p, batch, x, w, psi0, psi_final, grad_expz, grad_x,
@@ -1135,6 +1228,10 @@ size_t vqc_workspace_bytes(const vqc_plan* plan, int32_t batch, int32_t mode) {
                 need = std::max(need, bwd_workspace(p, L));
             }
         }
+        if (batch > 0 && use_cluster(p, 1)) {   // [either call's workspace | final states]
+            const size_t cs = p.dtype == VQC_C128 ? 16 : 8;
+            need = align256(need) + align256(((size_t)batch << p.n) * cs);
+        }
         g_err = saved;
         return need;
     }
@@ -1146,7 +1243,12 @@ size_t vqc_workspace_bytes(const vqc_plan* plan, int32_t batch, int32_t mode) {
     }
     if ((mode != 0 && mode != 1) || batch <= 0) return 0;
     const HostPlan& p = plan->hp;
-    if (use_cluster(p, mode)) return 0;
+    if (use_cluster(p, mode)) {
+        if (mode == 0) return 0;
+        Launch L;
+        if (plan_cluster(p, 1, batch, L) != VQC_OK) return 0;
+        return cluster_bwd_workspace(p, L);
+    }
     if (use_hbm(p, mode, batch)) {
         PassGeo L;
         if (plan_hbm(p, mode, batch, L) != VQC_OK) return 0;
@@ -1255,6 +1357,13 @@ vqc_status vqc_backward(const vqc_plan* plan, int32_t batch, const void* x, cons
         if (!grad_expz) return fail(VQC_ERR_INVALID_ARG, "grad_expz is NULL");
         st = check_out_ptrs(p, {grad_expz, grad_x, grad_w}, {});
         if (st != VQC_OK) return st;
+        if (use_cluster(p, 1)) {
+            if (p.dtype == VQC_C64)
+                return run_cluster_backward<float>(p, batch, x, w, psi0, psi_final, grad_expz, grad_x,
+                                                   grad_w, workspace, workspace_bytes, s);
+            return run_cluster_backward<double>(p, batch, x, w, psi0, psi_final, grad_expz, grad_x,
+                                                grad_w, workspace, workspace_bytes, s);
+        }
         if (use_hbm(p, 1, batch)) {
             if (p.dtype == VQC_C64)
                 return run_hbm_backward<float>(p, batch, x, w, psi0, psi_final, grad_expz, grad_x,
@@ -1313,6 +1422,21 @@ vqc_status vqc_forward_backward(const vqc_plan* plan, int32_t batch, const void*
                                   grad_w, workspace, workspace_bytes, s);
             return run<double>(p, 2, batch, x, w, psi0, nullptr, grad_expz, expz_out, nullptr, grad_x,
                                grad_w, workspace, workspace_bytes, s);
+        }
+        if (use_cluster(p, 1)) {
+            // the forward leaves the final states after the larger of the two calls'
+            // workspaces; the cluster backward starts from them
+            const size_t need = vqc_workspace_bytes(plan, batch, 3);
+            if (!workspace || workspace_bytes < need || misaligned(workspace, 256))
+                return fail(VQC_ERR_WORKSPACE, "workspace must be >= " + std::to_string(need) +
+                                                   " bytes and 256-byte aligned");
+            const size_t cs = p.dtype == VQC_C128 ? 16 : 8;
+            const size_t soff = need - align256(((size_t)batch << p.n) * cs);
+            void* psi_final = static_cast<char*>(workspace) + soff;
+            st = vqc_forward(plan, batch, x, w, psi0, expz_out, psi_final, workspace, soff, stream);
+            if (st != VQC_OK) return st;
+            return vqc_backward(plan, batch, x, w, psi0, psi_final, grad_expz, grad_x, grad_w, workspace,
+                                soff, stream);
         }
         // states beyond one SM: the forward (passes or cluster) leaves the final
         // states in the psi region of the backward's HBM layout, in this

@@ -656,19 +656,20 @@ vqc_status compile_host(const vqc_gate* gates, int32_t G, int32_t n, int32_t nx,
             p.scheds.push_back(std::move(s));
         }
     }
-    // Cluster schedules (forward): states up to 16 qubits over 2..8 CTAs of a
-    // thread-block cluster, one register block per thread (2^(n-K) threads) and
-    // at most 128 KiB of state per CTA.  CTAs of 512 threads (2^cta_bits):
-    // 256-thread CTAs, two clusters' CTAs per SM, measured 12% slower on the
-    // 16-qubit workload (more cross-CTA stages, wider cluster barriers).
-    {
-        const int K = max_k(0, dtype);
+    // Cluster schedules: states up to 16 qubits over 2..8 CTAs of a thread-block
+    // cluster, one register block per thread (2^(n-K) threads) and at most 128
+    // KiB of state per CTA (the backward holds psi and lam: two slices).  CTAs of
+    // 512 threads (2^cta_bits): 256-thread CTAs, two clusters' CTAs per SM,
+    // measured 12% slower on the 16-qubit forward (more cross-CTA stages, wider
+    // cluster barriers).
+    for (int mode = 0; mode < 2; ++mode) {
+        const int K = max_k(mode, dtype);
         const size_t cs = dtype == VQC_C128 ? 16 : 8;
         const int ctb = 9, cl = n - K - ctb;
-        if (n > resident_max_qubits(0, dtype) && n <= 16 && cl >= 1 && cl <= 3 &&
-            (((size_t)1 << (n - cl)) * cs) <= 128 * 1024) {
+        if (n > resident_max_qubits(mode, dtype) && n <= 16 && cl >= 1 && cl <= 3 &&
+            (((size_t)(mode + 1) << (n - cl)) * cs) <= 128 * 1024) {
             Schedule s;
-            s.mode = 0;
+            s.mode = mode;
             s.K = K;
             s.path = VQC_PATH_CLUSTER;
             s.cta_bits = ctb;

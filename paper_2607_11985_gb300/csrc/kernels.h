@@ -35,6 +35,7 @@ const void* reduce_dw_ptr(bool dbl);
 const void* reduce_cols_ptr(bool dbl);
 const void* abs2_ptr(bool dbl);   // |psi|^2, elementwise
 const void* cluster_ptr(bool dbl);   // cluster-path forward (K = 5 / 4 for complex64 / 128)
+const void* cluster_bwd_ptr(bool dbl, bool dfloat);   // cluster-path backward (K = 4 / 3)
 
 // Largest block (threads) each instantiation is compiled for.
 inline int sweep_max_threads(bool is_double, int mode, int K) {

@@ -483,15 +483,36 @@ def hbm_passes(L, s):
             break
 
 
+def cluster_locality(st, K, n, cl):
+    """cl_local of a cluster-schedule stage, by enumerating every (thread,
+    register) slot of both maps: bit 0 (loads) / bit 1 (stores) when each slot
+    lies in the slice of the CTA whose rank is the thread's top cl index bits
+    (slices of 2^(n - cl) slots, in rank order)."""
+    nb = int(st["nthreadbits"])
+    t = np.arange(1 << nb, dtype=np.int64)
+    r = np.arange(1 << K, dtype=np.int64)
+    flags = 0
+    for bit, (sig, tau) in enumerate((("sigma", "tau"), ("sigma_st", "tau_st"))):
+        base = np.zeros_like(t)
+        for i in range(nb):
+            base ^= np.where((t >> i) & 1, int(st[tau][i]), 0)
+        off = np.zeros_like(r)
+        for j in range(K):
+            off ^= np.where((r >> j) & 1, int(st[sig][j]), 0)
+        slots = base[:, None] ^ off[None, :]
+        if np.all((slots >> (n - cl)) == (t >> (nb - cl))[:, None]):
+            flags |= 1 << bit
+    return flags
+
+
 def schedules(L):
-    """Resident schedules for every usable (mode, K), then HBM passes (cluster
-    schedules exist only for 15-16-qubit states and are not built here)."""
+    """Resident schedules for every usable (mode, K), cluster schedules (one
+    sample over 2-8 CTAs of 512 threads), then HBM passes."""
     c64 = L.dtype == C64
     max_k = {(0, True): 5, (1, True): 4, (0, False): 4, (1, False): 3}
     res_max = {(0, True): 14, (1, True): 13, (0, False): 13, (1, False): 12}
     tile_q = {(0, True): 13, (1, True): 12, (0, False): 12, (1, False): 11}
     n = L.n
-    assert n <= 14, "golden plans cover states below the cluster range"
     out = []
     for mode in (0, 1):
         for K in range(1, min(max_k[mode, c64], n) + 1):
@@ -500,6 +521,20 @@ def schedules(L):
             s = Schedule(mode, K, n, 0)
             cut_stages(L, range(len(L.ops)), list(range(n)), K, s,
                        {i: e["slot"] for i, e in enumerate(L.entries)}, {i: i for i in range(len(L.accs))})
+            out.append(s)
+    for mode in (0, 1):
+        # one register block per thread, 512-thread CTAs, <= 128 KiB of state
+        # (psi, and lam for the backward) per CTA
+        K = max_k[mode, c64]
+        cl = n - K - 9
+        if n > res_max[mode, c64] and n <= 16 and 1 <= cl <= 3 and \
+                ((mode + 1) << (n - cl)) * (8 if c64 else 16) <= 128 * 1024:
+            s = Schedule(mode, K, n, 2)
+            s.cta_bits = 9
+            cut_stages(L, range(len(L.ops)), list(range(n)), K, s,
+                       {i: e["slot"] for i, e in enumerate(L.entries)}, {i: i for i in range(len(L.accs))})
+            for st in s.stages:
+                st["cl_local"] = cluster_locality(st, K, n, cl)
             out.append(s)
     for mode in (0, 1):
         m = min(tile_q[mode, c64], n - 1)

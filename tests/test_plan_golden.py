@@ -43,6 +43,22 @@ def test_workload_plans(cfg, dtype):
     assert_same(wl.config(cfg, dtype=dtype)[0].spec, dtype)
 
 
+@pytest.mark.parametrize("dtype", ["c64", "c128"])
+def test_sixteen_qubit_workload_plan(dtype):
+    """Cluster schedules (forward and backward, with their CTA-locality flags)
+    and the HBM passes of the 16-qubit / 8-layer workload."""
+    assert_same(wl.config(5, dtype=dtype)[0].spec, dtype)
+
+
+@pytest.mark.parametrize("n,dtype", [(13, "c128"), (14, "c64"), (14, "c128"), (15, "c64"), (15, "c128")])
+def test_cluster_range_plans(n, dtype):
+    """Every state size with a cluster schedule, on a layered circuit with a
+    CX ring, a CZ and a phase gate."""
+    spec = wl.layered(n, 2, ("RX", "RY"), "CX")
+    spec.add("CZ", (0, n - 1)).add("RZZ", (2, n - 2), [("w", 0)]).add("CRZ", (n - 1, 1), [("x", 0)])
+    assert_same(spec, dtype)
+
+
 def test_random_circuit_workload_plans():
     for w_ in wl.config(4)[::4]:
         assert_same(w_.spec, "c64")
