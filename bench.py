@@ -611,8 +611,9 @@ def run_ours(args, rank, world, local_rank):
                                          "fwd_bound": r["roofline"]["fwd"]["bound"]}
         out["configs"] = subs
     if not args.no_subrecords:
-        out["f4_tensor_core_stage"] = tc_stage_measurement(torch, torch.empty(256 << 20, dtype=torch.uint8,
-                                                                              device="cuda"), torch.cuda.current_stream())
+        flush_buf = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+        out["f4_tensor_core_stage"] = tc_stage_measurement(torch, flush_buf, torch.cuda.current_stream())
+        out["cluster_vs_passes"] = cluster_measurement(torch, flush_buf, torch.cuda.current_stream())
     if args.ablation:
         out["ablation"] = ablation(torch, wl_config(2))
     if args.regime:
@@ -652,6 +653,51 @@ def tc_stage_measurement(torch, flush, stream, repeats=32, n=16, batch=512):
     res["tc_over_fp32_speedup"] = res["fp32_cores"]["ms_per_application"] / res["tcgen05_tf32x3"]["ms_per_application"]
     res["max_abs_diff_after_%d" % repeats] = float((outs["fp32_cores"] - outs["tcgen05_tf32x3"]).abs().max())
     res["workload"] = "%d-qubit states x %d, %d applications on chip per call" % (n, batch, repeats)
+    return res
+
+
+def cluster_measurement(torch, flush, stream, n_calls=3):
+    """The thread-block-cluster path against the HBM-tiled passes on the same
+    batch (VQC_FORCE_PATH), complex64: forward (final states saved) and backward
+    from them, device time per call; the 16-qubit / 8-layer workload and
+    layered 8-layer circuits at 14 and 15 qubits (batch 128)."""
+    import os
+    from paper_2607_11985_gb300.circuit import Circuit
+    from paper_2607_11985_gb300 import workloads as wl
+    paths = {0: "resident", 1: "hbm-tiled", 2: "cluster"}
+    cases = [("16q_8L_B512 (the timed workload)", wl_config(5).spec, 512)]
+    for n in (14, 15):
+        cases.append(("%dq_8L_B128" % n, wl.layered(n, 8, ("RX", "RY", "RZ"), "CX"), 128))
+    saved = os.environ.get("VQC_FORCE_PATH")
+    res = {}
+    try:
+        for name, spec, B in cases:
+            rng = np.random.default_rng(7)
+            x = torch.tensor(rng.uniform(-np.pi, np.pi, (B, spec.num_x)), dtype=torch.float32, device="cuda")
+            w = torch.tensor(rng.uniform(-np.pi, np.pi, spec.num_w), dtype=torch.float32, device="cuda")
+            gE = torch.tensor(rng.standard_normal((B, spec.n)), dtype=torch.float32, device="cuda")
+            r = {}
+            for force in ("hbm", "cluster"):
+                os.environ["VQC_FORCE_PATH"] = force
+                c = Circuit(spec, "c64")
+                inf = c.info(B)
+                E, st = c.forward(x, w, want_state=True)
+                dx, dw = c.backward(x, w, gE, psi_final=st)
+                f = statistics.median(time_calls(torch, lambda: c.forward(x, w, out=E, state_out=st),
+                                                 n_calls, flush, stream))
+                b = statistics.median(time_calls(torch, lambda: c.backward(x, w, gE, psi_final=st, grad_x=dx,
+                                                                           grad_w=dw), n_calls, flush, stream))
+                r[force] = {"fwd_ms": f, "bwd_ms": b, "path_fwd_bwd": [paths[inf["fwd_path"]], paths[inf["bwd_path"]]],
+                            "dw": dw.double()}
+                del c, E, st
+            r["dw_max_abs_diff"] = float((r["hbm"].pop("dw") - r["cluster"].pop("dw")).abs().max())
+            r["cluster_over_passes_speedup"] = {k: r["hbm"][k + "_ms"] / r["cluster"][k + "_ms"] for k in ("fwd", "bwd")}
+            res[name] = r
+    finally:
+        if saved is None:
+            os.environ.pop("VQC_FORCE_PATH", None)
+        else:
+            os.environ["VQC_FORCE_PATH"] = saved
     return res
 
 
