@@ -7,8 +7,9 @@ a fixed device-memory budget): it takes no workspace and uses scratch built
 into the library instead.  It runs the same kernels with the same fixed-order
 reductions as the workspace entry point, so its gradients must be bit-identical
 to those of vqc_backward, on two calls in a row (the second call finds the first
-call's leftovers in the shared scratch): on the resident path and on the
-HBM-tiled passes (15 qubits), from a saved final state and recomputing it.  A
+call's leftovers in the shared scratch): on the resident path, on the
+HBM-tiled passes (15 qubits) and on the thread-block-cluster backward (14
+qubits), from a saved final state and recomputing it.  A
 batch whose scratch need exceeds the built-in size must be rejected with
 VQC_ERR_WORKSPACE.
 
@@ -93,6 +94,29 @@ def test_noalloc_backward_hbm_passes(saved_state):
     x = torch.tensor(rng.uniform(-3, 3, (1, 15)), dtype=torch.float32, device="cuda")
     w = torch.tensor(rng.uniform(-3, 3, spec.num_w), dtype=torch.float32, device="cuda")
     gE = torch.tensor(rng.standard_normal((1, 15)), dtype=torch.float32, device="cuda")
+    st = c.forward(x, w, want_state=True)[1] if saved_state else None
+    dx_ref, dw_ref = _workspace_backward(B, c, x, w, gE, st)
+    for _ in range(2):
+        dx, dw = _noalloc_backward(B, c, x, w, gE, st)
+        torch.cuda.synchronize()
+        assert torch.isfinite(dx).all() and torch.isfinite(dw).all()
+        assert torch.equal(dx, dx_ref) and torch.equal(dw, dw_ref)
+
+
+@pytest.mark.parametrize("saved_state", [True, False])
+def test_noalloc_backward_cluster(saved_state):
+    # 14 qubits complex64: the backward runs on 2-CTA thread-block clusters; the
+    # built-in scratch holds its per-cluster dw partials
+    from paper_2607_11985_gb300 import binding as B
+    from paper_2607_11985_gb300.circuit import Circuit
+    spec = wl.layered(14, 2, ("RX", "RY", "RZ"), "CX")
+    rng = np.random.default_rng(1414)
+    b = 40
+    c = Circuit(spec, "c64")
+    assert c.info(b)["bwd_path"] == 2
+    x = torch.tensor(rng.uniform(-3, 3, (b, 14)), dtype=torch.float32, device="cuda")
+    w = torch.tensor(rng.uniform(-3, 3, spec.num_w), dtype=torch.float32, device="cuda")
+    gE = torch.tensor(rng.standard_normal((b, 14)), dtype=torch.float32, device="cuda")
     st = c.forward(x, w, want_state=True)[1] if saved_state else None
     dx_ref, dw_ref = _workspace_backward(B, c, x, w, gE, st)
     for _ in range(2):
