@@ -7,6 +7,7 @@ way) against the oracle and against the device-memory calls.
 * forward only (no gE), complex128, a batch that grows and shrinks (the arena
   is reallocated and its workspaces re-initialised), batch 0;
 * a 16-qubit circuit on the HBM-tiled path (both workspaces in the arena);
+* a 14-qubit circuit whose backward runs on thread-block clusters;
 * argument errors.
 """
 import numpy as np
@@ -113,6 +114,31 @@ def test_hbm_path_circuit(access):
     assert np.array_equal(E, E_d) and np.array_equal(dx, dx_d) and np.array_equal(dw, dw_d)
     E_ref = orc.forward(spec, x.astype(np.float64), w.astype(np.float64))
     assert maxerr(E, E_ref) <= TOL["c64"]["E"]
+
+
+def test_cluster_backward_circuit(access):
+    """14 qubits complex64: resident forward, backward on 2-CTA thread-block
+    clusters (the final states in the arena's workspace); three calls, so the
+    later ones replay the captured graph."""
+    n = 14
+    spec = wl.layered(n, 2, ("RX", "RY", "RZ"), "CX", ring_range=lambda l: 2 * l + 1)
+    rng = np.random.default_rng(1414)
+    b = 5
+    x = rng.uniform(-np.pi, np.pi, (b, n)).astype(np.float32)
+    w = rng.uniform(-np.pi, np.pi, spec.num_w).astype(np.float32)
+    gE = rng.standard_normal((b, n)).astype(np.float32)
+    c = C(spec, "c64")
+    info = c.info(b)
+    assert info["fwd_path"] == 0 and info["bwd_path"] == 2
+    w_ = wl.Workload("cluster14", spec, b, x.astype(np.float64), w.astype(np.float64),
+                     gE.astype(np.float64), "c64", 1414)
+    E_d, st = run_fwd(c, w_)
+    dx_d, dw_d = run_bwd(c, w_, psi_final=torch.tensor(st, device="cuda"))
+    for _ in range(3):
+        E, dx, dw = c.evaluate_host(x, w, gE)
+        assert np.array_equal(E, E_d) and np.array_equal(dx, dx_d) and np.array_equal(dw, dw_d)
+    dx_ref, dw_ref = orc.backward(spec, x.astype(np.float64), w.astype(np.float64), gE.astype(np.float64))
+    assert maxerr(dx, dx_ref) <= TOL["c64"]["grad"] and maxerr(dw, dw_ref) <= TOL["c64"]["grad"]
 
 
 def test_argument_errors():
