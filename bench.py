@@ -404,6 +404,8 @@ def measure_workload(torch, ws_list, steps, warmup, flush, stream, fma, pk, pk_k
                         "call": "vqc_forward_backward (gE known before the call)"}
         rec["time_stats_ms"]["bwd"] = stats([sum(t) for t in zip(*bwd_ms)])
         rec["time_stats_ms"]["fused"] = stats([sum(t) for t in zip(*fused_ms)])
+    if len(benches) > 1:
+        rec["concurrent"] = concurrent_steps(torch, benches, steps, flush, stream, world, evals)
     parts = [(b.info, b.Bt, statistics.mean(f) / 1e3,
               statistics.mean(bw) / 1e3 if has_bwd else None)
              for b, f, bw in zip(benches, fwd_ms, bwd_ms if has_bwd else [None] * len(benches))]
@@ -414,6 +416,43 @@ def measure_workload(torch, ws_list, steps, warmup, flush, stream, fma, pk, pk_k
         rec["cpu_baseline"] = cpu_baseline(ws_list, cpu_seconds, has_bwd)
     rec["_benches"] = benches
     return rec
+
+
+def concurrent_steps(torch, benches, steps, flush, stream, world, evals, nstreams=8):
+    """A workload of several independent circuits with their steps issued on
+    `nstreams` streams at once (each circuit on its own buffers; fork and join
+    through events on the launch stream), so that small launches share the
+    GPU: device time per step, L2 flushed before each."""
+    streams = [torch.cuda.Stream() for _ in range(nstreams)]
+    saved = [b.sp for b in benches]
+    ms = []
+    try:
+        for j, b in enumerate(benches):
+            b.sp = streams[j % nstreams].cuda_stream
+        for i in range(steps + 2):
+            flush.zero_()
+            a = torch.cuda.Event(enable_timing=True)
+            e = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for st in streams:
+                st.wait_event(a)
+            for b in benches:
+                b.step()
+            for st in streams:
+                j = torch.cuda.Event()
+                j.record(st)
+                stream.wait_event(j)
+            e.record(stream)
+            torch.cuda.synchronize()
+            if i >= 2:
+                ms.append(a.elapsed_time(e))
+    finally:
+        for b, sp in zip(benches, saved):
+            b.sp = sp
+    t = statistics.mean(ms)
+    return {"value": world * evals / (t / 1e3), "ms_per_step": t, "streams": nstreams,
+            "unit": "circuit evals/s (%s)" % ("fwd+adjoint bwd" if benches[0].w_.backward else "fwd"),
+            "basis": "every circuit's step issued on %d streams at once (2 untimed rounds first)" % nstreams}
 
 
 def e2e_rate(torch, benches, steps, stream, world):
@@ -576,6 +615,7 @@ def run_ours(args, rank, world, local_rank):
         "fwd": rec["fwd"],
         "bwd": rec.get("bwd"),
         "fused": rec.get("fused"),
+        "concurrent": rec.get("concurrent"),
         "time_stats_ms": rec["time_stats_ms"],
         "roofline": {"kernel": kernel_name(info, args.dtype, dom), "bound": rl["bound"],
                      "achieved": main["achieved"], "peak": main["peak"], "unit": main["unit"],
