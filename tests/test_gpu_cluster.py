@@ -8,7 +8,9 @@ psi and lam of one sample spread over the shared memory of 2, 4 or 8 CTAs.
   forward + backward; a batch larger than the resident clusters (each cluster
   takes several samples);
 * the 16-qubit / 8-layer complex64 workload at its full batch (512 rows): dx
-  and dw of every row against the batch-parallel oracle.
+  and dw of every row against the batch-parallel oracle;
+* a circuit whose accumulators do not fit beside the two slices falls back to
+  the HBM passes.
 """
 import numpy as np
 import pytest
@@ -116,3 +118,24 @@ def test_config5_cluster_backward_full_batch(monkeypatch):
     report(w_.name + "_cluster", **errs)
     for k, v in errs.items():
         assert v <= TOL["c64"]["grad"], (k, v)
+
+
+def test_cluster_backward_falls_back_when_accumulators_do_not_fit(monkeypatch):
+    """A deep 14-qubit circuit (420 parametrised runs): the cluster backward's
+    per-warp rho partials would not fit one CTA's shared memory next to psi and
+    lam, so the backward takes the HBM passes, by default and when the cluster
+    is asked for; its gradients still match the oracle."""
+    n = 14
+    spec = wl.layered(n, 30, ("RX", "RY"), "CX")
+    rng = np.random.default_rng(3014)
+    B = 2
+    w_ = wl.Workload("deep_n14", spec, B, wl._round(rng.uniform(-np.pi, np.pi, (B, n)), "c64"),
+                     wl._round(rng.uniform(-np.pi, np.pi, spec.num_w), "c64"),
+                     wl._round(rng.standard_normal((B, n)), "c64"), "c64", 3014)
+    c = C(spec, "c64")
+    assert c.info(B)["bwd_path"] == 1
+    monkeypatch.setenv("VQC_FORCE_PATH", "cluster")
+    assert c.info(B)["bwd_path"] == 1
+    dx, dw = run_bwd(c, w_)
+    dx_ref, dw_ref = orc.backward(spec, w_.x, w_.w, w_.gE)
+    assert maxerr(dx, dx_ref) <= TOL["c64"]["grad"] and maxerr(dw, dw_ref) <= TOL["c64"]["grad"]
