@@ -1,7 +1,8 @@
-// cluster.cuh -- forward sweep with a sample's state spread over a thread-block
-// cluster (distributed shared memory), for states larger than one SM's shared
-// memory but small enough for 2..8 SMs (complex64: 15-17 qubits, complex128:
-// 14-16 qubits).
+// cluster.cuh -- forward and backward sweeps with a sample's state (forward) or
+// its psi and lam (backward) spread over a thread-block cluster (distributed
+// shared memory), for states larger than one SM's shared memory but small
+// enough for 2..8 SMs (forward: complex64 15-16 qubits, complex128 14-16;
+// backward: complex64 14-16, complex128 13-15).
 //
 // Same stage program as the resident path (sweep.cuh): the stage maps give
 // every register amplitude a slot in [0, 2^n); slot s lives in the shared memory
@@ -11,9 +12,11 @@
 // the cluster window (mapa + ld/st.shared::cluster); a cluster barrier replaces
 // the group barrier between stages.  A stage whose maps keep every block inside
 // its thread's own CTA (the compiler's cl_local flags) uses plain shared loads
-// and stores and, when no data crosses CTAs at its end, the CTA barrier.  One sample per cluster at a time; the
-// 2^(n-K) threads of its group are spread over the cluster's CTAs in rank
-// order.  The <Z> sums go from each CTA to rank 0, which writes E.
+// and stores and, when no data crosses CTAs at its end, the CTA barrier.  One
+// sample per cluster at a time; the 2^(n-K) threads of its group are spread
+// over the cluster's CTAs in rank order.  The forward's <Z> sums go from each
+// CTA to rank 0, which writes E; the backward's rho sums likewise (rank 0
+// writes dx and the cluster's dw partial).
 #pragma once
 
 #include "sweep.cuh"

@@ -110,12 +110,11 @@ template <> struct VecSel<dd, true> { using t = Vec16Raw; };
 // and of k, and both the index deposit into global qubits and the swizzle are
 // linear in those fields, so each is a per-thread part XOR a per-k part
 // (tabulated once per pass in shared memory: koff[k] = (global, slot)).
-template <typename R, bool RAW = false>
+template <typename R, bool RAW = false, int U = 8>
 __device__ __forceinline__ void tile_gather(C2<R>* sm, const SC2<R>* gs, uint32_t gt, uint32_t st,
                                             const uint2* koff, int nk, int T, int t) {
     using V = typename VecSel<R, RAW>::t;
     constexpr int APV = 16 / sizeof(C2<R>);
-    constexpr int U = 8;
     int k = 0;
     for (; k + U <= nk; k += U) {
         V v[U];
@@ -149,6 +148,18 @@ __device__ __forceinline__ void tile_scatter(const C2<R>* sm, SC2<R>* gs, uint32
         for (int e = 0; e < APV; ++e) v.a[e] = sm[sl ^ e];
         v.st(gs + (gt | koff[k].x));
     }
+}
+
+// Bring a tile's 128-byte lines into L2 ahead of its gather (a hint: no result,
+// no wait).  With T >= 8 (every production tile) vectors t .. t+7 of one k
+// share a line, so every eighth thread takes the lines; smaller groups touch
+// some lines more than once.
+template <typename R>
+__device__ __forceinline__ void tile_prefetch(const SC2<R>* gs, uint32_t gt, const uint2* koff, int nk,
+                                              int t) {
+    if (t & 7) return;
+    for (int k = 0; k < nk; ++k)
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(gs + (gt | koff[k].x)));
 }
 
 // FULL: tile groups span whole warps (2^(m-K) >= 32 threads; every production
@@ -254,11 +265,23 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
         const uint32_t gt = tile_global(u_t, tile_base, A.tile_q, G);
         if (A.src_psi) {
             if (DDK && A.src_raw) tile_gather<R, DDK>(psi, A.src_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
-            else tile_gather<R>(psi, A.src_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
+            else   // 16 loads in flight where one state is gathered, 8 beside lam's registers
+                tile_gather<R, false, MODE == 0 ? 16 : 8>(psi, A.src_psi + sbase, gt, st_t, koff, nk, q.T, q.t);
         }
         if (MODE == 1 && A.src_lam) {
             if (DDK && A.lam_raw) tile_gather<R, DDK>(lam, A.src_lam + sbase, gt, st_t, koff, nk, q.T, q.t);
             else tile_gather<R>(lam, A.src_lam + sbase, gt, st_t, koff, nk, q.T, q.t);
+        }
+        if (unit + gridDim.x < A.nunits) {   // the CTA's next tile into L2 during this one's stages
+            const long long nt = min((unit + gridDim.x) * A.S + q.g, total_tiles - 1);
+            const int nb = (int)(nt / A.ntiles), ntau = (int)(nt % A.ntiles);
+            uint32_t nbase = 0;
+            for (int j = 0; j < A.nout; ++j)
+                if ((ntau >> j) & 1) nbase |= 1u << A.out_q[j];
+            const uint32_t ngt = tile_global(u_t, nbase, A.tile_q, G);
+            const size_t nsb = (size_t)nb << n;
+            if (A.src_psi) tile_prefetch<R>(A.src_psi + nsb, ngt, koff, nk, q.t);
+            if (MODE == 1 && A.src_lam) tile_prefetch<R>(A.src_lam + nsb, ngt, koff, nk, q.t);
         }
         __syncthreads();
 
