@@ -792,7 +792,7 @@ void forget_plan(const HostPlan* p) {
 // Workspace of the HBM path.  Forward: [control | working state | <Z> partials].
 // Backward: [control | psi | lam | gradient-term partials].
 struct HbmWs {
-    size_t state = 0, lam = 0, part = 0, total = 0;
+    size_t state = 0, lam = 0, part = 0, terms = 0, total = 0;
 };
 
 HbmWs hbm_layout(const HostPlan& p, int mode, int B, int ntiles) {
@@ -803,10 +803,11 @@ HbmWs hbm_layout(const HostPlan& p, int mode, int B, int ntiles) {
     if (mode == 0) {
         w.part = w.state + sbytes;
         w.total = w.part + align256((size_t)B * ntiles * p.n * rs);
-    } else {
+    } else {   // per-tile rho sums [B * ntiles][accs][4], then the per-sample terms [B][terms]
         w.lam = w.state + sbytes;
         w.part = w.lam + sbytes;
-        w.total = w.part + align256((size_t)B * ntiles * std::max<size_t>(p.term_src.size(), 1) * rs);
+        w.terms = w.part + align256((size_t)B * ntiles * std::max<size_t>(p.accs.size(), 1) * 4 * rs);
+        w.total = w.terms + align256((size_t)B * std::max<size_t>(p.term_src.size(), 1) * rs);
     }
     return w;
 }
@@ -840,7 +841,7 @@ void fill_pass_args(const HostPlan& p, const PassGeo& L, const DPass& ps, PArgs<
     a.sh_count = ps.sh_count;
     a.acc_begin = ps.acc_begin;
     a.acc_count = ps.acc_count;
-    a.n_terms = (int)p.term_src.size();
+    a.n_accs = (int)p.accs.size();
     a.Px = p.num_x;
     a.nunits = L.nunits;
     for (int i = 0; i < 24; ++i) {
@@ -920,7 +921,8 @@ vqc_status run_hbm_backward(const HostPlan& p, int B, const void* x, const void*
     char* wsc = static_cast<char*>(ws);
     C* Psi = reinterpret_cast<C*>(wsc + lay.state);
     C* Lam = reinterpret_cast<C*>(wsc + lay.lam);
-    R* terms = reinterpret_cast<R*>(wsc + lay.part);
+    R* rho = reinterpret_cast<R*>(wsc + lay.part);
+    R* terms = reinterpret_cast<R*>(wsc + lay.terms);
     const C* src0 = static_cast<const C*>(psi_final);
     if (!src0) {
         // recompute the final state into Psi (the forward passes need no <Z>)
@@ -959,16 +961,33 @@ vqc_status run_hbm_backward(const HostPlan& p, int B, const void* x, const void*
         a.src_raw = first ? psi_final == nullptr : 1;   // recomputed states are raw
         a.lam_raw = 1;
         a.dst_raw = 1;
-        a.terms = terms;
+        a.rho = rho;
         void* args[] = {&a};
         VQC_CUDA(launch(L.fn, dim3(L.grid), dim3(L.block), args, L.smem, stream));
     }
     const char* base = static_cast<const char*>(p.dbuf);
     const bool dbl = p.dtype == VQC_C128;
     int nt = (int)p.term_src.size();
+    const bool want = (dx && p.num_x > 0) || (dw && p.num_w > 0);
+    if (want && !p.accs.empty()) {   // per-sample gradient terms from the per-tile rho sums
+        const R* r = rho;
+        int Bi = B, ntl = L.ntiles, na = (int)p.accs.size(), Px = p.num_x;
+        const DAcc* accs = reinterpret_cast<const DAcc*>(base + p.dev_accs);
+        const DEntry* entries = reinterpret_cast<const DEntry*>(base + p.dev_entries);
+        const DConst* consts = reinterpret_cast<const DConst*>(base + p.dev_consts);
+        const R* cang = reinterpret_cast<const R*>(base + p.dev_cang);
+        const R* cmat = reinterpret_cast<const R*>(base + p.dev_cmat);
+        const R* xr = static_cast<const R*>(x);
+        const R* wr = static_cast<const R*>(w);
+        R* o = terms;
+        void* args[] = {&r, &Bi, &ntl, &na, &accs, &entries, &consts, &cang, &cmat, &xr, &Px, &wr, &nt, &o};
+        const int blocks = (int)std::min<long long>(4096, ((long long)B * na + 255) / 256);
+        VQC_CUDA(launch(p.dfloat ? reduce_terms_ptr_dd() : reduce_terms_ptr(dbl), dim3(std::max(blocks, 1)),
+                        dim3(256), args, 0, stream));
+    }
     if (dx && p.num_x > 0) {
         const R* t = terms;
-        int Bi = B, ntl = L.ntiles, Px = p.num_x;
+        int Bi = B, ntl = 1, Px = p.num_x;
         const int32_t* ptr = reinterpret_cast<const int32_t*>(base + p.dev_xocc_ptr);
         const int32_t* occ = reinterpret_cast<const int32_t*>(base + p.dev_xocc);
         R* o = static_cast<R*>(dx);
@@ -979,7 +998,7 @@ vqc_status run_hbm_backward(const HostPlan& p, int B, const void* x, const void*
     }
     if (dw && p.num_w > 0) {
         const R* t = terms;
-        long long rows = (long long)B * L.ntiles;
+        long long rows = B;
         const int32_t* ptr = reinterpret_cast<const int32_t*>(base + p.dev_wocc_ptr);
         const int32_t* occ = reinterpret_cast<const int32_t*>(base + p.dev_wocc);
         R* o = static_cast<R*>(dw);

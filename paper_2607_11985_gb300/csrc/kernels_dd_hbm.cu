@@ -1,6 +1,6 @@
 // kernels_dd_hbm.cu -- double-float (complex128 storage) instantiations of the
-// HBM-tiled pass kernels (K = 4 forward, 3 backward, as complex128) and of the
-// cluster-path forward (K = 4).
+// HBM-tiled pass kernels (K = 4 forward, 3 backward, as complex128), of the
+// per-sample gradient-term reduction and of the cluster-path forward (K = 4).
 #include "cluster.cuh"
 #include "kernels.h"
 #include "pass.cuh"
@@ -16,5 +16,6 @@ const void* pass_ptr_dd(int mode, int K, bool full) {
 }
 
 const void* cluster_ptr_dd() { return reinterpret_cast<const void*>(&cluster_fwd_kernel<dd, 4>); }
+const void* reduce_terms_ptr_dd() { return reinterpret_cast<const void*>(&reduce_terms<dd>); }
 
 }  // namespace vqc

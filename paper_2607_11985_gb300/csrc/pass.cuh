@@ -8,8 +8,10 @@
 // One launch per pass: each CTA loads S tiles (the other n - m qubits fix the
 // tile), runs the pass's register-block stages on them in shared memory
 // exactly as the resident path does, and writes them back.  The forward's last
-// pass emits per-tile <Z> partials; the backward emits per-tile gradient
-// terms.  reduce_* kernels sum partials in a fixed order (deterministic).
+// pass emits per-tile <Z> partials; the backward emits per-tile rho sums of
+// the pass's accumulators, which reduce_terms adds up per sample and turns into
+// gradient terms.  reduce_* kernels sum partials in a fixed order
+// (deterministic).
 #pragma once
 
 #include "sweep.cuh"
@@ -30,7 +32,7 @@ struct PArgs {
     const DAcc* accs;
     int n, m, K, tbits, G, S, nout, ntiles;
     int stage_begin, stage_end;
-    int ps_begin, ps_count, sh_begin, sh_count, acc_begin, acc_count, n_terms, Px;
+    int ps_begin, ps_count, sh_begin, sh_count, acc_begin, acc_count, n_accs, Px;
     int B;
     long long nunits;
     uint8_t tile_q[24], out_q[24];
@@ -42,7 +44,7 @@ struct PArgs {
     const C2<R>* src_lam;   // backward: lam tiles (nullptr: lam = O psi in the first stage)
     C2<R>* dst_lam;
     R* E_part;              // forward, last pass: [B * ntiles, n]
-    R* terms;               // backward: [B * ntiles, n_terms]
+    R* rho;                 // backward: per-tile rho sums [B * ntiles][n_accs][4] (3 used)
     int sm_sh, sm_ps, sm_psi, sm_lam, sm_acc, sm_red;
     const unsigned char* plan;   // plan regions copied to shared memory (see KArgs)
     int tab_off, tab_bytes, sched_off, sched_bytes, sm_plan, plan_smem;
@@ -200,7 +202,6 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
         rebase(reinterpret_cast<const unsigned char*>(A.cmat), A.plan, A.tab_off, smt));
     const R* P_cang = reinterpret_cast<const R*>(
         rebase(reinterpret_cast<const unsigned char*>(A.cang), A.plan, A.tab_off, smt));
-    const DAcc* P_accs = rebase(A.accs, A.plan, A.tab_off, smt);
     if (A.plan_smem) __syncthreads();
 
     const int n = A.n, G = A.G, tdim = 1 << A.m;
@@ -366,15 +367,16 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
                 tile_scatter<R>(lam, A.dst_lam + sbase, gt, st_t, koff, nk, q.T, q.t);
             }
         }
-        for (int i = threadIdx.x; i < A.S * A.acc_count; i += nthr) {
-            const int gg = i / A.acc_count, k = i % A.acc_count;
+        // the tile's rho sums (warps in order), in parallel over accumulators and
+        // components; the per-sample turn into terms is reduce_terms' work
+        for (int i = threadIdx.x; i < A.S * A.acc_count * 3; i += nthr) {
+            const int gg = i / (A.acc_count * 3), r = i % (A.acc_count * 3), k = r / 3, c = r % 3;
             const long long tt = unit * A.S + gg;
             if (tt >= total_tiles) continue;
-            const int bb = (int)(tt / A.ntiles);
-            const DAcc ac = P_accs[vqc_ld(&P_pass_accs[A.acc_begin + k])];
-            acc_terms<R>(ac, P_entries[ac.entry], acc_all + ((size_t)gg * A.acc_count + k) * q.wg * 8,
-                         q.wg, P_consts, A.x ? A.x + (size_t)bb * A.Px : static_cast<const St<R>*>(nullptr), A.w, P_cang,
-                         P_cmat, A.terms + tt * A.n_terms);
+            const R* ap = acc_all + ((size_t)gg * A.acc_count + k) * q.wg * 8 + c;
+            R sum = 0;
+            for (int wi = 0; wi < q.wg; ++wi) sum += ap[wi * 8];
+            A.rho[((size_t)tt * A.n_accs + vqc_ld(&P_pass_accs[A.acc_begin + k])) * 4 + c] = as_out<St<R>>(sum);
         }
         __syncthreads();
     }
@@ -391,6 +393,35 @@ __global__ void reduce_expz(const R* E_part, int B, int ntiles, int n, R* E) {
         R s = 0;
         for (int t = 0; t < ntiles; ++t) s += E_part[(b * ntiles + t) * n + j];
         E[i] = s;
+    }
+}
+
+// Gradient terms of every accumulator of every sample: the sample's per-tile
+// rho sums added in tile order, then the constituent walk of acc_terms (one
+// partial), in the kernels' arithmetic R (the plan's constants are stored as R:
+// (hi, lo) float pairs for double-float plans).  terms: [B, n_terms].
+template <typename R>
+__global__ void __launch_bounds__(256) reduce_terms(const St<R>* rho, int B, int ntiles, int n_accs,
+                                                    const DAcc* accs, const DEntry* entries,
+                                                    const DConst* consts, const R* cang, const R* cmat,
+                                                    const St<R>* x, int Px, const St<R>* w, int n_terms,
+                                                    St<R>* terms) {
+    grid_dep_wait();
+    grid_dep_launch();
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < (long long)B * n_accs;
+         i += (long long)gridDim.x * blockDim.x) {
+        const long long b = i / n_accs;
+        const int k = (int)(i % n_accs);
+        R t[4] = {0, 0, 0, 0};
+        for (int tau = 0; tau < ntiles; ++tau) {
+            const St<R>* r = rho + ((b * ntiles + tau) * n_accs + k) * 4;
+            t[0] += as_r<R>(r[0]);
+            t[1] += as_r<R>(r[1]);
+            t[2] += as_r<R>(r[2]);
+        }
+        const DAcc ac = accs[k];
+        acc_terms<R>(ac, entries[ac.entry], t, 1, consts,
+                     x ? x + b * Px : static_cast<const St<R>*>(nullptr), w, cang, cmat, terms + b * n_terms);
     }
 }
 
