@@ -297,12 +297,16 @@ class CircuitBench:
     def launches(self):
         """Library kernels per step: resident forward 1, resident backward 2
         (sweep + fixed-order dw sum); HBM-tiled: one launch per pass plus the
-        partial sums (E; dx and dw); cluster forward 1."""
+        partial sums (E; the per-sample gradient terms, dx and dw); cluster
+        forward 1, cluster backward 2."""
         inf, nx, nw = self.info, self.w_.spec.num_x > 0, self.w_.spec.num_w > 0
         f = inf["fwd_passes"] + 1 if inf["fwd_path"] == 1 else 1
         if not self.w_.backward:
             return f
-        b = inf["bwd_passes"] + int(nx) + int(nw) if inf["bwd_path"] == 1 else 1 + int(nw)
+        if inf["bwd_path"] == 1:
+            b = inf["bwd_passes"] + int(nx or nw) + int(nx) + int(nw)
+        else:
+            b = 1 + int(nw)
         return f + b
 
     def host_step(self, stream_ptr):
