@@ -326,6 +326,7 @@ void fill_plan_args(const HostPlan& p, const Launch& L, KArgs<R>& a) {
     a.n_ps = p.n_ps;
     a.n_sh = p.n_sh;
     a.n_accs = (int)p.accs.size();
+    a.n_ps = p.n_ps;
     a.n_terms = (int)p.term_src.size();
     a.Px = p.num_x;
     a.Pw = p.num_w;
@@ -792,7 +793,7 @@ void forget_plan(const HostPlan* p) {
 // Workspace of the HBM path.  Forward: [control | working state | <Z> partials].
 // Backward: [control | psi | lam | gradient-term partials].
 struct HbmWs {
-    size_t state = 0, lam = 0, part = 0, terms = 0, total = 0;
+    size_t state = 0, lam = 0, part = 0, terms = 0, ps = 0, total = 0;
 };
 
 HbmWs hbm_layout(const HostPlan& p, int mode, int B, int ntiles) {
@@ -802,14 +803,38 @@ HbmWs hbm_layout(const HostPlan& p, int mode, int B, int ntiles) {
     w.state = 256;
     if (mode == 0) {
         w.part = w.state + sbytes;
-        w.total = w.part + align256((size_t)B * ntiles * p.n * rs);
+        w.ps = w.part + align256((size_t)B * ntiles * p.n * rs);
     } else {   // per-tile rho sums [B * ntiles][accs][4], then the per-sample terms [B][terms]
         w.lam = w.state + sbytes;
         w.part = w.lam + sbytes;
         w.terms = w.part + align256((size_t)B * ntiles * std::max<size_t>(p.accs.size(), 1) * 4 * rs);
-        w.total = w.terms + align256((size_t)B * std::max<size_t>(p.term_src.size(), 1) * rs);
+        w.ps = w.terms + align256((size_t)B * std::max<size_t>(p.term_src.size(), 1) * rs);
     }
+    // every sample's per-sample table entries [B][n_ps][entry words]
+    w.total = w.ps + align256((size_t)B * p.n_ps * (p.dtype == VQC_C128 ? 8 : 32) * rs);
     return w;
+}
+
+// Every sample's per-sample table entries into `out` (ps_tables), read by the
+// passes instead of evaluating them once per tile.
+template <typename R>
+vqc_status launch_ps_tables(const HostPlan& p, int B, const void* x, const void* w, void* out,
+                            cudaStream_t stream) {
+    if (p.n_ps == 0) return VQC_OK;
+    const char* base = static_cast<const char*>(p.dbuf);
+    const DEntry* entries = reinterpret_cast<const DEntry*>(base + p.dev_entries);
+    const int32_t* ps_list = reinterpret_cast<const int32_t*>(base + p.dev_ps_list);
+    const DConst* consts = reinterpret_cast<const DConst*>(base + p.dev_consts);
+    const R* cang = reinterpret_cast<const R*>(base + p.dev_cang);
+    const R* cmat = reinterpret_cast<const R*>(base + p.dev_cmat);
+    const R* xr = static_cast<const R*>(x);
+    const R* wr = static_cast<const R*>(w);
+    int Px = p.num_x, Bi = B, nps = p.n_ps;
+    void* args[] = {&entries, &ps_list, &consts, &cang, &cmat, &xr, &Px, &wr, &Bi, &nps, &out};
+    const int blocks = (int)std::min<long long>(4096, ((long long)B * nps + 255) / 256);
+    VQC_CUDA(launch(p.dfloat ? ps_tables_ptr_dd() : ps_tables_ptr(p.dtype == VQC_C128), dim3(std::max(blocks, 1)),
+                    dim3(256), args, 0, stream));
+    return VQC_OK;
 }
 
 template <typename R>
@@ -842,6 +867,7 @@ void fill_pass_args(const HostPlan& p, const PassGeo& L, const DPass& ps, PArgs<
     a.acc_begin = ps.acc_begin;
     a.acc_count = ps.acc_count;
     a.n_accs = (int)p.accs.size();
+    a.n_ps = p.n_ps;
     a.Px = p.num_x;
     a.nunits = L.nunits;
     for (int i = 0; i < 24; ++i) {
@@ -874,10 +900,14 @@ vqc_status run_hbm_forward(const HostPlan& p, int B, const void* x, const void* 
     char* wsc = static_cast<char*>(ws);
     C* W = state_out ? static_cast<C*>(state_out) : reinterpret_cast<C*>(wsc + lay.state);
     R* E_part = reinterpret_cast<R*>(wsc + lay.part);
+    void* ps_g = wsc + lay.ps;
+    st = launch_ps_tables<R>(p, B, x, w, ps_g, stream);
+    if (st != VQC_OK) return st;
     const int np = (int)L.s->passes.size();
     for (int i = 0; i < np; ++i) {
         PArgs<R> a{};
         fill_pass_args<R>(p, L, L.s->passes[i], a);
+        a.ps_g = ps_g;
         a.B = B;
         a.x = static_cast<const R*>(x);
         a.w = static_cast<const R*>(w);
@@ -923,6 +953,11 @@ vqc_status run_hbm_backward(const HostPlan& p, int B, const void* x, const void*
     C* Lam = reinterpret_cast<C*>(wsc + lay.lam);
     R* rho = reinterpret_cast<R*>(wsc + lay.part);
     R* terms = reinterpret_cast<R*>(wsc + lay.terms);
+    void* ps_g = wsc + lay.ps;
+    if (p.dtype == VQC_C128 || !psi_final) {   // complex64 backward passes evaluate their own entries
+        st = launch_ps_tables<R>(p, B, x, w, ps_g, stream);
+        if (st != VQC_OK) return st;
+    }
     const C* src0 = static_cast<const C*>(psi_final);
     if (!src0) {
         // recompute the final state into Psi (the forward passes need no <Z>)
@@ -933,6 +968,7 @@ vqc_status run_hbm_backward(const HostPlan& p, int B, const void* x, const void*
         for (int i = 0; i < npf; ++i) {
             PArgs<R> a{};
             fill_pass_args<R>(p, Lf, Lf.s->passes[i], a);
+            a.ps_g = ps_g;
             a.B = B;
             a.x = static_cast<const R*>(x);
             a.w = static_cast<const R*>(w);
@@ -949,6 +985,7 @@ vqc_status run_hbm_backward(const HostPlan& p, int B, const void* x, const void*
     for (int i = np - 1; i >= 0; --i) {
         PArgs<R> a{};
         fill_pass_args<R>(p, L, L.s->passes[i], a);
+        a.ps_g = ps_g;
         a.B = B;
         a.x = static_cast<const R*>(x);
         a.w = static_cast<const R*>(w);

@@ -27,6 +27,7 @@ const void* sweep_ptr_dd_fused(int K, bool full);
 const void* pass_ptr_dd(int mode, int K, bool full);
 const void* cluster_ptr_dd();
 const void* reduce_terms_ptr_dd();
+const void* ps_tables_ptr_dd();
 
 // HBM-tiled pass kernels (K fixed per type and mode) and partial reductions.
 const void* pass_ptr(bool dbl, int mode, int K, bool full);   // full: tile groups >= 32 threads
@@ -34,6 +35,7 @@ const void* reduce_expz_ptr(bool dbl);
 const void* reduce_dx_ptr(bool dbl);
 const void* reduce_dw_ptr(bool dbl);
 const void* reduce_terms_ptr(bool dbl);   // per-sample gradient terms from per-tile rho sums
+const void* ps_tables_ptr(bool dbl);      // per-sample table entries of every sample (HBM passes)
 const void* reduce_cols_ptr(bool dbl);
 const void* abs2_ptr(bool dbl);   // |psi|^2, elementwise
 const void* cluster_ptr(bool dbl);   // cluster-path forward (K = 5 / 4 for complex64 / 128)

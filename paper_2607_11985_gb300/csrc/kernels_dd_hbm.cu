@@ -1,6 +1,7 @@
 // kernels_dd_hbm.cu -- double-float (complex128 storage) instantiations of the
 // HBM-tiled pass kernels (K = 4 forward, 3 backward, as complex128), of the
-// per-sample gradient-term reduction and of the cluster-path forward (K = 4).
+// per-sample tables and gradient-term reduction and of the cluster-path forward
+// (K = 4).
 #include "cluster.cuh"
 #include "kernels.h"
 #include "pass.cuh"
@@ -17,5 +18,6 @@ const void* pass_ptr_dd(int mode, int K, bool full) {
 
 const void* cluster_ptr_dd() { return reinterpret_cast<const void*>(&cluster_fwd_kernel<dd, 4>); }
 const void* reduce_terms_ptr_dd() { return reinterpret_cast<const void*>(&reduce_terms<dd>); }
+const void* ps_tables_ptr_dd() { return reinterpret_cast<const void*>(&ps_tables<dd>); }
 
 }  // namespace vqc

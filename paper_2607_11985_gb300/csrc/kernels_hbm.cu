@@ -36,6 +36,10 @@ const void* abs2_ptr(bool dbl) {
     return dbl ? reinterpret_cast<const void*>(&abs2_kernel<double>)
                : reinterpret_cast<const void*>(&abs2_kernel<float>);
 }
+const void* ps_tables_ptr(bool dbl) {
+    return dbl ? reinterpret_cast<const void*>(&ps_tables<double>)
+               : reinterpret_cast<const void*>(&ps_tables<float>);
+}
 const void* reduce_terms_ptr(bool dbl) {
     return dbl ? reinterpret_cast<const void*>(&reduce_terms<double>)
                : reinterpret_cast<const void*>(&reduce_terms<float>);

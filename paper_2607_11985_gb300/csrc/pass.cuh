@@ -33,6 +33,9 @@ struct PArgs {
     int n, m, K, tbits, G, S, nout, ntiles;
     int stage_begin, stage_end;
     int ps_begin, ps_count, sh_begin, sh_count, acc_begin, acc_count, n_accs, Px;
+    const void* ps_g;       // per-sample tables of every sample [B][n_ps][entry words] (ps_tables),
+                            // kernel real type (not read by the complex64 backward)
+    int n_ps;
     int B;
     long long nunits;
     uint8_t tile_q[24], out_q[24];
@@ -254,13 +257,29 @@ __global__ void __launch_bounds__(256, 2) pass_kernel(const __grid_constant__ PA
         for (int j = 0; j < A.nout; ++j)
             if ((tau >> j) & 1) tile_base |= 1u << A.out_q[j];
 
-        for (int i = threadIdx.x; i < A.S * A.ps_count; i += nthr) {
-            const int gg = i / A.ps_count, k = i % A.ps_count;
-            const long long tt = min(unit * A.S + gg, total_tiles - 1);
-            const int bb = (int)(tt / A.ntiles);
-            const DEntry e = P_entries[vqc_ld(&P_pass_entries[A.ps_begin + k])];
-            eval_entry<R>(e, P_consts, A.x + (size_t)bb * A.Px, A.w, P_cang, P_cmat,
-                          ps_all + ((size_t)gg * A.ps_count + k) * EntryWords<R>::value);
+        if (MODE == 1 && std::is_same<R, float>::value) {
+            // the complex64 backward evaluates its per-sample entries itself: with
+            // the table copy instead its register allocation spilled more and it
+            // measured 0.7% slower (the other kernels read the table)
+            for (int i = threadIdx.x; i < A.S * A.ps_count; i += nthr) {
+                const int gg = i / A.ps_count, k = i % A.ps_count;
+                const long long tt = min(unit * A.S + gg, total_tiles - 1);
+                const int bb = (int)(tt / A.ntiles);
+                const DEntry e = P_entries[vqc_ld(&P_pass_entries[A.ps_begin + k])];
+                eval_entry<R>(e, P_consts, A.x + (size_t)bb * A.Px, A.w, P_cang, P_cmat,
+                              ps_all + ((size_t)gg * A.ps_count + k) * EntryWords<R>::value);
+            }
+        } else if (A.ps_count) {   // the pass's per-sample entries, copied from the sample's precomputed table
+            constexpr int V = EntryWords<R>::value * (int)sizeof(R) / 16;   // 16-byte vectors per entry
+            const int4* gtab = static_cast<const int4*>(A.ps_g);
+            int4* stab = reinterpret_cast<int4*>(ps_all);
+            const int per = A.ps_count * V;
+            for (int i = threadIdx.x; i < A.S * per; i += nthr) {
+                const int gg = i / per, r = i - gg * per, k = r / V, v = r - k * V;
+                const int bb = (int)(min(unit * A.S + gg, total_tiles - 1) / A.ntiles);
+                const int slot = P_entries[vqc_ld(&P_pass_entries[A.ps_begin + k])].slot;
+                stab[((size_t)gg * A.ps_count + k) * V + v] = gtab[((size_t)bb * A.n_ps + slot) * V + v];
+            }
         }
         const size_t sbase = (size_t)b << n;
         const uint32_t gt = tile_global(u_t, tile_base, A.tile_q, G);
@@ -393,6 +412,25 @@ __global__ void reduce_expz(const R* E_part, int B, int ntiles, int n, R* E) {
         R s = 0;
         for (int t = 0; t < ntiles; ++t) s += E_part[(b * ntiles + t) * n + j];
         E[i] = s;
+    }
+}
+
+// Per-sample table entries of every sample (the x-dependent runs), evaluated
+// once per call for all passes: out [B][n_ps][entry words], in the kernels'
+// real type R (slot order = ps_list order).
+template <typename R>
+__global__ void __launch_bounds__(256) ps_tables(const DEntry* entries, const int32_t* ps_list,
+                                                 const DConst* consts, const R* cang, const R* cmat,
+                                                 const St<R>* x, int Px, const St<R>* w, int B, int n_ps,
+                                                 R* out) {
+    grid_dep_wait();
+    grid_dep_launch();
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < (long long)B * n_ps;
+         i += (long long)gridDim.x * blockDim.x) {
+        const long long b = i / n_ps;
+        const DEntry e = entries[vqc_ld(&ps_list[i % n_ps])];
+        eval_entry<R>(e, consts, x + b * Px, w, cang, cmat,
+                      out + ((size_t)b * n_ps + e.slot) * EntryWords<R>::value);
     }
 }
 
