@@ -297,14 +297,15 @@ class CircuitBench:
     def launches(self):
         """Library kernels per step: resident forward 1, resident backward 2
         (sweep + fixed-order dw sum); HBM-tiled: one launch per pass plus the
-        partial sums (E; the per-sample gradient terms, dx and dw); cluster
-        forward 1, cluster backward 2."""
+        per-sample tables (circuits with x; the complex64 backward from a saved
+        state evaluates its own) and the partial sums (E; the per-sample
+        gradient terms, dx and dw); cluster forward 1, cluster backward 2."""
         inf, nx, nw = self.info, self.w_.spec.num_x > 0, self.w_.spec.num_w > 0
-        f = inf["fwd_passes"] + 1 if inf["fwd_path"] == 1 else 1
+        f = inf["fwd_passes"] + 1 + int(nx) if inf["fwd_path"] == 1 else 1
         if not self.w_.backward:
             return f
         if inf["bwd_path"] == 1:
-            b = inf["bwd_passes"] + int(nx or nw) + int(nx) + int(nw)
+            b = inf["bwd_passes"] + int(nx or nw) + int(nx) + int(nw) + int(nx and self.w_.dtype != "c64")
         else:
             b = 1 + int(nw)
         return f + b

@@ -47,19 +47,23 @@ def test_roofline_bound_is_the_closer_ceiling():
 
 def test_launch_count_per_step():
     """gpu_launches: every library kernel of a step (the driver compares this
-    claim with the ncu launch list): HBM forward = passes + the <Z> sum; HBM
-    backward = passes + per-sample terms + dx sum + dw sum; resident forward 1,
-    backward 2 (sweep + dw sum); cluster backward 2."""
+    claim with the ncu launch list): HBM forward = per-sample tables + passes +
+    the <Z> sum; HBM backward = passes + per-sample terms + dx sum + dw sum
+    (+ the tables outside complex64); resident forward 1, backward 2 (sweep +
+    dw sum); cluster backward 2."""
     class Spec:
         num_x, num_w = 16, 384
 
     class W:
-        spec, backward = Spec(), True
+        spec, backward, dtype = Spec(), True, "c64"
 
     b = bench.CircuitBench.__new__(bench.CircuitBench)
     b.w_ = W()
     b.info = {"fwd_path": 1, "bwd_path": 1, "fwd_passes": 11, "bwd_passes": 12}
-    assert b.launches() == (11 + 1) + (12 + 1 + 1 + 1)
+    assert b.launches() == (11 + 1 + 1) + (12 + 1 + 1 + 1)
+    b.w_.dtype = "c128"   # the complex128 backward reads the per-sample tables too
+    assert b.launches() == (11 + 1 + 1) + (12 + 1 + 1 + 1 + 1)
+    b.w_.dtype = "c64"
     b.info = {"fwd_path": 0, "bwd_path": 0, "fwd_passes": 1, "bwd_passes": 1}
     assert b.launches() == 1 + 2
     b.info = {"fwd_path": 0, "bwd_path": 2, "fwd_passes": 1, "bwd_passes": 1}
